@@ -1,0 +1,192 @@
+"""ctypes front of the C oracle (oracle/tppsd_oracle.c) -- test infrastructure.
+
+Argument marshalling only; every computation happens in the C file.
+"""
+import ctypes as C
+import os
+
+import numpy as np
+
+from . import build as _build
+
+FLAG_NO_BONUS = 1
+_lib = None
+
+_i32p = np.ctypeslib.ndpointer(np.int32, flags="C_CONTIGUOUS")
+_f32p = np.ctypeslib.ndpointer(np.float32, flags="C_CONTIGUOUS")
+_f64p = np.ctypeslib.ndpointer(np.float64, flags="C_CONTIGUOUS")
+_i64p = np.ctypeslib.ndpointer(np.int64, flags="C_CONTIGUOUS")
+_u32p = np.ctypeslib.ndpointer(np.uint32, flags="C_CONTIGUOUS")
+
+
+def _opt(p):
+    """ndpointer that also accepts None."""
+    class _P(p):
+        @classmethod
+        def from_param(cls, obj):
+            if obj is None:
+                return None
+            return p.from_param(obj)
+    return _P
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        path = _build.build()
+        L = C.CDLL(path)
+        L.oracle_philox4x32.argtypes = [_u32p, _u32p, _u32p]
+        L.oracle_uniforms.argtypes = [C.c_uint64, C.c_uint32, C.c_uint32, C.c_uint32, _f64p]
+        L.oracle_round_bf16.argtypes = [C.c_double]
+        L.oracle_round_bf16.restype = C.c_double
+        L.oracle_temporal_encoding.argtypes = [C.c_int32, C.c_double, _f64p]
+        L.oracle_score.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p, _i32p,
+                                   _opt(_f64p), _opt(_f64p), _opt(_f64p), C.c_int32, C.c_int32]
+        L.oracle_sample_ar.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p, _i32p,
+                                       C.c_int32, C.c_uint64, C.c_int32,
+                                       _f64p, _f64p, _i32p, _f64p, C.c_int32]
+        L.oracle_sample_sd.argtypes = [_i32p, _f32p, C.c_int64, _i32p, _f32p, C.c_int64,
+                                       C.c_int32, C.c_int32, _f32p, _i32p, C.c_int32, C.c_int32,
+                                       C.c_uint64, C.c_uint32, C.c_int32,
+                                       _f64p, _f64p, _i32p, _f64p, _i64p, C.c_int32]
+        L.oracle_log_g.argtypes = [C.c_int32, _f64p, C.c_double]
+        L.oracle_log_g.restype = C.c_double
+        L.oracle_log_f.argtypes = [C.c_int32, _f64p, C.c_int32]
+        L.oracle_log_f.restype = C.c_double
+        L.oracle_sample_head.argtypes = [C.c_int32, C.c_int32, _f64p, C.c_int32, C.c_uint64,
+                                         _f64p, _opt(_i32p)]
+        L.oracle_resample_time.argtypes = [C.c_int32, _f64p, _f64p, C.c_int32, C.c_uint64,
+                                           _f64p, _opt(_i32p)]
+        L.oracle_resample_mark.argtypes = [C.c_int32, C.c_int32, _f64p, _f64p, C.c_int32,
+                                           C.c_uint64, _i32p]
+        L.oracle_toy_sd.argtypes = [C.c_int32, C.c_int32, _f64p, _f64p, C.c_int32, C.c_int32,
+                                    C.c_int32, C.c_uint64, C.c_uint32, _f64p, _i32p, _i64p]
+        L.oracle_toy_ar.argtypes = [C.c_int32, C.c_int32, _f64p, C.c_int32, C.c_int32,
+                                    C.c_uint64, _f64p, _i32p]
+        for f in ("oracle_score", "oracle_sample_ar", "oracle_sample_sd", "oracle_toy_sd",
+                  "oracle_toy_ar"):
+            getattr(L, f).restype = C.c_int
+        _lib = L
+    return _lib
+
+
+def _cfg(cfg):
+    return np.array([cfg.layers, cfg.d_model, cfg.heads, cfg.d_ffn, cfg.n_mix, cfg.n_marks,
+                     cfg.dtype], np.int32)
+
+
+def _c(a, dt):
+    return np.ascontiguousarray(a, dtype=dt)
+
+
+def _check(rc, what):
+    if rc != 0:
+        raise ValueError(f"{what} rejected its arguments (rc={rc})")
+
+
+def philox4x32(ctr, key):
+    out = np.zeros(4, np.uint32)
+    lib().oracle_philox4x32(_c(ctr, np.uint32), _c(key, np.uint32), out)
+    return out
+
+
+def uniforms(seed, seq, pos, block):
+    u = np.zeros(4)
+    lib().oracle_uniforms(seed, seq, pos, block, u)
+    return u
+
+
+def round_bf16(x: float) -> float:
+    return lib().oracle_round_bf16(float(x))
+
+
+def temporal_encoding(d: int, t: float):
+    out = np.zeros(d)
+    lib().oracle_temporal_encoding(d, float(t), out)
+    return out
+
+
+def head_width(cfg):
+    return 3 * cfg.n_mix + cfg.n_marks
+
+
+def score(cfg, blob, tau, marks, recompute=False, nthreads=0, heads=True):
+    """Teacher-forced heads and per-event log g / log f of one model."""
+    tau = _c(tau, np.float32)
+    marks = _c(marks, np.int32)
+    B, n = tau.shape
+    hd = np.full((B, n, head_width(cfg)), np.nan) if heads else None
+    lg = np.zeros((B, n))
+    lf = np.zeros((B, n))
+    _check(lib().oracle_score(_cfg(cfg), _c(blob, np.float32), blob.size, B, n, tau, marks,
+                              hd, lg, lf, int(recompute), nthreads), "oracle_score")
+    return hd, lg, lf
+
+
+def sample_ar(cfg_t, blob_t, hist_tau, hist_marks, n_events, seed, recompute=False, nthreads=0):
+    hist_tau = _c(hist_tau, np.float32)
+    hist_marks = _c(hist_marks, np.int32)
+    B, H = hist_tau.shape
+    tau = np.zeros((B, n_events)); t = np.zeros((B, n_events))
+    k = np.zeros((B, n_events), np.int32); mg = np.zeros((B, n_events))
+    _check(lib().oracle_sample_ar(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size, B, H,
+                                  hist_tau, hist_marks, n_events, seed, int(recompute),
+                                  tau, t, k, mg, nthreads), "oracle_sample_ar")
+    return dict(tau=tau, t=t, k=k, margin=mg)
+
+
+def sample_sd(cfg_t, blob_t, cfg_d, blob_d, hist_tau, hist_marks, n_events, gamma, seed,
+              flags=0, recompute=False, nthreads=0):
+    hist_tau = _c(hist_tau, np.float32)
+    hist_marks = _c(hist_marks, np.int32)
+    B, H = hist_tau.shape
+    tau = np.zeros((B, n_events)); t = np.zeros((B, n_events))
+    k = np.zeros((B, n_events), np.int32); mg = np.zeros((B, n_events))
+    st = np.zeros((B, 5), np.int64)
+    _check(lib().oracle_sample_sd(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size,
+                                  _cfg(cfg_d), _c(blob_d, np.float32), blob_d.size, B, H,
+                                  hist_tau, hist_marks, n_events, gamma, seed, flags,
+                                  int(recompute), tau, t, k, mg, st, nthreads),
+           "oracle_sample_sd")
+    return dict(tau=tau, t=t, k=k, margin=mg, stats=st)
+
+
+def log_g(M, head, tau):
+    head = _c(head, np.float64)
+    return np.array([lib().oracle_log_g(M, head, float(x)) for x in np.atleast_1d(tau)])
+
+
+def sample_head(M, K, head, n, seed):
+    tau = np.zeros(n); k = np.zeros(n, np.int32)
+    lib().oracle_sample_head(M, K, _c(head, np.float64), n, seed, tau, k)
+    return tau, k
+
+
+def resample_time(M, head_t, head_d, n, seed):
+    tau = np.zeros(n); it = np.zeros(n, np.int32)
+    lib().oracle_resample_time(M, _c(head_t, np.float64), _c(head_d, np.float64), n, seed, tau, it)
+    return tau, it
+
+
+def resample_mark(M, K, head_t, head_d, n, seed):
+    k = np.zeros(n, np.int32)
+    lib().oracle_resample_mark(M, K, _c(head_t, np.float64), _c(head_d, np.float64), n, seed, k)
+    return k
+
+
+def toy_sd(M, K, table_t, table_d, B, N, gamma, seed, flags=0):
+    tau = np.zeros((B, N)); k = np.zeros((B, N), np.int32); st = np.zeros((B, 5), np.int64)
+    _check(lib().oracle_toy_sd(M, K, _c(table_t, np.float64), _c(table_d, np.float64), B, N,
+                               gamma, seed, flags, tau, k, st), "oracle_toy_sd")
+    return tau, k, st
+
+
+def toy_ar(M, K, table_t, B, N, seed):
+    tau = np.zeros((B, N)); k = np.zeros((B, N), np.int32)
+    _check(lib().oracle_toy_ar(M, K, _c(table_t, np.float64), B, N, seed, tau, k),
+           "oracle_toy_ar")
+    return tau, k
+
+
+def cores() -> int:
+    return os.cpu_count() or 1
