@@ -1,0 +1,167 @@
+/*
+ * tppsd.h -- C ABI of the GB300 TPP-SD sampler.
+ *
+ * TPP-SD (arxiv 2507.09252) samples a marked temporal point process from a
+ * large "target" Transformer TPP by letting a small "draft" Transformer TPP
+ * propose gamma events, verifying all of them with one causal target pass,
+ * and resampling the first rejected event from the adjusted distribution
+ * (Sec. 4.3, Alg. 1, Eq. 3-4, Theorem 1).  The output has the law of plain
+ * autoregressive sampling from the target (App. A.2).
+ *
+ * Conventions for every entry point:
+ *  - Status codes are returned; nothing throws or exits across the ABI.  On
+ *    an error the context stays usable and outputs are unspecified.
+ *  - A context must not be used by two host threads at once.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Work is enqueued on it; calls return before the GPU is done
+ *    unless stated otherwise.
+ *  - Array arguments are caller-owned.  Unless stated otherwise they may be
+ *    host memory (pageable or pinned) or device memory: the library detects
+ *    which and stages host data through its own device buffers on `stream`.
+ *    Host outputs are complete when the stream has been synchronised
+ *    (tppsd_wait); pageable host outputs are complete on return.
+ *  - Sequences are independent; sequence b uses random slots keyed by b.
+ */
+#ifndef TPPSD_H
+#define TPPSD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct tppsd_ctx tppsd_ctx; /* opaque, owned by the library */
+
+typedef enum {
+    TPPSD_OK = 0,
+    TPPSD_ERR_INVALID_ARG = -1,  /* bad size, pointer, config or call order */
+    TPPSD_ERR_OOM = -2,          /* device or host allocation failed */
+    TPPSD_ERR_CUDA = -3,         /* a CUDA call failed; see tppsd_last_error */
+    TPPSD_ERR_UNSUPPORTED = -4,  /* shape outside the compiled kernels' range */
+    TPPSD_ERR_ROUND_LIMIT = -5,  /* the round loop stopped at its safety cap */
+    TPPSD_ERR_TIMEOUT = -6,      /* tppsd_wait gave up before the GPU finished */
+    TPPSD_ERR_NO_DEVICE = -7,    /* no CUDA device / driver */
+    TPPSD_WARN_RESAMPLE_CAP = 1  /* a Theorem-1 loop hit its iteration cap */
+} tppsd_status_t;
+
+/* Model shape.  Weight blob layout (float32 values, row-major [out][in],
+ * y = W x + b), in this order:
+ *   type_emb [K][d]                                  (W of Sec. 4.2)
+ *   for each layer: w_qkv [3d][d], b_qkv [3d], w_o [d][d], b_o [d],
+ *                   ln1_g [d], ln1_b [d], w_1 [F][d], b_1 [F],
+ *                   w_2 [d][F], b_2 [d], ln2_g [d], ln2_b [d]
+ *   E [3d][d]                                        (e = E h, no bias)
+ *   v_w [M][d], b_w [M], v_mu [M][d], b_mu [M], v_s [M][d], b_s [M]
+ *   v_k1 [d][d], b_k1 [d], v_k2 [K][d], b_k2 [K]
+ * Model (Sec. 4.2): x_i = z(t_i) + W[k_i] with the THP temporal encoding
+ * z_2j = sin(t w_j), z_2j+1 = cos(t w_j), w_j = 10000^(-2j/d), t absolute
+ * (App. D.4); post-LN layers h <- LN(h + MHA(h)), h <- LN(h + W2 ReLU(W1 h
+ * + b1) + b2) with causal softmax attention (scale 1/sqrt(d/heads)),
+ * LayerNorm eps 1e-5; heads: w = softmax(v_w e1 + b_w), mu = v_mu e2 + b_mu,
+ * sigma = exp(v_s e3 + b_s), f = softmax(v_k2 tanh(v_k1 h + b_k1) + b_k2).
+ * dtype 0 = fp32 throughout.  dtype 1 = bf16: the blob's values must be
+ * bf16-representable; GEMM inputs and Q/K/V are rounded to bf16 (nearest
+ * even), accumulation, LayerNorm, softmax, heads and sampling are fp32. */
+typedef struct {
+    int32_t layers;   /* 1..16 */
+    int32_t d_model;  /* multiple of 16, <= 512 */
+    int32_t heads;    /* 1..8 (draft: 1, 2 or 4); d_model / heads in {8, 16, 32, 64} */
+    int32_t d_ffn;    /* multiple of 16, <= 4096 */
+    int32_t n_mix;    /* M, 1..64 */
+    int32_t n_marks;  /* K, 1..256; equal for target and draft */
+    int32_t dtype;    /* 0 fp32, 1 bf16 */
+} tppsd_model_cfg;
+
+/* Counters of the last tppsd_sample / tppsd_sample_autoregressive call. */
+typedef struct {
+    int64_t rounds;          /* (sequence, round) pairs; AR: events sampled */
+    int64_t drafted;         /* draft events proposed (gamma per pair) */
+    int64_t accepted;        /* drafts accepted before the first rejection */
+    int64_t emitted;         /* events written, before truncation to n_events */
+    int64_t resample_iters;  /* Theorem-1 loop iterations */
+    int64_t cap_hits;        /* Theorem-1 loops stopped by the cap */
+    int64_t loop_iters;      /* device round-loop iterations */
+    int64_t kernel_launches; /* kernels launched by the call */
+    int64_t target_keys;     /* sum over (sequence, target pass) of cached keys read per layer */
+    int64_t draft_keys;      /* sum over draft positions encoded of keys read per layer */
+    int64_t prefill_launches;/* kernels launched by the last tppsd_prefill */
+} tppsd_stats;
+
+/* Number of floats a blob of this shape must hold (0 if unsupported). */
+size_t tppsd_blob_floats(const tppsd_model_cfg* cfg);
+
+/* Uploads both models and allocates KV caches and buffers for up to
+ * max_batch sequences of max_positions events (history + generated +
+ * gamma + 1) and draft length up to max_gamma.  Blobs: host or device
+ * float arrays of tppsd_blob_floats() values, copied.  *out receives the
+ * context, or NULL on error. */
+tppsd_status_t tppsd_create_models(const tppsd_model_cfg* target, const tppsd_model_cfg* draft,
+                                   const float* target_blob, size_t target_floats,
+                                   const float* draft_blob, size_t draft_floats,
+                                   int32_t max_batch, int32_t max_positions, int32_t max_gamma,
+                                   tppsd_ctx** out);
+
+/* Binds the history of `batch` sequences and encodes it with both models
+ * (KV caches of events 0..hist_len-2; event hist_len-1 is encoded by the
+ * first verify pass).  hist_tau [batch][hist_len] inter-event times
+ * (t_1 = tau_1, t_i = t_{i-1} + tau_i, summed in fp64), hist_marks
+ * [batch][hist_len] in 0..K-1 (values outside are clamped into range).
+ * hist_len >= 1. */
+tppsd_status_t tppsd_prefill(tppsd_ctx* ctx, int32_t batch, const float* hist_tau,
+                             const int32_t* hist_marks, int32_t hist_len, void* stream);
+
+#define TPPSD_FLAG_NO_BONUS 1u  /* no extra target event after a full accept */
+#define TPPSD_FLAG_HOST_LOOP 2u /* round loop driven from the host (debug) */
+#define TPPSD_FLAG_PROFILE 4u   /* host-driven loop with CUDA events around every kernel */
+
+/* TPP-SD (Sec. 4.3, Alg. 1): draws n_events events after the prefilled
+ * history of each of the first `batch` sequences, with gamma drafts per
+ * round.  Uniforms: Philox4x32-10 keyed by `seed`, counter (event index,
+ * block, sequence, 0).  Outputs [batch][n_events]: out_tau inter-event
+ * times (fp32), out_t absolute times (fp64), out_marks.  Each call restarts
+ * from the prefilled history. */
+tppsd_status_t tppsd_sample(tppsd_ctx* ctx, int32_t batch, int32_t n_events, int32_t gamma,
+                            uint64_t seed, uint32_t flags, float* out_tau, double* out_t,
+                            int32_t* out_marks, void* stream);
+
+/* Target-only autoregressive sampling (Sec. 4.2), same slots and outputs. */
+tppsd_status_t tppsd_sample_autoregressive(tppsd_ctx* ctx, int32_t batch, int32_t n_events,
+                                           uint64_t seed, uint32_t flags, float* out_tau,
+                                           double* out_t, int32_t* out_marks, void* stream);
+
+/* Teacher-forced scoring with one model (which 0 = target, 1 = draft): for
+ * sequences tau/marks [batch][len], out_heads [batch][len][3M+K] (may be
+ * NULL) gets the head after events 0..i at row i (row len-1 untouched):
+ * [log w | mu | log sigma | log f]; out_logg / out_logf [batch][len] (may
+ * be NULL) get log g(tau_i | h_{i-1}) and log f(k_i | h_{i-1}) (Eq. 2
+ * terms), NaN at i = 0.  Overwrites the caches: prefill again before
+ * sampling. */
+tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
+                           const float* tau, const int32_t* marks, float* out_heads,
+                           float* out_logg, float* out_logf, void* stream);
+
+/* Synchronises the last stream used and copies the last call's counters.
+ * Returns that call's status (OK, WARN_RESAMPLE_CAP or ERR_ROUND_LIMIT). */
+tppsd_status_t tppsd_get_stats(tppsd_ctx* ctx, tppsd_stats* out);
+
+/* Per-kernel-class device time of the last call made with
+ * TPPSD_FLAG_PROFILE (synchronises): ms[TPPSD_KERNEL_CLASSES] total
+ * milliseconds measured with CUDA events on the call's stream, launches[]
+ * counts.  Class names: tppsd_kernel_class_name(i). */
+#define TPPSD_KERNEL_CLASSES 13
+tppsd_status_t tppsd_kernel_times(tppsd_ctx* ctx, double* ms, int64_t* launches);
+const char* tppsd_kernel_class_name(int32_t cls);
+
+/* Host watchdog: waits at most timeout_ms for the last call's work. */
+tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms);
+
+const char* tppsd_status_str(tppsd_status_t status);
+const char* tppsd_last_error(const tppsd_ctx* ctx); /* "" if none */
+void tppsd_destroy(tppsd_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -43,11 +43,11 @@ def lib():
         L.oracle_score.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p, _i32p,
                                    _opt(_f64p), _opt(_f64p), _opt(_f64p), C.c_int32, C.c_int32]
         L.oracle_sample_ar.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p, _i32p,
-                                       C.c_int32, C.c_uint64, C.c_int32,
+                                       C.c_int32, C.c_uint64, C.c_int32, _opt(_i32p),
                                        _f64p, _f64p, _i32p, _f64p, C.c_int32]
         L.oracle_sample_sd.argtypes = [_i32p, _f32p, C.c_int64, _i32p, _f32p, C.c_int64,
                                        C.c_int32, C.c_int32, _f32p, _i32p, C.c_int32, C.c_int32,
-                                       C.c_uint64, C.c_uint32, C.c_int32,
+                                       C.c_uint64, C.c_uint32, C.c_int32, _opt(_i32p),
                                        _f64p, _f64p, _i32p, _f64p, _i64p, C.c_int32]
         L.oracle_log_g.argtypes = [C.c_int32, _f64p, C.c_double]
         L.oracle_log_g.restype = C.c_double
@@ -123,7 +123,17 @@ def score(cfg, blob, tau, marks, recompute=False, nthreads=0, heads=True):
     return hd, lg, lf
 
 
-def sample_ar(cfg_t, blob_t, hist_tau, hist_marks, n_events, seed, recompute=False, nthreads=0):
+def _ids(seq_ids, B):
+    if seq_ids is None:
+        return None
+    ids = np.ascontiguousarray(seq_ids, np.int32)
+    if ids.shape != (B,):
+        raise ValueError("seq_ids must have one entry per sequence")
+    return ids
+
+
+def sample_ar(cfg_t, blob_t, hist_tau, hist_marks, n_events, seed, recompute=False, nthreads=0,
+              seq_ids=None):
     hist_tau = _c(hist_tau, np.float32)
     hist_marks = _c(hist_marks, np.int32)
     B, H = hist_tau.shape
@@ -131,12 +141,12 @@ def sample_ar(cfg_t, blob_t, hist_tau, hist_marks, n_events, seed, recompute=Fal
     k = np.zeros((B, n_events), np.int32); mg = np.zeros((B, n_events))
     _check(lib().oracle_sample_ar(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size, B, H,
                                   hist_tau, hist_marks, n_events, seed, int(recompute),
-                                  tau, t, k, mg, nthreads), "oracle_sample_ar")
+                                  _ids(seq_ids, B), tau, t, k, mg, nthreads), "oracle_sample_ar")
     return dict(tau=tau, t=t, k=k, margin=mg)
 
 
 def sample_sd(cfg_t, blob_t, cfg_d, blob_d, hist_tau, hist_marks, n_events, gamma, seed,
-              flags=0, recompute=False, nthreads=0):
+              flags=0, recompute=False, nthreads=0, seq_ids=None):
     hist_tau = _c(hist_tau, np.float32)
     hist_marks = _c(hist_marks, np.int32)
     B, H = hist_tau.shape
@@ -146,7 +156,7 @@ def sample_sd(cfg_t, blob_t, cfg_d, blob_d, hist_tau, hist_marks, n_events, gamm
     _check(lib().oracle_sample_sd(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size,
                                   _cfg(cfg_d), _c(blob_d, np.float32), blob_d.size, B, H,
                                   hist_tau, hist_marks, n_events, gamma, seed, flags,
-                                  int(recompute), tau, t, k, mg, st, nthreads),
+                                  int(recompute), _ids(seq_ids, B), tau, t, k, mg, st, nthreads),
            "oracle_sample_sd")
     return dict(tau=tau, t=t, k=k, margin=mg, stats=st)
 

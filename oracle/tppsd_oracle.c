@@ -569,7 +569,7 @@ static void store_out(const evbuf *ev, int H, int N, int64_t b, double *o_tau, d
 
 int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
-                     int32_t N, uint64_t seed, int32_t recompute,
+                     int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                      int32_t nthreads)
 {
@@ -584,7 +584,7 @@ int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
         evbuf_alloc(&ev, cap);
         tstate_init(&ts, &mT, cap, recompute);
         load_history(&ev, hist_tau + (int64_t)b * H, hist_marks + (int64_t)b * H, H);
-        ar_sequence(&TRANSFORMER_OPS, &ts, &ev, H, N, seed, (uint32_t)b);
+        ar_sequence(&TRANSFORMER_OPS, &ts, &ev, H, N, seed, (uint32_t)(seq_ids ? seq_ids[b] : b));
         store_out(&ev, H, N, b, out_tau, out_t, out_k, out_margin);
         tstate_free(&ts);
         evbuf_free(&ev);
@@ -596,6 +596,7 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      const int32_t cfgD[7], const float *blobD, int64_t nD,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
+                     const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                      int64_t *stats, int32_t nthreads)
 {
@@ -613,7 +614,7 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
         tstate_init(&ds, &mD, cap, recompute);
         load_history(&ev, hist_tau + (int64_t)b * H, hist_marks + (int64_t)b * H, H);
         sd_sequence(&TRANSFORMER_OPS, &ts, &TRANSFORMER_OPS, &ds, &ev, H, N, gamma, seed,
-                    (uint32_t)b, flags, st);
+                    (uint32_t)(seq_ids ? seq_ids[b] : b), flags, st);
         store_out(&ev, H, N, b, out_tau, out_t, out_k, out_margin);
         if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
         tstate_free(&ts);

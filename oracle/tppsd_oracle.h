@@ -40,10 +40,12 @@ int oracle_score(const int32_t cfg[7], const float *blob, int64_t blob_floats,
 
 /* Naive autoregressive sampling from the target (Sec. 4.2).  History
  * tau/marks are [B][H]; outputs [B][N]: inter-event time, absolute time,
- * mark, and the smallest decision margin taken at that event. */
+ * mark, and the smallest decision margin taken at that event.  seq_ids
+ * (may be NULL = 0..B-1) gives each row's sequence index, which keys its
+ * random slots. */
 int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
-                     int32_t N, uint64_t seed, int32_t recompute,
+                     int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                      int32_t nthreads);
 
@@ -54,6 +56,7 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      const int32_t cfgD[7], const float *blobD, int64_t nD,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
+                     const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                      int64_t *stats, int32_t nthreads);
 

@@ -1,0 +1,719 @@
+// C ABI of the TPP-SD sampler (include/tppsd.h): context, weight upload,
+// prefill, the device-resident round loop, scoring, status and stats.
+//
+// The sampling loop of Alg. 1 runs without host round trips: one round
+// (draft -> verify forward -> heads -> epilogue -> control) is captured once
+// into the body of a CUDA-graph WHILE node; k_round_control sets the loop
+// condition from the device.  Per-call values (history length, event count,
+// seed, output pointers) live in device memory, so one instantiated graph
+// serves every call with the same (batch, gamma, flags).
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <chrono>
+#include <map>
+#include <new>
+#include <string>
+#include <thread>
+#include <tuple>
+#include <vector>
+
+#include "../../include/tppsd.h"
+#include "engine.h"
+
+using namespace tppsd;
+
+namespace {
+
+struct HostModel {
+    tppsd_model_cfg cfg{};
+    DevModel dm{};
+    void* dbuf = nullptr;
+};
+
+struct GraphEntry {
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    int launches_per_round = 0;
+};
+
+// CUDA events around every launch of a profiled call, accumulated per class.
+struct Profiler {
+    std::vector<cudaEvent_t> pool;
+    std::vector<std::pair<int, int>> spans;  // (class, index of begin event)
+    size_t used = 0;
+    int open_cls = -1, open_ev = -1;
+    cudaError_t err = cudaSuccess;
+    cudaEvent_t next() {
+        if (used == pool.size()) {
+            cudaEvent_t e;
+            cudaError_t r = cudaEventCreate(&e);
+            if (r != cudaSuccess) { err = r; return nullptr; }
+            pool.push_back(e);
+        }
+        return pool[used++];
+    }
+    void reset() { used = 0; spans.clear(); err = cudaSuccess; }
+    static void mark(void* self, int cls, int begin, cudaStream_t st) {
+        Profiler* p = (Profiler*)self;
+        cudaEvent_t e = p->next();
+        if (!e) return;
+        cudaError_t r = cudaEventRecord(e, st);
+        if (r != cudaSuccess) p->err = r;
+        if (begin) p->spans.emplace_back(cls, (int)(p->used - 1));
+    }
+};
+
+}  // namespace
+
+struct tppsd_ctx {
+    int device = 0;
+    HostModel T, D;
+    int max_batch = 0, n_max = 0, max_gamma = 0;
+    SeqState ss{};
+    KVCache kvT{}, kvD{};
+    Work work{};
+    float* draft_heads = nullptr;
+    CallParams* d_params = nullptr;
+    DevStats* d_stats = nullptr;
+    int* d_active = nullptr;
+    int* h_active = nullptr;  // pinned
+    cudaStream_t cap_stream = nullptr;
+    cudaEvent_t done_event = nullptr;
+    cudaStream_t last_stream = nullptr;
+    std::map<std::tuple<int, int, int, unsigned>, GraphEntry> graphs;
+    // staging of host outputs
+    void* stage = nullptr;
+    size_t stage_bytes = 0;
+    // state
+    int prefill_batch = 0, hist_len = 0;
+    bool prefilled = false;
+    int last_launches = 0;
+    int prefill_launches = 0;
+    Profiler prof;
+    bool profiled = false;
+    std::string err;
+    std::vector<void*> allocs;
+};
+
+// ---------------------------------------------------------------- helpers
+static const char* fault_mode() {
+    const char* f = getenv("TPPSD_FAULT");
+    return f ? f : "";
+}
+
+#define CK(expr)                                                                   \
+    do {                                                                           \
+        cudaError_t e_ = (expr);                                                   \
+        if (e_ != cudaSuccess) {                                                   \
+            if (ctx) ctx->err = std::string(#expr) + ": " + cudaGetErrorString(e_); \
+            return e_ == cudaErrorMemoryAllocation ? TPPSD_ERR_OOM : TPPSD_ERR_CUDA; \
+        }                                                                          \
+    } while (0)
+
+static bool is_device_ptr(const void* p) {
+    if (!p) return false;
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+static bool cfg_ok(const tppsd_model_cfg* c) {
+    if (!c) return false;
+    if (c->layers < 1 || c->layers > MAX_LAYERS) return false;
+    if (c->d_model < 16 || c->d_model > MAX_D || c->d_model % 16) return false;
+    if (c->heads < 1 || c->heads > 8 || c->d_model % c->heads) return false;
+    const int dh = c->d_model / c->heads;
+    if (dh != 8 && dh != 16 && dh != 32 && dh != 64) return false;
+    if (c->d_ffn < 16 || c->d_ffn > 4096 || c->d_ffn % 16) return false;
+    if (c->n_mix < 1 || c->n_mix > MAX_MIX) return false;
+    if (c->n_marks < 1 || c->n_marks > MAX_MARKS) return false;
+    return c->dtype == 0 || c->dtype == 1;
+}
+
+extern "C" size_t tppsd_blob_floats(const tppsd_model_cfg* c) {
+    if (!cfg_ok(c)) return 0;
+    const size_t L = c->layers, d = c->d_model, F = c->d_ffn, M = c->n_mix, K = c->n_marks;
+    const size_t layer = 3 * d * d + 3 * d + d * d + d + 2 * d + F * d + F + d * F + d + 2 * d;
+    return K * d + L * layer + 3 * d * d + 3 * (M * d + M) + d * d + d + K * d + K;
+}
+
+static uint16_t f32_to_bf16_bits(float f) {
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    u += 0x7FFFu + ((u >> 16) & 1u);  // nearest, ties to even (finite inputs)
+    return (uint16_t)(u >> 16);
+}
+
+// Lays one model out in a single device buffer: storage-type GEMM matrices
+// first, then fp32 vectors, embeddings and head, then the fp64 frequency
+// table; every piece 16-byte aligned.
+static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_model_cfg* cfg,
+                                   const float* blob_any, size_t nfloats) {
+    hm.cfg = *cfg;
+    const int L = cfg->layers, d = cfg->d_model, F = cfg->d_ffn, M = cfg->n_mix, K = cfg->n_marks;
+    std::vector<float> blob(nfloats);
+    if (is_device_ptr(blob_any)) {
+        CK(cudaMemcpy(blob.data(), blob_any, nfloats * sizeof(float), cudaMemcpyDeviceToHost));
+    } else {
+        memcpy(blob.data(), blob_any, nfloats * sizeof(float));
+    }
+    // blob offsets (include/tppsd.h layout)
+    size_t o = 0;
+    auto take = [&](size_t n) { size_t r = o; o += n; return r; };
+    const size_t o_emb = take((size_t)K * d);
+    struct LO { size_t wqkv, bqkv, wo, bo, g1, b1n, w1, b1, w2, b2, g2, b2n; };
+    std::vector<LO> lo(L);
+    for (int l = 0; l < L; ++l) {
+        lo[l].wqkv = take(3 * (size_t)d * d); lo[l].bqkv = take(3 * d);
+        lo[l].wo = take((size_t)d * d); lo[l].bo = take(d);
+        lo[l].g1 = take(d); lo[l].b1n = take(d);
+        lo[l].w1 = take((size_t)F * d); lo[l].b1 = take(F);
+        lo[l].w2 = take((size_t)d * F); lo[l].b2 = take(d);
+        lo[l].g2 = take(d); lo[l].b2n = take(d);
+    }
+    const size_t oE = take(3 * (size_t)d * d);
+    const size_t ovw = take((size_t)M * d), obw = take(M), ovm = take((size_t)M * d), obm = take(M);
+    const size_t ovs = take((size_t)M * d), obs = take(M);
+    const size_t ok1 = take((size_t)d * d), obk1 = take(d), ok2 = take((size_t)K * d), obk2 = take(K);
+    if (o != nfloats) {
+        ctx->err = "blob size does not match the model shape";
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    std::vector<char> buf;
+    auto add = [&](const void* src, size_t bytes) {
+        size_t off = (buf.size() + 15) & ~(size_t)15;
+        buf.resize(off + bytes);
+        memcpy(buf.data() + off, src, bytes);
+        return off;
+    };
+    const bool bf = cfg->dtype == 1;
+    auto add_mat = [&](size_t off, size_t n) {
+        if (!bf) return add(blob.data() + off, n * sizeof(float));
+        std::vector<uint16_t> t(n);
+        for (size_t i = 0; i < n; ++i) t[i] = f32_to_bf16_bits(blob[off + i]);
+        return add(t.data(), n * 2);
+    };
+    auto add_vec = [&](size_t off, size_t n) { return add(blob.data() + off, n * sizeof(float)); };
+    struct LB { size_t wqkv, bqkv, wo, bo, g1, b1n, w1, b1, w2, b2, g2, b2n; };
+    std::vector<LB> lb(L);
+    for (int l = 0; l < L; ++l) {
+        lb[l].wqkv = add_mat(lo[l].wqkv, 3 * (size_t)d * d);
+        lb[l].wo = add_mat(lo[l].wo, (size_t)d * d);
+        lb[l].w1 = add_mat(lo[l].w1, (size_t)F * d);
+        lb[l].w2 = add_mat(lo[l].w2, (size_t)d * F);
+    }
+    for (int l = 0; l < L; ++l) {
+        lb[l].bqkv = add_vec(lo[l].bqkv, 3 * d); lb[l].bo = add_vec(lo[l].bo, d);
+        lb[l].g1 = add_vec(lo[l].g1, d); lb[l].b1n = add_vec(lo[l].b1n, d);
+        lb[l].b1 = add_vec(lo[l].b1, F); lb[l].b2 = add_vec(lo[l].b2, d);
+        lb[l].g2 = add_vec(lo[l].g2, d); lb[l].b2n = add_vec(lo[l].b2n, d);
+    }
+    const size_t b_emb = add_vec(o_emb, (size_t)K * d);
+    const size_t bE = add_vec(oE, 3 * (size_t)d * d);
+    const size_t bvw = add_vec(ovw, (size_t)M * d), bbw = add_vec(obw, M);
+    const size_t bvm = add_vec(ovm, (size_t)M * d), bbm = add_vec(obm, M);
+    const size_t bvs = add_vec(ovs, (size_t)M * d), bbs = add_vec(obs, M);
+    const size_t bk1 = add_vec(ok1, (size_t)d * d), bbk1 = add_vec(obk1, d);
+    const size_t bk2 = add_vec(ok2, (size_t)K * d), bbk2 = add_vec(obk2, K);
+    std::vector<double> omega(d / 2);
+    for (int i = 0; i < d / 2; ++i) omega[i] = pow(10000.0, -2.0 * i / (double)d);
+    const size_t b_om = add(omega.data(), omega.size() * sizeof(double));
+    buf.resize((buf.size() + 15) & ~(size_t)15);
+    CK(cudaMalloc(&hm.dbuf, buf.size()));
+    ctx->allocs.push_back(hm.dbuf);
+    CK(cudaMemcpy(hm.dbuf, buf.data(), buf.size(), cudaMemcpyHostToDevice));
+    const char* b = (const char*)hm.dbuf;
+    DevModel& m = hm.dm;
+    m.L = L; m.d = d; m.nh = cfg->heads; m.dh = d / cfg->heads; m.F = F; m.M = M; m.K = K;
+    m.dtype = cfg->dtype;
+    m.type_emb = (const float*)(b + b_emb);
+    m.omega = (const double*)(b + b_om);
+    for (int l = 0; l < L; ++l) {
+        LayerW& w = m.layer[l];
+        w.w_qkv = b + lb[l].wqkv; w.b_qkv = (const float*)(b + lb[l].bqkv);
+        w.w_o = b + lb[l].wo; w.b_o = (const float*)(b + lb[l].bo);
+        w.ln1_g = (const float*)(b + lb[l].g1); w.ln1_b = (const float*)(b + lb[l].b1n);
+        w.w_1 = b + lb[l].w1; w.b_1 = (const float*)(b + lb[l].b1);
+        w.w_2 = b + lb[l].w2; w.b_2 = (const float*)(b + lb[l].b2);
+        w.ln2_g = (const float*)(b + lb[l].g2); w.ln2_b = (const float*)(b + lb[l].b2n);
+    }
+    HeadW& h = m.head;
+    h.E = (const float*)(b + bE);
+    h.v_w = (const float*)(b + bvw); h.b_w = (const float*)(b + bbw);
+    h.v_mu = (const float*)(b + bvm); h.b_mu = (const float*)(b + bbm);
+    h.v_s = (const float*)(b + bvs); h.b_s = (const float*)(b + bbs);
+    h.v_k1 = (const float*)(b + bk1); h.b_k1 = (const float*)(b + bbk1);
+    h.v_k2 = (const float*)(b + bk2); h.b_k2 = (const float*)(b + bbk2);
+    m.base = b;
+    m.bytes = buf.size();
+    return TPPSD_OK;
+}
+
+template <typename P>
+static tppsd_status_t dalloc(tppsd_ctx* ctx, P** p, size_t bytes) {
+    void* q = nullptr;
+    CK(cudaMalloc(&q, bytes ? bytes : 16));
+    ctx->allocs.push_back(q);
+    *p = (P*)q;
+    return TPPSD_OK;
+}
+
+#define TRY(x)                               \
+    do {                                     \
+        tppsd_status_t s_ = (x);             \
+        if (s_ != TPPSD_OK) return s_;       \
+    } while (0)
+
+static tppsd_status_t alloc_kv(tppsd_ctx* ctx, KVCache& kv, const tppsd_model_cfg& c) {
+    const size_t el = c.dtype == 1 ? 2 : 4;
+    const size_t n = (size_t)c.layers * ctx->max_batch * ctx->n_max * c.d_model;
+    TRY(dalloc(ctx, &kv.k, n * el));
+    TRY(dalloc(ctx, &kv.v, n * el));
+    kv.Bmax = ctx->max_batch;
+    kv.n_max = ctx->n_max;
+    return TPPSD_OK;
+}
+
+static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
+                                  const tppsd_model_cfg* draft, const float* tb, size_t tn,
+                                  const float* db, size_t dn) {
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) {
+        cudaGetLastError();
+        ctx->err = "no CUDA device";
+        return TPPSD_ERR_NO_DEVICE;
+    }
+    CK(cudaGetDevice(&ctx->device));
+    TRY(upload_model(ctx, ctx->T, target, tb, tn));
+    TRY(upload_model(ctx, ctx->D, draft, db, dn));
+    const int B = ctx->max_batch, nm = ctx->n_max;
+    SeqState& ss = ctx->ss;
+    ss.n_max = nm;
+    TRY(dalloc(ctx, &ss.tau, sizeof(float) * (size_t)B * nm));
+    TRY(dalloc(ctx, &ss.t, sizeof(double) * (size_t)B * nm));
+    TRY(dalloc(ctx, &ss.k, sizeof(int) * (size_t)B * nm));
+    TRY(dalloc(ctx, &ss.n_emit, sizeof(int) * B));
+    TRY(dalloc(ctx, &ss.n_draft, sizeof(int) * B));
+    TRY(dalloc(ctx, &ss.done, sizeof(int) * B));
+    CK(cudaMemset(ss.tau, 0, sizeof(float) * (size_t)B * nm));
+    CK(cudaMemset(ss.t, 0, sizeof(double) * (size_t)B * nm));
+    CK(cudaMemset(ss.k, 0, sizeof(int) * (size_t)B * nm));
+    CK(cudaMemset(ss.done, 1, sizeof(int) * B));
+    TRY(alloc_kv(ctx, ctx->kvT, *target));
+    TRY(alloc_kv(ctx, ctx->kvD, *draft));
+    Work& w = ctx->work;
+    w.R = B * (ctx->max_gamma + 1);
+    if (w.R < 2048) w.R = 2048;
+    const int dmax = target->d_model > draft->d_model ? target->d_model : draft->d_model;
+    const int fmax = target->d_ffn > draft->d_ffn ? target->d_ffn : draft->d_ffn;
+    const int hwT = 3 * target->n_mix + target->n_marks, hwD = 3 * draft->n_mix + draft->n_marks;
+    const int hw = hwT > hwD ? hwT : hwD;
+    const size_t R = w.R;
+    TRY(dalloc(ctx, &w.row_seq, sizeof(int) * R));
+    TRY(dalloc(ctx, &w.row_pos, sizeof(int) * R));
+    TRY(dalloc(ctx, &w.x, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.y, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.xb, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.q, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.att, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.hid, sizeof(float) * R * fmax));
+    TRY(dalloc(ctx, &w.heads, sizeof(float) * R * hw));
+    TRY(dalloc(ctx, &ctx->draft_heads, sizeof(float) * (size_t)B * ctx->max_gamma * hwD));
+    TRY(dalloc(ctx, &ctx->d_params, sizeof(CallParams)));
+    TRY(dalloc(ctx, &ctx->d_stats, sizeof(DevStats)));
+    TRY(dalloc(ctx, &ctx->d_active, sizeof(int)));
+    CK(cudaMemset(ctx->d_stats, 0, sizeof(DevStats)));
+    CK(cudaMallocHost(&ctx->h_active, sizeof(int)));
+    CK(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking));
+    CK(cudaEventCreateWithFlags(&ctx->done_event, cudaEventDisableTiming));
+    CK(cudaDeviceSynchronize());
+    return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_create_models(const tppsd_model_cfg* target,
+                                              const tppsd_model_cfg* draft,
+                                              const float* target_blob, size_t target_floats,
+                                              const float* draft_blob, size_t draft_floats,
+                                              int32_t max_batch, int32_t max_positions,
+                                              int32_t max_gamma, tppsd_ctx** out) {
+    if (!out) return TPPSD_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (!cfg_ok(target) || !cfg_ok(draft) || !target_blob || !draft_blob)
+        return TPPSD_ERR_INVALID_ARG;
+    if (target->n_marks != draft->n_marks) return TPPSD_ERR_INVALID_ARG;
+    if (target_floats != tppsd_blob_floats(target) || draft_floats != tppsd_blob_floats(draft))
+        return TPPSD_ERR_INVALID_ARG;
+    if (max_batch < 1 || max_positions < 2 || max_gamma < 1 || max_gamma > 31)
+        return TPPSD_ERR_INVALID_ARG;
+    const int dhD = draft->d_model / draft->heads;
+    if (!(draft->heads == 1 || draft->heads == 2 || draft->heads == 4) || dhD < 8)
+        return TPPSD_ERR_UNSUPPORTED;
+    if (!strcmp(fault_mode(), "alloc")) return TPPSD_ERR_OOM;  // injected allocation failure
+    tppsd_ctx* ctx = new (std::nothrow) tppsd_ctx();
+    if (!ctx) return TPPSD_ERR_OOM;
+    ctx->max_batch = max_batch;
+    ctx->n_max = max_positions;
+    ctx->max_gamma = max_gamma;
+    tppsd_status_t st = create_impl(ctx, target, draft, target_blob, target_floats, draft_blob,
+                                    draft_floats);
+    if (st != TPPSD_OK) {
+        fprintf(stderr, "tppsd_create_models: %s\n", ctx->err.c_str());
+        tppsd_destroy(ctx);
+        return st;
+    }
+    *out = ctx;
+    return TPPSD_OK;
+}
+
+// Forward pass of rows [0, total) in ROWS_SPAN mode, q rows per sequence, in
+// chunks that fit the row workspace.  after(g0, rows) runs after each chunk.
+template <typename F>
+static tppsd_status_t span_forward(tppsd_ctx* ctx, HostModel& hm, KVCache& kv, int B, int q,
+                                   bool heads, cudaStream_t st, F after, int* launches) {
+    const long long total = (long long)B * q;
+    long long chunk = ctx->work.R;
+    if (q <= chunk) chunk = (chunk / q) * q;
+    for (long long g0 = 0; g0 < total; g0 += chunk) {
+        RowSpec rs{ROWS_SPAN, q, (int)(total - g0 < chunk ? total - g0 : chunk), (int)g0};
+        CK(launch_forward(hm.dm, kv, ctx->ss, ctx->work, rs, heads, st, launches, nullptr));
+        TRY(after((int)g0, rs.count));
+    }
+    return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_prefill(tppsd_ctx* ctx, int32_t batch, const float* hist_tau,
+                                        const int32_t* hist_marks, int32_t hist_len,
+                                        void* stream) {
+    if (!ctx || !hist_tau || !hist_marks) return TPPSD_ERR_INVALID_ARG;
+    if (batch < 1 || batch > ctx->max_batch || hist_len < 1 || hist_len + 2 > ctx->n_max)
+        return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    cudaStream_t st = (cudaStream_t)stream;
+    SeqState& ss = ctx->ss;
+    const size_t pitch_f = sizeof(float) * ss.n_max, pitch_i = sizeof(int) * ss.n_max;
+    CK(cudaMemcpy2DAsync(ss.tau, pitch_f, hist_tau, sizeof(float) * hist_len,
+                         sizeof(float) * hist_len, batch, cudaMemcpyDefault, st));
+    CK(cudaMemcpy2DAsync(ss.k, pitch_i, hist_marks, sizeof(int) * hist_len,
+                         sizeof(int) * hist_len, batch, cudaMemcpyDefault, st));
+    CK(launch_history_times(ss, batch, hist_len, st));
+    int nl = 1;
+    if (hist_len >= 2) {
+        auto none = [](int, int) { return TPPSD_OK; };
+        TRY(span_forward(ctx, ctx->T, ctx->kvT, batch, hist_len - 1, false, st, none, &nl));
+        TRY(span_forward(ctx, ctx->D, ctx->kvD, batch, hist_len - 1, false, st, none, &nl));
+    }
+    ctx->prefill_launches = nl;
+    CK(cudaEventRecord(ctx->done_event, st));
+    ctx->last_stream = st;
+    ctx->prefill_batch = batch;
+    ctx->hist_len = hist_len;
+    ctx->prefilled = true;
+    return TPPSD_OK;
+}
+
+// One round: SD (mode 0) or AR (mode 1).  Returns launches in *nl.
+static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, cudaStream_t st,
+                                   unsigned long long cond, int use_cond, int* nl,
+                                   const Prof* prof) {
+    int n = 0;
+    Work& w = ctx->work;
+    if (mode == 0) {
+        PROF_MARK(prof, KC_DRAFT, 1, st);
+        CK(launch_draft(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma, ctx->draft_heads,
+                        ctx->max_gamma, ctx->d_stats, st));
+        PROF_MARK(prof, KC_DRAFT, 0, st);
+        ++n;
+        RowSpec rs{ROWS_STEP, gamma + 1, B * (gamma + 1), 0};
+        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof));
+        PROF_MARK(prof, KC_EPILOGUE, 1, st);
+        CK(launch_verify_epilogue(ctx->T.dm, ctx->D.dm, ctx->ss, ctx->d_params, B, gamma, w.heads,
+                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, st));
+        PROF_MARK(prof, KC_EPILOGUE, 0, st);
+        ++n;
+    } else {
+        RowSpec rs{ROWS_STEP, 1, B, 0};
+        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof));
+        PROF_MARK(prof, KC_AR_SAMPLE, 1, st);
+        CK(launch_ar_sample(ctx->T.dm, ctx->ss, ctx->d_params, B, w.heads, ctx->d_stats, st));
+        PROF_MARK(prof, KC_AR_SAMPLE, 0, st);
+        ++n;
+    }
+    PROF_MARK(prof, KC_CONTROL, 1, st);
+    CK(launch_round_control(ctx->ss, ctx->d_params, B, ctx->d_stats, cond, use_cond,
+                            use_cond ? nullptr : ctx->d_active, st));
+    PROF_MARK(prof, KC_CONTROL, 0, st);
+    ++n;
+    if (nl) *nl = n;
+    return TPPSD_OK;
+}
+
+static tppsd_status_t get_graph(tppsd_ctx* ctx, int mode, int B, int gamma, unsigned flags,
+                                GraphEntry** out) {
+    auto key = std::make_tuple(mode, B, gamma, flags);
+    auto it = ctx->graphs.find(key);
+    if (it != ctx->graphs.end()) {
+        *out = &it->second;
+        return TPPSD_OK;
+    }
+    GraphEntry ge;
+    CK(cudaGraphCreate(&ge.graph, 0));
+    cudaGraphConditionalHandle h;
+    CK(cudaGraphConditionalHandleCreate(&h, ge.graph, 1, cudaGraphCondAssignDefault));
+    cudaGraphNodeParams cp{};
+    cp.type = cudaGraphNodeTypeConditional;
+    cp.conditional.handle = h;
+    cp.conditional.type = cudaGraphCondTypeWhile;
+    cp.conditional.size = 1;
+    cudaGraphNode_t node;
+    CK(cudaGraphAddNode(&node, ge.graph, nullptr, nullptr, 0, &cp));
+    cudaGraph_t body = cp.conditional.phGraph_out[0];
+    CK(cudaStreamBeginCaptureToGraph(ctx->cap_stream, body, nullptr, nullptr, 0,
+                                     cudaStreamCaptureModeRelaxed));
+    tppsd_status_t rs = record_round(ctx, mode, B, gamma, ctx->cap_stream, (unsigned long long)h, 1,
+                                     &ge.launches_per_round, nullptr);
+    cudaGraph_t captured = nullptr;
+    cudaError_t ce = cudaStreamEndCapture(ctx->cap_stream, &captured);
+    TRY(rs);
+    CK(ce);
+    CK(cudaGraphInstantiate(&ge.exec, ge.graph, 0));
+    auto res = ctx->graphs.emplace(key, ge);
+    *out = &res.first->second;
+    return TPPSD_OK;
+}
+
+static tppsd_status_t ensure_stage(tppsd_ctx* ctx, size_t bytes) {
+    if (bytes <= ctx->stage_bytes) return TPPSD_OK;
+    if (ctx->stage) cudaFree(ctx->stage);
+    ctx->stage = nullptr;
+    ctx->stage_bytes = 0;
+    CK(cudaMalloc(&ctx->stage, bytes));
+    ctx->stage_bytes = bytes;
+    return TPPSD_OK;
+}
+
+static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int gamma, uint64_t seed,
+                                  uint32_t flags, float* out_tau, double* out_t, int32_t* out_k,
+                                  void* stream) {
+    if (!ctx) return TPPSD_ERR_INVALID_ARG;
+    if (N > 0 && (!out_tau || !out_t || !out_k)) return TPPSD_ERR_INVALID_ARG;
+    if (!ctx->prefilled || B < 1 || B > ctx->prefill_batch || N < 0) return TPPSD_ERR_INVALID_ARG;
+    if (mode == 0 && (gamma < 1 || gamma > ctx->max_gamma)) return TPPSD_ERR_INVALID_ARG;
+    const int H = ctx->hist_len;
+    if ((long long)H + N + (mode == 0 ? gamma : 0) + 2 > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    if (!strcmp(fault_mode(), "launch")) {
+        ctx->err = "injected launch failure (TPPSD_FAULT=launch)";
+        return TPPSD_ERR_CUDA;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    const size_t nb = (size_t)B * (N > 0 ? N : 1);
+    const bool host_out[3] = {N > 0 && !is_device_ptr(out_tau), N > 0 && !is_device_ptr(out_t),
+                              N > 0 && !is_device_ptr(out_k)};
+    const bool any_host = host_out[0] || host_out[1] || host_out[2];
+    if (any_host) TRY(ensure_stage(ctx, nb * (4 + 8 + 4) + 64));
+    char* sb = (char*)ctx->stage;
+    CallParams p{};
+    p.B = B; p.H = H; p.N = N; p.gamma = mode == 0 ? gamma : 0; p.n_max = ctx->n_max;
+    p.flags = flags; p.seed = seed;
+    p.out_t = host_out[1] ? (double*)sb : out_t;
+    p.out_tau = host_out[0] ? (float*)(sb + nb * 8) : out_tau;
+    p.out_k = host_out[2] ? (int*)(sb + nb * 12) : out_k;
+    p.max_loops = N + 2;
+    const bool profile = (flags & TPPSD_FLAG_PROFILE) != 0;
+    Prof prof{&Profiler::mark, &ctx->prof};
+    const Prof* pp = profile ? &prof : nullptr;
+    if (profile) ctx->prof.reset();
+    ctx->profiled = profile;
+    PROF_MARK(pp, KC_BEGIN, 1, st);
+    CK(launch_begin(p, ctx->d_params, ctx->ss, ctx->d_stats, st));
+    PROF_MARK(pp, KC_BEGIN, 0, st);
+    int launches = 1;
+    if (N > 0) {
+        if (flags & (TPPSD_FLAG_HOST_LOOP | TPPSD_FLAG_PROFILE)) {
+            for (int it = 0; it < N + 2; ++it) {
+                int nl = 0;
+                TRY(record_round(ctx, mode, B, gamma, st, 0, 0, &nl, pp));
+                launches += nl;
+                CK(cudaMemcpyAsync(ctx->h_active, ctx->d_active, sizeof(int), cudaMemcpyDeviceToHost, st));
+                CK(cudaStreamSynchronize(st));
+                if (!*ctx->h_active) break;
+            }
+        } else {
+            GraphEntry* ge = nullptr;
+            TRY(get_graph(ctx, mode, B, mode == 0 ? gamma : 0, flags & TPPSD_FLAG_NO_BONUS, &ge));
+            CK(cudaGraphLaunch(ge->exec, st));
+            launches = -ge->launches_per_round;  // resolved from loop_iters in get_stats
+        }
+    }
+    if (host_out[1]) CK(cudaMemcpyAsync(out_t, p.out_t, (size_t)B * N * 8, cudaMemcpyDeviceToHost, st));
+    if (host_out[0]) CK(cudaMemcpyAsync(out_tau, p.out_tau, (size_t)B * N * 4, cudaMemcpyDeviceToHost, st));
+    if (host_out[2]) CK(cudaMemcpyAsync(out_k, p.out_k, (size_t)B * N * 4, cudaMemcpyDeviceToHost, st));
+    CK(cudaEventRecord(ctx->done_event, st));
+    ctx->last_stream = st;
+    ctx->last_launches = launches;
+    return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_sample(tppsd_ctx* ctx, int32_t batch, int32_t n_events,
+                                       int32_t gamma, uint64_t seed, uint32_t flags,
+                                       float* out_tau, double* out_t, int32_t* out_marks,
+                                       void* stream) {
+    return run_sampler(ctx, 0, batch, n_events, gamma, seed, flags, out_tau, out_t, out_marks,
+                       stream);
+}
+
+extern "C" tppsd_status_t tppsd_sample_autoregressive(tppsd_ctx* ctx, int32_t batch,
+                                                      int32_t n_events, uint64_t seed,
+                                                      uint32_t flags, float* out_tau,
+                                                      double* out_t, int32_t* out_marks,
+                                                      void* stream) {
+    return run_sampler(ctx, 1, batch, n_events, 0, seed, flags, out_tau, out_t, out_marks, stream);
+}
+
+extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
+                                      const float* tau, const int32_t* marks, float* out_heads,
+                                      float* out_logg, float* out_logf, void* stream) {
+    if (!ctx || !tau || !marks || (which != 0 && which != 1)) return TPPSD_ERR_INVALID_ARG;
+    if (batch < 1 || batch > ctx->max_batch || len < 2 || len > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    cudaStream_t st = (cudaStream_t)stream;
+    HostModel& hm = which == 0 ? ctx->T : ctx->D;
+    KVCache& kv = which == 0 ? ctx->kvT : ctx->kvD;
+    SeqState& ss = ctx->ss;
+    ctx->prefilled = false;
+    CK(cudaMemcpy2DAsync(ss.tau, sizeof(float) * ss.n_max, tau, sizeof(float) * len,
+                         sizeof(float) * len, batch, cudaMemcpyDefault, st));
+    CK(cudaMemcpy2DAsync(ss.k, sizeof(int) * ss.n_max, marks, sizeof(int) * len, sizeof(int) * len,
+                         batch, cudaMemcpyDefault, st));
+    CK(launch_history_times(ss, batch, len, st));
+    const int W = 3 * hm.cfg.n_mix + hm.cfg.n_marks;
+    const size_t nh = (size_t)batch * len * W, nl = (size_t)batch * len;
+    const bool hh = out_heads && !is_device_ptr(out_heads);
+    const bool hg = out_logg && !is_device_ptr(out_logg);
+    const bool hf = out_logf && !is_device_ptr(out_logf);
+    if (hh || hg || hf) TRY(ensure_stage(ctx, (nh + 2 * nl) * sizeof(float) + 64));
+    float* sb = (float*)ctx->stage;
+    float* d_heads = hh ? sb : out_heads;
+    float* d_logg = hg ? sb + nh : out_logg;
+    float* d_logf = hf ? sb + nh + nl : out_logf;
+    auto after = [&](int g0, int rows) -> tppsd_status_t {
+        CK(launch_score_logs(hm.dm, ss, ctx->work, batch, len, g0, rows, d_heads, d_logg, d_logf, st));
+        return TPPSD_OK;
+    };
+    int launches = 0;
+    TRY(span_forward(ctx, hm, kv, batch, len - 1, true, st, after, &launches));
+    if (hh) CK(cudaMemcpyAsync(out_heads, d_heads, nh * 4, cudaMemcpyDeviceToHost, st));
+    if (hg) CK(cudaMemcpyAsync(out_logg, d_logg, nl * 4, cudaMemcpyDeviceToHost, st));
+    if (hf) CK(cudaMemcpyAsync(out_logf, d_logf, nl * 4, cudaMemcpyDeviceToHost, st));
+    CK(cudaEventRecord(ctx->done_event, st));
+    ctx->last_stream = st;
+    return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms) {
+    if (!ctx) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    const auto t0 = std::chrono::steady_clock::now();
+    for (;;) {
+        const cudaError_t e = cudaEventQuery(ctx->done_event);
+        if (e == cudaSuccess) return TPPSD_OK;
+        if (e != cudaErrorNotReady) CK(e);
+        const auto ms = std::chrono::duration_cast<std::chrono::milliseconds>(
+                            std::chrono::steady_clock::now() - t0).count();
+        if (ms >= timeout_ms) {
+            ctx->err = "tppsd_wait: timed out";
+            return TPPSD_ERR_TIMEOUT;
+        }
+        std::this_thread::sleep_for(std::chrono::microseconds(200));
+    }
+}
+
+extern "C" tppsd_status_t tppsd_get_stats(tppsd_ctx* ctx, tppsd_stats* out) {
+    if (!ctx || !out) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    CK(cudaEventSynchronize(ctx->done_event));
+    DevStats s{};
+    CK(cudaMemcpy(&s, ctx->d_stats, sizeof(s), cudaMemcpyDeviceToHost));
+    out->rounds = (int64_t)s.rounds;
+    out->drafted = (int64_t)s.drafted;
+    out->accepted = (int64_t)s.accepted;
+    out->emitted = (int64_t)s.emitted;
+    out->resample_iters = (int64_t)s.resample_iters;
+    out->cap_hits = (int64_t)s.cap_hits;
+    out->loop_iters = (int64_t)s.loop_iters;
+    out->prefill_launches = ctx->prefill_launches;
+    out->target_keys = (int64_t)s.target_keys;
+    out->draft_keys = (int64_t)s.draft_keys;
+    out->kernel_launches = ctx->last_launches >= 0
+                               ? ctx->last_launches
+                               : 1 + (int64_t)s.loop_iters * (-ctx->last_launches);
+    if (s.round_limit_hit) return TPPSD_ERR_ROUND_LIMIT;
+    if (s.cap_hits) return TPPSD_WARN_RESAMPLE_CAP;
+    return TPPSD_OK;
+}
+
+static const char* KC_NAMES[KC_COUNT] = {"draft", "embed", "gemm_qkv", "attention", "gemm_o",
+                                         "layernorm", "gemm_ffn1", "gemm_ffn2", "head",
+                                         "epilogue", "ar_sample", "control", "begin"};
+
+extern "C" const char* tppsd_kernel_class_name(int32_t cls) {
+    return cls >= 0 && cls < KC_COUNT ? KC_NAMES[cls] : "";
+}
+
+extern "C" tppsd_status_t tppsd_kernel_times(tppsd_ctx* ctx, double* ms, int64_t* launches) {
+    if (!ctx || !ms || !launches) return TPPSD_ERR_INVALID_ARG;
+    for (int i = 0; i < KC_COUNT; ++i) { ms[i] = 0.0; launches[i] = 0; }
+    if (!ctx->profiled) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    CK(ctx->prof.err);
+    CK(cudaEventSynchronize(ctx->done_event));
+    for (auto& sp : ctx->prof.spans) {
+        float t = 0.f;
+        CK(cudaEventElapsedTime(&t, ctx->prof.pool[sp.second], ctx->prof.pool[sp.second + 1]));
+        ms[sp.first] += t;
+        launches[sp.first] += 1;
+    }
+    return TPPSD_OK;
+}
+
+extern "C" const char* tppsd_status_str(tppsd_status_t s) {
+    switch (s) {
+        case TPPSD_OK: return "ok";
+        case TPPSD_ERR_INVALID_ARG: return "invalid argument";
+        case TPPSD_ERR_OOM: return "out of memory";
+        case TPPSD_ERR_CUDA: return "CUDA error";
+        case TPPSD_ERR_UNSUPPORTED: return "unsupported shape";
+        case TPPSD_ERR_ROUND_LIMIT: return "round limit reached";
+        case TPPSD_ERR_TIMEOUT: return "timeout";
+        case TPPSD_ERR_NO_DEVICE: return "no CUDA device";
+        case TPPSD_WARN_RESAMPLE_CAP: return "resample cap reached";
+    }
+    return "unknown status";
+}
+
+extern "C" const char* tppsd_last_error(const tppsd_ctx* ctx) { return ctx ? ctx->err.c_str() : ""; }
+
+extern "C" void tppsd_destroy(tppsd_ctx* ctx) {
+    if (!ctx) return;
+    cudaSetDevice(ctx->device);
+    cudaDeviceSynchronize();
+    for (auto& kv : ctx->graphs) {
+        if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+        if (kv.second.graph) cudaGraphDestroy(kv.second.graph);
+    }
+    for (void* p : ctx->allocs) cudaFree(p);
+    if (ctx->stage) cudaFree(ctx->stage);
+    if (ctx->h_active) cudaFreeHost(ctx->h_active);
+    for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
+    if (ctx->cap_stream) cudaStreamDestroy(ctx->cap_stream);
+    if (ctx->done_event) cudaEventDestroy(ctx->done_event);
+    cudaGetLastError();
+    delete ctx;
+}

@@ -1,0 +1,145 @@
+// Internal interface between the C-ABI layer (api.cu) and the kernels
+// (kernels.cu): device model descriptors, per-call parameters, launchers.
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace tppsd {
+
+constexpr int MAX_LAYERS = 16;
+constexpr int MAX_MIX = 64;
+constexpr int MAX_MARKS = 256;
+constexpr int MAX_D = 512;
+
+struct LayerW {
+    const void* w_qkv; const float* b_qkv;   // [3d][d] storage type, [3d]
+    const void* w_o;   const float* b_o;     // [d][d], [d]
+    const float* ln1_g; const float* ln1_b;  // [d]
+    const void* w_1;   const float* b_1;     // [F][d], [F]
+    const void* w_2;   const float* b_2;     // [d][F], [d]
+    const float* ln2_g; const float* ln2_b;  // [d]
+};
+
+struct HeadW {  // all fp32 (exact copies of the blob values)
+    const float *E, *v_w, *b_w, *v_mu, *b_mu, *v_s, *b_s, *v_k1, *b_k1, *v_k2, *b_k2;
+};
+
+// One model on the device.  Every pointer lies in [base, base + bytes), so a
+// kernel can copy the whole model to shared memory and rebase the pointers.
+struct DevModel {
+    int L, d, nh, dh, F, M, K, dtype;
+    const float* type_emb;   // [K][d] fp32
+    const double* omega;     // [d/2] temporal-encoding frequencies
+    LayerW layer[MAX_LAYERS];
+    HeadW head;
+    const char* base;
+    size_t bytes;
+    __host__ __device__ int head_width() const { return 3 * M + K; }
+};
+
+// KV cache of one model: K and V each [L][Bmax][nh][n_max][dh] (storage type).
+struct KVCache {
+    void* k;
+    void* v;
+    int Bmax, n_max;
+};
+
+// Parameters of one sampling call, kept in device memory so that one
+// captured graph serves every call with the same (batch, gamma, flags).
+struct CallParams {
+    int B, H, N, gamma, n_max;
+    uint32_t flags;
+    uint64_t seed;
+    float* out_tau;
+    double* out_t;
+    int* out_k;
+    int max_loops;
+};
+
+// Device counters of the current call (mirrors tppsd_stats + status).
+struct DevStats {
+    unsigned long long rounds, drafted, accepted, emitted, resample_iters, cap_hits, loop_iters;
+    unsigned long long target_keys;  // sum over (sequence, target pass) of keys per layer
+    unsigned long long draft_keys;   // sum over draft encode steps of keys per layer
+    int round_limit_hit;
+};
+
+// Kernel classes timed by the profiling loop.
+enum KernelClass {
+    KC_DRAFT = 0, KC_EMBED, KC_GEMM_QKV, KC_ATTENTION, KC_GEMM_O, KC_LAYERNORM, KC_GEMM_FFN1,
+    KC_GEMM_FFN2, KC_HEAD, KC_EPILOGUE, KC_AR_SAMPLE, KC_CONTROL, KC_BEGIN, KC_COUNT
+};
+
+// Optional launch timer: mark(cls, 1) before a launch, mark(cls, 0) after.
+struct Prof {
+    void (*mark)(void* self, int cls, int begin, cudaStream_t st);
+    void* self;
+};
+#define PROF_MARK(prof, cls, b, st) \
+    do {                            \
+        if (prof) (prof)->mark((prof)->self, (cls), (b), (st)); \
+    } while (0)
+
+// Per-sequence state of the sampler.
+struct SeqState {
+    float* tau;   // [Bmax][n_max] inter-event times
+    double* t;    // [Bmax][n_max] absolute times
+    int* k;       // [Bmax][n_max] marks
+    int* n_emit;  // [Bmax] events so far (history + generated)
+    int* n_draft; // [Bmax] positions encoded in the draft cache
+    int* done;    // [Bmax]
+    int n_max;
+};
+
+// Row workspace of the batched forward.
+struct Work {
+    int R;               // capacity in rows
+    int* row_seq;        // [R] sequence of the row, -1 = inactive
+    int* row_pos;        // [R] absolute position of the row
+    float* x;            // [R][dmax] residual stream (fp32)
+    void* xb;            // [R][dmax] GEMM input copy (storage type)
+    void* q;             // [R][dmax]
+    void* att;           // [R][dmax]
+    void* hid;           // [R][Fmax]
+    float* y;            // [R][dmax] pre-LayerNorm sums
+    float* heads;        // [R][hw_max]
+};
+
+// Row modes of a forward pass.
+enum RowMode { ROWS_STEP = 0, ROWS_SPAN = 1 };
+struct RowSpec {
+    int mode;   // ROWS_STEP: r = s*q + l at position n_emit[s]-1+l (skips done s)
+                // ROWS_SPAN: g = g0 + r, s = g / q, position g % q
+    int q;      // rows per sequence
+    int count;  // rows in this pass
+    int g0;
+};
+
+// ---------------------------------------------------------------- launchers
+// All return cudaGetLastError() of their launches.
+cudaError_t launch_forward(const DevModel& m, const KVCache& kv, const SeqState& ss,
+                           const Work& w, const RowSpec& rs, bool want_heads,
+                           cudaStream_t st, int* launches, const Prof* prof);
+cudaError_t launch_history_times(const SeqState& ss, int B, int H, cudaStream_t st);
+cudaError_t launch_begin(const CallParams& p, CallParams* dp, const SeqState& ss,
+                         DevStats* stats, cudaStream_t st);
+cudaError_t launch_draft(const DevModel& m, const KVCache& kv, const SeqState& ss,
+                         const CallParams* dp, int B, int gamma, float* draft_heads,
+                         int gamma_max, DevStats* stats, cudaStream_t st);
+cudaError_t launch_verify_epilogue(const DevModel& mT, const DevModel& mD, const SeqState& ss,
+                                   const CallParams* dp, int B, int gamma, const float* t_heads,
+                                   const float* d_heads, int gamma_max, DevStats* stats,
+                                   cudaStream_t st);
+cudaError_t launch_ar_sample(const DevModel& mT, const SeqState& ss, const CallParams* dp,
+                             int B, const float* heads, DevStats* stats, cudaStream_t st);
+cudaError_t launch_round_control(const SeqState& ss, const CallParams* dp, int B,
+                                 DevStats* stats, unsigned long long cond_handle, int use_cond,
+                                 int* active_out, cudaStream_t st);
+cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work& w, int B,
+                              int len, int s0, int rows, float* out_heads, float* out_logg,
+                              float* out_logf, cudaStream_t st);
+size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
+int draft_supported(const DevModel& m);
+
+}  // namespace tppsd

@@ -110,3 +110,22 @@ def torch_reference_heads(cfg, blob, tau, marks):
         a = torch.tanh(Fn.linear(x, P("head.v_k1"), P("head.b_k1")))
         lf = torch.log_softmax(Fn.linear(a, P("head.v_k2"), P("head.b_k2")), -1)
     return torch.cat([lw, mu, s, lf], -1).numpy()
+
+
+def pit_times(rows, M, taus):
+    """u_i = G(tau_i | head_i): iid Uniform(0,1) when each tau_i is drawn from
+    its head's mixture given the past (probability integral transform; the
+    time-rescaling statistic of App. A.4 with the model as ground truth)."""
+    w = np.exp(rows[:, :M]); mu = rows[:, M:2 * M]; sg = np.exp(rows[:, 2 * M:3 * M])
+    lt = np.log(np.asarray(taus, np.float64))[:, None]
+    return (w * stats.norm.cdf((lt - mu) / sg)).sum(1)
+
+
+def pit_marks(rows, M, ks, rng):
+    """Randomised PIT of discrete marks: F(k-1) + V f(k), V ~ U(0,1), is iid
+    Uniform(0,1) when each k_i is drawn from its head's f given the past."""
+    f = np.exp(rows[:, 3 * M:])
+    f = f / f.sum(1, keepdims=True)
+    cdf_below = np.cumsum(f, 1) - f
+    idx = np.arange(len(ks))
+    return cdf_below[idx, ks] + rng.uniform(size=len(ks)) * f[idx, ks]

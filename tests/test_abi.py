@@ -1,0 +1,93 @@
+"""The C-ABI library builds, loads and exports every declared symbol; host-side
+argument checks and injected faults work without a GPU."""
+import os
+import re
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+
+from paper_2507_09252_gb300 import configs as CF
+from paper_2507_09252_gb300 import inputs as IN
+from paper_2507_09252_gb300 import tppsd as T
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "tppsd.h")).read()
+    return sorted(set(re.findall(r"\b(tppsd_[a-z_]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_symbol():
+    L = T.load()
+    names = _declared()
+    assert "tppsd_sample" in names and "tppsd_prefill" in names and len(names) >= 11
+    for n in names:
+        assert hasattr(L, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", T.lib_path()], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (tppsd_\w+)", out))
+    assert set(names) <= exported
+
+
+@pytest.mark.parametrize("wl", CF.BY_INDEX)
+def test_blob_size_agrees_with_generator(wl):
+    for cfg in (wl.target, wl.draft) + tuple(wl.drafts):
+        assert T.tppsd_blob_floats(cfg) == IN.blob_size(cfg) == IN.model_blob(cfg, 0, 0).size
+
+
+def test_invalid_shapes_rejected():
+    bad = CF.ModelCfg(2, 30, 2, 64, 4, 1, 0)      # d not a multiple of 16
+    assert T.tppsd_blob_floats(bad) == 0
+    bad = CF.ModelCfg(2, 32, 3, 64, 4, 1, 0)      # heads do not divide d
+    assert T.tppsd_blob_floats(bad) == 0
+    bad = CF.ModelCfg(2, 32, 2, 64, 65, 1, 0)     # too many components
+    assert T.tppsd_blob_floats(bad) == 0
+
+
+def _try_create(**kw):
+    wl = CF.C1
+    bt = IN.model_blob(wl.target, 0, 0)
+    bd = IN.model_blob(wl.draft, 0, 1)
+    args = dict(target=wl.target, draft=wl.draft, target_blob=bt, draft_blob=bd,
+                max_batch=4, max_positions=100, max_gamma=4)
+    args.update(kw)
+    return T.tppsd_create_models(**args)
+
+
+def test_argument_errors_before_any_device_work():
+    with pytest.raises(T.TppsdError) as e:
+        _try_create(max_batch=0)
+    assert e.value.status == T.TPPSD_ERR_INVALID_ARG
+    with pytest.raises(T.TppsdError) as e:
+        _try_create(max_gamma=40)
+    assert e.value.status == T.TPPSD_ERR_INVALID_ARG
+    wl = CF.C1
+    with pytest.raises(T.TppsdError) as e:   # mark spaces differ
+        _try_create(draft=CF.ModelCfg(1, 16, 1, 32, 4, 3, 0),
+                    draft_blob=IN.model_blob(CF.ModelCfg(1, 16, 1, 32, 4, 3, 0), 0, 1))
+    assert e.value.status == T.TPPSD_ERR_INVALID_ARG
+    # null context
+    assert T.load().tppsd_prefill(None, 1, None, None, 1, None) == T.TPPSD_ERR_INVALID_ARG
+    assert T.load().tppsd_sample(None, 1, 1, 1, 0, 0, None, None, None, None) == T.TPPSD_ERR_INVALID_ARG
+    assert T.status_str(T.TPPSD_ERR_ROUND_LIMIT) == "round limit reached"
+
+
+def test_injected_allocation_failure():
+    code = ("import sys; sys.path.insert(0, %r)\n"
+            "from tests.test_abi import _try_create\n"
+            "from paper_2507_09252_gb300 import tppsd as T\n"
+            "try:\n    _try_create()\nexcept T.TppsdError as e:\n    print('STATUS', e.status)\n") % ROOT
+    env = dict(os.environ, TPPSD_FAULT="alloc")
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, cwd=ROOT)
+    assert f"STATUS {T.TPPSD_ERR_OOM}" in out.stdout, out.stdout + out.stderr
+
+
+def test_no_device_is_reported_not_crashed():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(T.TppsdError) as e:
+        _try_create()
+    assert e.value.status == T.TPPSD_ERR_NO_DEVICE

@@ -1,0 +1,313 @@
+"""CUDA path vs the oracle, through the C ABI (needs a GB300)."""
+import numpy as np
+import pytest
+from scipy import stats
+
+from oracle import oracle as O
+from paper_2507_09252_gb300 import configs as CF
+from paper_2507_09252_gb300 import inputs as IN
+from paper_2507_09252_gb300 import tppsd as T
+from tests import gpu_common as G
+from tests import helpers as HP
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    T.load()
+
+
+# ------------------------------------------------------------------ scoring
+def _score_case(tcfg, dcfg, bt, bd, B, n, K, tol, seed=0):
+    tau, mk = G.hist(B, n, K, seed)
+    s = G.make_sampler(tcfg, dcfg, bt, bd, B, n + 4, 2)
+    for which, cfg, blob in ((0, tcfg, bt), (1, dcfg, bd)):
+        hd, lg, lf = s.score(which, tau, mk)
+        hd, lg, lf = hd.cpu().numpy(), lg.cpu().numpy(), lf.cpu().numpy()
+        ohd, olg, olf = O.score(cfg, blob, tau, mk)
+        M = cfg.n_mix
+        dh = np.abs(hd[:, :-1] - ohd[:, :-1]).max()
+        df = np.abs(lf[:, 1:] - olf[:, 1:]).max()
+        # log g(tau) amplifies head differences by ~|log tau - mu| / sigma^2, so
+        # it is compared absolutely where it is well conditioned, and
+        # everywhere against the exact log density of the GPU's own heads.
+        well = (tau[:, 1:] >= 0.1) & (tau[:, 1:] <= 10.0)
+        dg = np.abs(lg[:, 1:] - olg[:, 1:])[well].max()
+        own = np.array([[O.log_g(M, hd[b, i - 1].astype(np.float64), tau[b, i])[0]
+                         for i in range(1, n)] for b in range(B)])
+        de = np.abs(lg[:, 1:] - own).max()
+        assert dh < tol and dg < tol and df < tol and de < 1e-4, (which, dh, dg, df, de)
+        assert np.isnan(lg[:, 0]).all()
+    s.close()
+
+
+def test_score_parity_fp32_tiny_workload():
+    wl = CF.C1
+    bt, bd, _, _ = IN.workload_inputs(wl)
+    _score_case(wl.target, wl.draft, bt, bd, 4, 90, 1, G.TOL_FP32)
+
+
+def test_score_parity_fp32_history_dependent_heads():
+    tcfg, dcfg, bt, bd = G.small_models()
+    _score_case(tcfg, dcfg, bt, bd, 5, 150, 3, G.TOL_FP32)
+
+
+@pytest.mark.parametrize("idx,B,n", [(1, 3, 130), (2, 2, 140), (3, 1, 530), (4, 2, 80)])
+def test_score_parity_bf16_workloads(idx, B, n):
+    """Every workload's models (bf16, their own random-init weights) against
+    the oracle's bf16 emulation; the long one spans > 512 positions, several
+    64-key tiles and a ragged tail."""
+    wl = CF.BY_INDEX[idx]
+    bt, bd = IN.model_blob(wl.target, 0, 0), IN.model_blob(wl.draft, 0, 1)
+    _score_case(wl.target, wl.draft, bt, bd, B, n, wl.target.n_marks, G.TOL_BF16)
+
+
+@pytest.mark.parametrize("idx,B,n", [(1, 2, 100), (2, 2, 90), (3, 1, 150), (4, 2, 70)])
+def test_score_parity_fp32_large_shapes(idx, B, n):
+    """The workloads' shapes (d up to 512, 8 heads, d_head 64, M 16, K 100)
+    in fp32 with strongly history-dependent heads: checks indexing at every
+    size against the fp64 oracle at the fp32 tolerance."""
+    wl = CF.BY_INDEX[idx]
+    tcfg = CF.ModelCfg(**{**wl.target.__dict__, "dtype": CF.FP32})
+    dcfg = CF.ModelCfg(**{**wl.draft.__dict__, "dtype": CF.FP32})
+    bt = IN.model_blob(tcfg, 0, 0, head_gain=4.0)
+    bd = IN.model_blob(dcfg, 0, 1, head_gain=4.0)
+    _score_case(tcfg, dcfg, bt, bd, B, n, tcfg.n_marks, G.TOL_FP32)
+
+
+def test_score_parity_sweep_drafts():
+    wl = CF.C5
+    bt = IN.model_blob(wl.target, 0, 0)
+    for dcfg in wl.drafts:
+        bd = IN.model_blob(dcfg, 0, 1)
+        _score_case(wl.target, dcfg, bt, bd, 2, 70, wl.target.n_marks, G.TOL_BF16)
+
+
+# ------------------------------------------------------------------ sampling
+def _run_both(tcfg, dcfg, bt, bd, tau, mk, N, gamma, seed, flags=0, ar=False):
+    B, H = tau.shape
+    s = G.make_sampler(tcfg, dcfg, bt, bd, B, H + N + gamma + 4, max(gamma, 1))
+    s.prefill(tau, mk)
+    if ar:
+        g = G.to_np(s.sample_ar(N, seed, flags))
+        o = O.sample_ar(tcfg, bt, tau, mk, N, seed)
+    else:
+        g = G.to_np(s.sample(N, gamma, seed, flags))
+        o = O.sample_sd(tcfg, bt, dcfg, bd, tau, mk, N, gamma, seed, flags=flags)
+    st, stats = s.stats()
+    s.close()
+    return g, o, st, stats
+
+
+@pytest.mark.parametrize("ar", [False, True])
+def test_sequence_parity_fp32_tiny_workload(ar):
+    wl = CF.C1
+    bt, bd, tau, mk = IN.workload_inputs(wl)
+    g, o, st, stats = _run_both(wl.target, wl.draft, bt, bd, tau, mk, wl.n_events, wl.gamma, 1234, ar=ar)
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32)
+    assert not fails, fails
+    assert ident >= 3
+    assert np.allclose(g["t"], o["t"], rtol=1e-4) or exc
+    assert st == T.TPPSD_OK and stats["emitted"] >= wl.batch * wl.n_events
+    if not ar:
+        assert stats["accepted"] == o["stats"][:, 2].sum() or exc
+        assert stats["rounds"] == o["stats"][:, 0].sum() or exc
+
+
+@pytest.mark.parametrize("gamma,flags", [(4, 0), (1, 0), (7, 0), (4, T.TPPSD_FLAG_NO_BONUS)])
+def test_sequence_parity_fp32_with_rejections(gamma, flags):
+    """Draft and target differ: rejections of both kinds, Theorem-1 loops and
+    mark residual draws all happen, and the GPU reproduces the oracle."""
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5)
+    tau, mk = G.hist(24, 7, 3, 5)
+    g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 60, gamma, 77, flags=flags)
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32)
+    assert not fails, fails
+    assert ident >= 20
+    assert stats["resample_iters"] > 0 and stats["accepted"] < stats["drafted"]
+    ostats = o["stats"]
+    if exc == 0:
+        assert stats["accepted"] == ostats[:, 2].sum()
+        assert stats["resample_iters"] == ostats[:, 3].sum()
+
+
+def test_sequence_parity_bf16_prefix():
+    """bf16: teacher-forced parity is the strict check; sampled sequences
+    agree until a decision within bf16 noise of its threshold."""
+    wl = CF.C2
+    tcfg, dcfg = wl.target, wl.draft
+    bt = IN.model_blob(tcfg, 0, 0, head_gain=4.0)
+    bd = IN.shift_blob(dcfg, IN.model_blob(dcfg, 0, 1, head_gain=4.0), **{"head.b_mu": 0.3})
+    tau, mk = IN.histories(wl, batch=6)
+    g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 48, wl.gamma, 9)
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_BF16, rtol=2e-2)
+    assert not fails, fails
+
+
+def test_identical_draft_gives_autoregressive_output():
+    tcfg, _, bt, _ = G.small_models(gain=1.5)
+    tau, mk = G.hist(8, 5, 3, 1)
+    s = G.make_sampler(tcfg, tcfg, bt, bt, 8, 5 + 40 + 8, 6)
+    s.prefill(tau, mk)
+    sd = G.to_np(s.sample(40, 6, 3))
+    _, st_sd = s.stats()
+    ar = G.to_np(s.sample_ar(40, 3))
+    s.close()
+    assert st_sd["accepted"] >= 0.999 * st_sd["drafted"]
+    assert (sd["k"] == ar["k"]).mean() > 0.99
+    assert np.allclose(sd["tau"], ar["tau"], rtol=1e-4)
+
+
+def test_no_bonus_output_independent_of_gamma():
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5)
+    tau, mk = G.hist(16, 6, 3, 2)
+    s = G.make_sampler(tcfg, dcfg, bt, bd, 16, 6 + 40 + 10, 8)
+    s.prefill(tau, mk)
+    ref = G.to_np(s.sample(40, 1, 5, T.TPPSD_FLAG_NO_BONUS))
+    for gamma in (3, 8):
+        out = G.to_np(s.sample(40, gamma, 5, T.TPPSD_FLAG_NO_BONUS))
+        assert (out["k"] == ref["k"]).mean() > 0.99
+        assert np.allclose(out["tau"], ref["tau"], rtol=1e-4)
+    s.close()
+
+
+# ------------------------------------------------------------------ law
+def test_distribution_sd_equals_ar_on_gpu():
+    """1e5 events with a mismatched draft: the PIT of GPU SD times and the
+    randomised PIT of its marks against the target's conditional law (oracle
+    heads, teacher-forced on the GPU output) are iid Uniform(0,1); SD and AR
+    agree at fixed event indices across independent sequences."""
+    tcfg, dcfg, bt, bd = G.small_models()
+    B, H, N, gamma = 2000, 8, 50, 4
+    tau, mk = G.hist(B, H, 3, 0)
+    s = G.make_sampler(tcfg, dcfg, bt, bd, B, H + N + gamma + 4, gamma)
+    s.prefill(tau, mk)
+    sd = G.to_np(s.sample(N, gamma, 21))
+    _, st = s.stats()
+    ar = G.to_np(s.sample_ar(N, 22))
+    s.close()
+    assert 0.05 < st["accepted"] / st["drafted"] < 0.95 and st["resample_iters"] > 0
+    for j in (0, 9, 24, 49):
+        assert stats.ks_2samp(sd["tau"][:, j], ar["tau"][:, j]).pvalue > 1e-3
+        ct = np.stack([np.bincount(sd["k"][:, j], minlength=3), np.bincount(ar["k"][:, j], minlength=3)])
+        assert stats.chi2_contingency(ct)[1] > 1e-3
+    full_tau = np.concatenate([tau, sd["tau"]], 1)
+    full_k = np.concatenate([mk, sd["k"]], 1)
+    hd, _, _ = O.score(tcfg, bt, full_tau, full_k)
+    M = tcfg.n_mix
+    rows = hd[:, H - 1:H + N - 1].reshape(-1, hd.shape[-1])
+    assert stats.kstest(HP.pit_times(rows, M, full_tau[:, H:].ravel()), "uniform").pvalue > 1e-3
+    rng = np.random.default_rng(0)
+    assert stats.kstest(HP.pit_marks(rows, M, full_k[:, H:].ravel(), rng), "uniform").pvalue > 1e-3
+
+
+def test_distribution_bf16_headline_shape():
+    """Headline model shapes in bf16, mismatched draft, 256 x 512 events: the
+    PITs of GPU SD output against the GPU target's teacher-forced heads are
+    Uniform(0,1); on 8 sequences also against the oracle's bf16 heads."""
+    wl = CF.C2
+    tcfg, dcfg = wl.target, wl.draft
+    bt = IN.model_blob(tcfg, 0, 0, head_gain=4.0)
+    bd = IN.shift_blob(dcfg, IN.model_blob(dcfg, 0, 1, head_gain=4.0), **{"head.b_mu": 0.3, "head.b_s": 0.2})
+    tau, mk = IN.histories(wl, batch=256)
+    H, N = wl.hist_len, 512
+    s = G.make_sampler(tcfg, dcfg, bt, bd, 256, H + N + wl.gamma + 4, wl.gamma)
+    s.prefill(tau, mk)
+    sd = G.to_np(s.sample(N, wl.gamma, 31))
+    _, st = s.stats()
+    full_tau = np.concatenate([tau, sd["tau"]], 1)
+    full_k = np.concatenate([mk, sd["k"]], 1)
+    hd, _, _ = s.score(0, full_tau, full_k)
+    hd = hd.cpu().numpy()
+    s.close()
+    assert st["accepted"] < st["drafted"]
+    M = tcfg.n_mix
+    rows = hd[:, H - 1:H + N - 1].reshape(-1, hd.shape[-1]).astype(np.float64)
+    rng = np.random.default_rng(1)
+    assert stats.kstest(HP.pit_times(rows, M, full_tau[:, H:].ravel()), "uniform").pvalue > 1e-3
+    assert stats.kstest(HP.pit_marks(rows, M, full_k[:, H:].ravel(), rng), "uniform").pvalue > 1e-3
+    ohd, _, _ = O.score(tcfg, bt, full_tau[:8], full_k[:8])
+    orows = ohd[:, H - 1:H + N - 1].reshape(-1, ohd.shape[-1])
+    assert stats.kstest(HP.pit_times(orows, M, full_tau[:8, H:].ravel()), "uniform").pvalue > 1e-3
+
+
+# ------------------------------------------------------------------ full size
+def test_full_size_headline_workload():
+    """The benchmarked launch (256 x 512 events, gamma 8, bf16): outputs are
+    valid, sampled sequences agree with the oracle on their prefix, and the
+    GPU's teacher-forced scores of its own output match the oracle's."""
+    wl = CF.C2
+    bt, bd, tau, mk = IN.workload_inputs(wl)
+    B, H, N, g = wl.batch, wl.hist_len, wl.n_events, wl.gamma
+    s = G.make_sampler(wl.target, wl.draft, bt, bd, B, H + N + g + 4, g)
+    s.prefill(tau, mk)
+    out = G.to_np(s.sample(N, g, 2024))
+    st, stats_ = s.stats()
+    assert st == T.TPPSD_OK
+    assert np.isfinite(out["tau"]).all() and (out["tau"] > 0).all()
+    assert (out["k"] >= 0).all() and (out["k"] < wl.target.n_marks).all()
+    t_hist = tau.astype(np.float64).sum(1)
+    assert np.allclose(out["t"][:, 0], t_hist + out["tau"][:, 0], rtol=1e-9)
+    assert (np.diff(out["t"], axis=1) > 0).all()
+    assert stats_["emitted"] >= B * N and stats_["loop_iters"] <= N + 1
+    pick = [0, 97, 255]
+    o = O.sample_sd(wl.target, bt, wl.draft, bd, tau[pick], mk[pick], 40, g, 2024, seq_ids=pick)
+    sub = {k: out[k][pick, :40] for k in ("tau", "k")}
+    _, _, fails = G.compare_sequences(sub, {**o, "margin": o["margin"]}, G.MARGIN_BF16, rtol=2e-2)
+    assert not fails, fails
+    full_tau = np.concatenate([tau[pick], out["tau"][pick]], 1)
+    full_k = np.concatenate([mk[pick], out["k"][pick]], 1)
+    hd, lg, lf = s.score(0, full_tau, full_k)
+    _, olg, olf = O.score(wl.target, bt, full_tau, full_k, heads=False)
+    assert np.abs(lg.cpu().numpy()[:, 1:] - olg[:, 1:]).max() < G.TOL_BF16
+    assert np.abs(lf.cpu().numpy()[:, 1:] - olf[:, 1:]).max() < G.TOL_BF16
+    s.close()
+
+
+# ------------------------------------------------------------------ edge cases
+def test_edge_cases_and_call_paths():
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5)
+    tau, mk = G.hist(5, 4, 3, 9)
+    s = G.make_sampler(tcfg, dcfg, bt, bd, 5, 4 + 30 + 8, 6)
+    s.prefill(tau, mk)
+    # zero events: nothing happens, status ok
+    z = s.sample(0, 3, 1)
+    assert z["tau"].numel() == 0
+    a = G.to_np(s.sample(30, 3, 1))
+    b = G.to_np(s.sample(30, 3, 1))                    # restart from the prefill
+    assert all(np.array_equal(a[k], b[k]) for k in a)
+    c = G.to_np(s.sample(30, 3, 1, flags=T.TPPSD_FLAG_HOST_LOOP))
+    assert all(np.array_equal(a[k], c[k]) for k in a)
+    part = G.to_np(s.sample(30, 3, 1, batch=2))       # fewer sequences than prefilled
+    assert all(np.array_equal(a[k][:2], part[k]) for k in a)
+    # host (numpy) outputs through the same entry point
+    ht = np.zeros((5, 30), np.float32); htt = np.zeros((5, 30)); hk = np.zeros((5, 30), np.int32)
+    T.tppsd_sample(s.ctx, 5, 30, 3, 1, 0, ht, htt, hk)
+    assert T.tppsd_wait(s.ctx, 10000) == T.TPPSD_OK
+    assert np.array_equal(ht, a["tau"]) and np.array_equal(hk, a["k"]) and np.array_equal(htt, a["t"])
+    one = G.to_np(s.sample(1, 6, 1))
+    assert np.array_equal(one["k"][:, 0], a["k"][:, 0])
+    with pytest.raises(T.TppsdError):
+        s.sample(30, 7, 1)                             # gamma above max_gamma
+    with pytest.raises(T.TppsdError):
+        s.sample(60, 3, 1)                             # beyond max_positions
+    s.close()
+    # history of a single event: no prefill forward at all
+    tau1, mk1 = G.hist(3, 1, 3, 4)
+    g, o, st, _ = _run_both(tcfg, dcfg, bt, bd, tau1, mk1, 20, 3, 8)
+    _, _, fails = G.compare_sequences(g, o, G.MARGIN_FP32)
+    assert not fails
+
+
+def test_prefill_in_chunks_matches_oracle():
+    """More history rows than the row workspace: prefill runs in chunks that
+    split sequences; sampling afterwards still matches the oracle."""
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5)
+    tau, mk = G.hist(2, 2300, 3, 3)
+    g, o, st, _ = _run_both(tcfg, dcfg, bt, bd, tau, mk, 20, 3, 4)
+    _, _, fails = G.compare_sequences(g, o, G.MARGIN_FP32)
+    assert not fails
