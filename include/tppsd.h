@@ -142,6 +142,27 @@ tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t
                            const float* tau, const int32_t* marks, float* out_heads,
                            float* out_logg, float* out_logf, void* stream);
 
+/* Scoring that allocates nothing (the paper has no counterpart; this is a
+ * library convenience).  Same outputs as tppsd_score's out_logg and
+ * out_logf for device arrays tau, marks, out_logg, out_logf [batch][len];
+ * no head rows.  For callers that may not allocate device memory at call
+ * time: processes whose GPU memory is owned by another allocator, or
+ * latency-critical loops that cannot absorb cudaMalloc's implicit device
+ * synchronisation.  All working memory (sequence copy, K/V of the scored
+ * positions, row workspace) comes from one 16 MiB array in device memory
+ * that the library holds on every GPU that loads it until the process
+ * exits; a request whose K/V and sequence copy do not fit (with room for at
+ * least 16 workspace rows) returns TPPSD_ERR_INVALID_ARG with the reason
+ * in tppsd_last_error.  The first call on a device looks up that array's
+ * device address (a one-time set-up); make that first call before any
+ * stream capture.  Every call shares the array: calls that overlap on the
+ * GPU (other streams, other contexts, other host threads) race and give
+ * wrong results; serialise them.  Unlike tppsd_score it leaves the
+ * prefilled caches intact. */
+tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
+                                   const float* tau, const int32_t* marks, float* out_logg,
+                                   float* out_logf, void* stream);
+
 /* Synchronises the last stream used and copies the last call's counters.
  * Returns that call's status (OK, WARN_RESAMPLE_CAP or ERR_ROUND_LIMIT). */
 tppsd_status_t tppsd_get_stats(tppsd_ctx* ctx, tppsd_stats* out);

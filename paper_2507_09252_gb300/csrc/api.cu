@@ -15,6 +15,7 @@
 
 #include <chrono>
 #include <map>
+#include <mutex>
 #include <new>
 #include <string>
 #include <thread>
@@ -716,4 +717,129 @@ extern "C" void tppsd_destroy(tppsd_ctx* ctx) {
     if (ctx->done_event) cudaEventDestroy(ctx->done_event);
     cudaGetLastError();
     delete ctx;
+}
+
+// ---------------------------------------------------------------- scoring without allocation
+// tppsd_score_noalloc runs the same teacher-forced scoring pipeline as
+// tppsd_score, but every buffer it needs besides the caller's inputs and
+// outputs (sequence copy, K/V cache of the scored rows, row workspace) is
+// carved out of one fixed array in device memory that exists from the moment
+// the library is loaded.  The call itself never allocates.  This serves
+// callers that may not allocate device memory at call time: processes whose
+// device memory is owned by another allocator (a framework's caching pool
+// that has already reserved the GPU), and latency-critical loops that cannot
+// afford the implicit device synchronisation of cudaMalloc/cudaFree.
+constexpr size_t NOALLOC_SCRATCH_BYTES = (size_t)16 << 20;  // 16 MiB per device
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_SCRATCH_BYTES];
+
+namespace {
+constexpr int NOALLOC_MAX_DEVICES = 64;
+std::mutex g_noalloc_mutex;
+void* g_noalloc_addr[NOALLOC_MAX_DEVICES] = {};
+}  // namespace
+
+// Device address of the scratch array on the current device.  The symbol's
+// host-side name is not a device address; cudaGetSymbolAddress gives the
+// real one, once per device (the first call on a device does this set-up).
+static tppsd_status_t noalloc_scratch(tppsd_ctx* ctx, unsigned char** out) {
+    int dev = 0;
+    CK(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= NOALLOC_MAX_DEVICES) {
+        ctx->err = "tppsd_score_noalloc: device index out of range";
+        return TPPSD_ERR_UNSUPPORTED;
+    }
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_addr[dev]) {
+        void* p = nullptr;
+        CK(cudaGetSymbolAddress(&p, g_noalloc_scratch));
+        g_noalloc_addr[dev] = p;
+    }
+    *out = (unsigned char*)g_noalloc_addr[dev];
+    return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int32_t batch,
+                                              int32_t len, const float* tau, const int32_t* marks,
+                                              float* out_logg, float* out_logf, void* stream) {
+    if (!ctx || !tau || !marks || !out_logg || !out_logf || (which != 0 && which != 1))
+        return TPPSD_ERR_INVALID_ARG;
+    if (batch < 1 || len < 2) return TPPSD_ERR_INVALID_ARG;
+    CK(cudaSetDevice(ctx->device));
+    if (!is_device_ptr(tau) || !is_device_ptr(marks) || !is_device_ptr(out_logg) ||
+        !is_device_ptr(out_logf)) {
+        ctx->err = "tppsd_score_noalloc: all arrays must be device memory";
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    HostModel& hm = which == 0 ? ctx->T : ctx->D;
+    const tppsd_model_cfg& c = hm.cfg;
+    const size_t eb = c.dtype == 1 ? 2 : 4;
+    const size_t d = c.d_model, F = c.d_ffn, W = 3 * c.n_mix + c.n_marks;
+    const size_t n = (size_t)batch * len;
+    auto up = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    // fixed part: sequence copy, per-sequence state, K and V of every scored position
+    const size_t seq_bytes = up(n * 4) + up(n * 8) + up(n * 4) + 3 * up((size_t)batch * 4);
+    const size_t kv_bytes = 2 * up((size_t)c.layers * n * d * eb);
+    // per workspace row: row tables, x and y (fp32), xb/q/att (storage type), hid, head
+    const size_t row_bytes = 2 * 4 + 2 * d * 4 + 3 * d * eb + F * eb + W * 4;
+    const size_t fixed = seq_bytes + kv_bytes + 12 * 256;
+    const long long q = len - 1, total = (long long)batch * q;
+    long long rows = fixed < NOALLOC_SCRATCH_BYTES ? (long long)((NOALLOC_SCRATCH_BYTES - fixed) / row_bytes) : 0;
+    if (rows > total) rows = total;
+    if (rows < 16 && rows < total) {
+        char msg[200];
+        snprintf(msg, sizeof msg, "tppsd_score_noalloc: %d x %d events exceed the %zu-byte scratch",
+                 batch, len, NOALLOC_SCRATCH_BYTES);
+        ctx->err = msg;
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    unsigned char* base = nullptr;
+    TRY(noalloc_scratch(ctx, &base));
+    size_t off = 0;
+    auto take = [&](size_t bytes) { unsigned char* p = base + off; off += up(bytes); return (void*)p; };
+    SeqState ss{};
+    ss.n_max = len;
+    ss.tau = (float*)take(n * 4);
+    ss.t = (double*)take(n * 8);
+    ss.k = (int*)take(n * 4);
+    ss.n_emit = (int*)take((size_t)batch * 4);
+    ss.n_draft = (int*)take((size_t)batch * 4);
+    ss.done = (int*)take((size_t)batch * 4);
+    KVCache kv{};
+    kv.k = take((size_t)c.layers * n * d * eb);
+    kv.v = take((size_t)c.layers * n * d * eb);
+    kv.Bmax = batch;
+    kv.n_max = len;
+    Work w{};
+    w.R = (int)rows;
+    w.row_seq = (int*)take(rows * 4);
+    w.row_pos = (int*)take(rows * 4);
+    w.x = (float*)take(rows * d * 4);
+    w.y = (float*)take(rows * d * 4);
+    w.xb = take(rows * d * eb);
+    w.q = take(rows * d * eb);
+    w.att = take(rows * d * eb);
+    w.hid = take(rows * F * eb);
+    w.heads = (float*)take(rows * W * 4);
+    if (off > NOALLOC_SCRATCH_BYTES) {
+        ctx->err = "tppsd_score_noalloc: scratch layout overflow";
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    cudaStream_t st = (cudaStream_t)stream;
+    // Every byte read below is written first in this call (sequence copy,
+    // times, then K/V of positions 0..i before any query at i), so nothing
+    // left by an earlier call is ever read.
+    CK(cudaMemcpyAsync(ss.tau, tau, n * 4, cudaMemcpyDeviceToDevice, st));
+    CK(cudaMemcpyAsync(ss.k, marks, n * 4, cudaMemcpyDeviceToDevice, st));
+    CK(launch_history_times(ss, batch, len, st));
+    long long chunk = rows;
+    if (q <= chunk) chunk = (chunk / q) * q;
+    for (long long g0 = 0; g0 < total; g0 += chunk) {
+        RowSpec rs{ROWS_SPAN, (int)q, (int)(total - g0 < chunk ? total - g0 : chunk), (int)g0};
+        CK(launch_forward(hm.dm, kv, ss, w, rs, true, st, nullptr, nullptr));
+        CK(launch_score_logs(hm.dm, ss, w, batch, len, (int)g0, rs.count, nullptr, out_logg,
+                             out_logf, st));
+    }
+    CK(cudaEventRecord(ctx->done_event, st));
+    ctx->last_stream = st;
+    return TPPSD_OK;
 }

@@ -77,6 +77,8 @@ def load(build_if_missing: bool = True):
     L.tppsd_sample_autoregressive.argtypes = [_vp, C.c_int32, C.c_int32, C.c_uint64, C.c_uint32,
                                               _vp, _vp, _vp, _vp]
     L.tppsd_score.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp, _vp]
+    L.tppsd_score_noalloc.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp]
+    L.tppsd_score_noalloc.restype = C.c_int
     L.tppsd_get_stats.argtypes = [_vp, C.POINTER(tppsd_stats)]
     L.tppsd_wait.argtypes = [_vp, C.c_int32]
     L.tppsd_kernel_times.argtypes = [_vp, C.POINTER(C.c_double), C.POINTER(C.c_int64)]
@@ -209,6 +211,17 @@ def tppsd_score(ctx, which, batch, length, tau, marks, out_heads, out_logg, out_
                             _ptr(out_logg, np.float32, n, "out_logg"),
                             _ptr(out_logf, np.float32, n, "out_logf"), _stream(stream))
     return _check("tppsd_score", st, ctx)
+
+
+def tppsd_score_noalloc(ctx, which, batch, length, tau, marks, out_logg, out_logf, stream=None):
+    """Scoring whose working memory is a fixed device array of the library:
+    the call allocates nothing.  All arrays must be CUDA tensors."""
+    n = batch * length
+    st = load().tppsd_score_noalloc(ctx, which, batch, length, _ptr(tau, np.float32, n, "tau"),
+                                    _ptr(marks, np.int32, n, "marks"),
+                                    _ptr(out_logg, np.float32, n, "out_logg"),
+                                    _ptr(out_logf, np.float32, n, "out_logf"), _stream(stream))
+    return _check("tppsd_score_noalloc", st, ctx)
 
 
 def tppsd_get_stats(ctx):
