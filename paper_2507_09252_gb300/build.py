@@ -14,8 +14,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libtppsd.so")
-UNITS = ["kernels.cu", "api.cu"]
-HEADERS = ["common.cuh", "engine.h"]
+UNITS = ["kernels.cu", "draft.cu", "gemm_tc.cu", "attn.cu", "api.cu"]
+HEADERS = ["common.cuh", "engine.h", "tc_ptx.cuh"]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-fast-math",

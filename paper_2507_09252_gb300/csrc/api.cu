@@ -33,6 +33,7 @@ struct HostModel {
     tppsd_model_cfg cfg{};
     DevModel dm{};
     void* dbuf = nullptr;
+    void* tbuf = nullptr;
 };
 
 struct GraphEntry {
@@ -96,6 +97,8 @@ struct tppsd_ctx {
     int prefill_launches = 0;
     Profiler prof;
     bool profiled = false;
+    TcPlan tc{};          // tensor-core GEMM plan of the target model (enabled if supported)
+    int* d_err = nullptr; // sticky device error code (pipeline wait timeouts)
     std::string err;
     std::vector<void*> allocs;
 };
@@ -254,6 +257,74 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     h.v_k2 = (const float*)(b + bk2); h.b_k2 = (const float*)(b + bbk2);
     m.base = b;
     m.bytes = buf.size();
+    // transposed, self-contained copy ([in][out] matrices)
+    std::vector<char> tb;
+    auto tadd = [&](const void* src, size_t bytes) {
+        size_t off = (tb.size() + 15) & ~(size_t)15;
+        tb.resize(off + bytes);
+        memcpy(tb.data() + off, src, bytes);
+        return off;
+    };
+    auto tmat = [&](size_t off, size_t rows, size_t cols, bool storage) {  // blob [rows][cols] -> [cols][rows]
+        if (storage && bf) {
+            std::vector<uint16_t> t(rows * cols);
+            for (size_t r = 0; r < rows; ++r)
+                for (size_t c2 = 0; c2 < cols; ++c2) t[c2 * rows + r] = f32_to_bf16_bits(blob[off + r * cols + c2]);
+            return tadd(t.data(), t.size() * 2);
+        }
+        std::vector<float> t(rows * cols);
+        for (size_t r = 0; r < rows; ++r)
+            for (size_t c2 = 0; c2 < cols; ++c2) t[c2 * rows + r] = blob[off + r * cols + c2];
+        return tadd(t.data(), t.size() * 4);
+    };
+    auto tvec = [&](size_t off, size_t n) { return tadd(blob.data() + off, n * sizeof(float)); };
+    std::vector<LB> tl(L);
+    for (int l = 0; l < L; ++l) {
+        tl[l].wqkv = tmat(lo[l].wqkv, 3 * (size_t)d, d, true);
+        tl[l].wo = tmat(lo[l].wo, d, d, true);
+        tl[l].w1 = tmat(lo[l].w1, F, d, true);
+        tl[l].w2 = tmat(lo[l].w2, d, F, true);
+    }
+    for (int l = 0; l < L; ++l) {
+        tl[l].bqkv = tvec(lo[l].bqkv, 3 * d); tl[l].bo = tvec(lo[l].bo, d);
+        tl[l].g1 = tvec(lo[l].g1, d); tl[l].b1n = tvec(lo[l].b1n, d);
+        tl[l].b1 = tvec(lo[l].b1, F); tl[l].b2 = tvec(lo[l].b2, d);
+        tl[l].g2 = tvec(lo[l].g2, d); tl[l].b2n = tvec(lo[l].b2n, d);
+    }
+    const size_t t_emb = tvec(o_emb, (size_t)K * d);
+    const size_t tE = tmat(oE, 3 * (size_t)d, d, false);
+    const size_t tvw = tmat(ovw, M, d, false), tbw = tvec(obw, M);
+    const size_t tvm = tmat(ovm, M, d, false), tbm = tvec(obm, M);
+    const size_t tvs = tmat(ovs, M, d, false), tbs = tvec(obs, M);
+    const size_t tk1 = tmat(ok1, d, d, false), tbk1 = tvec(obk1, d);
+    const size_t tk2 = tmat(ok2, K, d, false), tbk2 = tvec(obk2, K);
+    const size_t t_om = tadd(omega.data(), omega.size() * sizeof(double));
+    tb.resize((tb.size() + 15) & ~(size_t)15);
+    CK(cudaMalloc(&hm.tbuf, tb.size()));
+    ctx->allocs.push_back(hm.tbuf);
+    CK(cudaMemcpy(hm.tbuf, tb.data(), tb.size(), cudaMemcpyHostToDevice));
+    const char* tbp = (const char*)hm.tbuf;
+    DevModelT& mt = m.t;
+    mt.type_emb = (const float*)(tbp + t_emb);
+    mt.omega = (const double*)(tbp + t_om);
+    for (int l = 0; l < L; ++l) {
+        LayerW& w = mt.layer[l];
+        w.w_qkv = tbp + tl[l].wqkv; w.b_qkv = (const float*)(tbp + tl[l].bqkv);
+        w.w_o = tbp + tl[l].wo; w.b_o = (const float*)(tbp + tl[l].bo);
+        w.ln1_g = (const float*)(tbp + tl[l].g1); w.ln1_b = (const float*)(tbp + tl[l].b1n);
+        w.w_1 = tbp + tl[l].w1; w.b_1 = (const float*)(tbp + tl[l].b1);
+        w.w_2 = tbp + tl[l].w2; w.b_2 = (const float*)(tbp + tl[l].b2);
+        w.ln2_g = (const float*)(tbp + tl[l].g2); w.ln2_b = (const float*)(tbp + tl[l].b2n);
+    }
+    HeadW& th = mt.head;
+    th.E = (const float*)(tbp + tE);
+    th.v_w = (const float*)(tbp + tvw); th.b_w = (const float*)(tbp + tbw);
+    th.v_mu = (const float*)(tbp + tvm); th.b_mu = (const float*)(tbp + tbm);
+    th.v_s = (const float*)(tbp + tvs); th.b_s = (const float*)(tbp + tbs);
+    th.v_k1 = (const float*)(tbp + tk1); th.b_k1 = (const float*)(tbp + tbk1);
+    th.v_k2 = (const float*)(tbp + tk2); th.b_k2 = (const float*)(tbp + tbk2);
+    mt.base = tbp;
+    mt.bytes = tb.size();
     return TPPSD_OK;
 }
 
@@ -280,6 +351,44 @@ static tppsd_status_t alloc_kv(tppsd_ctx* ctx, KVCache& kv, const tppsd_model_cf
     kv.Bmax = ctx->max_batch;
     kv.n_max = ctx->n_max;
     return TPPSD_OK;
+}
+
+// bn for an N-wide GEMM tile: 128 when it gives several tiles, else 256.
+static int pick_bn(int N) {
+    if (N % 128 == 0 && N <= 512) return 128;
+    if (N % 256 == 0) return 256;
+    if (N % 128 == 0) return 128;
+    if (N % 64 == 0) return 64;
+    return 0;
+}
+
+// Tensor maps for the target model's tensor-core GEMMs (bf16 models whose
+// widths are multiples of 64 and whose heads are >= 16 wide).
+static void build_tc_plan(tppsd_ctx* ctx) {
+    TcPlan& p = ctx->tc;
+    p.enabled = 0;
+    const DevModel& m = ctx->T.dm;
+    const tppsd_model_cfg& c = ctx->T.cfg;
+    if (getenv("TPPSD_NO_TC") || c.dtype != 1) return;
+    const int d = c.d_model, F = c.d_ffn;
+    if (d % 64 || F % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
+    p.bn_qkv = pick_bn(3 * d);
+    p.bn_ffn1 = pick_bn(F);
+    p.bn_o = d;
+    if (!p.bn_qkv || !p.bn_ffn1) return;
+    const Work& w = ctx->work;
+    bool ok = make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128) &&
+              make_tmap_bf16(&p.a_hid, w.hid, F, w.R, 128);
+    const int bo = d < 256 ? d : 256;
+    for (int l = 0; l < m.L && ok; ++l) {
+        const LayerW& L = m.layer[l];
+        ok = make_tmap_bf16(&p.layer[l].wqkv, L.w_qkv, d, 3 * d, p.bn_qkv < 256 ? p.bn_qkv : 256) &&
+             make_tmap_bf16(&p.layer[l].wo, L.w_o, d, d, bo) &&
+             make_tmap_bf16(&p.layer[l].w1, L.w_1, d, F, p.bn_ffn1 < 256 ? p.bn_ffn1 : 256) &&
+             make_tmap_bf16(&p.layer[l].w2, L.w_2, F, d, bo);
+    }
+    p.err = ctx->d_err;
+    p.enabled = ok ? 1 : 0;
 }
 
 static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
@@ -331,6 +440,10 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &ctx->d_stats, sizeof(DevStats)));
     TRY(dalloc(ctx, &ctx->d_active, sizeof(int)));
     CK(cudaMemset(ctx->d_stats, 0, sizeof(DevStats)));
+    TRY(dalloc(ctx, &ctx->d_err, sizeof(int)));
+    CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
+    w.err = ctx->d_err;
+    build_tc_plan(ctx);
     CK(cudaMallocHost(&ctx->h_active, sizeof(int)));
     CK(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking));
     CK(cudaEventCreateWithFlags(&ctx->done_event, cudaEventDisableTiming));
@@ -383,7 +496,8 @@ static tppsd_status_t span_forward(tppsd_ctx* ctx, HostModel& hm, KVCache& kv, i
     if (q <= chunk) chunk = (chunk / q) * q;
     for (long long g0 = 0; g0 < total; g0 += chunk) {
         RowSpec rs{ROWS_SPAN, q, (int)(total - g0 < chunk ? total - g0 : chunk), (int)g0};
-        CK(launch_forward(hm.dm, kv, ctx->ss, ctx->work, rs, heads, st, launches, nullptr));
+        CK(launch_forward(hm.dm, kv, ctx->ss, ctx->work, rs, heads, st, launches, nullptr,
+                          &hm == &ctx->T ? &ctx->tc : nullptr));
         TRY(after((int)g0, rs.count));
     }
     return TPPSD_OK;
@@ -427,12 +541,16 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
     Work& w = ctx->work;
     if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
-        CK(launch_draft(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma, ctx->draft_heads,
-                        ctx->max_gamma, ctx->d_stats, st));
+        if (draft_warp_supported(ctx->D.dm) && !getenv("TPPSD_DRAFT_CTA"))
+            CK(launch_draft_warp(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
+                                 ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
+        else
+            CK(launch_draft(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma, ctx->draft_heads,
+                            ctx->max_gamma, ctx->d_stats, st));
         PROF_MARK(prof, KC_DRAFT, 0, st);
         ++n;
         RowSpec rs{ROWS_STEP, gamma + 1, B * (gamma + 1), 0};
-        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof));
+        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof, &ctx->tc));
         PROF_MARK(prof, KC_EPILOGUE, 1, st);
         CK(launch_verify_epilogue(ctx->T.dm, ctx->D.dm, ctx->ss, ctx->d_params, B, gamma, w.heads,
                                   ctx->draft_heads, ctx->max_gamma, ctx->d_stats, st));
@@ -440,7 +558,7 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
         ++n;
     } else {
         RowSpec rs{ROWS_STEP, 1, B, 0};
-        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof));
+        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof, &ctx->tc));
         PROF_MARK(prof, KC_AR_SAMPLE, 1, st);
         CK(launch_ar_sample(ctx->T.dm, ctx->ss, ctx->d_params, B, w.heads, ctx->d_stats, st));
         PROF_MARK(prof, KC_AR_SAMPLE, 0, st);
@@ -624,7 +742,15 @@ extern "C" tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms) {
     const auto t0 = std::chrono::steady_clock::now();
     for (;;) {
         const cudaError_t e = cudaEventQuery(ctx->done_event);
-        if (e == cudaSuccess) return TPPSD_OK;
+        if (e == cudaSuccess) {
+            int derr = 0;
+            CK(cudaMemcpy(&derr, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+            if (derr) {
+                ctx->err = "a tensor-core pipeline wait timed out on the device";
+                return TPPSD_ERR_TIMEOUT;
+            }
+            return TPPSD_OK;
+        }
         if (e != cudaErrorNotReady) CK(e);
         const auto ms = std::chrono::duration_cast<std::chrono::milliseconds>(
                             std::chrono::steady_clock::now() - t0).count();
@@ -655,6 +781,12 @@ extern "C" tppsd_status_t tppsd_get_stats(tppsd_ctx* ctx, tppsd_stats* out) {
     out->kernel_launches = ctx->last_launches >= 0
                                ? ctx->last_launches
                                : 1 + (int64_t)s.loop_iters * (-ctx->last_launches);
+    int derr = 0;
+    CK(cudaMemcpy(&derr, ctx->d_err, sizeof(int), cudaMemcpyDeviceToHost));
+    if (derr) {
+        ctx->err = "a tensor-core pipeline wait timed out on the device (code " + std::to_string(derr) + ")";
+        return TPPSD_ERR_TIMEOUT;
+    }
     if (s.round_limit_hit) return TPPSD_ERR_ROUND_LIMIT;
     if (s.cap_hits) return TPPSD_WARN_RESAMPLE_CAP;
     return TPPSD_OK;

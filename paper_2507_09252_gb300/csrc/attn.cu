@@ -1,0 +1,284 @@
+// Causal attention of the target model for bf16 caches (verify pass: gamma+1
+// queries per sequence; AR step: 1 query; prefill: chunks of 16 queries).
+//
+// CTA = (up to 16 query rows of one sequence, one head), four warps.  The
+// K and V of one (sequence, layer, head) are contiguous [position][d_head]
+// in HBM, so every key tile is one bulk copy (cp.async.bulk) into the
+// warp's own double-buffered shared stage, completing on an mbarrier; warp
+// w streams tiles w, w+4, ... and keeps its own online-softmax state
+// (flash-decoding split inside the CTA).  S = Q K^T uses mma.sync
+// m16n8k16 with bf16 inputs (exact products, fp32 accumulation); P V uses
+// fp16 P and V (V converted in shared memory) with fp32 accumulation.  The
+// four partial results are merged through shared memory.
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+#include "engine.h"
+#include "tc_ptx.cuh"
+
+namespace tppsd {
+
+template <int DH>
+struct AttnShape {
+    static constexpr int KT = 2048 / DH;             // keys per tile: 4 KB of K, 4 KB of V
+    static constexpr int TILE_BYTES = KT * DH * 2;
+    static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
+    static constexpr int WARP_BYTES = 2 * STAGE_BYTES + 32;  // two stages + two mbarriers
+    static constexpr int MERGE_BYTES = 4 * (16 * DH + 32) * 4;
+    static constexpr int SMEM = 4 * WARP_BYTES + MERGE_BYTES + 16 * 4 + 64;
+};
+
+__device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_f16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ uint32_t pack_half2(float x, float y) {
+    const __half2 h = __floats2half2_rn(x, y);
+    return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+template <int DH>
+__global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
+    using S = AttnShape<DH>;
+    constexpr int KT = S::KT, NT = KT / 8, KS = DH / 16;
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int g = lane >> 2, t4 = lane & 3;
+    const int h = blockIdx.y;
+    const int seq = a.g0 / a.q_per_seq + blockIdx.z;
+    const int r_lo = max(0, seq * a.q_per_seq - a.g0);
+    const int r_hi = min(a.count, (seq + 1) * a.q_per_seq - a.g0);
+    const int rb = r_lo + blockIdx.x * 16;
+    const int re = min(rb + 16, r_hi);
+    if (rb >= re) return;
+    const int s = a.row_seq[rb];
+    if (s < 0) return;  // rows of one sequence are all active or all inactive
+    const int nq = re - rb;
+    unsigned char* wbase = smem + warp * S::WARP_BYTES;
+    uint64_t* bars = (uint64_t*)(wbase + 2 * S::STAGE_BYTES);
+    float* merge = (float*)(smem + 4 * S::WARP_BYTES);
+    int* qpos = (int*)(smem + 4 * S::WARP_BYTES + S::MERGE_BYTES);
+    if (threadIdx.x < 16) qpos[threadIdx.x] = threadIdx.x < nq ? a.row_pos[rb + threadIdx.x] : -1;
+    if (lane == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    const int maxpos = qpos[nq - 1];
+    const int pos_g = qpos[g], pos_g8 = qpos[g + 8];  // -1 for padding rows
+    const int ntiles = (maxpos + KT) / KT;
+    const size_t base = ((((size_t)a.layer * a.kv.Bmax + s) * a.nh + h) * (size_t)a.kv.n_max) * DH;
+    const bf16* kg = a.kc + base;
+    const bf16* vg = a.vc + base;
+
+    // Q fragments (rows g and g+8 of this CTA, all DH columns), bf16 pairs
+    uint32_t qa[KS][4];
+#pragma unroll
+    for (int k = 0; k < KS; ++k) {
+        const int c0 = 16 * k + 2 * t4;
+        auto ld = [&](int row, int col) -> uint32_t {
+            if (row >= nq) return 0u;
+            return *reinterpret_cast<const uint32_t*>(a.q + (size_t)(rb + row) * a.d + h * DH + col);
+        };
+        qa[k][0] = ld(g, c0);
+        qa[k][1] = ld(g + 8, c0);
+        qa[k][2] = ld(g, c0 + 8);
+        qa[k][3] = ld(g + 8, c0 + 8);
+    }
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;  // rows g, g+8
+    float o[DH / 8][4];
+#pragma unroll
+    for (int n = 0; n < DH / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+
+    auto issue = [&](int tile, int stage) {
+        const int k0 = tile * KT, cnt = min(KT, maxpos + 1 - k0);
+        const uint32_t bytes = (uint32_t)cnt * DH * 2;
+        unsigned char* st = wbase + stage * S::STAGE_BYTES;
+        mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
+        bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
+        bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
+    };
+    if (lane == 0 && warp < ntiles) issue(warp, 0);
+    int it = 0;
+    bool ok = true;
+    for (int tile = warp; tile < ntiles && ok; tile += 4, ++it) {
+        const int stage = it & 1;
+        if (lane == 0 && tile + 4 < ntiles) issue(tile + 4, stage ^ 1);
+        ok = __all_sync(0xffffffffu, mbar_wait(&bars[stage], (it >> 1) & 1, err, 21));
+        if (!ok) break;
+        unsigned char* st = wbase + stage * S::STAGE_BYTES;
+        const bf16* ks = (const bf16*)st;
+        __half* vs = (__half*)(st + S::TILE_BYTES);
+        const int k0 = tile * KT, cnt = min(KT, maxpos + 1 - k0);
+        // V tile: bf16 -> fp16 in place; rows past the copied keys -> 0
+        for (int i = lane; i < KT * DH / 8; i += 32) {
+            uint4* p = reinterpret_cast<uint4*>(vs) + i;
+            uint4 w = *p;
+            if (i * 8 / DH >= cnt) {
+                w = make_uint4(0, 0, 0, 0);
+            } else {
+                __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&w);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 f = __bfloat1622float2(b[j]);
+                    *reinterpret_cast<__half2*>(&b[j]) = __floats2half2_rn(f.x, f.y);
+                }
+            }
+            *p = w;
+        }
+        __syncwarp();
+        // S = Q K^T for KT keys
+        float sc[NT][4];
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
+            const int key = 8 * n + g;
+            const bool kin = key < cnt;
+#pragma unroll
+            for (int k = 0; k < KS; ++k) {
+                const uint32_t b0 = kin ? *reinterpret_cast<const uint32_t*>(ks + key * DH + 16 * k + 2 * t4) : 0u;
+                const uint32_t b1 = kin ? *reinterpret_cast<const uint32_t*>(ks + key * DH + 16 * k + 8 + 2 * t4) : 0u;
+                mma_bf16(sc[n], qa[k], b0, b1);
+            }
+        }
+        // scale, causal mask, online softmax (rows g and g+8; quad reductions)
+        float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            const int key = k0 + 8 * n + 2 * t4;
+            sc[n][0] = (key <= pos_g) ? sc[n][0] * a.scale : -INFINITY;
+            sc[n][1] = (key + 1 <= pos_g) ? sc[n][1] * a.scale : -INFINITY;
+            sc[n][2] = (key <= pos_g8) ? sc[n][2] * a.scale : -INFINITY;
+            sc[n][3] = (key + 1 <= pos_g8) ? sc[n][3] * a.scale : -INFINITY;
+            mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
+            mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
+        }
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+        const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+        const float ref0 = mn0 == -INFINITY ? 0.f : mn0, ref1 = mn1 == -INFINITY ? 0.f : mn1;
+        const float c0 = expf(m0 - ref0), c1 = expf(m1 - ref1);
+        float rs0 = 0.f, rs1 = 0.f;
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            sc[n][0] = expf(sc[n][0] - ref0);
+            sc[n][1] = expf(sc[n][1] - ref0);
+            sc[n][2] = expf(sc[n][2] - ref1);
+            sc[n][3] = expf(sc[n][3] - ref1);
+            rs0 += sc[n][0] + sc[n][1];
+            rs1 += sc[n][2] + sc[n][3];
+        }
+        rs0 += __shfl_xor_sync(0xffffffffu, rs0, 1);
+        rs0 += __shfl_xor_sync(0xffffffffu, rs0, 2);
+        rs1 += __shfl_xor_sync(0xffffffffu, rs1, 1);
+        rs1 += __shfl_xor_sync(0xffffffffu, rs1, 2);
+        l0 = l0 * c0 + rs0;
+        l1 = l1 * c1 + rs1;
+        m0 = mn0;
+        m1 = mn1;
+#pragma unroll
+        for (int n = 0; n < DH / 8; ++n) {
+            o[n][0] *= c0; o[n][1] *= c0;
+            o[n][2] *= c1; o[n][3] *= c1;
+        }
+        // O += P V: P (fp16) from the S accumulators, V fragments by ldmatrix.trans
+        const uint32_t vbase = smem_u32(vs);
+#pragma unroll
+        for (int kk = 0; kk < KT / 16; ++kk) {
+            uint32_t pa[4];
+            pa[0] = pack_half2(sc[2 * kk][0], sc[2 * kk][1]);
+            pa[1] = pack_half2(sc[2 * kk][2], sc[2 * kk][3]);
+            pa[2] = pack_half2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+            pa[3] = pack_half2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+            for (int n = 0; n < DH / 8; n += 2) {
+                // lanes 0-15: keys 16kk + (lane & 15) at columns 8n; lanes 16-31 at 8(n+1)
+                const int key = 16 * kk + (lane & 15);
+                const int col = 8 * n + (lane >> 4) * 8;
+                uint32_t vb[4];
+                ldsm_x4_trans(vb, vbase + (uint32_t)(key * DH + col) * 2);
+                mma_f16(o[n], pa, vb[0], vb[1]);
+                mma_f16(o[n + 1], pa, vb[2], vb[3]);
+            }
+        }
+        __syncwarp();
+    }
+    // per-warp partial results -> shared memory
+    float* mw = merge + warp * (16 * DH + 32);
+    if (t4 == 0) {
+        mw[g] = m0; mw[g + 8] = m1;
+        mw[16 + g] = l0; mw[16 + g + 8] = l1;
+    }
+#pragma unroll
+    for (int n = 0; n < DH / 8; ++n) {
+        const int col = 8 * n + 2 * t4;
+        mw[32 + g * DH + col] = o[n][0];
+        mw[32 + g * DH + col + 1] = o[n][1];
+        mw[32 + (g + 8) * DH + col] = o[n][2];
+        mw[32 + (g + 8) * DH + col + 1] = o[n][3];
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < nq * DH; i += blockDim.x) {
+        const int row = i / DH, col = i % DH;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) M = fmaxf(M, merge[w * (16 * DH + 32) + row]);
+        float L = 0.f, O = 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const float* p = merge + w * (16 * DH + 32);
+            if (p[row] == -INFINITY) continue;
+            const float e = expf(p[row] - M);
+            L += p[16 + row] * e;
+            O += p[32 + row * DH + col] * e;
+        }
+        a.out[(size_t)(rb + row) * a.d + h * DH + col] = __float2bfloat16_rn(O / L);
+    }
+}
+
+cudaError_t launch_attn_mma(const AttArgs<bf16>& a, int dh, int nh, int nseg, int* err, cudaStream_t st) {
+    const dim3 grid((a.q_per_seq + 15) / 16, nh, nseg);
+    switch (dh) {
+        case 16: {
+            const int sm = AttnShape<16>::SMEM;
+            cudaFuncSetAttribute(k_attn_mma<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            k_attn_mma<16><<<grid, 128, sm, st>>>(a, err);
+            break;
+        }
+        case 32: {
+            const int sm = AttnShape<32>::SMEM;
+            cudaFuncSetAttribute(k_attn_mma<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            k_attn_mma<32><<<grid, 128, sm, st>>>(a, err);
+            break;
+        }
+        case 64: {
+            const int sm = AttnShape<64>::SMEM;
+            cudaFuncSetAttribute(k_attn_mma<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+            k_attn_mma<64><<<grid, 128, sm, st>>>(a, err);
+            break;
+        }
+        default:
+            return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace tppsd

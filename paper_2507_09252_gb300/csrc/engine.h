@@ -1,6 +1,8 @@
 // Internal interface between the C-ABI layer (api.cu) and the kernels
 // (kernels.cu): device model descriptors, per-call parameters, launchers.
 #pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -25,6 +27,19 @@ struct HeadW {  // all fp32 (exact copies of the blob values)
     const float *E, *v_w, *b_w, *v_mu, *b_mu, *v_s, *b_s, *v_k1, *b_k1, *v_k2, *b_k2;
 };
 
+// The same model with every matrix transposed to [in][out] (storage type for
+// the layer matrices, fp32 for the head) so that a warp whose lanes own
+// consecutive outputs reads consecutive words.  Self-contained: all vectors
+// are copied in too, and every pointer lies in [base, base + bytes).
+struct DevModelT {
+    const float* type_emb;   // [K][d]
+    const double* omega;     // [d/2]
+    LayerW layer[MAX_LAYERS];  // w_qkv [d][3d], w_o [d][d], w_1 [d][F], w_2 [F][d]
+    HeadW head;              // E [d][3d], v_w/v_mu/v_s [d][M], v_k1 [d][d], v_k2 [d][K]
+    const char* base;
+    size_t bytes;
+};
+
 // One model on the device.  Every pointer lies in [base, base + bytes), so a
 // kernel can copy the whole model to shared memory and rebase the pointers.
 struct DevModel {
@@ -35,6 +50,7 @@ struct DevModel {
     HeadW head;
     const char* base;
     size_t bytes;
+    DevModelT t;             // transposed copy (used by the warp-per-sequence draft)
     __host__ __device__ int head_width() const { return 3 * M + K; }
 };
 
@@ -94,6 +110,7 @@ struct SeqState {
 
 // Row workspace of the batched forward.
 struct Work {
+    int* err;            // device error flag for bounded waits (may be null)
     int R;               // capacity in rows
     int* row_seq;        // [R] sequence of the row, -1 = inactive
     int* row_pos;        // [R] absolute position of the row
@@ -116,11 +133,57 @@ struct RowSpec {
     int g0;
 };
 
+// Arguments of one attention launch (rows of q_per_seq queries per sequence).
+template <typename T>
+struct AttArgs {
+    const T* q;   // [R][d]
+    const T* kc;  // K cache base ([layer][seq][head][pos][d_head])
+    const T* vc;
+    T* out;       // [R][d]
+    const int* row_seq;
+    const int* row_pos;
+    int count, q_per_seq, g0, d, nh, layer;
+    KVCache kv;
+    float scale;
+};
+cudaError_t launch_attn_mma(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int nseg, int* err,
+                            cudaStream_t st);
+
+// ---------------------------------------------------------------- tensor-core GEMM
+enum { EPI_TC_QKV = 0, EPI_TC_RELU = 1, EPI_TC_RESID_LN = 2 };
+struct TcGemmArgs {
+    int R, N, K, epi;
+    const float* bias;
+    // EPI_TC_QKV
+    __nv_bfloat16* q_out; __nv_bfloat16* kc; __nv_bfloat16* vc;
+    const int* row_seq; const int* row_pos;
+    int d, nh, dh, layer, Bmax, n_max;
+    // EPI_TC_RELU
+    __nv_bfloat16* out_t;
+    // EPI_TC_RESID_LN
+    const float* resid; float* x_out; __nv_bfloat16* xb_out; const float* ln_g; const float* ln_b;
+    int* err;  // set (first error wins) if a pipeline wait times out
+};
+struct TcLayerMaps { CUtensorMap wqkv, wo, w1, w2; };
+// Tensor maps of one bf16 model's weights and of the row-workspace buffers it
+// reads (rows = Work.R), built once per context.
+struct TcPlan {
+    int enabled;
+    int bn_qkv, bn_o, bn_ffn1;
+    int* err;
+    CUtensorMap a_xb, a_att, a_hid;
+    TcLayerMaps layer[MAX_LAYERS];
+};
+bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows);
+cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
+                           cudaStream_t st);
+
 // ---------------------------------------------------------------- launchers
 // All return cudaGetLastError() of their launches.
 cudaError_t launch_forward(const DevModel& m, const KVCache& kv, const SeqState& ss,
                            const Work& w, const RowSpec& rs, bool want_heads,
-                           cudaStream_t st, int* launches, const Prof* prof);
+                           cudaStream_t st, int* launches, const Prof* prof,
+                           const TcPlan* tc = nullptr);
 cudaError_t launch_history_times(const SeqState& ss, int B, int H, cudaStream_t st);
 cudaError_t launch_begin(const CallParams& p, CallParams* dp, const SeqState& ss,
                          DevStats* stats, cudaStream_t st);
@@ -140,6 +203,11 @@ cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work&
                               int len, int s0, int rows, float* out_heads, float* out_logg,
                               float* out_logf, cudaStream_t st);
 size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
+// Warp-per-sequence draft (draft.cu) for the shapes it is compiled for.
+int draft_warp_supported(const DevModel& m);
+cudaError_t launch_draft_warp(const DevModel& m, const KVCache& kv, const SeqState& ss,
+                              const CallParams* dp, int B, int gamma, float* draft_heads,
+                              int gamma_max, DevStats* stats, int* err, cudaStream_t st);
 int draft_supported(const DevModel& m);
 
 }  // namespace tppsd

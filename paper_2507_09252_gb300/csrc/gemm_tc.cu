@@ -1,0 +1,279 @@
+// Tensor-core GEMM for the target model's linear layers (bf16 in, fp32
+// accumulate): Y[R][N] = A[R][K] W[N][K]^T + b, with the epilogue fused.
+//
+// One CTA computes a 128 x BN tile.  Warp 0 (one thread) streams 128x64 A
+// and BNx64 W tiles into shared memory with TMA (128-byte swizzle) through
+// a ring of stages guarded by mbarriers; warp 1 (one thread) issues
+// tcgen05.mma (M=128, N<=256 per instruction, K=16) into a TMEM
+// accumulator and releases each stage with tcgen05.commit; then all four
+// warps read the accumulator back (thread t owns row t of the tile: TMEM
+// lane t) and apply the epilogue:
+//   EPI_QKV      bias, bf16 round, Q to the row buffer, K/V scattered into the
+//                KV cache at each row's (sequence, position)
+//   EPI_RELU     bias, ReLU, bf16 round
+//   EPI_RESID_LN bias + residual, LayerNorm over the full row (BN = N = d),
+//                fp32 row and its bf16 copy
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "engine.h"
+#include "tc_ptx.cuh"
+
+namespace tppsd {
+
+template <int BN>
+struct TcShape {
+    static constexpr int BM = 128, BK = 64;
+    static constexpr int STAGES = BN >= 512 ? 2 : 4;
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
+    static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE + 1024 + 256;
+};
+
+__device__ __forceinline__ void st_bf16x16(bf16* dst, const float (&v)[16]) {
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    d[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(128, 1)
+    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, TcGemmArgs a) {
+    using S = TcShape<BN>;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* full = (uint64_t*)(smem + S::STAGES * S::STAGE);
+    uint64_t* empty = full + S::STAGES;
+    uint64_t* done = empty + S::STAGES;
+    uint32_t* tslot = (uint32_t*)(done + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n0 = blockIdx.x * BN, m0 = blockIdx.y * S::BM;
+    const int KB = a.K / S::BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(done, 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, S::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // producer: TMA loads of the A and W tiles of every K block
+        for (int kb = 0; kb < KB; ++kb) {
+            const int s = kb % S::STAGES, round = kb / S::STAGES;
+            if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
+            mbar_arrive_expect_tx(&full[s], S::STAGE);
+            unsigned char* st = smem + s * S::STAGE;
+            tma_load_2d(st, &mapA, &full[s], kb * S::BK, m0);
+#pragma unroll
+            for (int c = 0; c < BN; c += 256)
+                tma_load_2d(st + S::A_BYTES + c * 128, &mapB, &full[s], kb * S::BK, n0 + c);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // MMA issuer
+        constexpr int NI = BN < 256 ? BN : 256;
+        const uint32_t idesc = idesc_bf16(128, NI);
+        for (int kb = 0; kb < KB; ++kb) {
+            const int s = kb % S::STAGES, round = kb / S::STAGES;
+            if (!mbar_wait(&full[s], round & 1, a.err, 2)) break;
+            tc_fence_after();
+            const uint32_t abase = smem_u32(smem + s * S::STAGE), bbase = abase + S::A_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < S::BK / 16; ++kk) {
+                const uint64_t ad = sw128_desc(abase + kk * 32);
+#pragma unroll
+                for (int c = 0; c < BN; c += 256)
+                    tc_mma_bf16(tmem + c, ad, sw128_desc(bbase + c * 128 + kk * 32), idesc,
+                                (kb | kk) != 0);
+            }
+            tc_commit(&empty[s]);
+        }
+        tc_commit(done);  // arrives when every MMA above has completed
+    }
+    __syncwarp();
+    const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
+    tc_fence_after();
+
+    const int r = m0 + warp * 32 + lane;
+    const bool live = ok && r < a.R;
+    const uint32_t tw = tmem + ((uint32_t)(warp * 32) << 16);
+    if (ok) {
+        if (a.epi == EPI_TC_RELU) {
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+                if (live) {
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) v[i] = fmaxf(v[i] + a.bias[n0 + c0 + i], 0.f);
+                    st_bf16x16(a.out_t + (size_t)r * a.N + n0 + c0, v);
+                }
+            }
+        } else if (a.epi == EPI_TC_QKV) {
+            const int s = live ? a.row_seq[r] : -1, pos = live ? a.row_pos[r] : 0;
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+                if (!live) continue;
+                const int col = n0 + c0, which = col / a.d, cc = col - which * a.d;
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[i] += a.bias[col + i];
+                if (which == 0) {
+                    st_bf16x16(a.q_out + (size_t)r * a.d + cc, v);
+                } else if (s >= 0) {
+                    const int h = cc / a.dh, e = cc - h * a.dh;
+                    bf16* dst = (which == 1 ? a.kc : a.vc) +
+                                ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
+                    st_bf16x16(dst, v);
+                }
+            }
+        } else if (BN <= 256) {  // EPI_TC_RESID_LN, BN == N == d
+            // TMEM -> shared tile [128][BN+1] (stages are free: every MMA is
+            // done), then one warp per row: coalesced residual reads and
+            // coalesced x / xb writes, warp-reduced mean and variance.
+            float* tile = (float*)smem;
+            constexpr int LD = BN + 1;
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+                float* dst = tile + (size_t)(warp * 32 + lane) * LD + c0;
+#pragma unroll
+                for (int i = 0; i < 16; ++i) dst[i] = v[i];
+            }
+            __syncthreads();
+            constexpr int PL = BN / 32;  // columns per lane
+            float bias[PL], g[PL], b[PL];
+#pragma unroll
+            for (int j = 0; j < PL; ++j) {
+                bias[j] = a.bias[lane + 32 * j];
+                g[j] = a.ln_g[lane + 32 * j];
+                b[j] = a.ln_b[lane + 32 * j];
+            }
+            for (int rr = warp; rr < 128; rr += 4) {
+                const int row = m0 + rr;
+                if (row >= a.R) break;
+                float y[PL];
+                float sum = 0.f;
+#pragma unroll
+                for (int j = 0; j < PL; ++j) {
+                    const int c = lane + 32 * j;
+                    y[j] = tile[rr * LD + c] + bias[j] + a.resid[(size_t)row * BN + c];
+                    sum += y[j];
+                }
+                const float mean = warp_sum(sum) / BN;
+                float var = 0.f;
+#pragma unroll
+                for (int j = 0; j < PL; ++j) var += (y[j] - mean) * (y[j] - mean);
+                const float inv = 1.0f / sqrtf(warp_sum(var) / BN + LN_EPS);
+#pragma unroll
+                for (int j = 0; j < PL; ++j) {
+                    const int c = lane + 32 * j;
+                    const float o = (y[j] - mean) * inv * g[j] + b[j];
+                    a.x_out[(size_t)row * BN + c] = o;
+                    a.xb_out[(size_t)row * BN + c] = __float2bfloat16_rn(o);
+                }
+            }
+        } else {  // EPI_TC_RESID_LN with BN = 512: row per thread, three passes over TMEM
+            const float* res = a.resid + (size_t)(live ? r : 0) * a.N;
+            float sum = 0.f;
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) sum += v[i] + a.bias[c0 + i] + (live ? res[c0 + i] : 0.f);
+            }
+            const float mean = sum / BN;
+            float var = 0.f;
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const float y = v[i] + a.bias[c0 + i] + (live ? res[c0 + i] : 0.f) - mean;
+                    var += y * y;
+                }
+            }
+            const float inv = 1.0f / sqrtf(var / BN + LN_EPS);
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+                if (!live) continue;
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    v[i] = (v[i] + a.bias[c0 + i] + res[c0 + i] - mean) * inv * a.ln_g[c0 + i] + a.ln_b[c0 + i];
+                float4* xo = reinterpret_cast<float4*>(a.x_out + (size_t)r * a.N + c0);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) xo[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                st_bf16x16(a.xb_out + (size_t)r * a.N + c0, v);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------- host side
+static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    }
+    return fn;
+}
+
+bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tmap_encoder();
+    if (!enc || K % 64 || ((uintptr_t)ptr & 15)) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN>
+static cudaError_t launch_bn(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, cudaStream_t st) {
+    const size_t sm = TcShape<BN>::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    const dim3 grid(a.N / BN, (a.R + 127) / 128);
+    k_gemm_tc<BN><<<grid, 128, sm, st>>>(A, W, a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
+                           cudaStream_t st) {
+    if (a.R <= 0) return cudaSuccess;
+    switch (BN) {
+        case 64: return launch_bn<64>(A, W, a, st);
+        case 128: return launch_bn<128>(A, W, a, st);
+        case 256: return launch_bn<256>(A, W, a, st);
+        case 512: return launch_bn<512>(A, W, a, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace tppsd

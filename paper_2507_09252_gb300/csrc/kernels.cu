@@ -195,19 +195,6 @@ __global__ void k_layernorm(const float* y, const float* g, const float* b, floa
     }
 }
 
-template <typename T>
-struct AttArgs {
-    const T* q;   // [R][d]
-    const T* kc;  // layer-independent base; index with kv_index
-    const T* vc;
-    T* out;       // [R][d]
-    const int* row_seq;
-    const int* row_pos;
-    int count, q_per_seq, g0, d, nh, layer;
-    KVCache kv;
-    float scale;
-};
-
 // Multi-query causal attention: CTA = (16 rows of one sequence, one head).
 // K/V tiles of 64 positions are staged in shared memory and shared by the
 // CTA's queries; each warp runs an online softmax for its queries.
@@ -892,10 +879,27 @@ __global__ void k_score_logs(SeqState ss, Work w, int M, int K, int len, int g0,
         default: return cudaErrorInvalidValue;                         \
     }
 
+// Attention of one layer: bf16 caches use the bulk-copy / mma kernel of
+// attn.cu; fp32 caches (the fp32 models) use the SIMT kernels above.
+template <typename T>
+static cudaError_t attention_launch(const AttArgs<T>& aa, const DevModel& m, const RowSpec& rs, int R,
+                                    int nseg, int* err, cudaStream_t st) {
+    if constexpr (sizeof(T) == 2) {
+        if (m.dh >= 16) return launch_attn_mma(aa, m.dh, m.nh, nseg, err, st);
+    }
+    if (rs.q == 1) {
+        DISPATCH_DH(m.dh, (k_attention_single<T, DH><<<R, 256, 0, st>>>(aa)));
+    } else {
+        const dim3 ag((rs.q + 15) / 16, m.nh, nseg);
+        DISPATCH_DH(m.dh, (k_attention<T, DH><<<ag, 128, 0, st>>>(aa)));
+    }
+    return cudaGetLastError();
+}
+
 template <typename T>
 static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqState& ss,
                              const Work& w, const RowSpec& rs, bool want_heads, cudaStream_t st,
-                             int* launches, const Prof* prof) {
+                             int* launches, const Prof* prof, const TcPlan* tc) {
     const int R = rs.count, d = m.d, F = m.F;
     if (R <= 0) return cudaSuccess;
     int nl = 0;
@@ -915,8 +919,51 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
     const dim3 blk(256);
     auto grid = [&](int N) { return dim3((N + 63) / 64, (R + 63) / 64); };
     const int nseg = (int)((rs.g0 + (long long)R - 1) / rs.q - rs.g0 / rs.q + 1);
+    const bool use_tc = tc && tc->enabled && m.dtype == 1;
     for (int l = 0; l < m.L; ++l) {
         const LayerW& L = m.layer[l];
+        if (use_tc) {
+            cudaError_t e;
+            TcGemmArgs g{};
+            g.R = R; g.N = 3 * d; g.K = d; g.epi = EPI_TC_QKV; g.bias = L.b_qkv;
+            g.q_out = (bf16*)q; g.kc = (bf16*)kv.k; g.vc = (bf16*)kv.v;
+            g.row_seq = w.row_seq; g.row_pos = w.row_pos;
+            g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+            g.err = tc->err;
+            PROF_MARK(prof, KC_GEMM_QKV, 1, st);
+            if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].wqkv, g, tc->bn_qkv, st)) != cudaSuccess) return e;
+            PROF_MARK(prof, KC_GEMM_QKV, 0, st);
+            AttArgs<T> aa{};
+            aa.q = q; aa.kc = (const T*)kv.k; aa.vc = (const T*)kv.v; aa.out = att;
+            aa.row_seq = w.row_seq; aa.row_pos = w.row_pos; aa.count = R; aa.q_per_seq = rs.q;
+            aa.g0 = rs.g0; aa.d = d; aa.nh = m.nh; aa.layer = l; aa.kv = kv;
+            aa.scale = 1.0f / sqrtf((float)m.dh);
+            PROF_MARK(prof, KC_ATTENTION, 1, st);
+            if ((e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st)) != cudaSuccess) return e;
+            PROF_MARK(prof, KC_ATTENTION, 0, st);
+            TcGemmArgs go{};
+            go.R = R; go.N = d; go.K = d; go.epi = EPI_TC_RESID_LN; go.bias = L.b_o;
+            go.resid = w.x; go.x_out = w.x; go.xb_out = (bf16*)xb; go.ln_g = L.ln1_g; go.ln_b = L.ln1_b;
+            go.err = tc->err;
+            PROF_MARK(prof, KC_GEMM_O, 1, st);
+            if ((e = launch_gemm_tc(tc->a_att, tc->layer[l].wo, go, tc->bn_o, st)) != cudaSuccess) return e;
+            PROF_MARK(prof, KC_GEMM_O, 0, st);
+            TcGemmArgs g1{};
+            g1.R = R; g1.N = F; g1.K = d; g1.epi = EPI_TC_RELU; g1.bias = L.b_1; g1.out_t = (bf16*)hid;
+            g1.err = tc->err;
+            PROF_MARK(prof, KC_GEMM_FFN1, 1, st);
+            if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].w1, g1, tc->bn_ffn1, st)) != cudaSuccess) return e;
+            PROF_MARK(prof, KC_GEMM_FFN1, 0, st);
+            TcGemmArgs g2{};
+            g2.R = R; g2.N = d; g2.K = F; g2.epi = EPI_TC_RESID_LN; g2.bias = L.b_2;
+            g2.resid = w.x; g2.x_out = w.x; g2.xb_out = (bf16*)xb; g2.ln_g = L.ln2_g; g2.ln_b = L.ln2_b;
+            g2.err = tc->err;
+            PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
+            if ((e = launch_gemm_tc(tc->a_hid, tc->layer[l].w2, g2, tc->bn_o, st)) != cudaSuccess) return e;
+            PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
+            nl += 5;
+            continue;
+        }
         GemmArgs<T> g{};
         g.A = xb; g.W = (const T*)L.w_qkv; g.bias = L.b_qkv; g.R = R; g.N = 3 * d; g.K = d;
         g.q_out = q; g.kc = (T*)kv.k; g.vc = (T*)kv.v; g.row_seq = w.row_seq; g.row_pos = w.row_pos;
@@ -930,11 +977,9 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         aa.g0 = rs.g0; aa.d = d; aa.nh = m.nh; aa.layer = l; aa.kv = kv;
         aa.scale = 1.0f / sqrtf((float)m.dh);
         PROF_MARK(prof, KC_ATTENTION, 1, st);
-        if (rs.q == 1) {
-            DISPATCH_DH(m.dh, (k_attention_single<T, DH><<<R, 256, 0, st>>>(aa)));
-        } else {
-            const dim3 ag((rs.q + 15) / 16, m.nh, nseg);
-            DISPATCH_DH(m.dh, (k_attention<T, DH><<<ag, 128, 0, st>>>(aa)));
+        {
+            const cudaError_t e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st);
+            if (e != cudaSuccess) return e;
         }
         PROF_MARK(prof, KC_ATTENTION, 0, st);
         GemmArgs<T> go{};
@@ -976,9 +1021,9 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
 
 cudaError_t launch_forward(const DevModel& m, const KVCache& kv, const SeqState& ss, const Work& w,
                            const RowSpec& rs, bool want_heads, cudaStream_t st, int* launches,
-                           const Prof* prof) {
-    return m.dtype == 1 ? forward_t<bf16>(m, kv, ss, w, rs, want_heads, st, launches, prof)
-                        : forward_t<float>(m, kv, ss, w, rs, want_heads, st, launches, prof);
+                           const Prof* prof, const TcPlan* tc) {
+    return m.dtype == 1 ? forward_t<bf16>(m, kv, ss, w, rs, want_heads, st, launches, prof, tc)
+                        : forward_t<float>(m, kv, ss, w, rs, want_heads, st, launches, prof, tc);
 }
 
 cudaError_t launch_history_times(const SeqState& ss, int B, int H, cudaStream_t st) {
