@@ -229,6 +229,23 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     std::vector<double> omega(d / 2);
     for (int i = 0; i < d / 2; ++i) omega[i] = pow(10000.0, -2.0 * i / (double)d);
     const size_t b_om = add(omega.data(), omega.size() * sizeof(double));
+    // head matrices regrouped for the batched head: [E; v_k1] (4d x d) with
+    // bias [0; b_k1], and the output maps transposed side by side (d x (3M+K))
+    std::vector<float> ek((size_t)4 * d * d), ekb((size_t)4 * d, 0.f);
+    memcpy(ek.data(), blob.data() + oE, sizeof(float) * 3 * (size_t)d * d);
+    memcpy(ek.data() + 3 * (size_t)d * d, blob.data() + ok1, sizeof(float) * (size_t)d * d);
+    memcpy(ekb.data() + 3 * d, blob.data() + obk1, sizeof(float) * d);
+    const int WO = 3 * M + K;
+    std::vector<float> ho((size_t)d * WO), hob(WO);
+    const size_t src_off[4] = {ovw, ovm, ovs, ok2}, bsrc[4] = {obw, obm, obs, obk2};
+    const int cnt[4] = {M, M, M, K};
+    for (int part = 0, col0 = 0; part < 4; col0 += cnt[part], ++part)
+        for (int o2 = 0; o2 < cnt[part]; ++o2) {
+            hob[col0 + o2] = blob[bsrc[part] + o2];
+            for (int i = 0; i < d; ++i) ho[(size_t)i * WO + col0 + o2] = blob[src_off[part] + (size_t)o2 * d + i];
+        }
+    const size_t b_ek = add(ek.data(), ek.size() * 4), b_ekb = add(ekb.data(), ekb.size() * 4);
+    const size_t b_ho = add(ho.data(), ho.size() * 4), b_hob = add(hob.data(), hob.size() * 4);
     buf.resize((buf.size() + 15) & ~(size_t)15);
     CK(cudaMalloc(&hm.dbuf, buf.size()));
     ctx->allocs.push_back(hm.dbuf);
@@ -255,6 +272,10 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     h.v_s = (const float*)(b + bvs); h.b_s = (const float*)(b + bbs);
     h.v_k1 = (const float*)(b + bk1); h.b_k1 = (const float*)(b + bbk1);
     h.v_k2 = (const float*)(b + bk2); h.b_k2 = (const float*)(b + bbk2);
+    m.head_ek_w = (const float*)(b + b_ek);
+    m.head_ek_b = (const float*)(b + b_ekb);
+    m.head_out_t = (const float*)(b + b_ho);
+    m.head_out_b = (const float*)(b + b_hob);
     m.base = b;
     m.bytes = buf.size();
     // transposed, self-contained copy ([in][out] matrices)
@@ -435,6 +456,7 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &w.att, sizeof(float) * R * dmax));
     TRY(dalloc(ctx, &w.hid, sizeof(float) * R * fmax));
     TRY(dalloc(ctx, &w.heads, sizeof(float) * R * hw));
+    TRY(dalloc(ctx, &w.hd4, sizeof(float) * R * 4 * dmax));
     TRY(dalloc(ctx, &ctx->draft_heads, sizeof(float) * (size_t)B * ctx->max_gamma * hwD));
     TRY(dalloc(ctx, &ctx->d_params, sizeof(CallParams)));
     TRY(dalloc(ctx, &ctx->d_stats, sizeof(DevStats)));
@@ -912,8 +934,8 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     const size_t seq_bytes = up(n * 4) + up(n * 8) + up(n * 4) + 3 * up((size_t)batch * 4);
     const size_t kv_bytes = 2 * up((size_t)c.layers * n * d * eb);
     // per workspace row: row tables, x and y (fp32), xb/q/att (storage type), hid, head
-    const size_t row_bytes = 2 * 4 + 2 * d * 4 + 3 * d * eb + F * eb + W * 4;
-    const size_t fixed = seq_bytes + kv_bytes + 12 * 256;
+    const size_t row_bytes = 2 * 4 + 2 * d * 4 + 3 * d * eb + F * eb + W * 4 + 4 * d * 4;
+    const size_t fixed = seq_bytes + kv_bytes + 13 * 256;
     const long long q = len - 1, total = (long long)batch * q;
     long long rows = fixed < NOALLOC_SCRATCH_BYTES ? (long long)((NOALLOC_SCRATCH_BYTES - fixed) / row_bytes) : 0;
     if (rows > total) rows = total;
@@ -952,6 +974,7 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     w.att = take(rows * d * eb);
     w.hid = take(rows * F * eb);
     w.heads = (float*)take(rows * W * 4);
+    w.hd4 = (float*)take(rows * 4 * d * 4);
     if (off > NOALLOC_SCRATCH_BYTES) {
         ctx->err = "tppsd_score_noalloc: scratch layout overflow";
         return TPPSD_ERR_INVALID_ARG;

@@ -201,7 +201,7 @@ struct DraftWarp {
     static constexpr int RM = 2;                // M <= 64
     static constexpr int RK = 8;                // K <= 256
 
-    const DevModelT& m;
+    const DevModelT& m;   // pointer table in shared memory (rebased when staged)
     const DraftWArgs& a;
     int s, lane, L, M, K, n_max;
     T* kv_s;                                    // per-warp resident KV: [L][2][NH][n_max][DH]
@@ -378,33 +378,39 @@ struct DraftWarp {
 template <typename T, int D, int F, int DH, bool KVS>
 __global__ void __launch_bounds__(128) k_draft_warp(DraftWArgs a) {
     extern __shared__ __align__(16) char smem[];
+    __shared__ DevModelT m;  // one pointer table per CTA, read by every thread
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    DevModelT m = a.m.t;
     if (a.w_smem) {
-        const int4* src = (const int4*)m.base;
+        const int4* src = (const int4*)a.m.t.base;
         int4* dst = (int4*)smem;
-        for (size_t i = threadIdx.x; i < m.bytes / 16; i += blockDim.x) dst[i] = src[i];
-        auto rb = [&](const void* p) { return (const char*)smem + ((const char*)p - m.base); };
-        m.type_emb = (const float*)rb(m.type_emb);
-        m.omega = (const double*)rb(m.omega);
-        for (int l = 0; l < a.m.L; ++l) {
-            LayerW& L = m.layer[l];
-            L.w_qkv = rb(L.w_qkv); L.b_qkv = (const float*)rb(L.b_qkv);
-            L.w_o = rb(L.w_o);     L.b_o = (const float*)rb(L.b_o);
-            L.ln1_g = (const float*)rb(L.ln1_g); L.ln1_b = (const float*)rb(L.ln1_b);
-            L.w_1 = rb(L.w_1);     L.b_1 = (const float*)rb(L.b_1);
-            L.w_2 = rb(L.w_2);     L.b_2 = (const float*)rb(L.b_2);
-            L.ln2_g = (const float*)rb(L.ln2_g); L.ln2_b = (const float*)rb(L.ln2_b);
-        }
-        HeadW& H = m.head;
-        H.E = (const float*)rb(H.E);
-        H.v_w = (const float*)rb(H.v_w);   H.b_w = (const float*)rb(H.b_w);
-        H.v_mu = (const float*)rb(H.v_mu); H.b_mu = (const float*)rb(H.b_mu);
-        H.v_s = (const float*)rb(H.v_s);   H.b_s = (const float*)rb(H.b_s);
-        H.v_k1 = (const float*)rb(H.v_k1); H.b_k1 = (const float*)rb(H.b_k1);
-        H.v_k2 = (const float*)rb(H.v_k2); H.b_k2 = (const float*)rb(H.b_k2);
-        __syncthreads();
+        for (size_t i = threadIdx.x; i < a.m.t.bytes / 16; i += blockDim.x) dst[i] = src[i];
     }
+    if (threadIdx.x == 0) {
+        m = a.m.t;
+        if (a.w_smem) {
+            const char* ob = a.m.t.base;
+            auto rb = [&](const void* p) { return (const char*)smem + ((const char*)p - ob); };
+            m.type_emb = (const float*)rb(m.type_emb);
+            m.omega = (const double*)rb(m.omega);
+            for (int l = 0; l < a.m.L; ++l) {
+                LayerW& L = m.layer[l];
+                L.w_qkv = rb(L.w_qkv); L.b_qkv = (const float*)rb(L.b_qkv);
+                L.w_o = rb(L.w_o);     L.b_o = (const float*)rb(L.b_o);
+                L.ln1_g = (const float*)rb(L.ln1_g); L.ln1_b = (const float*)rb(L.ln1_b);
+                L.w_1 = rb(L.w_1);     L.b_1 = (const float*)rb(L.b_1);
+                L.w_2 = rb(L.w_2);     L.b_2 = (const float*)rb(L.b_2);
+                L.ln2_g = (const float*)rb(L.ln2_g); L.ln2_b = (const float*)rb(L.ln2_b);
+            }
+            HeadW& H = m.head;
+            H.E = (const float*)rb(H.E);
+            H.v_w = (const float*)rb(H.v_w);   H.b_w = (const float*)rb(H.b_w);
+            H.v_mu = (const float*)rb(H.v_mu); H.b_mu = (const float*)rb(H.b_mu);
+            H.v_s = (const float*)rb(H.v_s);   H.b_s = (const float*)rb(H.b_s);
+            H.v_k1 = (const float*)rb(H.v_k1); H.b_k1 = (const float*)rb(H.b_k1);
+            H.v_k2 = (const float*)rb(H.v_k2); H.b_k2 = (const float*)rb(H.b_k2);
+        }
+    }
+    __syncthreads();
     const CallParams& P = *a.P;
     const int s = blockIdx.x * a.wpc + warp;
     if (s >= P.B || a.ss.done[s]) return;  // no block barrier below
@@ -481,7 +487,7 @@ int draft_warp_supported(const DevModel& m) {
 cudaError_t launch_draft_warp(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st) {
-    const size_t SMEM_MAX = 227 * 1024;
+    const size_t SMEM_MAX = 224 * 1024;  // dynamic part; the pointer table is static
     DraftWArgs a{};
     a.m = m; a.kv = kv; a.ss = ss; a.P = dp; a.st = stats; a.heads = draft_heads;
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;

@@ -50,6 +50,10 @@ struct DevModel {
     HeadW head;
     const char* base;
     size_t bytes;
+    const float* head_ek_w;  // [4d][d] fp32: rows of E then rows of v_k1
+    const float* head_ek_b;  // [4d]: zeros then b_k1
+    const float* head_out_t; // [d][3M+K] fp32: v_w, v_mu, v_s, v_k2 transposed side by side
+    const float* head_out_b; // [3M+K]: b_w, b_mu, b_s, b_k2
     DevModelT t;             // transposed copy (used by the warp-per-sequence draft)
     __host__ __device__ int head_width() const { return 3 * M + K; }
 };
@@ -121,6 +125,7 @@ struct Work {
     void* hid;           // [R][Fmax]
     float* y;            // [R][dmax] pre-LayerNorm sums
     float* heads;        // [R][hw_max]
+    float* hd4;          // [R][4 dmax] head pre-activations (e = E h, V_k1 h + b_k1)
 };
 
 // Row modes of a forward pass.

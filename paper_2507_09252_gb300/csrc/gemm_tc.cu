@@ -164,28 +164,42 @@ __global__ void __launch_bounds__(128, 1)
                 g[j] = a.ln_g[lane + 32 * j];
                 b[j] = a.ln_b[lane + 32 * j];
             }
-            for (int rr = warp; rr < 128; rr += 4) {
-                const int row = m0 + rr;
-                if (row >= a.R) break;
-                float y[PL];
-                float sum = 0.f;
+            // rows in batches of 8: the residual is the output buffer, so the
+            // loads of a batch are all issued before any of its stores
+            constexpr int RB = 8;
+            for (int rr0 = warp; rr0 < 128; rr0 += 4 * RB) {
+                float y[RB][PL];
 #pragma unroll
-                for (int j = 0; j < PL; ++j) {
-                    const int c = lane + 32 * j;
-                    y[j] = tile[rr * LD + c] + bias[j] + a.resid[(size_t)row * BN + c];
-                    sum += y[j];
+                for (int bq = 0; bq < RB; ++bq) {
+                    const int rr = rr0 + 4 * bq, row = m0 + rr;
+#pragma unroll
+                    for (int j = 0; j < PL; ++j) {
+                        const int c = lane + 32 * j;
+                        y[bq][j] = (rr < 128 && row < a.R)
+                                       ? tile[rr * LD + c] + bias[j] + a.resid[(size_t)row * BN + c]
+                                       : 0.f;
+                    }
                 }
-                const float mean = warp_sum(sum) / BN;
-                float var = 0.f;
 #pragma unroll
-                for (int j = 0; j < PL; ++j) var += (y[j] - mean) * (y[j] - mean);
-                const float inv = 1.0f / sqrtf(warp_sum(var) / BN + LN_EPS);
+                for (int bq = 0; bq < RB; ++bq) {
+                    const int rr = rr0 + 4 * bq, row = m0 + rr;
+                    float sum = 0.f;
 #pragma unroll
-                for (int j = 0; j < PL; ++j) {
-                    const int c = lane + 32 * j;
-                    const float o = (y[j] - mean) * inv * g[j] + b[j];
-                    a.x_out[(size_t)row * BN + c] = o;
-                    a.xb_out[(size_t)row * BN + c] = __float2bfloat16_rn(o);
+                    for (int j = 0; j < PL; ++j) sum += y[bq][j];
+                    const float mean = warp_sum(sum) / BN;
+                    float var = 0.f;
+#pragma unroll
+                    for (int j = 0; j < PL; ++j) var += (y[bq][j] - mean) * (y[bq][j] - mean);
+                    const float inv = 1.0f / sqrtf(warp_sum(var) / BN + LN_EPS);
+                    if (rr < 128 && row < a.R) {
+#pragma unroll
+                        for (int j = 0; j < PL; ++j) {
+                            const int c = lane + 32 * j;
+                            const float o = (y[bq][j] - mean) * inv * g[j] + b[j];
+                            a.x_out[(size_t)row * BN + c] = o;
+                            a.xb_out[(size_t)row * BN + c] = __float2bfloat16_rn(o);
+                        }
+                    }
                 }
             }
         } else {  // EPI_TC_RESID_LN with BN = 512: row per thread, three passes over TMEM

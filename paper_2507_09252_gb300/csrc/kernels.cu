@@ -79,7 +79,7 @@ __global__ void k_embed(DevModel m, SeqState ss, RowSpec rs, Work w) {
     }
 }
 
-enum { EPI_QKV = 0, EPI_RELU = 1, EPI_RESID = 2 };
+enum { EPI_QKV = 0, EPI_RELU = 1, EPI_RESID = 2, EPI_F32 = 3 };
 
 template <typename T>
 struct GemmArgs {
@@ -153,6 +153,8 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs<T> a) {
                 }
             } else if (EPI == EPI_RELU) {
                 St<T>::st(a.out_t + (size_t)r * a.N + c, fmaxf(v, 0.f));
+            } else if (EPI == EPI_F32) {
+                a.out_f[(size_t)r * a.N + c] = v;
             } else {
                 a.out_f[(size_t)r * a.N + c] = v + a.resid[(size_t)r * a.N + c];
             }
@@ -470,6 +472,67 @@ __global__ void __launch_bounds__(128) k_head(DevModel m, Work w, int count) {
     __syncthreads();
     cta_head(m.head, d, m.M, m.K, h, e, a, out);
     for (int i = threadIdx.x; i < W; i += blockDim.x) w.heads[(size_t)r * W + i] = out[i];
+}
+
+// Head outputs from the batched pre-activations hd4 = [E h | V_k1 h + b_k1]
+// (Sec. 4.2): w, mu, sigma logits from e1, e2, e3 and mark logits from
+// tanh(.), then the two log-softmaxes.  One warp per row; the output maps
+// (transposed, [d][3M+K]) are staged in shared memory when they fit.
+__global__ void __launch_bounds__(256) k_head_out(DevModel m, Work w, int count, int stage) {
+    extern __shared__ float hsm[];
+    const int d = m.d, M = m.M, K = m.K, WO = 3 * M + K;
+    const float* Wt = m.head_out_t;
+    if (stage) {
+        for (int i = threadIdx.x; i < d * WO; i += blockDim.x) hsm[i] = Wt[i];
+        Wt = hsm;
+        __syncthreads();
+    }
+    float* xs = hsm + (stage ? d * WO : 0) + (threadIdx.x >> 5) * 4 * d;  // per-warp row copy
+    const int lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+    for (int r = blockIdx.x * nw + (threadIdx.x >> 5); r < count; r += gridDim.x * nw) {
+        if (w.row_seq[r] < 0) continue;
+        const float* src = w.hd4 + (size_t)r * 4 * d;
+        for (int i = lane; i < 4 * d; i += 32) xs[i] = i < 3 * d ? src[i] : tanhf(src[i]);
+        __syncwarp();
+        float out[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int o = lane + 32 * j;
+            out[j] = 0.f;
+            if (o >= WO) continue;
+            // which input block feeds output o: e1 (w), e2 (mu), e3 (sigma), tanh part (marks)
+            const int part = o < M ? 0 : (o < 2 * M ? 1 : (o < 3 * M ? 2 : 3));
+            const float* xin = xs + part * d;
+            float acc = m.head_out_b[o];
+            for (int i = 0; i < d; ++i) acc = fmaf(Wt[(size_t)i * WO + o], xin[i], acc);
+            out[j] = acc;
+        }
+        // log-softmax over [0, M) and [3M, 3M+K)
+        float mx_w = -INFINITY, mx_k = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int o = lane + 32 * j;
+            if (o < M) mx_w = fmaxf(mx_w, out[j]);
+            else if (o >= 3 * M && o < WO) mx_k = fmaxf(mx_k, out[j]);
+        }
+        mx_w = warp_max(mx_w);
+        mx_k = warp_max(mx_k);
+        float sw = 0.f, sk = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int o = lane + 32 * j;
+            if (o < M) sw += expf(out[j] - mx_w);
+            else if (o >= 3 * M && o < WO) sk += expf(out[j] - mx_k);
+        }
+        const float lzw = mx_w + logf(warp_sum(sw)), lzk = mx_k + logf(warp_sum(sk));
+        float* dst = w.heads + (size_t)r * WO;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int o = lane + 32 * j;
+            if (o < WO) dst[o] = o < M ? out[j] - lzw : (o >= 3 * M ? out[j] - lzk : out[j]);
+        }
+        __syncwarp();
+    }
 }
 
 // ======================================================================
@@ -1009,11 +1072,21 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         nl += 7;
     }
     if (want_heads) {
-        const size_t sm = sizeof(float) * (size_t)(5 * d + m.head_width());
+        // e | V_k1 h + b_k1 for all rows (fp32 tiled GEMM), then the small maps
         PROF_MARK(prof, KC_HEAD, 1, st);
-        k_head<<<R, 128, sm, st>>>(m, w, R);
+        GemmArgs<float> gh{};
+        gh.A = w.x; gh.W = m.head_ek_w; gh.bias = m.head_ek_b; gh.R = R; gh.N = 4 * d; gh.K = d;
+        gh.out_f = w.hd4;
+        k_gemm<float, EPI_F32><<<dim3((4 * d + 63) / 64, (R + 63) / 64), 256, 0, st>>>(gh);
+        const int WO = m.head_width();
+        const size_t wbytes = sizeof(float) * (size_t)d * WO;
+        const int stage = wbytes <= 96 * 1024;
+        const size_t sm = (stage ? wbytes : 0) + sizeof(float) * 8 * 4 * d;
+        if (sm > 48 * 1024) cudaFuncSetAttribute(k_head_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        const int blocks = min((R + 7) / 8, 152 * 2);
+        k_head_out<<<blocks, 256, sm, st>>>(m, w, R, stage);
         PROF_MARK(prof, KC_HEAD, 0, st);
-        ++nl;
+        nl += 2;
     }
     if (launches) *launches += nl;
     return cudaGetLastError();
