@@ -59,6 +59,29 @@ def dist_env():
     return rank, world, local
 
 
+def rank_histories(wl, rank):
+    """Histories of one rank: every rank samples its own batch of
+    independent sequences (seed offset by the rank), so nothing is exchanged
+    on the data path."""
+    return IN.histories(wl, seed=wl.seed + rank)
+
+
+def max_over_ranks(ms, world, device):
+    """Step time of the whole job: the slowest rank's (MAX all-reduce)."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(world, batch, n_events, ms):
+    """Events per second over all ranks (weak scaling: batch per rank)."""
+    return world * batch * n_events / (ms / 1e3)
+
+
 def workload_config(wl, rank_seed):
     return {"workload": wl.name, "batch_per_gpu": wl.batch, "hist_len": wl.hist_len,
             "n_events": wl.n_events, "gamma": wl.gamma,
@@ -132,7 +155,7 @@ def roofline(kt, stats, wl, peaks):
                 layer) + Q read + output write:  target_keys * 2 d eb + 2 R d eb
     draft:      draft K/V of every encoded position + weights staged once
                 per CTA + draft heads written
-    gemm_*:     2 R N K FLOPs (SIMT fp32 FMA path)
+    gemm_*:     2 R N K FLOPs per layer (tcgen05 bf16 path for bf16 models)
     others:     bytes of their inputs and outputs
     """
     T, D = wl.target, wl.draft
@@ -156,7 +179,7 @@ def roofline(kt, stats, wl, peaks):
     elif name.startswith("gemm"):
         nk = {"gemm_qkv": (3 * d, d), "gemm_o": (d, d), "gemm_ffn1": (F, d), "gemm_ffn2": (d, F)}[name]
         total = 2.0 * rows * nk[0] * nk[1] * L
-        bound, unit = "alu", "TFLOP/s"
+        bound, unit = "tensor", "TFLOP/s"
     else:
         total = rows * d * 4 * 2
     per_launch = total / max(launches, 1)
@@ -165,8 +188,8 @@ def roofline(kt, stats, wl, peaks):
         peak = peaks.get("hbm_gbs", 6800.0)
     else:
         achieved = per_launch / per_launch_s / 1e12
-        # fp32 FFMA on CUDA cores: 152 SMs x 128 lanes x 2 FLOP x max clock
-        peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        # dense bf16 tensor peak, sustained (the kernel runs inside a long step)
+        peak = peaks.get("bf16_tflops_sustained", 1700.0)
     share = ms / sum(v[0] for v in kt.values())
     return {"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": round(peak, 1),
             "unit": unit, "frac": round(achieved / peak, 4), "traffic": None,
@@ -252,7 +275,7 @@ def main():
         dist.init_process_group("nccl", init_method="env://")
     B, H, N, g = wl.batch, wl.hist_len, wl.n_events, wl.gamma
     bt, bd = IN.model_blob(wl.target, wl.seed, 0), IN.model_blob(wl.draft, wl.seed, 1)
-    tau_np, mk_np = IN.histories(wl, seed=wl.seed + rank)
+    tau_np, mk_np = rank_histories(wl, rank)
     s = Sampler(wl.target, wl.draft, bt, bd, B, H + N + g + 4, g)
     tau = torch.from_numpy(tau_np).cuda()
     mk = torch.from_numpy(mk_np).cuda()
@@ -286,11 +309,7 @@ def main():
             e1.record(stream)
         barrier()
         ms = sum(e0.elapsed_time(e1) for e0, e1 in ev) / K
-        if world > 1:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms
+        return max_over_ranks(ms, world, "cuda")
 
     with ClockSampler(local) as clk:
         ms_sd = timed(step_sd, args.steps, args.warmup)
@@ -322,7 +341,7 @@ def main():
     roof = roofline(kt, st_prof, wl, peaks)
 
     events = world * B * N
-    value = events / (ms_sd / 1e3)
+    value = job_rate(world, B, N, ms_sd)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_sd, 3),

@@ -563,8 +563,8 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
     Work& w = ctx->work;
     if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
-        if (draft_warp_supported(ctx->D.dm) && !getenv("TPPSD_DRAFT_CTA"))
-            CK(launch_draft_warp(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
+        if (draft_team_supported(ctx->D.dm) && !getenv("TPPSD_DRAFT_CTA"))
+            CK(launch_draft_team(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
         else
             CK(launch_draft(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma, ctx->draft_heads,

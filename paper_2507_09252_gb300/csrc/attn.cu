@@ -4,8 +4,10 @@
 // CTA = (up to 16 query rows of one sequence, one head), four warps.  The
 // K and V of one (sequence, layer, head) are contiguous [position][d_head]
 // in HBM, so every key tile is one bulk copy (cp.async.bulk) into the
-// warp's own double-buffered shared stage, completing on an mbarrier; warp
-// w streams tiles w, w+4, ... and keeps its own online-softmax state
+// warp's own double-buffered shared stage, completing on an mbarrier.  The
+// keys 0..maxpos are cut into four contiguous ranges of equal length (a
+// multiple of 8 keys), one per warp, so all four warps work even when the
+// context is a single tile; each warp keeps its own online-softmax state
 // (flash-decoding split inside the CTA).  S = Q K^T uses mma.sync
 // m16n8k16 with bf16 inputs (exact products, fp32 accumulation); P V uses
 // fp16 P and V (V converted in shared memory) with fp32 accumulation.  The
@@ -82,7 +84,11 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
     __syncthreads();
     const int maxpos = qpos[nq - 1];
     const int pos_g = qpos[g], pos_g8 = qpos[g + 8];  // -1 for padding rows
-    const int ntiles = (maxpos + KT) / KT;
+    // this warp's key range [klo, khi)
+    const int nkeys = maxpos + 1;
+    const int share = (((nkeys + 3) / 4) + 7) & ~7;
+    const int klo = min(nkeys, warp * share), khi = min(nkeys, klo + share);
+    const int ntl = (khi - klo + KT - 1) / KT;
     const size_t base = ((((size_t)a.layer * a.kv.Bmax + s) * a.nh + h) * (size_t)a.kv.n_max) * DH;
     const bf16* kg = a.kc + base;
     const bf16* vg = a.vc + base;
@@ -107,25 +113,24 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
     for (int n = 0; n < DH / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
 
     auto issue = [&](int tile, int stage) {
-        const int k0 = tile * KT, cnt = min(KT, maxpos + 1 - k0);
+        const int k0 = klo + tile * KT, cnt = min(KT, khi - k0);
         const uint32_t bytes = (uint32_t)cnt * DH * 2;
         unsigned char* st = wbase + stage * S::STAGE_BYTES;
         mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
         bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
         bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
     };
-    if (lane == 0 && warp < ntiles) issue(warp, 0);
-    int it = 0;
+    if (lane == 0 && ntl > 0) issue(0, 0);
     bool ok = true;
-    for (int tile = warp; tile < ntiles && ok; tile += 4, ++it) {
+    for (int it = 0; it < ntl && ok; ++it) {
         const int stage = it & 1;
-        if (lane == 0 && tile + 4 < ntiles) issue(tile + 4, stage ^ 1);
+        if (lane == 0 && it + 1 < ntl) issue(it + 1, stage ^ 1);
         ok = __all_sync(0xffffffffu, mbar_wait(&bars[stage], (it >> 1) & 1, err, 21));
         if (!ok) break;
         unsigned char* st = wbase + stage * S::STAGE_BYTES;
         const bf16* ks = (const bf16*)st;
         __half* vs = (__half*)(st + S::TILE_BYTES);
-        const int k0 = tile * KT, cnt = min(KT, maxpos + 1 - k0);
+        const int k0 = klo + it * KT, cnt = min(KT, khi - k0);
         // V tile: bf16 -> fp16 in place; rows past the copied keys -> 0
         for (int i = lane; i < KT * DH / 8; i += 32) {
             uint4* p = reinterpret_cast<uint4*>(vs) + i;
@@ -157,15 +162,17 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
                 mma_bf16(sc[n], qa[k], b0, b1);
             }
         }
-        // scale, causal mask, online softmax (rows g and g+8; quad reductions)
+        // scale, mask (keys past the copied ones, and causal), online
+        // softmax (rows g and g+8; quad reductions)
         float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
-            const int key = k0 + 8 * n + 2 * t4;
-            sc[n][0] = (key <= pos_g) ? sc[n][0] * a.scale : -INFINITY;
-            sc[n][1] = (key + 1 <= pos_g) ? sc[n][1] * a.scale : -INFINITY;
-            sc[n][2] = (key <= pos_g8) ? sc[n][2] * a.scale : -INFINITY;
-            sc[n][3] = (key + 1 <= pos_g8) ? sc[n][3] * a.scale : -INFINITY;
+            const int kt = 8 * n + 2 * t4, key = k0 + kt;
+            const bool in0 = kt < cnt, in1 = kt + 1 < cnt;
+            sc[n][0] = (in0 && key <= pos_g) ? sc[n][0] * a.scale : -INFINITY;
+            sc[n][1] = (in1 && key + 1 <= pos_g) ? sc[n][1] * a.scale : -INFINITY;
+            sc[n][2] = (in0 && key <= pos_g8) ? sc[n][2] * a.scale : -INFINITY;
+            sc[n][3] = (in1 && key + 1 <= pos_g8) ? sc[n][3] * a.scale : -INFINITY;
             mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
             mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
         }

@@ -54,7 +54,7 @@ struct DevModel {
     const float* head_ek_b;  // [4d]: zeros then b_k1
     const float* head_out_t; // [d][3M+K] fp32: v_w, v_mu, v_s, v_k2 transposed side by side
     const float* head_out_b; // [3M+K]: b_w, b_mu, b_s, b_k2
-    DevModelT t;             // transposed copy (used by the warp-per-sequence draft)
+    DevModelT t;             // transposed copy (read by the per-sequence draft kernel)
     __host__ __device__ int head_width() const { return 3 * M + K; }
 };
 
@@ -208,9 +208,9 @@ cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work&
                               int len, int s0, int rows, float* out_heads, float* out_logg,
                               float* out_logf, cudaStream_t st);
 size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
-// Warp-per-sequence draft (draft.cu) for the shapes it is compiled for.
-int draft_warp_supported(const DevModel& m);
-cudaError_t launch_draft_warp(const DevModel& m, const KVCache& kv, const SeqState& ss,
+// One-CTA-per-sequence draft (draft.cu) for the shapes it is compiled for.
+int draft_team_supported(const DevModel& m);
+cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st);
 int draft_supported(const DevModel& m);

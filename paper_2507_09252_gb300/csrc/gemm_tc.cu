@@ -30,7 +30,9 @@ struct TcShape {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE = A_BYTES + B_BYTES;
     static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
-    static constexpr size_t SMEM = (size_t)STAGES * STAGE + 1024 + 256;
+    // residual rows of the LayerNorm epilogue, prefetched during the main loop
+    static constexpr int RES_BYTES = BN <= 128 ? BM * BN * 4 : 0;
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE + RES_BYTES + 1024 + 256;
 };
 
 __device__ __forceinline__ void st_bf16x16(bf16* dst, const float (&v)[16]) {
@@ -51,10 +53,13 @@ __global__ void __launch_bounds__(128, 1)
     using S = TcShape<BN>;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    uint64_t* full = (uint64_t*)(smem + S::STAGES * S::STAGE);
+    float* resid_s = (float*)(smem + S::STAGES * S::STAGE);
+    uint64_t* full = (uint64_t*)(smem + S::STAGES * S::STAGE + S::RES_BYTES);
     uint64_t* empty = full + S::STAGES;
     uint64_t* done = empty + S::STAGES;
-    uint32_t* tslot = (uint32_t*)(done + 1);
+    uint64_t* resbar = done + 1;
+    uint32_t* tslot = (uint32_t*)(resbar + 1);
+    const bool res_pref = S::RES_BYTES > 0 && a.epi == EPI_TC_RESID_LN;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n0 = blockIdx.x * BN, m0 = blockIdx.y * S::BM;
     const int KB = a.K / S::BK;
@@ -65,6 +70,7 @@ __global__ void __launch_bounds__(128, 1)
             mbar_init(&empty[s], 1);
         }
         mbar_init(done, 1);
+        mbar_init(resbar, 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(tslot, S::TMEM_COLS);
@@ -74,7 +80,13 @@ __global__ void __launch_bounds__(128, 1)
     const uint32_t tmem = *tslot;
 
     if (warp == 0 && lane == 0) {
-        // producer: TMA loads of the A and W tiles of every K block
+        // producer: the tile's residual rows (contiguous, since N == BN),
+        // then TMA loads of the A and W tiles of every K block
+        if (res_pref) {
+            const uint32_t bytes = (uint32_t)min(S::BM, a.R - m0) * BN * 4;
+            mbar_arrive_expect_tx(resbar, bytes);
+            bulk_load(resid_s, a.resid + (size_t)m0 * BN, bytes, resbar);
+        }
         for (int kb = 0; kb < KB; ++kb) {
             const int s = kb % S::STAGES, round = kb / S::STAGES;
             if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
@@ -109,6 +121,8 @@ __global__ void __launch_bounds__(128, 1)
     __syncwarp();
     const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
     tc_fence_after();
+    // every thread waits for the residual copy, so none is in flight at exit
+    const bool have_res = res_pref && mbar_wait(resbar, 0, a.err, 4);
 
     const int r = m0 + warp * 32 + lane;
     const bool live = ok && r < a.R;
@@ -144,7 +158,8 @@ __global__ void __launch_bounds__(128, 1)
             }
         } else if (BN <= 256) {  // EPI_TC_RESID_LN, BN == N == d
             // TMEM -> shared tile [128][BN+1] (stages are free: every MMA is
-            // done), then one warp per row: coalesced residual reads and
+            // done), then one warp per row: residual rows from the prefetched
+            // shared copy (global reads if the copy timed out),
             // coalesced x / xb writes, warp-reduced mean and variance.
             float* tile = (float*)smem;
             constexpr int LD = BN + 1;
@@ -175,9 +190,10 @@ __global__ void __launch_bounds__(128, 1)
 #pragma unroll
                     for (int j = 0; j < PL; ++j) {
                         const int c = lane + 32 * j;
-                        y[bq][j] = (rr < 128 && row < a.R)
-                                       ? tile[rr * LD + c] + bias[j] + a.resid[(size_t)row * BN + c]
-                                       : 0.f;
+                        y[bq][j] = 0.f;
+                        if (rr < 128 && row < a.R)
+                            y[bq][j] = tile[rr * LD + c] + bias[j] +
+                                       (have_res ? resid_s[rr * BN + c] : a.resid[(size_t)row * BN + c]);
                     }
                 }
 #pragma unroll

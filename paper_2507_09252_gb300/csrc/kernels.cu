@@ -715,6 +715,7 @@ __device__ void write_outputs(const SeqState& ss, const CallParams& P, int s, in
 // sequential loop), k from f' (Eq. 4).  A full accept adds the bonus event
 // from the target head after the last draft (unless NO_BONUS).
 __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
+    __shared__ float epi_consts[4 * 8 * MAX_MIX];
     const int lane = threadIdx.x & 31;
     const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
     const CallParams& P = *a.P;
@@ -753,13 +754,64 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
         const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
         if (!at) {
+            // Per-component constants of both heads, computed once per
+            // sequence: running sums of w_T (the component pick), mu, sigma,
+            // 1/sigma and log w - log sigma.  The log tau and log(2 pi)/2
+            // terms of log g_T and log g_D cancel in their difference.
+            float* cs = epi_consts + (threadIdx.x >> 5) * 8 * MAX_MIX;
+            float *cumT = cs, *muT = cs + MAX_MIX, *sgT = cs + 2 * MAX_MIX, *isT = cs + 3 * MAX_MIX;
+            float *cT = cs + 4 * MAX_MIX, *muD = cs + 5 * MAX_MIX, *isD = cs + 6 * MAX_MIX, *cD = cs + 7 * MAX_MIX;
+            const int MT = a.MT, MD = a.MD;
+            for (int m = lane; m < MT; m += 32) {
+                muT[m] = hT[MT + m];
+                sgT[m] = expf(hT[2 * MT + m]);
+                isT[m] = expf(-hT[2 * MT + m]);
+                cT[m] = hT[m] - hT[2 * MT + m];
+            }
+            for (int m = lane; m < MD; m += 32) {
+                muD[m] = hD[MD + m];
+                isD[m] = expf(-hD[2 * MD + m]);
+                cD[m] = hD[m] - hD[2 * MD + m];
+            }
+            if (lane == 0) {
+                float run = 0.f;
+                for (int m = 0; m < MT; ++m) { run += expf(hT[m]); cumT[m] = run; }
+            }
+            __syncwarp();
+            const float totT = cumT[MT - 1];
             bool found = false;
             float last = 0.f;
             for (int base = 0; base < RESAMPLE_CAP && !found; base += 32) {
                 const int it = base + lane;
                 const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 2u + (uint32_t)it);
-                const float tp = draw_tau(hT, a.MT, u.x, u.y, u.z);
-                const float al = fmaxf(0.f, 1.f - expf(head_log_g(hD, a.MD, tp) - head_log_g(hT, a.MT, tp)));
+                // proposal tau ~ g_T (Theorem 1): component, then log-normal
+                const float target = u.x * totT;
+                int z = MT - 1;
+                for (int m = 0; m < MT; ++m)
+                    if (cumT[m] >= target) { z = m; break; }
+                const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
+                const float lt = fmaf(sgT[z], eps, muT[z]);
+                float mT = -INFINITY, mD = -INFINITY;
+                for (int m = 0; m < MT; ++m) {
+                    const float q = (lt - muT[m]) * isT[m];
+                    mT = fmaxf(mT, cT[m] - 0.5f * q * q);
+                }
+                for (int m = 0; m < MD; ++m) {
+                    const float q = (lt - muD[m]) * isD[m];
+                    mD = fmaxf(mD, cD[m] - 0.5f * q * q);
+                }
+                float sT = 0.f, sD = 0.f;
+                for (int m = 0; m < MT; ++m) {
+                    const float q = (lt - muT[m]) * isT[m];
+                    sT += expf(cT[m] - 0.5f * q * q - mT);
+                }
+                for (int m = 0; m < MD; ++m) {
+                    const float q = (lt - muD[m]) * isD[m];
+                    sD += expf(cD[m] - 0.5f * q * q - mD);
+                }
+                // acceptance probability max(0, 1 - g_D / g_T)
+                const float al = fmaxf(0.f, 1.f - expf((mD + logf(sD)) - (mT + logf(sT))));
+                const float tp = expf(lt);
                 const unsigned ok = __ballot_sync(0xffffffffu, u.w < al);
                 if (ok) {
                     const int j = __ffs(ok) - 1;

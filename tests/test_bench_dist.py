@@ -1,0 +1,70 @@
+"""Multi-rank logic of bench.py on CPU: two gloo ranks, each with its own
+independent batch, whole-job time = the slowest rank's, whole-job rate =
+all ranks' events over that time."""
+import os
+import socket
+import sys
+
+import numpy as np
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank(rank, world, port, q):
+    sys.path.insert(0, ROOT)
+    import torch.distributed as dist
+
+    import bench
+    from paper_2507_09252_gb300 import configs as CF
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        wl = CF.C1
+        tau, mk = bench.rank_histories(wl, rank)
+        ms = 10.0 + 5.0 * rank                # rank 1 is the slow one
+        job_ms = bench.max_over_ranks(ms, world, "cpu")
+        q.put((rank, job_ms, bench.job_rate(world, wl.batch, wl.n_events, job_ms),
+               tau.tobytes(), mk.tobytes()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks():
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_rank, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = [q.get(timeout=120) for _ in range(2)]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    res.sort()
+    sys.path.insert(0, ROOT)
+    from paper_2507_09252_gb300 import configs as CF
+    wl = CF.C1
+    for _, job_ms, rate, _, _ in res:
+        assert job_ms == pytest.approx(15.0)
+        assert rate == pytest.approx(2 * wl.batch * wl.n_events / 0.015)
+    # each rank's histories are its own (no shared units)
+    assert res[0][3] != res[1][3]
+
+
+def test_single_rank_identity():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.max_over_ranks(3.5, 1, "cpu") == 3.5
+    assert bench.job_rate(1, 256, 512, 1000.0) == pytest.approx(256 * 512)
+    from paper_2507_09252_gb300 import configs as CF
+    a = bench.rank_histories(CF.C1, 0)
+    b = bench.rank_histories(CF.C1, 0)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
