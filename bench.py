@@ -49,6 +49,9 @@ def parse():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--host-loop", action="store_true",
+                    help="launch every round's kernels from the host instead of one CUDA graph "
+                         "(same kernels; lets a per-launch profiler see them)")
     return ap.parse_args()
 
 
@@ -288,13 +291,15 @@ def main():
             dist.barrier()
         torch.cuda.synchronize()
 
+    fl = T.TPPSD_FLAG_HOST_LOOP if args.host_loop else 0
+
     def step_sd():
         T.tppsd_prefill(s.ctx, B, tau, mk, H, stream)
-        T.tppsd_sample(s.ctx, B, N, g, 1234, 0, *outs, stream)
+        T.tppsd_sample(s.ctx, B, N, g, 1234, fl, *outs, stream)
 
     def step_ar():
         T.tppsd_prefill(s.ctx, B, tau, mk, H, stream)
-        T.tppsd_sample_autoregressive(s.ctx, B, N, 1234, 0, *outs, stream)
+        T.tppsd_sample_autoregressive(s.ctx, B, N, 1234, fl, *outs, stream)
 
     def timed(step, K, W):
         for _ in range(W):
@@ -326,7 +331,7 @@ def main():
 
     def step_e2e():
         T.tppsd_prefill(s.ctx, B, h_tau, h_mk, H, stream)
-        T.tppsd_sample(s.ctx, B, N, g, 1234, 0, *h_out, stream)
+        T.tppsd_sample(s.ctx, B, N, g, 1234, fl, *h_out, stream)
 
     ms_e2e = timed(step_e2e, max(1, min(args.steps, 3)), 1)
     h2d = B * H * (4 + 4)
@@ -346,7 +351,8 @@ def main():
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_sd, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic", "config": workload_config(wl, wl.seed),
+        "data": "synthetic", "config": {**workload_config(wl, wl.seed),
+                                        "launch": "host loop" if args.host_loop else "one CUDA graph per call"},
         "mean_accepted_per_verify": round(st_sd["accepted"] / max(st_sd["rounds"], 1), 3),
         "alpha": round(st_sd["accepted"] / max(st_sd["drafted"], 1), 4),
         "rounds": st_sd["loop_iters"],

@@ -4,15 +4,17 @@
 // Each round a CTA catches its draft cache up to the last emitted event and
 // then drafts gamma events: head of the draft model -> direct sample
 // (z ~ Cat(w), eps ~ N(0,1), tau = exp(mu_z + sigma_z eps); k ~ f, Sec. 4.2)
-// -> encode the drafted event -> next head.  The critical path of a step is
-// a chain of small matrix-vector products; each is spread over the 128
-// threads (one thread per output, or input slices reduced through shared
-// memory when there are few outputs), and the attention over (head, key
-// range) pairs of the four warps.  Weights are read through L1 in an
-// [in][out] layout (consecutive threads read consecutive words); the
-// sequence's draft KV cache is loaded into shared memory once per round by
-// bulk copies and written through to HBM, so all gamma steps read keys on
-// chip.
+// -> encode the drafted event -> next head.  The critical path is a chain
+// of small matrix-vector products, each spread over the 128 threads: one
+// thread per output when there are many outputs, otherwise input slices
+// whose partial sums are reduced through shared memory, with the bias,
+// residual add and LayerNorm folded into that reduction (d <= 32).  The
+// attention runs over (head, key range) pairs of the four warps.  The two
+// components of the sample (time by warp 0, mark by warp 1) are drawn in
+// parallel with warp scans.  Weights are read through L1 in an [in][out]
+// layout (consecutive threads read consecutive words); the sequence's draft
+// KV cache is loaded into shared memory once per round by bulk copies and
+// written through to HBM, so all gamma steps read keys on chip.
 #include <math.h>
 
 #include "common.cuh"
@@ -59,46 +61,56 @@ __device__ __forceinline__ void load_row16(const T* p, float (&out)[DH]) {
     }
 }
 
-// y[o] = sum_{i<IN} WT[i][o] xs[i] + b[o] for o < OUT (xs, y in shared
-// memory).  Ends with a block barrier.
+// sum_{i<IN} WT[i][o] xs[i] (WT is [IN][OUT], xs in shared memory).
 template <typename TW>
-__device__ __forceinline__ void team_mv(const TW* __restrict__ WT, const float* __restrict__ b,
-                                        const float* xs, int IN, int OUT, float* y, float* part) {
-    const int t = threadIdx.x;
-    if (OUT >= 64) {
-        for (int o = t; o < OUT; o += 128) {
-            float acc = b ? __ldg(b + o) : 0.f;
+__device__ __forceinline__ float dot_col(const TW* __restrict__ WT, int OUT, int o, const float* xs, int IN) {
+    float acc = 0.f;
 #pragma unroll 8
-            for (int i = 0; i < IN; ++i) acc = fmaf(St<TW>::ld(WT + (size_t)i * OUT + o), xs[i], acc);
-            y[o] = acc;
-        }
-        __syncthreads();
-        return;
-    }
-    // few outputs: G input slices, partial sums reduced through shared memory
-    const int OP = OUT <= 32 ? 32 : 64, G = 128 / OP;
-    const int o = t % OP, g = t / OP;
+    for (int i = 0; i < IN; ++i) acc = fmaf(St<TW>::ld(WT + (size_t)i * OUT + o), xs[i], acc);
+    return acc;
+}
+
+// Partial sums of a product with few outputs: thread t takes output
+// ob + t % OP over input slice t / OP of 128 / OP; part[t] receives its sum.
+// Ends with a block barrier; the caller reduces part[g * OP + j] over g.
+template <typename TW>
+__device__ __forceinline__ void split_partials(const TW* __restrict__ WT, int OUT, int ob, const float* xs,
+                                               int IN, int OP, float* part) {
+    const int t = threadIdx.x, G = 128 / OP, o = ob + t % OP, g = t / OP;
     const int per = (IN + G - 1) / G, i0 = g * per, i1 = min(IN, i0 + per);
     float acc = 0.f;
     if (o < OUT) {
 #pragma unroll 8
         for (int i = i0; i < i1; ++i) acc = fmaf(St<TW>::ld(WT + (size_t)i * OUT + o), xs[i], acc);
     }
-    part[g * OP + o] = acc;
+    part[t] = acc;
     __syncthreads();
-    if (t < OUT) {
-        float s = b ? __ldg(b + t) : 0.f;
-        for (int gg = 0; gg < G; ++gg) s += part[gg * OP + t];
-        y[t] = s;
+}
+
+// Residual add + LayerNorm of d <= 32 values by warp 0 (lane j < d holds
+// the summed output j): x = LN(x + y), xin its rounded copy.
+template <typename T>
+__device__ __forceinline__ void warp_resid_ln(float yv, float* x, float* xin, int d, const float* g,
+                                              const float* b) {
+    const int lane = threadIdx.x & 31;
+    const bool live = lane < d;
+    const float v = live ? x[lane] + yv : 0.f;
+    const float mean = warp_sum(v) / d;
+    const float c = live ? v - mean : 0.f;
+    const float inv = 1.0f / sqrtf(warp_sum(c * c) / d + LN_EPS);
+    if (live) {
+        const float o = c * inv * g[lane] + b[lane];
+        x[lane] = o;
+        xin[lane] = St<T>::rnd(o);
     }
-    __syncthreads();
 }
 
 // Attention of one query (qs in shared memory, nh heads of DH) over keys
 // 0..n_keys-1 of K/V blocks [nh][stride][DH] (shared or global): warp w
 // takes head w % nh and key range w / nh of 4 / nh; lane-strided keys with
 // a private online softmax (exp2 units), warp merge by shuffles, then the
-// warps of a head merge through shared memory.  Ends with a barrier.
+// warps of a head merge through shared memory; the output is rounded to
+// the storage type.  Ends with a barrier.
 template <typename T, int DH>
 __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
                                             int n_keys, int nh, float* out, float* scratch) {
@@ -161,42 +173,71 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
             L += src[1] * e;
             O += src[2 + c] * e;
         }
-        out[t] = O / L;
+        out[t] = St<T>::rnd(O / L);
     }
     __syncthreads();
 }
 
-// Residual add + LayerNorm of x (shared, d) by warp 0; also its rounded copy.
-template <typename T>
-__device__ __forceinline__ void team_add_ln(float* x, const float* y, float* xin, int d, const float* g,
-                                            const float* b) {
-    if (threadIdx.x < 32) {
-        const int lane = threadIdx.x;
-        float sum = 0.f;
-        for (int i = lane; i < d; i += 32) { x[i] += y[i]; sum += x[i]; }
-        const float mean = warp_sum(sum) / d;
-        float var = 0.f;
-        for (int i = lane; i < d; i += 32) var += (x[i] - mean) * (x[i] - mean);
-        const float inv = 1.0f / sqrtf(warp_sum(var) / d + LN_EPS);
-        for (int i = lane; i < d; i += 32) {
-            const float v = (x[i] - mean) * inv * g[i] + b[i];
-            x[i] = v;
-            xin[i] = St<T>::rnd(v);
-        }
+// Warp-parallel log-softmax of n <= 32*R values v[] (shared) in place, then
+// the smallest index whose running sum of probabilities reaches u * total.
+template <int R>
+__device__ __forceinline__ int warp_logsoftmax_pick(float* v, int n, float u) {
+    const int lane = threadIdx.x & 31;
+    float x[R];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int i = lane + 32 * r;
+        x[r] = i < n ? v[i] : -INFINITY;
+        mx = fmaxf(mx, x[r]);
     }
-    __syncthreads();
+    mx = warp_max(mx);
+    float sm = 0.f;
+#pragma unroll
+    for (int r = 0; r < R; ++r) sm += lane + 32 * r < n ? expf(x[r] - mx) : 0.f;
+    const float lz = mx + logf(warp_sum(sm));
+    float p[R], tot = 0.f;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int i = lane + 32 * r;
+        p[r] = 0.f;
+        if (i < n) {
+            x[r] -= lz;
+            v[i] = x[r];
+            p[r] = expf(x[r]);
+        }
+        tot += p[r];
+    }
+    const float target = u * warp_sum(tot);
+    float base = 0.f;
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        float c = p[r];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float t = __shfl_up_sync(FULL, c, o);
+            if (lane >= o) c += t;
+        }
+        const unsigned hit = __ballot_sync(FULL, lane + 32 * r < n && base + c >= target);
+        if (hit) return 32 * r + __ffs(hit) - 1;
+        base += __shfl_sync(FULL, c, 31);
+    }
+    return n - 1;
 }
 
 template <typename T, int DH, bool KVS>
 __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
     extern __shared__ __align__(16) char smem[];
+    __shared__ double t_new;
+    __shared__ int k_new;
     const int s = blockIdx.x;
     const CallParams& P = *a.P;
     if (s >= P.B || a.ss.done[s]) return;
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const DevModelT& m = a.m.t;
     const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
     const int n_max = a.kv.n_max;
+    const int OPd = d <= 32 ? 32 : 64;  // output block of the few-output products
     // shared layout: [resident KV][mbarrier][work vectors]
     const size_t kvb = KVS ? (((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15) : 0;
     T* kvs = (T*)smem;
@@ -206,9 +247,9 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
     float* qkv = xin + d;
     float* att = qkv + 3 * d;
     float* hid = att + d;
-    float* e = hid + F;
-    float* av = e + 3 * d;
-    float* hd = av + d;
+    float* y = hid + F;
+    float* e = y + d;  // E h (3d) | tanh(V_k1 h + b_k1) (d)
+    float* hd = e + 4 * d;
     float* part = hd + ((W + 3) & ~3);
     float* attn = part + 128;
     const SeqState& ss = a.ss;
@@ -232,28 +273,58 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
         __syncthreads();
         mbar_wait(bar, 0, a.err, 12);
     }
-    auto encode = [&](int p) {
-        const size_t so = (size_t)s * ss.n_max + p;
-        const double t = ss.t[so];
-        const int k = min(max(ss.k[so], 0), K - 1);
-        for (int i = tid; i < d; i += 128) {
-            const double ang = t * m.omega[i >> 1];
-            const double red = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
-            float sv, cv;
-            sincosf((float)red, &sv, &cv);
-            const float v = ((i & 1) ? cv : sv) + m.type_emb[(size_t)k * d + i];
-            x[i] = v;
-            xin[i] = St<T>::rnd(v);
+    // x = LN(x + W_T in + b): few-output product, then the residual add and
+    // LayerNorm (folded into the reduction when d <= 32).  Ends synced.
+    auto proj_resid_ln = [&](const T* WT, const float* bias, const float* in, int IN, const float* g,
+                             const float* b) {
+        split_partials<T>(WT, d, 0, in, IN, OPd, part);
+        if (d <= 32) {
+            if (warp == 0) {
+                float v = 0.f;
+                if (lane < d) {
+                    v = bias[lane];
+                    for (int gg = 0; gg < 128 / OPd; ++gg) v += part[gg * OPd + lane];
+                }
+                warp_resid_ln<T>(v, x, xin, d, g, b);
+            }
+            __syncthreads();
+            return;
+        }
+        for (int ob = 0; ob < d; ob += OPd) {
+            if (ob > 0) split_partials<T>(WT, d, ob, in, IN, OPd, part);
+            if (tid < OPd && ob + tid < d) {
+                float v = bias[ob + tid];
+                for (int gg = 0; gg < 128 / OPd; ++gg) v += part[gg * OPd + tid];
+                y[ob + tid] = v;
+            }
+            __syncthreads();
+        }
+        if (warp == 0) {
+            float sum = 0.f;
+            for (int i = lane; i < d; i += 32) { x[i] += y[i]; sum += x[i]; }
+            const float mean = warp_sum(sum) / d;
+            float var = 0.f;
+            for (int i = lane; i < d; i += 32) var += (x[i] - mean) * (x[i] - mean);
+            const float inv = 1.0f / sqrtf(warp_sum(var) / d + LN_EPS);
+            for (int i = lane; i < d; i += 32) {
+                const float v = (x[i] - mean) * inv * g[i] + b[i];
+                x[i] = v;
+                xin[i] = St<T>::rnd(v);
+            }
         }
         __syncthreads();
+    };
+    // Layers of the encode step at position p from x / xin (set and synced
+    // by the caller); leaves the final hidden state in x (synced).
+    auto layers = [&](int p) {
         for (int l = 0; l < L; ++l) {
             const LayerW& Wl = m.layer[l];
-            team_mv<T>((const T*)Wl.w_qkv, Wl.b_qkv, xin, d, 3 * d, qkv, part);
-            for (int i = tid; i < 3 * d; i += 128) {
-                const float v = St<T>::rnd(qkv[i]);
-                qkv[i] = v;
-                if (i >= d) {
-                    const int w = i < 2 * d ? 0 : 1, c = i - d - w * d, hh = c / DH, ee = c - hh * DH;
+            // Q, K, V; K and V appended to the cache at position p
+            for (int o = tid; o < 3 * d; o += 128) {
+                const float v = St<T>::rnd(dot_col<T>((const T*)Wl.w_qkv, 3 * d, o, xin, d) + Wl.b_qkv[o]);
+                qkv[o] = v;
+                if (o >= d) {
+                    const int w = o < 2 * d ? 0 : 1, c = o - d - w * d, hh = c / DH, ee = c - hh * DH;
                     const size_t off = ((size_t)hh * n_max + p) * DH + ee;
                     St<T>::st(gk(l, w) + off, v);
                     if (KVS) St<T>::st(sk(l, w) + off, v);
@@ -263,61 +334,105 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
             const T* kb = KVS ? sk(l, 0) : gk(l, 0);
             const T* vb = KVS ? sk(l, 1) : gk(l, 1);
             team_attend<T, DH>(qkv, kb, vb, n_max, p + 1, NH, att, attn);
-            for (int i = tid; i < d; i += 128) att[i] = St<T>::rnd(att[i]);
+            proj_resid_ln((const T*)Wl.w_o, Wl.b_o, att, d, Wl.ln1_g, Wl.ln1_b);
+            for (int o = tid; o < F; o += 128)
+                hid[o] = St<T>::rnd(fmaxf(dot_col<T>((const T*)Wl.w_1, F, o, xin, d) + Wl.b_1[o], 0.f));
             __syncthreads();
-            team_mv<T>((const T*)Wl.w_o, Wl.b_o, att, d, d, e, part);
-            team_add_ln<T>(x, e, xin, d, Wl.ln1_g, Wl.ln1_b);
-            team_mv<T>((const T*)Wl.w_1, Wl.b_1, xin, d, F, hid, part);
-            for (int i = tid; i < F; i += 128) hid[i] = St<T>::rnd(fmaxf(hid[i], 0.f));
-            __syncthreads();
-            team_mv<T>((const T*)Wl.w_2, Wl.b_2, hid, F, d, e, part);
-            team_add_ln<T>(x, e, xin, d, Wl.ln2_g, Wl.ln2_b);
+            proj_resid_ln((const T*)Wl.w_2, Wl.b_2, hid, F, Wl.ln2_g, Wl.ln2_b);
         }
     };
-    for (int p = nd; p < n; ++p) encode(p);
+    // Encoding of event (t, k) into x / xin (App. D.4 THP encoding, angle
+    // reduced mod 2 pi in fp64, plus the mark embedding).  Not synced.
+    auto embed = [&](double t, int k) {
+        for (int i = tid; i < d; i += 128) {
+            const double ang = t * m.omega[i >> 1];
+            const double red = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
+            float sv, cv;
+            sincosf((float)red, &sv, &cv);
+            const float v = ((i & 1) ? cv : sv) + m.type_emb[(size_t)k * d + i];
+            x[i] = v;
+            xin[i] = St<T>::rnd(v);
+        }
+    };
+    for (int p = nd; p < n; ++p) {  // catch-up over events already emitted
+        const size_t so = (size_t)s * ss.n_max + p;
+        embed(ss.t[so], min(max(ss.k[so], 0), K - 1));
+        __syncthreads();
+        layers(p);
+    }
     if (tid == 0) {
         const long long last = n + a.gamma - 2;  // last position the round encodes
         atomicAdd(&a.st->draft_keys, (unsigned long long)((last + 1) * (last + 2) / 2 - (long long)nd * (nd + 1) / 2));
     }
     const HeadW& H = m.head;
+    const int OPh = W <= 32 ? 32 : (W <= 64 ? 64 : 128);
     for (int l = 1; l <= a.gamma; ++l) {
         const int p = n + l - 1;  // index of the drafted event
-        // head (Sec. 4.2): e = E h, a = tanh(V_k1 h + b), then the small maps
-        team_mv<float>(H.E, nullptr, x, d, 3 * d, e, part);
-        team_mv<float>(H.v_k1, H.b_k1, x, d, d, av, part);
-        for (int i = tid; i < d; i += 128) av[i] = tanhf(av[i]);
+        // head (Sec. 4.2): e = E h | a = tanh(V_k1 h + b_k1)
+        for (int o = tid; o < 4 * d; o += 128)
+            e[o] = o < 3 * d ? dot_col<float>(H.E, 3 * d, o, x, d)
+                             : tanhf(dot_col<float>(H.v_k1, d, o - 3 * d, x, d) + H.b_k1[o - 3 * d]);
         __syncthreads();
-        team_mv<float>(H.v_w, H.b_w, e, d, M, hd, part);
-        team_mv<float>(H.v_mu, H.b_mu, e + d, d, M, hd + M, part);
-        team_mv<float>(H.v_s, H.b_s, e + 2 * d, d, M, hd + 2 * M, part);
-        team_mv<float>(H.v_k2, H.b_k2, av, d, K, hd + 3 * M, part);
-        const int warp = tid >> 5;
-        if (warp < 2) {  // log-softmax of w (warp 0) and f (warp 1)
-            float* v = warp == 0 ? hd : hd + 3 * M;
-            const int nn = warp == 0 ? M : K, lane = tid & 31;
-            float mx = -INFINITY;
-            for (int i = lane; i < nn; i += 32) mx = fmaxf(mx, v[i]);
-            mx = warp_max(mx);
-            float sm = 0.f;
-            for (int i = lane; i < nn; i += 32) sm += expf(v[i] - mx);
-            const float lz = mx + logf(warp_sum(sm));
-            __syncwarp();
-            for (int i = lane; i < nn; i += 32) v[i] -= lz;
+        // [w logits | mu | log sigma | mark logits] in blocks of OPh outputs;
+        // output j reads its own matrix and input segment
+        for (int ob = 0; ob < W; ob += OPh) {
+            {
+                const int G = 128 / OPh, o = ob + tid % OPh, g = tid / OPh;
+                const int per = (d + G - 1) / G, i0 = g * per, i1 = min(d, i0 + per);
+                float acc = 0.f;
+                if (o < W) {
+                    const float* WT;
+                    const float* in;
+                    int ld, oo;
+                    if (o < M) { WT = H.v_w; in = e; ld = M; oo = o; }
+                    else if (o < 2 * M) { WT = H.v_mu; in = e + d; ld = M; oo = o - M; }
+                    else if (o < 3 * M) { WT = H.v_s; in = e + 2 * d; ld = M; oo = o - 2 * M; }
+                    else { WT = H.v_k2; in = e + 3 * d; ld = K; oo = o - 3 * M; }
+#pragma unroll 8
+                    for (int i = i0; i < i1; ++i) acc = fmaf(WT[(size_t)i * ld + oo], in[i], acc);
+                }
+                part[tid] = acc;
+            }
+            __syncthreads();
+            if (tid < OPh && ob + tid < W) {
+                const int o = ob + tid;
+                float v = o < M ? H.b_w[o] : o < 2 * M ? H.b_mu[o - M] : o < 3 * M ? H.b_s[o - 2 * M] : H.b_k2[o - 3 * M];
+                for (int gg = 0; gg < 128 / OPh; ++gg) v += part[gg * OPh + tid];
+                hd[o] = v;
+            }
+            __syncthreads();
+        }
+        // direct sample: warp 0 the time (component, Box-Muller), warp 1 the
+        // mark; both normalise their logits in place
+        const size_t so = (size_t)s * ss.n_max + p;
+        if (warp < 2) {
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
+            if (warp == 0) {
+                const int z = warp_logsoftmax_pick<2>(hd, M, u.x);
+                if (lane == 0) {
+                    const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
+                    const float tau = expf(hd[M + z] + expf(hd[2 * M + z]) * eps);
+                    const double t = ss.t[so - 1] + (double)tau;
+                    ss.tau[so] = tau;
+                    ss.t[so] = t;
+                    t_new = t;
+                }
+            } else {
+                const int k = warp_logsoftmax_pick<8>(hd + 3 * M, K, u.w);
+                if (lane == 0) {
+                    ss.k[so] = k;
+                    k_new = k;
+                }
+            }
         }
         __syncthreads();
         float* rec = a.heads + ((size_t)s * a.gamma_max + (l - 1)) * W;
         for (int i = tid; i < W; i += 128) rec[i] = hd[i];
-        if (tid == 0) {
-            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
-            const float tau = draw_tau(hd, M, u.x, u.y, u.z);
-            const int k = pick_categorical_log(hd + 3 * M, K, u.w);
-            const size_t o = (size_t)s * ss.n_max + p;
-            ss.tau[o] = tau;
-            ss.t[o] = ss.t[o - 1] + (double)tau;
-            ss.k[o] = k;
+        if (l < a.gamma) {
+            embed(t_new, k_new);
+            __syncthreads();
+            layers(p);
         }
-        __syncthreads();
-        if (l < a.gamma) encode(p);
     }
 }
 
@@ -349,7 +464,7 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
     const size_t eb = m.dtype == 1 ? 2 : 4;
     const int W = 3 * m.M + m.K;
-    const size_t fl = sizeof(float) * (10 * (size_t)m.d + m.F + ((W + 3) & ~3) + 128 + 4 * 66) + 16;
+    const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + 128 + 4 * 66) + 16;
     const size_t kvb = ((size_t)m.L * 2 * kv.n_max * m.d * eb + 15) & ~(size_t)15;
     const int kvs = kvb + fl <= 110 * 1024;
     const size_t sm = (kvs ? kvb : 0) + fl;

@@ -175,6 +175,7 @@ struct TcLayerMaps { CUtensorMap wqkv, wo, w1, w2; };
 struct TcPlan {
     int enabled;
     int bn_qkv, bn_o, bn_ffn1;
+    int ln_cluster;  // LayerNorm GEMMs by column-split clusters (else one CTA per 128 full rows)
     int* err;
     CUtensorMap a_xb, a_att, a_hid;
     TcLayerMaps layer[MAX_LAYERS];
@@ -182,6 +183,12 @@ struct TcPlan {
 bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows);
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
                            cudaStream_t st);
+// Columns per CTA of the cluster LayerNorm GEMM for a row width N (0: unsupported).
+int ln_cluster_cols(int N);
+// EPI_TC_RESID_LN by a cluster of N / ln_cluster_cols(N) CTAs per 128 rows;
+// W's tensor map has boxes of ln_cluster_cols(N) rows.
+cudaError_t launch_gemm_ln_cluster(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a,
+                                   cudaStream_t st);
 
 // ---------------------------------------------------------------- launchers
 // All return cudaGetLastError() of their launches.

@@ -258,6 +258,148 @@ __global__ void __launch_bounds__(128, 1)
     if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
 }
 
+// ---------------------------------------------------------------- LayerNorm GEMM
+// Y = LayerNorm(A W^T + b + resid) over rows of N = CL * BNC columns.  A
+// cluster of CL CTAs shares 128 rows, CTA j computing columns j*BNC ..
+// (j+1)*BNC - 1 on the tensor cores, so a row's LayerNorm statistics are
+// summed over the cluster through distributed shared memory (two-pass:
+// mean, then the centred sum of squares).  Thread t owns row t of the tile.
+// The residual rows of the CTA's columns are prefetched by bulk copies
+// while the main loop runs.
+template <int BNC>
+struct LnShape {
+    static constexpr int BM = 128, BK = 64, STAGES = 4;
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = BNC * BK * 2;
+    static constexpr int STAGE = A_BYTES + B_BYTES;
+    static constexpr int RLD = BNC + 4;              // padded residual row (floats)
+    static constexpr int RES_BYTES = BM * RLD * 4;
+    static constexpr int TMEM_COLS = BNC;
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE + RES_BYTES + 2 * BM * 4 + 1024 + 256;
+};
+
+template <int BNC>
+__global__ void __launch_bounds__(128, 1)
+    k_gemm_ln_cl(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, TcGemmArgs a) {
+    using S = LnShape<BNC>;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    float* resid_s = (float*)(smem + S::STAGES * S::STAGE);
+    float* red1 = resid_s + S::BM * S::RLD;
+    float* red2 = red1 + S::BM;
+    uint64_t* full = (uint64_t*)(red2 + S::BM);
+    uint64_t* empty = full + S::STAGES;
+    uint64_t* done = empty + S::STAGES;
+    uint64_t* resbar = done + 1;
+    uint32_t* tslot = (uint32_t*)(resbar + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t crank = cluster_ctarank(), ncl = cluster_nctarank();
+    const int n0 = (int)crank * BNC, m0 = blockIdx.y * S::BM;
+    const int KB = a.K / S::BK, N = a.N;
+    const int rows = min(S::BM, a.R - m0);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(done, 1);
+        mbar_init(resbar, 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, S::TMEM_COLS);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // residual rows (BNC contiguous floats each), then the A / W tiles
+        mbar_arrive_expect_tx(resbar, (uint32_t)rows * BNC * 4);
+        for (int r = 0; r < rows; ++r)
+            bulk_load(resid_s + r * S::RLD, a.resid + (size_t)(m0 + r) * N + n0, BNC * 4, resbar);
+        for (int kb = 0; kb < KB; ++kb) {
+            const int s = kb % S::STAGES, round = kb / S::STAGES;
+            if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
+            mbar_arrive_expect_tx(&full[s], S::STAGE);
+            unsigned char* st = smem + s * S::STAGE;
+            tma_load_2d(st, &mapA, &full[s], kb * S::BK, m0);
+            tma_load_2d(st + S::A_BYTES, &mapB, &full[s], kb * S::BK, n0);
+        }
+    } else if (warp == 1 && lane == 0) {
+        const uint32_t idesc = idesc_bf16(128, BNC);
+        for (int kb = 0; kb < KB; ++kb) {
+            const int s = kb % S::STAGES, round = kb / S::STAGES;
+            if (!mbar_wait(&full[s], round & 1, a.err, 2)) break;
+            tc_fence_after();
+            const uint32_t abase = smem_u32(smem + s * S::STAGE), bbase = abase + S::A_BYTES;
+#pragma unroll
+            for (int kk = 0; kk < S::BK / 16; ++kk)
+                tc_mma_bf16(tmem, sw128_desc(abase + kk * 32), sw128_desc(bbase + kk * 32), idesc,
+                            (kb | kk) != 0);
+            tc_commit(&empty[s]);
+        }
+        tc_commit(done);
+    }
+    __syncwarp();
+    const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
+    tc_fence_after();
+    const bool have_res = mbar_wait(resbar, 0, a.err, 4);
+
+    const int t = warp * 32 + lane, r = m0 + t;
+    const bool live = ok && t < rows;
+    const uint32_t tw = tmem + ((uint32_t)(warp * 32) << 16);
+    float y[BNC];
+#pragma unroll
+    for (int c0 = 0; c0 < BNC; c0 += 16) {
+        float v[16];
+        tmem_ld16(tw + c0, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) y[c0 + i] = v[i] + a.bias[n0 + c0 + i];
+    }
+    float s1 = 0.f;
+    if (live) {
+#pragma unroll
+        for (int c = 0; c < BNC; c += 4) {
+            const float4 q = have_res ? *reinterpret_cast<const float4*>(resid_s + t * S::RLD + c)
+                                      : *reinterpret_cast<const float4*>(a.resid + (size_t)r * N + n0 + c);
+            y[c] += q.x; y[c + 1] += q.y; y[c + 2] += q.z; y[c + 3] += q.w;
+        }
+#pragma unroll
+        for (int c = 0; c < BNC; ++c) s1 += y[c];
+    }
+    red1[t] = s1;
+    cluster_sync();
+    float tot1 = 0.f;
+    for (uint32_t j = 0; j < ncl; ++j) tot1 += ld_dsmem_f32(red1 + t, j);
+    const float mean = tot1 / N;
+    float s2 = 0.f;
+#pragma unroll
+    for (int c = 0; c < BNC; ++c) s2 += (y[c] - mean) * (y[c] - mean);
+    red2[t] = s2;
+    cluster_sync();
+    float tot2 = 0.f;
+    for (uint32_t j = 0; j < ncl; ++j) tot2 += ld_dsmem_f32(red2 + t, j);
+    const float inv = 1.0f / sqrtf(tot2 / N + LN_EPS);
+    if (live) {
+#pragma unroll
+        for (int c0 = 0; c0 < BNC; c0 += 16) {
+            float o[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                o[i] = (y[c0 + i] - mean) * inv * a.ln_g[n0 + c0 + i] + a.ln_b[n0 + c0 + i];
+            float4* xo = reinterpret_cast<float4*>(a.x_out + (size_t)r * N + n0 + c0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) xo[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
+            st_bf16x16(a.xb_out + (size_t)r * N + n0 + c0, o);
+        }
+    }
+    cluster_sync();  // no CTA leaves while another may still read its red2
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
+}
+
 // ---------------------------------------------------------------- host side
 static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -292,6 +434,44 @@ static cudaError_t launch_bn(const CUtensorMap& A, const CUtensorMap& W, const T
     const dim3 grid(a.N / BN, (a.R + 127) / 128);
     k_gemm_tc<BN><<<grid, 128, sm, st>>>(A, W, a);
     return cudaGetLastError();
+}
+
+template <int BNC>
+static cudaError_t launch_ln_bnc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int CL,
+                                 cudaStream_t st) {
+    const size_t sm = LnShape<BNC>::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_ln_cl<BNC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(CL, (a.R + 127) / 128, 1);
+    cfg.blockDim = dim3(128, 1, 1);
+    cfg.dynamicSmemBytes = sm;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = CL;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, k_gemm_ln_cl<BNC>, A, W, a);
+}
+
+int ln_cluster_cols(int N) {
+    if (N % 32 || N < 32) return 0;
+    if (N <= 256) return 32;
+    if (N <= 512 && N % 64 == 0) return 64;
+    return 0;
+}
+
+cudaError_t launch_gemm_ln_cluster(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a,
+                                   cudaStream_t st) {
+    if (a.R <= 0) return cudaSuccess;
+    const int bnc = ln_cluster_cols(a.N);
+    if (!bnc || a.K % 64) return cudaErrorInvalidValue;
+    const int CL = a.N / bnc;
+    if (CL > 8) return cudaErrorInvalidValue;
+    return bnc == 32 ? launch_ln_bnc<32>(A, W, a, CL, st) : launch_ln_bnc<64>(A, W, a, CL, st);
 }
 
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,

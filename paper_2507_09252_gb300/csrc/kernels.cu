@@ -1,10 +1,13 @@
 // Kernels of the TPP-SD sampler (arxiv 2507.09252) for GB300 (sm_103a).
 //
-// One sampling round of Alg. 1 is: k_draft (gamma draft events per
-// sequence, Sec. 4.3 "Drafting") -> batched target forward over gamma+1
-// positions per sequence (Sec. 4.3 "Verification") -> k_head ->
-// k_verify_epilogue (ratio tests, first rejection, Theorem-1 / Eq. 4
-// resampling, commit and cache rollback) -> k_round_control.
+// One sampling round of Alg. 1 is: the draft kernel (gamma draft events per
+// sequence, Sec. 4.3 "Drafting": k_draft_team in draft.cu, or k_draft here
+// for shapes it does not cover) -> batched target forward over gamma+1
+// positions per sequence (Sec. 4.3 "Verification"; tensor-core GEMMs in
+// gemm_tc.cu and attention in attn.cu for bf16 models) -> heads (fp32 GEMM
+// + k_head_out) -> k_verify_epilogue (ratio tests, first rejection,
+// Theorem-1 / Eq. 4 resampling, commit and cache rollback) ->
+// k_round_control.
 #include <math.h>
 
 #include "common.cuh"
@@ -456,22 +459,6 @@ __global__ void __launch_bounds__(256) k_attention_single(AttArgs<T> a) {
     cta_attend_one<T, DH>(qs, a.kc + base, a.vc + base, a.row_pos[r] + 1, a.nh, a.kv.n_max,
                           a.scale, os, scratch);
     for (int i = threadIdx.x; i < a.d; i += blockDim.x) St<T>::st(a.out + (size_t)r * a.d + i, os[i]);
-}
-
-// Heads of every active row: CTA per row.
-__global__ void __launch_bounds__(128) k_head(DevModel m, Work w, int count) {
-    extern __shared__ float sh[];
-    const int r = blockIdx.x;
-    if (r >= count || w.row_seq[r] < 0) return;
-    const int d = m.d, W = m.head_width();
-    float* h = sh;
-    float* e = h + d;
-    float* a = e + 3 * d;
-    float* out = a + d;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) h[i] = w.x[(size_t)r * d + i];
-    __syncthreads();
-    cta_head(m.head, d, m.M, m.K, h, e, a, out);
-    for (int i = threadIdx.x; i < W; i += blockDim.x) w.heads[(size_t)r * W + i] = out[i];
 }
 
 // Head outputs from the batched pre-activations hd4 = [E h | V_k1 h + b_k1]
@@ -1061,7 +1048,9 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             go.resid = w.x; go.x_out = w.x; go.xb_out = (bf16*)xb; go.ln_g = L.ln1_g; go.ln_b = L.ln1_b;
             go.err = tc->err;
             PROF_MARK(prof, KC_GEMM_O, 1, st);
-            if ((e = launch_gemm_tc(tc->a_att, tc->layer[l].wo, go, tc->bn_o, st)) != cudaSuccess) return e;
+            e = tc->ln_cluster ? launch_gemm_ln_cluster(tc->a_att, tc->layer[l].wo, go, st)
+                               : launch_gemm_tc(tc->a_att, tc->layer[l].wo, go, tc->bn_o, st);
+            if (e != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_O, 0, st);
             TcGemmArgs g1{};
             g1.R = R; g1.N = F; g1.K = d; g1.epi = EPI_TC_RELU; g1.bias = L.b_1; g1.out_t = (bf16*)hid;
@@ -1074,7 +1063,9 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             g2.resid = w.x; g2.x_out = w.x; g2.xb_out = (bf16*)xb; g2.ln_g = L.ln2_g; g2.ln_b = L.ln2_b;
             g2.err = tc->err;
             PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
-            if ((e = launch_gemm_tc(tc->a_hid, tc->layer[l].w2, g2, tc->bn_o, st)) != cudaSuccess) return e;
+            e = tc->ln_cluster ? launch_gemm_ln_cluster(tc->a_hid, tc->layer[l].w2, g2, st)
+                               : launch_gemm_tc(tc->a_hid, tc->layer[l].w2, g2, tc->bn_o, st);
+            if (e != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
             nl += 5;
             continue;
