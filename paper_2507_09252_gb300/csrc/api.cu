@@ -395,8 +395,7 @@ static void build_tc_plan(tppsd_ctx* ctx) {
     if (d % 64 || F % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
     p.bn_qkv = pick_bn(3 * d);
     p.bn_ffn1 = pick_bn(F);
-    p.ln_cluster = getenv("TPPSD_LN_ROWS") ? 0 : 1;
-    p.bn_o = p.ln_cluster ? ln_cluster_cols(d) : d;
+    p.bn_o = ln_cluster_cols(d);
     if (!p.bn_qkv || !p.bn_ffn1 || !p.bn_o) return;
     const Work& w = ctx->work;
     bool ok = make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128) &&

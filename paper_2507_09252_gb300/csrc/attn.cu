@@ -22,7 +22,7 @@ namespace tppsd {
 
 template <int DH>
 struct AttnShape {
-    static constexpr int KT = 2048 / DH;             // keys per tile: 4 KB of K, 4 KB of V
+    static constexpr int KT = 1024 / DH;             // keys per tile: 2 KB of K, 2 KB of V
     static constexpr int TILE_BYTES = KT * DH * 2;
     static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
     static constexpr int WARP_BYTES = 2 * STAGE_BYTES + 32;  // two stages + two mbarriers
@@ -55,7 +55,7 @@ __device__ __forceinline__ uint32_t pack_half2(float x, float y) {
 }
 
 template <int DH>
-__global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
+__global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) {
     using S = AttnShape<DH>;
     constexpr int KT = S::KT, NT = KT / 8, KS = DH / 16;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -69,21 +69,13 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
     const int re = min(rb + 16, r_hi);
     if (rb >= re) return;
     const int s = a.row_seq[rb];
+    const int maxpos = a.row_pos[re - 1];  // rows of a sequence are in position order
     if (s < 0) return;  // rows of one sequence are all active or all inactive
     const int nq = re - rb;
     unsigned char* wbase = smem + warp * S::WARP_BYTES;
     uint64_t* bars = (uint64_t*)(wbase + 2 * S::STAGE_BYTES);
     float* merge = (float*)(smem + 4 * S::WARP_BYTES);
     int* qpos = (int*)(smem + 4 * S::WARP_BYTES + S::MERGE_BYTES);
-    if (threadIdx.x < 16) qpos[threadIdx.x] = threadIdx.x < nq ? a.row_pos[rb + threadIdx.x] : -1;
-    if (lane == 0) {
-        mbar_init(&bars[0], 1);
-        mbar_init(&bars[1], 1);
-        mbar_fence_init();
-    }
-    __syncthreads();
-    const int maxpos = qpos[nq - 1];
-    const int pos_g = qpos[g], pos_g8 = qpos[g + 8];  // -1 for padding rows
     // this warp's key range [klo, khi)
     const int nkeys = maxpos + 1;
     const int share = (((nkeys + 3) / 4) + 7) & ~7;
@@ -92,6 +84,22 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
     const size_t base = ((((size_t)a.layer * a.kv.Bmax + s) * a.nh + h) * (size_t)a.kv.n_max) * DH;
     const bf16* kg = a.kc + base;
     const bf16* vg = a.vc + base;
+    auto issue = [&](int tile, int stage) {
+        const int k0 = klo + tile * KT, cnt = min(KT, khi - k0);
+        const uint32_t bytes = (uint32_t)cnt * DH * 2;
+        unsigned char* st = wbase + stage * S::STAGE_BYTES;
+        mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
+        bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
+        bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
+    };
+    // the first tile's copy is in flight before anything else is loaded
+    if (lane == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        mbar_fence_init();
+        if (ntl > 0) issue(0, 0);
+    }
+    if (threadIdx.x < 16) qpos[threadIdx.x] = threadIdx.x < nq ? a.row_pos[rb + threadIdx.x] : -1;
 
     // Q fragments (rows g and g+8 of this CTA, all DH columns), bf16 pairs
     uint32_t qa[KS][4];
@@ -112,15 +120,8 @@ __global__ void __launch_bounds__(128) k_attn_mma(AttArgs<bf16> a, int* err) {
 #pragma unroll
     for (int n = 0; n < DH / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
 
-    auto issue = [&](int tile, int stage) {
-        const int k0 = klo + tile * KT, cnt = min(KT, khi - k0);
-        const uint32_t bytes = (uint32_t)cnt * DH * 2;
-        unsigned char* st = wbase + stage * S::STAGE_BYTES;
-        mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
-        bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
-        bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
-    };
-    if (lane == 0 && ntl > 0) issue(0, 0);
+    __syncthreads();  // qpos and the mbarrier inits are visible
+    const int pos_g = qpos[g], pos_g8 = qpos[g + 8];  // -1 for padding rows
     bool ok = true;
     for (int it = 0; it < ntl && ok; ++it) {
         const int stage = it & 1;

@@ -174,8 +174,7 @@ struct TcLayerMaps { CUtensorMap wqkv, wo, w1, w2; };
 // reads (rows = Work.R), built once per context.
 struct TcPlan {
     int enabled;
-    int bn_qkv, bn_o, bn_ffn1;
-    int ln_cluster;  // LayerNorm GEMMs by column-split clusters (else one CTA per 128 full rows)
+    int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
     int* err;
     CUtensorMap a_xb, a_att, a_hid;
     TcLayerMaps layer[MAX_LAYERS];

@@ -7,12 +7,12 @@
 // tcgen05.mma (M=128, N<=256 per instruction, K=16) into a TMEM
 // accumulator and releases each stage with tcgen05.commit; then all four
 // warps read the accumulator back (thread t owns row t of the tile: TMEM
-// lane t) and apply the epilogue:
+// lane t) and apply the epilogue; warps 2-3, idle during the main loop,
+// stage the epilogue's parameters in shared memory meanwhile:
 //   EPI_QKV      bias, bf16 round, Q to the row buffer, K/V scattered into the
 //                KV cache at each row's (sequence, position)
 //   EPI_RELU     bias, ReLU, bf16 round
-//   EPI_RESID_LN bias + residual, LayerNorm over the full row (BN = N = d),
-//                fp32 row and its bf16 copy
+// The residual + LayerNorm epilogue (rows of N = d) is k_gemm_ln_cl below.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -30,9 +30,9 @@ struct TcShape {
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE = A_BYTES + B_BYTES;
     static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
-    // residual rows of the LayerNorm epilogue, prefetched during the main loop
-    static constexpr int RES_BYTES = BN <= 128 ? BM * BN * 4 : 0;
-    static constexpr size_t SMEM = (size_t)STAGES * STAGE + RES_BYTES + 1024 + 256;
+    // epilogue parameters staged in shared memory: bias[BN], row seq/pos[BM]
+    static constexpr int PARAM_BYTES = BN * 4 + 2 * BM * 4;
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE + PARAM_BYTES + 1024 + 256;
 };
 
 __device__ __forceinline__ void st_bf16x16(bf16* dst, const float (&v)[16]) {
@@ -53,13 +53,13 @@ __global__ void __launch_bounds__(128, 1)
     using S = TcShape<BN>;
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    float* resid_s = (float*)(smem + S::STAGES * S::STAGE);
-    uint64_t* full = (uint64_t*)(smem + S::STAGES * S::STAGE + S::RES_BYTES);
+    float* bias_s = (float*)(smem + S::STAGES * S::STAGE);
+    int* rseq_s = (int*)(bias_s + BN);
+    int* rpos_s = rseq_s + S::BM;
+    uint64_t* full = (uint64_t*)(rpos_s + S::BM);
     uint64_t* empty = full + S::STAGES;
     uint64_t* done = empty + S::STAGES;
-    uint64_t* resbar = done + 1;
-    uint32_t* tslot = (uint32_t*)(resbar + 1);
-    const bool res_pref = S::RES_BYTES > 0 && a.epi == EPI_TC_RESID_LN;
+    uint32_t* tslot = (uint32_t*)(done + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n0 = blockIdx.x * BN, m0 = blockIdx.y * S::BM;
     const int KB = a.K / S::BK;
@@ -70,7 +70,6 @@ __global__ void __launch_bounds__(128, 1)
             mbar_init(&empty[s], 1);
         }
         mbar_init(done, 1);
-        mbar_init(resbar, 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(tslot, S::TMEM_COLS);
@@ -80,13 +79,7 @@ __global__ void __launch_bounds__(128, 1)
     const uint32_t tmem = *tslot;
 
     if (warp == 0 && lane == 0) {
-        // producer: the tile's residual rows (contiguous, since N == BN),
-        // then TMA loads of the A and W tiles of every K block
-        if (res_pref) {
-            const uint32_t bytes = (uint32_t)min(S::BM, a.R - m0) * BN * 4;
-            mbar_arrive_expect_tx(resbar, bytes);
-            bulk_load(resid_s, a.resid + (size_t)m0 * BN, bytes, resbar);
-        }
+        // producer: TMA loads of the A and W tiles of every K block
         for (int kb = 0; kb < KB; ++kb) {
             const int s = kb % S::STAGES, round = kb / S::STAGES;
             if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
@@ -117,14 +110,23 @@ __global__ void __launch_bounds__(128, 1)
             tc_commit(&empty[s]);
         }
         tc_commit(done);  // arrives when every MMA above has completed
+    } else if (warp >= 2) {
+        // idle during the main loop: stage the epilogue's parameters
+        const int t = threadIdx.x - 64;
+        for (int c = t; c < BN; c += 64) bias_s[c] = a.bias[n0 + c];
+        if (a.epi == EPI_TC_QKV) {
+            for (int r = t; r < S::BM; r += 64) {
+                const bool in = m0 + r < a.R;
+                rseq_s[r] = in ? a.row_seq[m0 + r] : -1;
+                rpos_s[r] = in ? a.row_pos[m0 + r] : 0;
+            }
+        }
     }
     __syncwarp();
     const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
     tc_fence_after();
-    // every thread waits for the residual copy, so none is in flight at exit
-    const bool have_res = res_pref && mbar_wait(resbar, 0, a.err, 4);
 
-    const int r = m0 + warp * 32 + lane;
+    const int t = warp * 32 + lane, r = m0 + t;
     const bool live = ok && r < a.R;
     const uint32_t tw = tmem + ((uint32_t)(warp * 32) << 16);
     if (ok) {
@@ -134,19 +136,19 @@ __global__ void __launch_bounds__(128, 1)
                 tmem_ld16(tw + c0, v);
                 if (live) {
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) v[i] = fmaxf(v[i] + a.bias[n0 + c0 + i], 0.f);
+                    for (int i = 0; i < 16; ++i) v[i] = fmaxf(v[i] + bias_s[c0 + i], 0.f);
                     st_bf16x16(a.out_t + (size_t)r * a.N + n0 + c0, v);
                 }
             }
-        } else if (a.epi == EPI_TC_QKV) {
-            const int s = live ? a.row_seq[r] : -1, pos = live ? a.row_pos[r] : 0;
+        } else {  // EPI_TC_QKV
+            const int s = live ? rseq_s[t] : -1, pos = rpos_s[t];
             for (int c0 = 0; c0 < BN; c0 += 16) {
                 float v[16];
                 tmem_ld16(tw + c0, v);
                 if (!live) continue;
                 const int col = n0 + c0, which = col / a.d, cc = col - which * a.d;
 #pragma unroll
-                for (int i = 0; i < 16; ++i) v[i] += a.bias[col + i];
+                for (int i = 0; i < 16; ++i) v[i] += bias_s[c0 + i];
                 if (which == 0) {
                     st_bf16x16(a.q_out + (size_t)r * a.d + cc, v);
                 } else if (s >= 0) {
@@ -155,101 +157,6 @@ __global__ void __launch_bounds__(128, 1)
                                 ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
                     st_bf16x16(dst, v);
                 }
-            }
-        } else if (BN <= 256) {  // EPI_TC_RESID_LN, BN == N == d
-            // TMEM -> shared tile [128][BN+1] (stages are free: every MMA is
-            // done), then one warp per row: residual rows from the prefetched
-            // shared copy (global reads if the copy timed out),
-            // coalesced x / xb writes, warp-reduced mean and variance.
-            float* tile = (float*)smem;
-            constexpr int LD = BN + 1;
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                float v[16];
-                tmem_ld16(tw + c0, v);
-                float* dst = tile + (size_t)(warp * 32 + lane) * LD + c0;
-#pragma unroll
-                for (int i = 0; i < 16; ++i) dst[i] = v[i];
-            }
-            __syncthreads();
-            constexpr int PL = BN / 32;  // columns per lane
-            float bias[PL], g[PL], b[PL];
-#pragma unroll
-            for (int j = 0; j < PL; ++j) {
-                bias[j] = a.bias[lane + 32 * j];
-                g[j] = a.ln_g[lane + 32 * j];
-                b[j] = a.ln_b[lane + 32 * j];
-            }
-            // rows in batches of 8: the residual is the output buffer, so the
-            // loads of a batch are all issued before any of its stores
-            constexpr int RB = 8;
-            for (int rr0 = warp; rr0 < 128; rr0 += 4 * RB) {
-                float y[RB][PL];
-#pragma unroll
-                for (int bq = 0; bq < RB; ++bq) {
-                    const int rr = rr0 + 4 * bq, row = m0 + rr;
-#pragma unroll
-                    for (int j = 0; j < PL; ++j) {
-                        const int c = lane + 32 * j;
-                        y[bq][j] = 0.f;
-                        if (rr < 128 && row < a.R)
-                            y[bq][j] = tile[rr * LD + c] + bias[j] +
-                                       (have_res ? resid_s[rr * BN + c] : a.resid[(size_t)row * BN + c]);
-                    }
-                }
-#pragma unroll
-                for (int bq = 0; bq < RB; ++bq) {
-                    const int rr = rr0 + 4 * bq, row = m0 + rr;
-                    float sum = 0.f;
-#pragma unroll
-                    for (int j = 0; j < PL; ++j) sum += y[bq][j];
-                    const float mean = warp_sum(sum) / BN;
-                    float var = 0.f;
-#pragma unroll
-                    for (int j = 0; j < PL; ++j) var += (y[bq][j] - mean) * (y[bq][j] - mean);
-                    const float inv = 1.0f / sqrtf(warp_sum(var) / BN + LN_EPS);
-                    if (rr < 128 && row < a.R) {
-#pragma unroll
-                        for (int j = 0; j < PL; ++j) {
-                            const int c = lane + 32 * j;
-                            const float o = (y[bq][j] - mean) * inv * g[j] + b[j];
-                            a.x_out[(size_t)row * BN + c] = o;
-                            a.xb_out[(size_t)row * BN + c] = __float2bfloat16_rn(o);
-                        }
-                    }
-                }
-            }
-        } else {  // EPI_TC_RESID_LN with BN = 512: row per thread, three passes over TMEM
-            const float* res = a.resid + (size_t)(live ? r : 0) * a.N;
-            float sum = 0.f;
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                float v[16];
-                tmem_ld16(tw + c0, v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) sum += v[i] + a.bias[c0 + i] + (live ? res[c0 + i] : 0.f);
-            }
-            const float mean = sum / BN;
-            float var = 0.f;
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                float v[16];
-                tmem_ld16(tw + c0, v);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const float y = v[i] + a.bias[c0 + i] + (live ? res[c0 + i] : 0.f) - mean;
-                    var += y * y;
-                }
-            }
-            const float inv = 1.0f / sqrtf(var / BN + LN_EPS);
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                float v[16];
-                tmem_ld16(tw + c0, v);
-                if (!live) continue;
-#pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    v[i] = (v[i] + a.bias[c0 + i] + res[c0 + i] - mean) * inv * a.ln_g[c0 + i] + a.ln_b[c0 + i];
-                float4* xo = reinterpret_cast<float4*>(a.x_out + (size_t)r * a.N + c0);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) xo[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-                st_bf16x16(a.xb_out + (size_t)r * a.N + c0, v);
             }
         }
     }
@@ -275,7 +182,7 @@ struct LnShape {
     static constexpr int RLD = BNC + 4;              // padded residual row (floats)
     static constexpr int RES_BYTES = BM * RLD * 4;
     static constexpr int TMEM_COLS = BNC;
-    static constexpr size_t SMEM = (size_t)STAGES * STAGE + RES_BYTES + 2 * BM * 4 + 1024 + 256;
+    static constexpr size_t SMEM = (size_t)STAGES * STAGE + RES_BYTES + 2 * BM * 4 + 3 * BNC * 4 + 1024 + 256;
 };
 
 template <int BNC>
@@ -287,7 +194,8 @@ __global__ void __launch_bounds__(128, 1)
     float* resid_s = (float*)(smem + S::STAGES * S::STAGE);
     float* red1 = resid_s + S::BM * S::RLD;
     float* red2 = red1 + S::BM;
-    uint64_t* full = (uint64_t*)(red2 + S::BM);
+    float* prm = red2 + S::BM;  // bias, LN gain, LN shift of the CTA's columns
+    uint64_t* full = (uint64_t*)(prm + 3 * BNC);
     uint64_t* empty = full + S::STAGES;
     uint64_t* done = empty + S::STAGES;
     uint64_t* resbar = done + 1;
@@ -340,6 +248,12 @@ __global__ void __launch_bounds__(128, 1)
             tc_commit(&empty[s]);
         }
         tc_commit(done);
+    } else if (warp >= 2) {
+        for (int c = threadIdx.x - 64; c < BNC; c += 64) {
+            prm[c] = a.bias[n0 + c];
+            prm[BNC + c] = a.ln_g[n0 + c];
+            prm[2 * BNC + c] = a.ln_b[n0 + c];
+        }
     }
     __syncwarp();
     const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
@@ -355,7 +269,7 @@ __global__ void __launch_bounds__(128, 1)
         float v[16];
         tmem_ld16(tw + c0, v);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) y[c0 + i] = v[i] + a.bias[n0 + c0 + i];
+        for (int i = 0; i < 16; ++i) y[c0 + i] = v[i] + prm[c0 + i];
     }
     float s1 = 0.f;
     if (live) {
@@ -387,7 +301,7 @@ __global__ void __launch_bounds__(128, 1)
             float o[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i)
-                o[i] = (y[c0 + i] - mean) * inv * a.ln_g[n0 + c0 + i] + a.ln_b[n0 + c0 + i];
+                o[i] = (y[c0 + i] - mean) * inv * prm[BNC + c0 + i] + prm[2 * BNC + c0 + i];
             float4* xo = reinterpret_cast<float4*>(a.x_out + (size_t)r * N + n0 + c0);
 #pragma unroll
             for (int i = 0; i < 4; ++i) xo[i] = make_float4(o[4 * i], o[4 * i + 1], o[4 * i + 2], o[4 * i + 3]);
@@ -477,6 +391,7 @@ cudaError_t launch_gemm_ln_cluster(const CUtensorMap& A, const CUtensorMap& W, c
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
                            cudaStream_t st) {
     if (a.R <= 0) return cudaSuccess;
+    if (a.epi != EPI_TC_QKV && a.epi != EPI_TC_RELU) return cudaErrorInvalidValue;
     switch (BN) {
         case 64: return launch_bn<64>(A, W, a, st);
         case 128: return launch_bn<128>(A, W, a, st);

@@ -1048,8 +1048,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             go.resid = w.x; go.x_out = w.x; go.xb_out = (bf16*)xb; go.ln_g = L.ln1_g; go.ln_b = L.ln1_b;
             go.err = tc->err;
             PROF_MARK(prof, KC_GEMM_O, 1, st);
-            e = tc->ln_cluster ? launch_gemm_ln_cluster(tc->a_att, tc->layer[l].wo, go, st)
-                               : launch_gemm_tc(tc->a_att, tc->layer[l].wo, go, tc->bn_o, st);
+            e = launch_gemm_ln_cluster(tc->a_att, tc->layer[l].wo, go, st);
             if (e != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_O, 0, st);
             TcGemmArgs g1{};
@@ -1063,8 +1062,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             g2.resid = w.x; g2.x_out = w.x; g2.xb_out = (bf16*)xb; g2.ln_g = L.ln2_g; g2.ln_b = L.ln2_b;
             g2.err = tc->err;
             PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
-            e = tc->ln_cluster ? launch_gemm_ln_cluster(tc->a_hid, tc->layer[l].w2, g2, st)
-                               : launch_gemm_tc(tc->a_hid, tc->layer[l].w2, g2, tc->bn_o, st);
+            e = launch_gemm_ln_cluster(tc->a_hid, tc->layer[l].w2, g2, st);
             if (e != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
             nl += 5;

@@ -36,11 +36,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Wait for the phase with the given parity to complete; ~0.3 s limit.
+// Wait for the phase with the given parity to complete.  Polls without
+// sleeping first (the pipelines' waits are short and on the critical path),
+// then backs off; gives up after 2^20 polls (well under a second).
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code) {
     for (int i = 0; i < (1 << 20); ++i) {
         if (mbar_try_wait(bar, parity)) return true;
-        if (i > 32) __nanosleep(256);
+        if (i > 4096) __nanosleep(128);
     }
     if (err) atomicCAS(err, 0, code);
     return false;
