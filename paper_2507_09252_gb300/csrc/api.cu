@@ -408,6 +408,13 @@ static void build_tc_plan(tppsd_ctx* ctx) {
              make_tmap_bf16(&p.layer[l].w1, L.w_1, d, F, p.bn_ffn1 < 256 ? p.bn_ffn1 : 256) &&
              make_tmap_bf16(&p.layer[l].w2, L.w_2, F, d, bo);
     }
+    p.mlp = ok && mlp_tc_supported(d, F) && !getenv("TPPSD_NO_MLP_FUSION");
+    for (int l = 0; l < m.L && p.mlp; ++l) {
+        const LayerW& L = m.layer[l];
+        p.mlp = make_tmap_bf16(&p.layer[l].wo_m, L.w_o, d, d, 128) &&
+                make_tmap_bf16(&p.layer[l].w1_m, L.w_1, d, F, 128) &&
+                make_tmap_bf16(&p.layer[l].w2_m, L.w_2, F, d, 128);
+    }
     p.err = ctx->d_err;
     p.enabled = ok ? 1 : 0;
 }

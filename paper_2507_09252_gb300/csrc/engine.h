@@ -169,12 +169,16 @@ struct TcGemmArgs {
     const float* resid; float* x_out; __nv_bfloat16* xb_out; const float* ln_g; const float* ln_b;
     int* err;  // set (first error wins) if a pipeline wait times out
 };
-struct TcLayerMaps { CUtensorMap wqkv, wo, w1, w2; };
+struct TcLayerMaps {
+    CUtensorMap wqkv, wo, w1, w2;      // boxes of the separate GEMMs
+    CUtensorMap wo_m, w1_m, w2_m;      // boxes of 128 rows for the fused block
+};
 // Tensor maps of one bf16 model's weights and of the row-workspace buffers it
 // reads (rows = Work.R), built once per context.
 struct TcPlan {
     int enabled;
     int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
+    int mlp;                    // post-attention block by the fused kernel
     int* err;
     CUtensorMap a_xb, a_att, a_hid;
     TcLayerMaps layer[MAX_LAYERS];
@@ -182,6 +186,20 @@ struct TcPlan {
 bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows);
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
                            cudaStream_t st);
+// Fused post-attention block of a layer (mlp_tc.cu): x1 = LN1(x + att W_o^T
+// + b_o); x = LN2(x1 + relu(x1 W_1^T + b_1) W_2^T + b_2); xb = bf16(x).
+struct MlpArgs {
+    int R, F;
+    const float *b_o, *ln1_g, *ln1_b, *b_1, *b_2, *ln2_g, *ln2_b;
+    float* x;             // [R][d] residual in, LN2 output out
+    __nv_bfloat16* xb;    // [R][d] bf16 copy of the output
+    int* err;
+};
+int mlp_tc_supported(int d, int F);
+// att: tensor map of the attention output rows (box 64 x 128); wo / w1 / w2:
+// weight maps with boxes of 64 x 128.
+cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
+                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st);
 // Columns per CTA of the cluster LayerNorm GEMM for a row width N (0: unsupported).
 int ln_cluster_cols(int N);
 // EPI_TC_RESID_LN by a cluster of N / ln_cluster_cols(N) CTAs per 128 rows;

@@ -1043,6 +1043,18 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             PROF_MARK(prof, KC_ATTENTION, 1, st);
             if ((e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st)) != cudaSuccess) return e;
             PROF_MARK(prof, KC_ATTENTION, 0, st);
+            if (tc->mlp) {
+                MlpArgs ma{};
+                ma.R = R; ma.F = F; ma.b_o = L.b_o; ma.ln1_g = L.ln1_g; ma.ln1_b = L.ln1_b;
+                ma.b_1 = L.b_1; ma.b_2 = L.b_2; ma.ln2_g = L.ln2_g; ma.ln2_b = L.ln2_b;
+                ma.x = w.x; ma.xb = (bf16*)xb; ma.err = tc->err;
+                PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
+                e = launch_mlp_tc(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st);
+                if (e != cudaSuccess) return e;
+                PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
+                nl += 3;
+                continue;
+            }
             TcGemmArgs go{};
             go.R = R; go.N = d; go.K = d; go.epi = EPI_TC_RESID_LN; go.bias = L.b_o;
             go.resid = w.x; go.x_out = w.x; go.xb_out = (bf16*)xb; go.ln_g = L.ln1_g; go.ln_b = L.ln1_b;

@@ -1,0 +1,340 @@
+// Fused post-attention block of one target layer on the tensor cores (bf16
+// operands, fp32 accumulation in TMEM), for d = 128 (reading of the layer:
+// post-LN Transformer block, ReLU FFN):
+//   x1 = LN1(x + att W_o^T + b_o)
+//   x  = LN2(x1 + relu(x1 W_1^T + b_1) W_2^T + b_2),   xb = bf16(x)
+// One CTA per 128-row tile, ten warps:
+//   warp 8     producer: the attention tile and every weight tile (TMA,
+//              128-byte swizzle) through a ring of stages
+//   warp 9     one thread issues tcgen05.mma; W tiles are consumed in the
+//              order O-proj, H_0, H_1, F2_0, H_2, F2_1, ... so the tensor
+//              core computes the next FFN1 chunk while the epilogue warps
+//              turn the current one into bf16 ReLU activations
+//   warps 0-7  epilogues: warps w and w+4 share TMEM lanes 32(w%4).. (row t
+//              = lane), each taking 64 of the row's 128 columns; LayerNorm
+//              partial sums meet in shared memory.  The residual tile is
+//              read and the output tile written with coalesced accesses
+//              through shared memory.
+// TMEM (512 columns): 0-127 the output projection, then (once LN1 has read
+// it) the FFN2 accumulator; 128-383 two FFN1 chunk buffers; 384-511 x1 in
+// fp32 (the LN2 residual).  Shared memory: the attention tile, then x1 in
+// bf16 (A operand of FFN1); the residual tile, then two buffers of chunk
+// activations (A operand of FFN2), then the output tile; the weight ring.
+// The FFN hidden layer (F columns) never leaves the SM.  Every wait is
+// bounded.
+#include <cuda.h>
+
+#include "common.cuh"
+#include "engine.h"
+#include "tc_ptx.cuh"
+
+namespace tppsd {
+
+struct MlpShape {
+    static constexpr int D = 128, BM = 128, BK = 64, CH = 128;
+    static constexpr int TILE = BM * BK * 2;            // 128 rows x 64 bf16 (16 KB)
+    static constexpr int STAGES = 6;
+    static constexpr int RLD = D + 4;                   // padded fp32 row (floats)
+    static constexpr int PF = 1024;                     // largest FFN width
+    static constexpr int OFF_A = 0;                     // attention tile, then x1 (2 k-blocks)
+    static constexpr int OFF_R = OFF_A + 2 * TILE;      // residual / 2 activation buffers / output
+    static constexpr int R_BYTES = ((BM * RLD * 4 + 1023) / 1024) * 1024;
+    static constexpr int OFF_W = OFF_R + R_BYTES;       // weight ring
+    static constexpr int OFF_P = OFF_W + STAGES * TILE; // b_o g1 be1 b_2 g2 be2 (D each), b_1 (F)
+    static constexpr int OFF_RED = OFF_P + (6 * D + PF) * 4;  // LayerNorm partials [2][4][BM]
+    static constexpr int OFF_B = OFF_RED + 8 * BM * 4;
+    static constexpr int NBAR = 23;
+    static constexpr size_t SMEM = (size_t)OFF_B + NBAR * 8 + 16 + 1024;
+    static_assert(R_BYTES >= 4 * TILE, "two activation buffers fit in the residual region");
+};
+
+// 16 consecutive columns c0.. of row t as bf16 into a K-major operand tile
+// pair (two 64-column k-blocks), 128-byte swizzle: the 16-byte chunk c of
+// row t sits at chunk c ^ (t & 7) of the row's 128 bytes.
+__device__ __forceinline__ void st_swizzled16(unsigned char* tiles, int t, int c0, const float* v) {
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
+    unsigned char* row = tiles + kb * MlpShape::TILE + t * 128;
+    *reinterpret_cast<uint4*>(row + (((ch + 0) ^ (t & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+    *reinterpret_cast<uint4*>(row + (((ch + 1) ^ (t & 7)) << 4)) = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+__device__ __forceinline__ void epi_sync() {  // the 256 epilogue threads only
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(320, 1)
+    k_mlp_tc(const __grid_constant__ CUtensorMap mapAtt, const __grid_constant__ CUtensorMap mapWo,
+             const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2, MlpArgs a) {
+    using S = MlpShape;
+    constexpr int D = S::D;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char* A = smem + S::OFF_A;
+    unsigned char* Rg = smem + S::OFF_R;
+    float* res = (float*)Rg;
+    unsigned char* Wr = smem + S::OFF_W;
+    float* prm = (float*)(smem + S::OFF_P);
+    float* red = (float*)(smem + S::OFF_RED);
+    uint64_t* bars = (uint64_t*)(smem + S::OFF_B);
+    uint64_t* full = bars;            // [STAGES]
+    uint64_t* empty = bars + 6;       // [STAGES]
+    uint64_t* abar = bars + 12;       // attention tile landed
+    uint64_t* o_done = bars + 13;     // output projection in TMEM
+    uint64_t* x1_ready = bars + 14;   // x1 operand written (256 arrivals)
+    uint64_t* h_done = bars + 15;     // [2] FFN1 chunk j in TMEM buffer j & 1
+    uint64_t* e2_done = bars + 17;    // [2] chunk j's activations in buffer j & 1 (256 arrivals)
+    uint64_t* hid_free = bars + 19;   // [2] FFN2 of chunk j done: buffer j & 1 reusable
+    uint64_t* y_done = bars + 21;     // FFN2 accumulator complete
+    uint32_t* tslot = (uint32_t*)(bars + 22);
+    static_assert(S::STAGES <= 6, "barrier slots");
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * S::BM, rows = min(S::BM, a.R - m0);
+    const int nc = a.F / S::CH;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S::STAGES; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_init(abar, 1);
+        mbar_init(o_done, 1);
+        mbar_init(x1_ready, 256);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&h_done[b], 1);
+            mbar_init(&e2_done[b], 256);
+            mbar_init(&hid_free[b], 1);
+        }
+        mbar_init(y_done, 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0) {
+            mbar_arrive_expect_tx(abar, 2 * S::TILE);
+            tma_load_2d(A, &mapAtt, abar, 0, m0);
+            tma_load_2d(A + S::TILE, &mapAtt, abar, 64, m0);
+            int q = 0;
+            bool ok = true;
+            auto load_w = [&](const CUtensorMap* map, int x, int y) {
+                if (!ok) return;
+                const int s = q % S::STAGES, round = q / S::STAGES;
+                ok = mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 31);
+                if (!ok) return;
+                mbar_arrive_expect_tx(&full[s], S::TILE);
+                tma_load_2d(Wr + s * S::TILE, map, &full[s], x, y);
+                ++q;
+            };
+            load_w(&mapWo, 0, 0);
+            load_w(&mapWo, 64, 0);
+            load_w(&mapW1, 0, 0);
+            load_w(&mapW1, 64, 0);
+            for (int j = 0; j < nc; ++j) {
+                if (j + 1 < nc) {
+                    load_w(&mapW1, 0, (j + 1) * S::CH);
+                    load_w(&mapW1, 64, (j + 1) * S::CH);
+                }
+                load_w(&mapW2, j * S::CH, 0);
+                load_w(&mapW2, j * S::CH + 64, 0);
+            }
+        }
+    } else if (warp == 9) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(128, 128);
+            int q = 0;
+            bool ok = true;
+            // one 128x128x64 step: A k-block at a_addr, W tile from the ring
+            auto mma_tile = [&](uint32_t a_addr, uint32_t d_tmem, bool acc) {
+                if (!ok) return;
+                const int s = q % S::STAGES, round = q / S::STAGES;
+                ok = mbar_wait(&full[s], round & 1, a.err, 32);
+                if (!ok) return;
+                tc_fence_after();
+                const uint32_t b_addr = smem_u32(Wr + s * S::TILE);
+#pragma unroll
+                for (int kk = 0; kk < S::BK / 16; ++kk)
+                    tc_mma_bf16(d_tmem, sw128_desc(a_addr + kk * 32), sw128_desc(b_addr + kk * 32), idesc,
+                                (acc || kk) ? 1u : 0u);
+                tc_commit(&empty[s]);
+                ++q;
+            };
+            const uint32_t a0 = smem_u32(A), r0 = smem_u32(Rg);
+            ok = mbar_wait(abar, 0, a.err, 33);
+            tc_fence_after();
+            mma_tile(a0, tmem, false);
+            mma_tile(a0 + S::TILE, tmem, true);
+            tc_commit(o_done);
+            if (ok) ok = mbar_wait(x1_ready, 0, a.err, 34);
+            tc_fence_after();
+            auto ffn1 = [&](int j) {
+                const uint32_t hb = tmem + 128 + (uint32_t)(j & 1) * 128;
+                mma_tile(a0, hb, false);
+                mma_tile(a0 + S::TILE, hb, true);
+                tc_commit(&h_done[j & 1]);
+            };
+            ffn1(0);
+            for (int j = 0; j < nc; ++j) {
+                if (j + 1 < nc) ffn1(j + 1);  // its TMEM buffer was released by chunk j-1's epilogue
+                if (ok) ok = mbar_wait(&e2_done[j & 1], (j >> 1) & 1, a.err, 35);
+                tc_fence_after();
+                const uint32_t hs = r0 + (uint32_t)(j & 1) * 2 * S::TILE;
+                mma_tile(hs, tmem, j > 0);
+                mma_tile(hs + S::TILE, tmem, true);
+                tc_commit(&hid_free[j & 1]);
+            }
+            tc_commit(y_done);
+        }
+    } else {
+        // epilogue warps 0-7: row t = 32 (warp % 4) + lane, columns cb..cb+63
+        const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * 64;
+        const bool live = t < rows;
+        for (int i = tid; i < 6 * D + a.F; i += 256) {
+            float v;
+            if (i < D) v = a.b_o[i];
+            else if (i < 2 * D) v = a.ln1_g[i - D];
+            else if (i < 3 * D) v = a.ln1_b[i - 2 * D];
+            else if (i < 4 * D) v = a.b_2[i - 3 * D];
+            else if (i < 5 * D) v = a.ln2_g[i - 4 * D];
+            else if (i < 6 * D) v = a.ln2_b[i - 5 * D];
+            else v = a.b_1[i - 6 * D];
+            prm[i] = v;
+        }
+        // residual tile, coalesced: float4 f of the tile -> row f / 32
+        for (int f = tid; f < S::BM * D / 4; f += 256) {
+            const int r = f >> 5, c4 = f & 31;
+            const float4 v = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+            *reinterpret_cast<float4*>(res + r * S::RLD + 4 * c4) = v;
+        }
+        epi_sync();
+        const float *p_bo = prm + cb, *p_g1 = prm + D + cb, *p_be1 = prm + 2 * D + cb, *p_b2 = prm + 3 * D + cb;
+        const float *p_g2 = prm + 4 * D + cb, *p_be2 = prm + 5 * D + cb, *p_b1 = prm + 6 * D + cb;
+        const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
+        float* xr = res + t * S::RLD + cb;
+        // mean and 1/sqrt(var + eps) of a row whose halves are held by the
+        // thread pairs (t, hh = 0 / 1); rd: this LayerNorm's [4][BM] partials
+        auto row_stats = [&](const float* y, float* rd, float& mean, float& inv) {
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+            for (int c = 0; c < 64; c += 4) {
+                s0 += y[c];
+                s1 += y[c + 1];
+                s2 += y[c + 2];
+                s3 += y[c + 3];
+            }
+            rd[hh * S::BM + t] = (s0 + s1) + (s2 + s3);
+            epi_sync();
+            mean = (rd[t] + rd[S::BM + t]) / D;
+            s0 = s1 = s2 = s3 = 0.f;
+#pragma unroll
+            for (int c = 0; c < 64; c += 4) {
+                s0 = fmaf(y[c] - mean, y[c] - mean, s0);
+                s1 = fmaf(y[c + 1] - mean, y[c + 1] - mean, s1);
+                s2 = fmaf(y[c + 2] - mean, y[c + 2] - mean, s2);
+                s3 = fmaf(y[c + 3] - mean, y[c + 3] - mean, s3);
+            }
+            rd[(2 + hh) * S::BM + t] = (s0 + s1) + (s2 + s3);
+            epi_sync();
+            inv = 1.0f / sqrtf((rd[2 * S::BM + t] + rd[3 * S::BM + t]) / D + LN_EPS);
+        };
+        mbar_wait(o_done, 0, a.err, 37);
+        tc_fence_after();
+        // y = O + b_o + x; LN1 -> x1: fp32 into TMEM columns 384.., bf16 into
+        // the A operand of FFN1 (columns cb.. are k-block hh)
+        float y[64];
+        tmem_ld64(tl + cb, y);
+#pragma unroll
+        for (int c = 0; c < 64; c += 4) {
+            const float4 r4 = *reinterpret_cast<const float4*>(xr + c);
+            y[c] += p_bo[c] + r4.x;
+            y[c + 1] += p_bo[c + 1] + r4.y;
+            y[c + 2] += p_bo[c + 2] + r4.z;
+            y[c + 3] += p_bo[c + 3] + r4.w;
+        }
+        float mean, inv;
+        row_stats(y, red, mean, inv);  // its barriers also end every read of the residual tile
+#pragma unroll
+        for (int c = 0; c < 64; ++c) y[c] = live ? (y[c] - mean) * inv * p_g1[c] + p_be1[c] : 0.f;
+        tmem_st64(tl + 384 + cb, y);
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(A, t, cb + c0, y + c0);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(x1_ready);
+        // FFN1 chunks: ReLU(H + b_1) -> bf16 operand of FFN2, buffer j & 1
+        for (int j = 0; j < nc; ++j) {
+            mbar_wait(&h_done[j & 1], (j >> 1) & 1, a.err, 38);
+            if (j >= 2) mbar_wait(&hid_free[j & 1], ((j >> 1) - 1) & 1, a.err, 39);
+            tc_fence_after();
+            tmem_ld64(tl + 128 + (uint32_t)(j & 1) * 128 + cb, y);
+            const float* b1 = p_b1 + j * S::CH;
+#pragma unroll
+            for (int c = 0; c < 64; ++c) y[c] = fmaxf(y[c] + b1[c], 0.f);
+            unsigned char* hs = Rg + (j & 1) * 2 * S::TILE;
+#pragma unroll
+            for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(hs, t, cb + c0, y + c0);
+            fence_proxy_async_smem();
+            tc_fence_before();
+            mbar_arrive(&e2_done[j & 1]);
+        }
+        // LN2 over y = F2 + b_2 + x1
+        mbar_wait(y_done, 0, a.err, 40);
+        tc_fence_after();
+        float x1[64];
+        tmem_ld64(tl + cb, y);
+        tmem_ld64(tl + 384 + cb, x1);
+#pragma unroll
+        for (int c = 0; c < 64; ++c) y[c] += p_b2[c] + x1[c];
+        row_stats(y, red + 4 * S::BM, mean, inv);
+        // output tile through shared memory (the activation buffers are free:
+        // every FFN2 step has completed), then coalesced row writes
+#pragma unroll
+        for (int c = 0; c < 64; c += 4) {
+            float4 o;
+            o.x = (y[c] - mean) * inv * p_g2[c] + p_be2[c];
+            o.y = (y[c + 1] - mean) * inv * p_g2[c + 1] + p_be2[c + 1];
+            o.z = (y[c + 2] - mean) * inv * p_g2[c + 2] + p_be2[c + 2];
+            o.w = (y[c + 3] - mean) * inv * p_g2[c + 3] + p_be2[c + 3];
+            *reinterpret_cast<float4*>(xr + c) = o;
+        }
+        epi_sync();
+        for (int f = tid; f < rows * D / 4; f += 256) {
+            const int r = f >> 5, c4 = f & 31;
+            const float4 v = *reinterpret_cast<const float4*>(res + r * S::RLD + 4 * c4);
+            *reinterpret_cast<float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4) = v;
+            const __nv_bfloat162 p0 = __floats2bfloat162_rn(v.x, v.y), p1 = __floats2bfloat162_rn(v.z, v.w);
+            uint2 w;
+            w.x = *reinterpret_cast<const uint32_t*>(&p0);
+            w.y = *reinterpret_cast<const uint32_t*>(&p1);
+            *reinterpret_cast<uint2*>(a.xb + (size_t)(m0 + r) * D + 4 * c4) = w;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+}
+
+int mlp_tc_supported(int d, int F) { return d == MlpShape::D && F % MlpShape::CH == 0 && F <= MlpShape::PF; }
+
+cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
+                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st) {
+    if (a.R <= 0) return cudaSuccess;
+    if (!mlp_tc_supported(MlpShape::D, a.F)) return cudaErrorInvalidValue;
+    const size_t sm = MlpShape::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(k_mlp_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    k_mlp_tc<<<(a.R + 127) / 128, 320, sm, st>>>(att, wo, w1, w2, a);
+    return cudaGetLastError();
+}
+
+}  // namespace tppsd
