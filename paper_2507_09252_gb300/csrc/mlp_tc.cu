@@ -198,23 +198,39 @@ __global__ void __launch_bounds__(320, 1)
         // epilogue warps 0-7: row t = 32 (warp % 4) + lane, columns cb..cb+63
         const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * 64;
         const bool live = t < rows;
-        for (int i = tid; i < 6 * D + a.F; i += 256) {
-            float v;
-            if (i < D) v = a.b_o[i];
-            else if (i < 2 * D) v = a.ln1_g[i - D];
-            else if (i < 3 * D) v = a.ln1_b[i - 2 * D];
-            else if (i < 4 * D) v = a.b_2[i - 3 * D];
-            else if (i < 5 * D) v = a.ln2_g[i - 4 * D];
-            else if (i < 6 * D) v = a.ln2_b[i - 5 * D];
-            else v = a.b_1[i - 6 * D];
-            prm[i] = v;
-        }
-        // residual tile, coalesced: float4 f of the tile -> row f / 32
-        for (int f = tid; f < S::BM * D / 4; f += 256) {
-            const int r = f >> 5, c4 = f & 31;
-            const float4 v = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
-                                      : make_float4(0.f, 0.f, 0.f, 0.f);
-            *reinterpret_cast<float4*>(res + r * S::RLD + 4 * c4) = v;
+        // residual tile (coalesced: float4 f of the tile is row f / 32) and the
+        // epilogue parameters; all loads are issued before any store
+        {
+            constexpr int NV = S::BM * D / 4 / 256;  // 16 float4 per thread
+            float4 v[NV];
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                v[k] = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            const float* src[6] = {a.b_o, a.ln1_g, a.ln1_b, a.b_2, a.ln2_g, a.ln2_b};
+            float pv[3];
+#pragma unroll
+            for (int k = 0; k < 3; ++k) {
+                const int i = tid + 256 * k;  // 768 = 6 D vector entries
+                pv[k] = src[i / D][i % D];
+            }
+            float b1v[S::PF / 256];
+#pragma unroll
+            for (int k = 0; k < S::PF / 256; ++k) {
+                const int i = tid + 256 * k;
+                b1v[k] = i < a.F ? a.b_1[i] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                *reinterpret_cast<float4*>(res + r * S::RLD + 4 * c4) = v[k];
+            }
+#pragma unroll
+            for (int k = 0; k < 3; ++k) prm[tid + 256 * k] = pv[k];
+#pragma unroll
+            for (int k = 0; k < S::PF / 256; ++k) prm[6 * D + tid + 256 * k] = b1v[k];
         }
         epi_sync();
         const float *p_bo = prm + cb, *p_g1 = prm + D + cb, *p_be1 = prm + 2 * D + cb, *p_b2 = prm + 3 * D + cb;
@@ -308,15 +324,26 @@ __global__ void __launch_bounds__(320, 1)
             *reinterpret_cast<float4*>(xr + c) = o;
         }
         epi_sync();
-        for (int f = tid; f < rows * D / 4; f += 256) {
-            const int r = f >> 5, c4 = f & 31;
-            const float4 v = *reinterpret_cast<const float4*>(res + r * S::RLD + 4 * c4);
-            *reinterpret_cast<float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4) = v;
-            const __nv_bfloat162 p0 = __floats2bfloat162_rn(v.x, v.y), p1 = __floats2bfloat162_rn(v.z, v.w);
-            uint2 w;
-            w.x = *reinterpret_cast<const uint32_t*>(&p0);
-            w.y = *reinterpret_cast<const uint32_t*>(&p1);
-            *reinterpret_cast<uint2*>(a.xb + (size_t)(m0 + r) * D + 4 * c4) = w;
+        {
+            constexpr int NV = S::BM * D / 4 / 256;
+            float4 v[NV];
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                v[k] = *reinterpret_cast<const float4*>(res + r * S::RLD + 4 * c4);
+            }
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                if (r >= rows) continue;
+                *reinterpret_cast<float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4) = v[k];
+                const __nv_bfloat162 p0 = __floats2bfloat162_rn(v[k].x, v[k].y);
+                const __nv_bfloat162 p1 = __floats2bfloat162_rn(v[k].z, v[k].w);
+                uint2 w;
+                w.x = *reinterpret_cast<const uint32_t*>(&p0);
+                w.y = *reinterpret_cast<const uint32_t*>(&p1);
+                *reinterpret_cast<uint2*>(a.xb + (size_t)(m0 + r) * D + 4 * c4) = w;
+            }
         }
     }
     tc_fence_before();
