@@ -321,6 +321,7 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const size_t tk2 = tmat(ok2, K, d, false), tbk2 = tvec(obk2, K);
     const size_t t_om = tadd(omega.data(), omega.size() * sizeof(double));
     tb.resize((tb.size() + 15) & ~(size_t)15);
+    tb.resize((tb.size() + 15) & ~(size_t)15);  // whole 16-byte chunks: one bulk copy stages it
     CK(cudaMalloc(&hm.tbuf, tb.size()));
     ctx->allocs.push_back(hm.tbuf);
     CK(cudaMemcpy(hm.tbuf, tb.data(), tb.size(), cudaMemcpyHostToDevice));

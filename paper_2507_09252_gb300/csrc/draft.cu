@@ -25,6 +25,13 @@ namespace tppsd {
 
 constexpr unsigned FULL = 0xffffffffu;
 
+// Barrier of the 128 threads that work on one sequence (named barrier 1 or
+// 2: a CTA holds one or two such teams).
+__device__ __forceinline__ void team_sync() {
+    if (threadIdx.x < 128) asm volatile("bar.sync 1, 128;" ::: "memory");
+    else asm volatile("bar.sync 2, 128;" ::: "memory");
+}
+
 struct DraftTeamArgs {
     DevModel m;
     KVCache kv;
@@ -61,13 +68,27 @@ __device__ __forceinline__ void load_row16(const T* p, float (&out)[DH]) {
     }
 }
 
-// sum_{i<IN} WT[i][o] xs[i] (WT is [IN][OUT], xs in shared memory).
+// sum_{i<i1} WT[i][o] xs[i] over i from i0, with four independent partial
+// sums (WT is [IN][OUT], xs in shared memory).
+template <typename TW>
+__device__ __forceinline__ float dot_range(const TW* __restrict__ WT, int OUT, int o, const float* xs, int i0,
+                                           int i1) {
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    const TW* w = WT + (size_t)i0 * OUT + o;
+    int i = i0;
+#pragma unroll 2
+    for (; i + 4 <= i1; i += 4, w += 4 * (size_t)OUT) {
+        a0 = fmaf(St<TW>::ld(w), xs[i], a0);
+        a1 = fmaf(St<TW>::ld(w + OUT), xs[i + 1], a1);
+        a2 = fmaf(St<TW>::ld(w + 2 * (size_t)OUT), xs[i + 2], a2);
+        a3 = fmaf(St<TW>::ld(w + 3 * (size_t)OUT), xs[i + 3], a3);
+    }
+    for (; i < i1; ++i, w += OUT) a0 = fmaf(St<TW>::ld(w), xs[i], a0);
+    return (a0 + a1) + (a2 + a3);
+}
 template <typename TW>
 __device__ __forceinline__ float dot_col(const TW* __restrict__ WT, int OUT, int o, const float* xs, int IN) {
-    float acc = 0.f;
-#pragma unroll 8
-    for (int i = 0; i < IN; ++i) acc = fmaf(St<TW>::ld(WT + (size_t)i * OUT + o), xs[i], acc);
-    return acc;
+    return dot_range<TW>(WT, OUT, o, xs, 0, IN);
 }
 
 // Partial sums of a product with few outputs: thread t takes output
@@ -76,15 +97,10 @@ __device__ __forceinline__ float dot_col(const TW* __restrict__ WT, int OUT, int
 template <typename TW>
 __device__ __forceinline__ void split_partials(const TW* __restrict__ WT, int OUT, int ob, const float* xs,
                                                int IN, int OP, float* part) {
-    const int t = threadIdx.x, G = 128 / OP, o = ob + t % OP, g = t / OP;
+    const int t = threadIdx.x & 127, G = 128 / OP, o = ob + t % OP, g = t / OP;
     const int per = (IN + G - 1) / G, i0 = g * per, i1 = min(IN, i0 + per);
-    float acc = 0.f;
-    if (o < OUT) {
-#pragma unroll 8
-        for (int i = i0; i < i1; ++i) acc = fmaf(St<TW>::ld(WT + (size_t)i * OUT + o), xs[i], acc);
-    }
-    part[t] = acc;
-    __syncthreads();
+    part[t] = o < OUT ? dot_range<TW>(WT, OUT, o, xs, i0, i1) : 0.f;
+    team_sync();
 }
 
 // Residual add + LayerNorm of d <= 32 values by warp 0 (lane j < d holds
@@ -114,7 +130,7 @@ __device__ __forceinline__ void warp_resid_ln(float yv, float* x, float* xin, in
 template <typename T, int DH>
 __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
                                             int n_keys, int nh, float* out, float* scratch) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31;
     const int h = warp % nh, split = warp / nh, S = 4 / nh;
     const int per = (n_keys + S - 1) / S, lo = split * per, hi = min(n_keys, lo + per);
     const float scale = 1.4426950408889634f / sqrtf((float)DH);
@@ -160,8 +176,8 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
 #pragma unroll
         for (int c = 0; c < DH; ++c) sw[2 + c] = o[c];
     }
-    __syncthreads();
-    for (int t = threadIdx.x; t < nh * DH; t += 128) {
+    team_sync();
+    for (int t = threadIdx.x & 127; t < nh * DH; t += 128) {
         const int hh = t / DH, c = t % DH;
         float M = -INFINITY;
         for (int sp = 0; sp < S; ++sp) M = fmaxf(M, scratch[(sp * nh + hh) * (DH + 2)]);
@@ -175,7 +191,7 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
         }
         out[t] = St<T>::rnd(O / L);
     }
-    __syncthreads();
+    team_sync();
 }
 
 // Warp-parallel log-softmax of n <= 32*R values v[] (shared) in place, then
@@ -225,24 +241,73 @@ __device__ __forceinline__ int warp_logsoftmax_pick(float* v, int n, float u) {
     return n - 1;
 }
 
-template <typename T, int DH, bool KVS>
-__global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
+// Copy of the transposed model's pointer table whose pointers are rebased
+// onto a staged copy of its bytes at dst.
+__device__ void rebase_model(DevModelT& m, const DevModelT& src, int L, const char* dst) {
+    m = src;
+    auto rb = [&](const void* p) { return dst + ((const char*)p - src.base); };
+    m.type_emb = (const float*)rb(m.type_emb);
+    m.omega = (const double*)rb(m.omega);
+    for (int l = 0; l < L; ++l) {
+        LayerW& w = m.layer[l];
+        w.w_qkv = rb(w.w_qkv); w.b_qkv = (const float*)rb(w.b_qkv);
+        w.w_o = rb(w.w_o);     w.b_o = (const float*)rb(w.b_o);
+        w.ln1_g = (const float*)rb(w.ln1_g); w.ln1_b = (const float*)rb(w.ln1_b);
+        w.w_1 = rb(w.w_1);     w.b_1 = (const float*)rb(w.b_1);
+        w.w_2 = rb(w.w_2);     w.b_2 = (const float*)rb(w.b_2);
+        w.ln2_g = (const float*)rb(w.ln2_g); w.ln2_b = (const float*)rb(w.ln2_b);
+    }
+    HeadW& h = m.head;
+    h.E = (const float*)rb(h.E);
+    h.v_w = (const float*)rb(h.v_w);   h.b_w = (const float*)rb(h.b_w);
+    h.v_mu = (const float*)rb(h.v_mu); h.b_mu = (const float*)rb(h.b_mu);
+    h.v_s = (const float*)rb(h.v_s);   h.b_s = (const float*)rb(h.b_s);
+    h.v_k1 = (const float*)rb(h.v_k1); h.b_k1 = (const float*)rb(h.b_k1);
+    h.v_k2 = (const float*)rb(h.v_k2); h.b_k2 = (const float*)rb(h.b_k2);
+    m.base = dst;
+}
+
+// TEAMS sequences per CTA, 128 threads each.  With WS the draft model is
+// staged once per CTA in shared memory (shared by its teams), so no weight
+// read leaves the SM; otherwise weights are read through L1.
+template <typename T, int DH, bool KVS, bool WS>
+__global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, int area_bytes) {
+    constexpr int TEAMS = WS ? 2 : 1;
     extern __shared__ __align__(16) char smem[];
-    __shared__ double t_new;
-    __shared__ int k_new;
-    const int s = blockIdx.x;
+    __shared__ double t_new_s[TEAMS];
+    __shared__ int k_new_s[TEAMS];
+    __shared__ DevModelT msh;
+    __shared__ uint64_t wbar;
+    const int team = threadIdx.x >> 7;
+    const int s = blockIdx.x * TEAMS + team;
     const CallParams& P = *a.P;
-    if (s >= P.B || a.ss.done[s]) return;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const DevModelT& m = a.m.t;
+    char* area = smem;
+    if (WS) {
+        const uint32_t wb = (uint32_t)a.m.t.bytes;
+        if (threadIdx.x == 0) {
+            mbar_init(&wbar, 1);
+            mbar_fence_init();
+            mbar_arrive_expect_tx(&wbar, wb);
+            bulk_load(smem, a.m.t.base, wb, &wbar);
+            rebase_model(msh, a.m.t, a.m.L, smem);
+        }
+        __syncthreads();
+        mbar_wait(&wbar, 0, a.err, 13);
+        area = smem + wb + (size_t)team * area_bytes;
+    }
+    if (s >= P.B || a.ss.done[s]) return;  // the rest synchronises within the team only
+    double& t_new = t_new_s[team];
+    int& k_new = k_new_s[team];
+    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
+    const DevModelT& m = WS ? msh : a.m.t;
     const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
     const int n_max = a.kv.n_max;
     const int OPd = d <= 32 ? 32 : 64;  // output block of the few-output products
-    // shared layout: [resident KV][mbarrier][work vectors]
+    // team area: [resident KV][mbarrier][work vectors]
     const size_t kvb = KVS ? (((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15) : 0;
-    T* kvs = (T*)smem;
-    uint64_t* bar = (uint64_t*)(smem + kvb);
-    float* x = (float*)(smem + kvb + 16);
+    T* kvs = (T*)area;
+    uint64_t* bar = (uint64_t*)(area + kvb);
+    float* x = (float*)(area + kvb + 16);
     float* xin = x + d;
     float* qkv = xin + d;
     float* att = qkv + 3 * d;
@@ -270,7 +335,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                     for (int h = 0; h < NH; ++h)
                         bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
         }
-        __syncthreads();
+        team_sync();
         mbar_wait(bar, 0, a.err, 12);
     }
     // x = LN(x + W_T in + b): few-output product, then the residual add and
@@ -287,7 +352,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                 }
                 warp_resid_ln<T>(v, x, xin, d, g, b);
             }
-            __syncthreads();
+            team_sync();
             return;
         }
         for (int ob = 0; ob < d; ob += OPd) {
@@ -297,7 +362,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                 for (int gg = 0; gg < 128 / OPd; ++gg) v += part[gg * OPd + tid];
                 y[ob + tid] = v;
             }
-            __syncthreads();
+            team_sync();
         }
         if (warp == 0) {
             float sum = 0.f;
@@ -312,7 +377,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                 xin[i] = St<T>::rnd(v);
             }
         }
-        __syncthreads();
+        team_sync();
     };
     // Layers of the encode step at position p from x / xin (set and synced
     // by the caller); leaves the final hidden state in x (synced).
@@ -330,14 +395,14 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                     if (KVS) St<T>::st(sk(l, w) + off, v);
                 }
             }
-            __syncthreads();
+            team_sync();
             const T* kb = KVS ? sk(l, 0) : gk(l, 0);
             const T* vb = KVS ? sk(l, 1) : gk(l, 1);
             team_attend<T, DH>(qkv, kb, vb, n_max, p + 1, NH, att, attn);
             proj_resid_ln((const T*)Wl.w_o, Wl.b_o, att, d, Wl.ln1_g, Wl.ln1_b);
             for (int o = tid; o < F; o += 128)
                 hid[o] = St<T>::rnd(fmaxf(dot_col<T>((const T*)Wl.w_1, F, o, xin, d) + Wl.b_1[o], 0.f));
-            __syncthreads();
+            team_sync();
             proj_resid_ln((const T*)Wl.w_2, Wl.b_2, hid, F, Wl.ln2_g, Wl.ln2_b);
         }
     };
@@ -357,7 +422,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
     for (int p = nd; p < n; ++p) {  // catch-up over events already emitted
         const size_t so = (size_t)s * ss.n_max + p;
         embed(ss.t[so], min(max(ss.k[so], 0), K - 1));
-        __syncthreads();
+        team_sync();
         layers(p);
     }
     if (tid == 0) {
@@ -372,7 +437,7 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
         for (int o = tid; o < 4 * d; o += 128)
             e[o] = o < 3 * d ? dot_col<float>(H.E, 3 * d, o, x, d)
                              : tanhf(dot_col<float>(H.v_k1, d, o - 3 * d, x, d) + H.b_k1[o - 3 * d]);
-        __syncthreads();
+        team_sync();
         // [w logits | mu | log sigma | mark logits] in blocks of OPh outputs;
         // output j reads its own matrix and input segment
         for (int ob = 0; ob < W; ob += OPh) {
@@ -388,19 +453,18 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                     else if (o < 2 * M) { WT = H.v_mu; in = e + d; ld = M; oo = o - M; }
                     else if (o < 3 * M) { WT = H.v_s; in = e + 2 * d; ld = M; oo = o - 2 * M; }
                     else { WT = H.v_k2; in = e + 3 * d; ld = K; oo = o - 3 * M; }
-#pragma unroll 8
-                    for (int i = i0; i < i1; ++i) acc = fmaf(WT[(size_t)i * ld + oo], in[i], acc);
+                    acc = dot_range<float>(WT, ld, oo, in, i0, i1);
                 }
                 part[tid] = acc;
             }
-            __syncthreads();
+            team_sync();
             if (tid < OPh && ob + tid < W) {
                 const int o = ob + tid;
                 float v = o < M ? H.b_w[o] : o < 2 * M ? H.b_mu[o - M] : o < 3 * M ? H.b_s[o - 2 * M] : H.b_k2[o - 3 * M];
                 for (int gg = 0; gg < 128 / OPh; ++gg) v += part[gg * OPh + tid];
                 hd[o] = v;
             }
-            __syncthreads();
+            team_sync();
         }
         // direct sample: warp 0 the time (component, Box-Muller), warp 1 the
         // mark; both normalise their logits in place
@@ -425,27 +489,32 @@ __global__ void __launch_bounds__(128) k_draft_team(DraftTeamArgs a) {
                 }
             }
         }
-        __syncthreads();
+        team_sync();
         float* rec = a.heads + ((size_t)s * a.gamma_max + (l - 1)) * W;
         for (int i = tid; i < W; i += 128) rec[i] = hd[i];
         if (l < a.gamma) {
             embed(t_new, k_new);
-            __syncthreads();
+            team_sync();
             layers(p);
         }
     }
 }
 
-template <typename T, int DH>
-static cudaError_t launch_team(DraftTeamArgs& a, int B, int kvs, size_t sm, cudaStream_t st) {
-    if (kvs) {
-        cudaFuncSetAttribute(k_draft_team<T, DH, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        k_draft_team<T, DH, true><<<B, 128, sm, st>>>(a);
-    } else {
-        cudaFuncSetAttribute(k_draft_team<T, DH, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        k_draft_team<T, DH, false><<<B, 128, sm, st>>>(a);
-    }
+template <typename T, int DH, bool KVS, bool WS>
+static cudaError_t launch_t(DraftTeamArgs& a, int B, int area, size_t sm, cudaStream_t st) {
+    constexpr int TEAMS = WS ? 2 : 1;
+    cudaError_t e = cudaFuncSetAttribute(k_draft_team<T, DH, KVS, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)sm);
+    if (e != cudaSuccess) return e;
+    k_draft_team<T, DH, KVS, WS><<<(B + TEAMS - 1) / TEAMS, 128 * TEAMS, sm, st>>>(a, area);
     return cudaGetLastError();
+}
+
+template <typename T, int DH>
+static cudaError_t launch_team(DraftTeamArgs& a, int B, int kvs, int ws, size_t area, size_t wb, cudaStream_t st) {
+    if (ws) return launch_t<T, DH, true, true>(a, B, (int)area, wb + 2 * area, st);
+    if (kvs) return launch_t<T, DH, true, false>(a, B, (int)area, area, st);
+    return launch_t<T, DH, false, false>(a, B, (int)area, area, st);
 }
 
 int draft_team_supported(const DevModel& m) {
@@ -455,7 +524,9 @@ int draft_team_supported(const DevModel& m) {
 }
 
 // The sequence's draft KV is kept in shared memory for the round when that
-// still leaves room for two CTAs per SM; otherwise it is read from HBM/L2.
+// still leaves room for two sequences per SM; then, if the model also fits,
+// two sequences share a CTA and a staged copy of the model.  Otherwise KV
+// and weights are read from HBM/L2.
 cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st) {
@@ -467,13 +538,15 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + 128 + 4 * 66) + 16;
     const size_t kvb = ((size_t)m.L * 2 * kv.n_max * m.d * eb + 15) & ~(size_t)15;
     const int kvs = kvb + fl <= 110 * 1024;
-    const size_t sm = (kvs ? kvb : 0) + fl;
+    const size_t area = ((kvs ? kvb : 0) + fl + 15) & ~(size_t)15;
+    const size_t wb = m.t.bytes;  // a whole number of 16-byte chunks
+    const int ws = kvs && wb % 16 == 0 && wb + 2 * area <= 224 * 1024;
     if (m.dtype == 0) {
-        if (m.dh == 16) return launch_team<float, 16>(a, B, kvs, sm, st);
-        return launch_team<float, 32>(a, B, kvs, sm, st);
+        if (m.dh == 16) return launch_team<float, 16>(a, B, kvs, ws, area, wb, st);
+        return launch_team<float, 32>(a, B, kvs, ws, area, wb, st);
     }
-    if (m.dh == 16) return launch_team<bf16, 16>(a, B, kvs, sm, st);
-    return launch_team<bf16, 32>(a, B, kvs, sm, st);
+    if (m.dh == 16) return launch_team<bf16, 16>(a, B, kvs, ws, area, wb, st);
+    return launch_team<bf16, 32>(a, B, kvs, ws, area, wb, st);
 }
 
 }  // namespace tppsd
