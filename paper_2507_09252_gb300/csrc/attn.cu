@@ -9,11 +9,10 @@
 // multiple of 8 keys), one per warp, so all four warps work even when the
 // context is a single tile; each warp keeps its own online-softmax state
 // (flash-decoding split inside the CTA).  S = Q K^T uses mma.sync
-// m16n8k16 with bf16 inputs (exact products, fp32 accumulation); P V uses
-// fp16 P and V (V converted in shared memory) with fp32 accumulation.  The
-// four partial results are merged through shared memory.
-#include <cuda_fp16.h>
-
+// m16n8k16 with bf16 inputs (exact products, fp32 accumulation); P V splits
+// P into two bf16 parts (P = P_hi + P_lo, 16 significant bits) against the
+// bf16 V tile as copied, with fp32 accumulation.  The four partial results
+// are merged through shared memory.
 #include "common.cuh"
 #include "engine.h"
 #include "tc_ptx.cuh"
@@ -37,21 +36,17 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-__device__ __forceinline__ void mma_f16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-        "{%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                  : "r"(addr));
 }
-__device__ __forceinline__ uint32_t pack_half2(float x, float y) {
-    const __half2 h = __floats2half2_rn(x, y);
-    return *reinterpret_cast<const uint32_t*>(&h);
+__device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uint32_t& lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(x, y);
+    const float2 hf = __bfloat1622float2(h);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(x - hf.x, y - hf.y);
+    hi = *reinterpret_cast<const uint32_t*>(&h);
+    lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
 template <int DH>
@@ -130,25 +125,13 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
         if (!ok) break;
         unsigned char* st = wbase + stage * S::STAGE_BYTES;
         const bf16* ks = (const bf16*)st;
-        __half* vs = (__half*)(st + S::TILE_BYTES);
+        const bf16* vs = (const bf16*)(st + S::TILE_BYTES);
         const int k0 = klo + it * KT, cnt = min(KT, khi - k0);
-        // V tile: bf16 -> fp16 in place; rows past the copied keys -> 0
-        for (int i = lane; i < KT * DH / 8; i += 32) {
-            uint4* p = reinterpret_cast<uint4*>(vs) + i;
-            uint4 w = *p;
-            if (i * 8 / DH >= cnt) {
-                w = make_uint4(0, 0, 0, 0);
-            } else {
-                __nv_bfloat162* b = reinterpret_cast<__nv_bfloat162*>(&w);
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const float2 f = __bfloat1622float2(b[j]);
-                    *reinterpret_cast<__half2*>(&b[j]) = __floats2half2_rn(f.x, f.y);
-                }
-            }
-            *p = w;
+        if (cnt < KT) {  // V rows past the copied keys -> 0 (their P is 0, and 0 * NaN bits is NaN)
+            for (int i = cnt * DH / 8 + lane; i < KT * DH / 8; i += 32)
+                reinterpret_cast<uint4*>(const_cast<bf16*>(vs))[i] = make_uint4(0, 0, 0, 0);
+            __syncwarp();
         }
-        __syncwarp();
         // S = Q K^T for KT keys
         float sc[NT][4];
 #pragma unroll
@@ -207,24 +190,26 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
             o[n][0] *= c0; o[n][1] *= c0;
             o[n][2] *= c1; o[n][3] *= c1;
         }
-        // O += P V: P (fp16) from the S accumulators, V fragments by ldmatrix.trans
+        // O += P V with P = P_hi + P_lo (two bf16 parts) and bf16 V fragments by
+        // ldmatrix.trans; keys past the copied ones have P = 0 (V there is masked)
         const uint32_t vbase = smem_u32(vs);
 #pragma unroll
         for (int kk = 0; kk < KT / 16; ++kk) {
-            uint32_t pa[4];
-            pa[0] = pack_half2(sc[2 * kk][0], sc[2 * kk][1]);
-            pa[1] = pack_half2(sc[2 * kk][2], sc[2 * kk][3]);
-            pa[2] = pack_half2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            pa[3] = pack_half2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+            uint32_t ph[4], pl[4];
+            split_bf16x2(sc[2 * kk][0], sc[2 * kk][1], ph[0], pl[0]);
+            split_bf16x2(sc[2 * kk][2], sc[2 * kk][3], ph[1], pl[1]);
+            split_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ph[2], pl[2]);
+            split_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ph[3], pl[3]);
 #pragma unroll
             for (int n = 0; n < DH / 8; n += 2) {
-                // lanes 0-15: keys 16kk + (lane & 15) at columns 8n; lanes 16-31 at 8(n+1)
                 const int key = 16 * kk + (lane & 15);
                 const int col = 8 * n + (lane >> 4) * 8;
                 uint32_t vb[4];
                 ldsm_x4_trans(vb, vbase + (uint32_t)(key * DH + col) * 2);
-                mma_f16(o[n], pa, vb[0], vb[1]);
-                mma_f16(o[n + 1], pa, vb[2], vb[3]);
+                mma_bf16(o[n], ph, vb[0], vb[1]);
+                mma_bf16(o[n], pl, vb[0], vb[1]);
+                mma_bf16(o[n + 1], ph, vb[2], vb[3]);
+                mma_bf16(o[n + 1], pl, vb[2], vb[3]);
             }
         }
         __syncwarp();
