@@ -156,8 +156,9 @@ def roofline(kt, stats, wl, peaks):
 
     attention:  K and V of every cached position read once per (sequence,
                 layer) + Q read + output write:  target_keys * 2 d eb + 2 R d eb
-    draft:      draft K/V of every encoded position + weights staged once
-                per CTA + draft heads written
+    draft:      draft K/V of each sequence loaded once per round (the kernel
+                keeps it in shared memory for the round) + draft heads
+                written + the draft model once per launch (L2-resident)
     gemm_*:     2 R N K FLOPs per layer (tcgen05 bf16 path for bf16 models)
     others:     bytes of their inputs and outputs
     """
@@ -175,8 +176,10 @@ def roofline(kt, stats, wl, peaks):
     elif name == "draft":
         from paper_2507_09252_gb300.tppsd import tppsd_blob_floats
         wbytes = tppsd_blob_floats(D) * 4
-        total = (stats["draft_keys"] * D.layers * 2 * D.d_model * eb
-                 + rounds * wbytes + stats["drafted"] * (3 * D.n_mix + D.n_marks) * 4)
+        # target_keys = sum over (sequence, round) of the context the round
+        # attends, i.e. the draft KV positions the round loads once
+        total = (stats["target_keys"] * D.layers * 2 * D.d_model * eb
+                 + launches * wbytes + stats["drafted"] * (3 * D.n_mix + D.n_marks) * 4)
     elif name == "head":
         total = rows * (d + W) * 4 + launches * (4 * d * d + (3 * T.n_mix + T.n_marks + d) * d) * 4
     elif name.startswith("gemm"):
