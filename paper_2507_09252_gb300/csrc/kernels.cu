@@ -694,60 +694,61 @@ __device__ void write_outputs(const SeqState& ss, const CallParams& P, int s, in
     }
 }
 
-// One warp per sequence.  Lane l-1 tests draft l (Sec. 4.3 "Verification"):
-// accept tau iff u_tau < min(1, g_T/g_D), k iff u_k < min(1, f_T/f_D); L =
-// first failing draft (ballot), gamma+1 if none.  At L the failing
-// component(s) are redrawn: tau from g' by Theorem 1 (warp-parallel: lane j
-// takes iteration base+j, the first accepting lane wins, which equals the
-// sequential loop), k from f' (Eq. 4).  A full accept adds the bonus event
-// from the target head after the last draft (unless NO_BONUS).
+// One CTA (four warps) per sequence.  Warp 0: lane l-1 tests draft l (Sec.
+// 4.3 "Verification"): accept tau iff u_tau < min(1, g_T/g_D), k iff u_k <
+// min(1, f_T/f_D); L = first failing draft (ballot), gamma+1 if none.  At L
+// the failing component(s) are redrawn: tau from g' by Theorem 1 (all 128
+// threads: thread j takes iteration base+j, the smallest accepting index
+// wins, which equals the sequential loop), k from f' (Eq. 4).  A full accept
+// adds the bonus event from the target head after the last draft (unless
+// NO_BONUS).
 __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
-    __shared__ float epi_consts[4 * 8 * MAX_MIX];
-    const int lane = threadIdx.x & 31;
-    const int s = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    // per-component constants of both mixtures for the Theorem-1 loop
+    __shared__ float cumT[MAX_MIX], muT[MAX_MIX], sgT[MAX_MIX], isT[MAX_MIX], cT[MAX_MIX];
+    __shared__ float muD[MAX_MIX], isD[MAX_MIX], cD[MAX_MIX];
+    __shared__ int sh_L, sh_at, sh_ak, sh_k;
+    __shared__ float sh_umr, sh_tau;
+    __shared__ int win_idx[4];
+    __shared__ float win_tau[4];
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int s = blockIdx.x;
     const CallParams& P = *a.P;
     const SeqState& ss = a.ss;
     if (s >= P.B || ss.done[s]) return;
     const int g = a.gamma, n = ss.n_emit[s];
     const size_t sb = (size_t)s * ss.n_max;
-    bool acc_t = true, acc_k = true;
-    float tau_hat = 0.f, u_mr = 0.f;
-    int k_hat = 0;
-    if (lane < g) {
-        const int p = n + lane;
-        tau_hat = ss.tau[sb + p];
-        k_hat = ss.k[sb + p];
-        const float* hT = a.th + ((size_t)s * (g + 1) + lane) * a.WT;
-        const float* hD = a.dh + ((size_t)s * a.gamma_max + lane) * a.WD;
-        const float rt = fminf(1.f, expf(head_log_g(hT, a.MT, tau_hat) - head_log_g(hD, a.MD, tau_hat)));
-        const float rk = fminf(1.f, expf(hT[3 * a.MT + k_hat] - hD[3 * a.MD + k_hat]));
-        const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 1u);
-        acc_t = u.x < rt;
-        acc_k = u.y < rk;
-        u_mr = u.z;
-    }
-    const unsigned fail = __ballot_sync(0xffffffffu, lane < g && !(acc_t && acc_k));
-    const int L = fail ? __ffs(fail) : g + 1;  // 1-based
-    const int A = L - 1;
-    int emitted;
-    unsigned long long iters = 0, cap = 0;
-    if (L <= g) {
-        const int p = n + L - 1, src = L - 1;
+    if (warp == 0) {
+        bool acc_t = true, acc_k = true;
+        float tau_hat = 0.f, u_mr = 0.f;
+        int k_hat = 0;
+        if (lane < g) {
+            const int p = n + lane;
+            tau_hat = ss.tau[sb + p];
+            k_hat = ss.k[sb + p];
+            const float* hT = a.th + ((size_t)s * (g + 1) + lane) * a.WT;
+            const float* hD = a.dh + ((size_t)s * a.gamma_max + lane) * a.WD;
+            const float rt = fminf(1.f, expf(head_log_g(hT, a.MT, tau_hat) - head_log_g(hD, a.MD, tau_hat)));
+            const float rk = fminf(1.f, expf(hT[3 * a.MT + k_hat] - hD[3 * a.MD + k_hat]));
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 1u);
+            acc_t = u.x < rt;
+            acc_k = u.y < rk;
+            u_mr = u.z;
+        }
+        const unsigned fail = __ballot_sync(0xffffffffu, lane < g && !(acc_t && acc_k));
+        const int L = fail ? __ffs(fail) : g + 1;  // 1-based
+        const int src = L <= g ? L - 1 : 0;
         const bool at = __shfl_sync(0xffffffffu, acc_t, src);
         const bool ak = __shfl_sync(0xffffffffu, acc_k, src);
         const float umr = __shfl_sync(0xffffffffu, u_mr, src);
-        float tau = __shfl_sync(0xffffffffu, tau_hat, src);
-        int k = __shfl_sync(0xffffffffu, k_hat, src);
-        const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
-        const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
-        if (!at) {
-            // Per-component constants of both heads, computed once per
-            // sequence: running sums of w_T (the component pick), mu, sigma,
-            // 1/sigma and log w - log sigma.  The log tau and log(2 pi)/2
-            // terms of log g_T and log g_D cancel in their difference.
-            float* cs = epi_consts + (threadIdx.x >> 5) * 8 * MAX_MIX;
-            float *cumT = cs, *muT = cs + MAX_MIX, *sgT = cs + 2 * MAX_MIX, *isT = cs + 3 * MAX_MIX;
-            float *cT = cs + 4 * MAX_MIX, *muD = cs + 5 * MAX_MIX, *isD = cs + 6 * MAX_MIX, *cD = cs + 7 * MAX_MIX;
+        const float tau = __shfl_sync(0xffffffffu, tau_hat, src);
+        const int k = __shfl_sync(0xffffffffu, k_hat, src);
+        if (L <= g && !at) {
+            // constants of the time resampler: running sums of w_T (the
+            // component pick), mu, sigma, 1/sigma and log w - log sigma.  The
+            // log tau and log(2 pi)/2 terms of log g_T and log g_D cancel in
+            // their difference.
+            const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
+            const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
             const int MT = a.MT, MD = a.MD;
             for (int m = lane; m < MT; m += 32) {
                 muT[m] = hT[MT + m];
@@ -764,54 +765,90 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
                 float run = 0.f;
                 for (int m = 0; m < MT; ++m) { run += expf(hT[m]); cumT[m] = run; }
             }
-            __syncwarp();
-            const float totT = cumT[MT - 1];
-            bool found = false;
-            float last = 0.f;
-            for (int base = 0; base < RESAMPLE_CAP && !found; base += 32) {
-                const int it = base + lane;
-                const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 2u + (uint32_t)it);
-                // proposal tau ~ g_T (Theorem 1): component, then log-normal
-                const float target = u.x * totT;
-                int z = MT - 1;
-                for (int m = 0; m < MT; ++m)
-                    if (cumT[m] >= target) { z = m; break; }
-                const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
-                const float lt = fmaf(sgT[z], eps, muT[z]);
-                float mT = -INFINITY, mD = -INFINITY;
-                for (int m = 0; m < MT; ++m) {
-                    const float q = (lt - muT[m]) * isT[m];
-                    mT = fmaxf(mT, cT[m] - 0.5f * q * q);
-                }
-                for (int m = 0; m < MD; ++m) {
-                    const float q = (lt - muD[m]) * isD[m];
-                    mD = fmaxf(mD, cD[m] - 0.5f * q * q);
-                }
-                float sT = 0.f, sD = 0.f;
-                for (int m = 0; m < MT; ++m) {
-                    const float q = (lt - muT[m]) * isT[m];
-                    sT += expf(cT[m] - 0.5f * q * q - mT);
-                }
-                for (int m = 0; m < MD; ++m) {
-                    const float q = (lt - muD[m]) * isD[m];
-                    sD += expf(cD[m] - 0.5f * q * q - mD);
-                }
-                // acceptance probability max(0, 1 - g_D / g_T)
-                const float al = fmaxf(0.f, 1.f - expf((mD + logf(sD)) - (mT + logf(sT))));
-                const float tp = expf(lt);
-                const unsigned ok = __ballot_sync(0xffffffffu, u.w < al);
-                if (ok) {
-                    const int j = __ffs(ok) - 1;
-                    tau = __shfl_sync(0xffffffffu, tp, j);
-                    iters = (unsigned long long)(base + j + 1);
-                    found = true;
-                }
-                last = __shfl_sync(0xffffffffu, tp, 31);
-            }
-            if (!found) { tau = last; iters = RESAMPLE_CAP; cap = 1; }
         }
-        if (!ak && lane == 0) {
+        if (lane == 0) {
+            sh_L = L;
+            sh_at = at;
+            sh_ak = ak;
+            sh_umr = umr;
+            sh_tau = tau;
+            sh_k = k;
+        }
+    }
+    __syncthreads();
+    const int L = sh_L, A = L - 1;
+    float tau = sh_tau;
+    unsigned long long iters = 0, cap = 0;
+    if (L <= g && !sh_at) {
+        // Theorem 1: proposals from g_T, accepted with max(0, 1 - g_D / g_T)
+        const int p = n + L - 1, MT = a.MT, MD = a.MD;
+        const float totT = cumT[MT - 1];
+        bool found = false;
+        float last = 0.f;
+        for (int base = 0; base < RESAMPLE_CAP && !found; base += 128) {
+            const int it = base + tid;
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 2u + (uint32_t)it);
+            const float target = u.x * totT;
+            int z = MT - 1;
+            for (int m = 0; m < MT; ++m)
+                if (cumT[m] >= target) { z = m; break; }
+            const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
+            const float lt = fmaf(sgT[z], eps, muT[z]);
+            float mT = -INFINITY, mD = -INFINITY;
+            for (int m = 0; m < MT; ++m) {
+                const float q = (lt - muT[m]) * isT[m];
+                mT = fmaxf(mT, cT[m] - 0.5f * q * q);
+            }
+            for (int m = 0; m < MD; ++m) {
+                const float q = (lt - muD[m]) * isD[m];
+                mD = fmaxf(mD, cD[m] - 0.5f * q * q);
+            }
+            float sT = 0.f, sD = 0.f;
+            for (int m = 0; m < MT; ++m) {
+                const float q = (lt - muT[m]) * isT[m];
+                sT += expf(cT[m] - 0.5f * q * q - mT);
+            }
+            for (int m = 0; m < MD; ++m) {
+                const float q = (lt - muD[m]) * isD[m];
+                sD += expf(cD[m] - 0.5f * q * q - mD);
+            }
+            const float al = fmaxf(0.f, 1.f - expf((mD + logf(sD)) - (mT + logf(sT))));
+            const float tp = expf(lt);
+            const unsigned okb = __ballot_sync(0xffffffffu, u.w < al);
+            if (lane == 0) {
+                win_idx[warp] = okb ? 32 * warp + __ffs(okb) - 1 : 1 << 30;
+            }
+            if (okb && lane == __ffs(okb) - 1) win_tau[warp] = tp;
+            if (tid == 127) last = tp;
+            __syncthreads();
+            int best = 1 << 30, bw = 0;
+            for (int w = 0; w < 4; ++w)
+                if (win_idx[w] < best) { best = win_idx[w]; bw = w; }
+            if (best < (1 << 30)) {
+                tau = win_tau[bw];
+                iters = (unsigned long long)(base + best + 1);
+                found = true;
+            }
+            __syncthreads();  // the winner slots are rewritten by the next step
+        }
+        if (!found) {  // the last proposal of the capped loop (thread 127's)
+            if (tid == 127) sh_tau = last;
+            __syncthreads();
+            tau = sh_tau;
+            iters = RESAMPLE_CAP;
+            cap = 1;
+        }
+    }
+    if (warp != 0) return;
+    int emitted;
+    if (L <= g) {
+        const int p = n + L - 1, src = L - 1;
+        int k = sh_k;
+        const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
+        const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
+        if (!sh_ak && lane == 0) {
             // f' = norm(max(0, f_T - f_D)); zero mass -> draw from f_T
+            const float umr = sh_umr;
             float tot = 0.f;
             for (int kk = 0; kk < a.K; ++kk) tot += fmaxf(0.f, expf(hT[3 * a.MT + kk]) - expf(hD[3 * a.MD + kk]));
             if (tot < 1e-12f) {
@@ -838,9 +875,9 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         if (lane == 0) {
             const float* hT = a.th + ((size_t)s * (g + 1) + g) * a.WT;
             const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
-            const float tau = draw_tau(hT, a.MT, u.x, u.y, u.z);
-            ss.tau[sb + p] = tau;
-            ss.t[sb + p] = ss.t[sb + p - 1] + (double)tau;
+            const float tb = draw_tau(hT, a.MT, u.x, u.y, u.z);
+            ss.tau[sb + p] = tb;
+            ss.t[sb + p] = ss.t[sb + p - 1] + (double)tb;
             ss.k[sb + p] = pick_categorical_log(hT + 3 * a.MT, a.K, u.w);
         }
         emitted = g + 1;
@@ -1209,7 +1246,7 @@ cudaError_t launch_verify_epilogue(const DevModel& mT, const DevModel& mD, const
     a.ss = ss; a.P = dp; a.th = t_heads; a.dh = d_heads;
     a.MT = mT.M; a.MD = mD.M; a.K = mT.K; a.WT = mT.head_width(); a.WD = mD.head_width();
     a.gamma = gamma; a.gamma_max = gamma_max; a.st = stats;
-    k_verify_epilogue<<<(B + 3) / 4, 128, 0, st>>>(a);
+    k_verify_epilogue<<<B, 128, 0, st>>>(a);
     return cudaGetLastError();
 }
 
