@@ -246,6 +246,16 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
         }
     const size_t b_ek = add(ek.data(), ek.size() * 4), b_ekb = add(ekb.data(), ekb.size() * 4);
     const size_t b_ho = add(ho.data(), ho.size() * 4), b_hob = add(hob.data(), hob.size() * 4);
+    // [E; v_k1] as a sum of two bf16 matrices (hi + lo) for the tensor-core head
+    std::vector<uint16_t> ekh(ek.size()), ekl(ek.size());
+    for (size_t i = 0; i < ek.size(); ++i) {
+        ekh[i] = f32_to_bf16_bits(ek[i]);
+        uint32_t hb = (uint32_t)ekh[i] << 16;
+        float hf;
+        memcpy(&hf, &hb, 4);
+        ekl[i] = f32_to_bf16_bits(ek[i] - hf);
+    }
+    const size_t b_ekh = add(ekh.data(), ekh.size() * 2), b_ekl = add(ekl.data(), ekl.size() * 2);
     buf.resize((buf.size() + 15) & ~(size_t)15);
     CK(cudaMalloc(&hm.dbuf, buf.size()));
     ctx->allocs.push_back(hm.dbuf);
@@ -276,6 +286,8 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     m.head_ek_b = (const float*)(b + b_ekb);
     m.head_out_t = (const float*)(b + b_ho);
     m.head_out_b = (const float*)(b + b_hob);
+    m.head_ek_hi = (const void*)(b + b_ekh);
+    m.head_ek_lo = (const void*)(b + b_ekl);
     m.base = b;
     m.bytes = buf.size();
     // transposed, self-contained copy ([in][out] matrices)
@@ -416,6 +428,9 @@ static void build_tc_plan(tppsd_ctx* ctx) {
                 make_tmap_bf16(&p.layer[l].w1_m, L.w_1, d, F, 128) &&
                 make_tmap_bf16(&p.layer[l].w2_m, L.w_2, F, d, 128);
     }
+    p.head = ok && head_tc_supported(m) &&
+             make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
+             make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
     p.err = ctx->d_err;
     p.enabled = ok ? 1 : 0;
 }

@@ -54,6 +54,8 @@ struct DevModel {
     const float* head_ek_b;  // [4d]: zeros then b_k1
     const float* head_out_t; // [d][3M+K] fp32: v_w, v_mu, v_s, v_k2 transposed side by side
     const float* head_out_b; // [3M+K]: b_w, b_mu, b_s, b_k2
+    const void* head_ek_hi;  // [4d][d] bf16: head_ek_w = hi + lo (split of each fp32 value)
+    const void* head_ek_lo;
     DevModelT t;             // transposed copy (read by the per-sequence draft kernel)
     __host__ __device__ int head_width() const { return 3 * M + K; }
 };
@@ -179,6 +181,8 @@ struct TcPlan {
     int enabled;
     int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
     int mlp;                    // post-attention block by the fused kernel
+    int head;                   // heads by the tensor-core head kernel
+    CUtensorMap head_hi, head_lo;
     int* err;
     CUtensorMap a_xb, a_att, a_hid;
     TcLayerMaps layer[MAX_LAYERS];
@@ -200,6 +204,12 @@ int mlp_tc_supported(int d, int F);
 // weight maps with boxes of 64 x 128.
 cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
                           const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st);
+// Target heads on the tensor cores (head_tc.cu) for bf16 models with d = 128:
+// reads the final hidden rows w.x, writes w.heads for rows with row_seq >= 0.
+// hi / lo: tensor maps of the split [E; V_k1] (boxes of 64 x 128).
+int head_tc_supported(const DevModel& m);
+cudaError_t launch_head_tc(const CUtensorMap& hi, const CUtensorMap& lo, const DevModel& m, const Work& w, int R,
+                           cudaStream_t st);
 // Columns per CTA of the cluster LayerNorm GEMM for a row width N (0: unsupported).
 int ln_cluster_cols(int N);
 // EPI_TC_RESID_LN by a cluster of N / ln_cluster_cols(N) CTAs per 128 rows;

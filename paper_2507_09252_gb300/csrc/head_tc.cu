@@ -1,0 +1,175 @@
+// Target heads on the tensor cores (Sec. 4.2) for d = 128.  The four
+// 128-column blocks of [E; V_k1] h feed disjoint head outputs: block 0 (e1)
+// the component logits, 1 (e2) mu, 2 (e3) log sigma, 3 (V_k1 h + b_k1, then
+// tanh) the mark logits.  So CTA (block nb, 128-row tile) computes block nb
+// with tcgen05 and then its own head outputs, with no exchange between
+// CTAs.  The head is fp32 arithmetic: h W^T is formed as
+// h_hi W_hi + h_hi W_lo + h_lo W_hi with both operands split into two bf16
+// parts (x = x_hi + x_lo), fp32 accumulation in TMEM (relative error about
+// 2^-16 of |h| |W|).  Warps 0-3 split the h rows (coalesced reads) into the
+// two swizzled A operands and later own one row each (TMEM lane); warp 4
+// loads the W_hi / W_lo tiles by TMA; one thread of warp 5 issues the MMAs.
+#include <cuda.h>
+
+#include "common.cuh"
+#include "engine.h"
+#include "tc_ptx.cuh"
+
+namespace tppsd {
+
+struct HeadShape {
+    static constexpr int D = 128, BM = 128, BK = 64, KB = D / BK;
+    static constexpr int TILE = BM * BK * 2;  // 16 KB
+    static constexpr int OFF_AH = 0, OFF_AL = KB * TILE, OFF_BH = 2 * KB * TILE, OFF_BL = 3 * KB * TILE;
+    static constexpr int OFF_BAR = 4 * KB * TILE;
+    static constexpr size_t SMEM = (size_t)OFF_BAR + 64 + 1024;
+};
+
+__global__ void __launch_bounds__(192, 1)
+    k_head_tc(const __grid_constant__ CUtensorMap mapHi, const __grid_constant__ CUtensorMap mapLo, DevModel m,
+              Work w, int R) {
+    using S = HeadShape;
+    constexpr int D = S::D;
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint64_t* bars = (uint64_t*)(smem + S::OFF_BAR);
+    uint64_t* a_ready = bars;      // both A operands written (128 arrivals)
+    uint64_t* b_full = bars + 1;   // W tiles landed
+    uint64_t* done = bars + 2;     // accumulator complete
+    uint32_t* tslot = (uint32_t*)(bars + 3);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nb = blockIdx.x, m0 = blockIdx.y * S::BM, rows = min(S::BM, R - m0);
+    if (threadIdx.x == 0) {
+        mbar_init(a_ready, 128);
+        mbar_init(b_full, 1);
+        mbar_init(done, 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, 128);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            mbar_arrive_expect_tx(b_full, 2 * S::KB * S::TILE);
+            for (int kb = 0; kb < S::KB; ++kb) {
+                tma_load_2d(smem + S::OFF_BH + kb * S::TILE, &mapHi, b_full, kb * S::BK, nb * 128);
+                tma_load_2d(smem + S::OFF_BL + kb * S::TILE, &mapLo, b_full, kb * S::BK, nb * 128);
+            }
+        }
+    } else if (warp == 5) {
+        if (lane == 0) {
+            bool ok = mbar_wait(a_ready, 0, w.err, 51);
+            ok = ok && mbar_wait(b_full, 0, w.err, 52);
+            tc_fence_after();
+            if (ok) {
+                const uint32_t idesc = idesc_bf16(128, 128);
+                const uint32_t ah = smem_u32(smem + S::OFF_AH), al = smem_u32(smem + S::OFF_AL);
+                const uint32_t bh = smem_u32(smem + S::OFF_BH), bl = smem_u32(smem + S::OFF_BL);
+                for (int kb = 0; kb < S::KB; ++kb)
+#pragma unroll
+                    for (int kk = 0; kk < S::BK / 16; ++kk) {
+                        const uint32_t o = kb * S::TILE + kk * 32;
+                        tc_mma_bf16(tmem, sw128_desc(ah + o), sw128_desc(bh + o), idesc, (kb | kk) != 0);
+                        tc_mma_bf16(tmem, sw128_desc(ah + o), sw128_desc(bl + o), idesc, 1u);
+                        tc_mma_bf16(tmem, sw128_desc(al + o), sw128_desc(bh + o), idesc, 1u);
+                    }
+            }
+            tc_commit(done);
+        }
+    } else {
+        const int t = threadIdx.x;
+        // A operands: h rows split into hi / lo bf16, written in the swizzled
+        // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7))
+        for (int f = t; f < S::BM * D / 4; f += 128) {
+            const int r = f >> 5, c4 = f & 31;
+            const float4 x = r < rows ? *reinterpret_cast<const float4*>(w.x + (size_t)(m0 + r) * D + 4 * c4)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float xs[4] = {x.x, x.y, x.z, x.w};
+            uint32_t hi[2], lo[2];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const __nv_bfloat162 h2 = __floats2bfloat162_rn(xs[2 * i], xs[2 * i + 1]);
+                const float2 hf = __bfloat1622float2(h2);
+                const __nv_bfloat162 l2 = __floats2bfloat162_rn(xs[2 * i] - hf.x, xs[2 * i + 1] - hf.y);
+                hi[i] = *reinterpret_cast<const uint32_t*>(&h2);
+                lo[i] = *reinterpret_cast<const uint32_t*>(&l2);
+            }
+            const int kb = c4 >> 4, ch = (c4 & 15) >> 1, half = c4 & 1;
+            const int off = kb * S::TILE + r * 128 + ((ch ^ (r & 7)) << 4) + half * 8;
+            *reinterpret_cast<uint2*>(smem + S::OFF_AH + off) = make_uint2(hi[0], hi[1]);
+            *reinterpret_cast<uint2*>(smem + S::OFF_AL + off) = make_uint2(lo[0], lo[1]);
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(a_ready);
+        // row t of the tile: its 128 columns of block nb, then its outputs
+        const bool live = t < rows && w.row_seq[m0 + t] >= 0;
+        mbar_wait(done, 0, w.err, 53);
+        tc_fence_after();
+        const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
+        const int M = m.M, K = m.K, WO = 3 * M + K;
+        const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M;
+        const float* bk1 = m.head_ek_b + 3 * D;
+        float* dst = w.heads + (size_t)(m0 + t) * WO + col0;
+        const float* Wt = m.head_out_t + col0;  // [d][WO]: column col0 + o holds output o's weights
+        float mx = -INFINITY, sum = 0.f;         // online log-sum-exp of the logits
+        for (int o0 = 0; o0 < cnt; o0 += 8) {
+            float acc[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] = o0 + j < cnt ? __ldg(m.head_out_b + col0 + o0 + j) : 0.f;
+            // the row's 128 columns, 64 at a time from TMEM (block 3: tanh(. + b_k1))
+            for (int hf = 0; hf < 2; ++hf) {
+                float v[64];
+                tmem_ld64(tl + 64 * hf, v);
+                if (nb == 3) {
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) v[i] = tanhf(v[i] + __ldg(bk1 + 64 * hf + i));
+                }
+#pragma unroll
+                for (int i = 0; i < 64; ++i) {
+                    const float* wr = Wt + (size_t)(64 * hf + i) * WO + o0;
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        if (o0 + j < cnt) acc[j] = fmaf(__ldg(wr + j), v[i], acc[j]);
+                }
+            }
+            if (!live) continue;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (o0 + j >= cnt) continue;
+                dst[o0 + j] = acc[j];
+                if (nb == 0 || nb == 3) {
+                    const float mn = fmaxf(mx, acc[j]);
+                    sum = sum * expf(mx - mn) + expf(acc[j] - mn);
+                    mx = mn;
+                }
+            }
+        }
+        if (live) {
+            if (nb == 0 || nb == 3) {  // log w, log f: subtract log sum exp
+                const float lz = mx + logf(sum);
+                for (int o = 0; o < cnt; ++o) dst[o] -= lz;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 128);
+}
+
+int head_tc_supported(const DevModel& m) { return m.dtype == 1 && m.d == HeadShape::D; }
+
+cudaError_t launch_head_tc(const CUtensorMap& hi, const CUtensorMap& lo, const DevModel& m, const Work& w, int R,
+                           cudaStream_t st) {
+    if (R <= 0) return cudaSuccess;
+    if (!head_tc_supported(m)) return cudaErrorInvalidValue;
+    const size_t sm = HeadShape::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(k_head_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    k_head_tc<<<dim3(4, (R + 127) / 128), 192, sm, st>>>(hi, lo, m, w, R);
+    return cudaGetLastError();
+}
+
+}  // namespace tppsd

@@ -1161,7 +1161,13 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         PROF_MARK(prof, KC_LAYERNORM, 0, st);
         nl += 7;
     }
-    if (want_heads) {
+    if (want_heads && use_tc && tc->head) {
+        PROF_MARK(prof, KC_HEAD, 1, st);
+        const cudaError_t e = launch_head_tc(tc->head_hi, tc->head_lo, m, w, R, st);
+        if (e != cudaSuccess) return e;
+        PROF_MARK(prof, KC_HEAD, 0, st);
+        nl += 1;
+    } else if (want_heads) {
         // e | V_k1 h + b_k1 for all rows (fp32 tiled GEMM), then the small maps
         PROF_MARK(prof, KC_HEAD, 1, st);
         GemmArgs<float> gh{};
