@@ -1,6 +1,6 @@
 """Per-kernel-class timing of one sampling call.
 
-    python -m paper_2507_09252_gb300.profile_call [--workload c2] [--calls 1]
+    python -m paper_2507_09252_gb300.profile_call [--workload c2] [--calls 2]
                                                   [--mode sd|ar] [--host-loop]
 
 Builds the workload's models and histories (seeded, synthetic), prefills,
@@ -27,8 +27,8 @@ def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--workload", default="c2", choices=sorted(WORKLOADS))
     ap.add_argument("--calls", type=int, default=2,
-                    help="calls to run; the per-class times are those of the last one (the first
-                         call also pays one-time kernel loading)")
+                    help="calls to run; the per-class times are those of the last one "
+                         "(the first call also pays one-time kernel loading)")
     ap.add_argument("--mode", default="sd", choices=["sd", "ar"])
     ap.add_argument("--host-loop", action="store_true")
     a = ap.parse_args(argv)
