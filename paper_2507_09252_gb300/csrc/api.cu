@@ -104,6 +104,10 @@ struct tppsd_ctx {
 };
 
 // ---------------------------------------------------------------- helpers
+namespace tppsd {
+int g_pdl = 1;
+}  // namespace tppsd
+
 static const char* fault_mode() {
     const char* f = getenv("TPPSD_FAULT");
     return f ? f : "";
@@ -515,6 +519,7 @@ extern "C" tppsd_status_t tppsd_create_models(const tppsd_model_cfg* target,
     if (!(draft->heads == 1 || draft->heads == 2 || draft->heads == 4) || dhD < 8)
         return TPPSD_ERR_UNSUPPORTED;
     if (!strcmp(fault_mode(), "alloc")) return TPPSD_ERR_OOM;  // injected allocation failure
+    g_pdl = getenv("TPPSD_NO_PDL") ? 0 : 1;
     tppsd_ctx* ctx = new (std::nothrow) tppsd_ctx();
     if (!ctx) return TPPSD_ERR_OOM;
     ctx->max_batch = max_batch;

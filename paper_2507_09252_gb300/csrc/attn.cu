@@ -53,6 +53,7 @@ template <int DH>
 __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) {
     using S = AttnShape<DH>;
     constexpr int KT = S::KT, NT = KT / 8, KS = DH / 16;
+    pdl_wait();
     extern __shared__ __align__(128) unsigned char smem[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane >> 2, t4 = lane & 3;
@@ -245,6 +246,7 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
         }
         a.out[(size_t)(rb + row) * a.d + h * DH + col] = __float2bfloat16_rn(O / L);
     }
+    pdl_trigger();
 }
 
 cudaError_t launch_attn_mma(const AttArgs<bf16>& a, int dh, int nh, int nseg, int* err, cudaStream_t st) {
@@ -253,19 +255,19 @@ cudaError_t launch_attn_mma(const AttArgs<bf16>& a, int dh, int nh, int nseg, in
         case 16: {
             const int sm = AttnShape<16>::SMEM;
             cudaFuncSetAttribute(k_attn_mma<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            k_attn_mma<16><<<grid, 128, sm, st>>>(a, err);
+            if (const cudaError_t e = launch_k(k_attn_mma<16>, grid, dim3(128), sm, st, a, err)) return e;
             break;
         }
         case 32: {
             const int sm = AttnShape<32>::SMEM;
             cudaFuncSetAttribute(k_attn_mma<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            k_attn_mma<32><<<grid, 128, sm, st>>>(a, err);
+            if (const cudaError_t e = launch_k(k_attn_mma<32>, grid, dim3(128), sm, st, a, err)) return e;
             break;
         }
         case 64: {
             const int sm = AttnShape<64>::SMEM;
             cudaFuncSetAttribute(k_attn_mma<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            k_attn_mma<64><<<grid, 128, sm, st>>>(a, err);
+            if (const cudaError_t e = launch_k(k_attn_mma<64>, grid, dim3(128), sm, st, a, err)) return e;
             break;
         }
         default:

@@ -12,6 +12,17 @@ constexpr uint32_t FLAG_NO_BONUS = 1u;
 
 typedef __nv_bfloat16 bf16;
 
+// ---------------------------------------------------------------- launch order
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while the previous kernel of the stream is still
+// finishing; pdl_wait() blocks until that kernel has completed and its
+// memory is visible, so every kernel calls it before its first access to
+// global memory.  pdl_trigger() lets the next kernel start launching once
+// every CTA of this one has called it or exited.  Both are no-ops for a
+// kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------------- storage
 // Storage type T of weights, GEMM inputs and KV: float (fp32 models) or bf16.
 template <typename T> struct St;

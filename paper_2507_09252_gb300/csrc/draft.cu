@@ -273,6 +273,7 @@ __device__ void rebase_model(DevModelT& m, const DevModelT& src, int L, const ch
 template <typename T, int DH, bool KVS, bool WS>
 __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, int area_bytes) {
     constexpr int TEAMS = WS ? 2 : 1;
+    pdl_wait();
     extern __shared__ __align__(16) char smem[];
     __shared__ double t_new_s[TEAMS];
     __shared__ int k_new_s[TEAMS];
@@ -498,6 +499,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             layers(p);
         }
     }
+    pdl_trigger();
 }
 
 template <typename T, int DH, bool KVS, bool WS>
@@ -506,8 +508,8 @@ static cudaError_t launch_t(DraftTeamArgs& a, int B, int area, size_t sm, cudaSt
     cudaError_t e = cudaFuncSetAttribute(k_draft_team<T, DH, KVS, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)sm);
     if (e != cudaSuccess) return e;
-    k_draft_team<T, DH, KVS, WS><<<(B + TEAMS - 1) / TEAMS, 128 * TEAMS, sm, st>>>(a, area);
-    return cudaGetLastError();
+    return launch_k(k_draft_team<T, DH, KVS, WS>, dim3((B + TEAMS - 1) / TEAMS), dim3(128 * TEAMS), sm, st, a,
+                    area);
 }
 
 template <typename T, int DH>

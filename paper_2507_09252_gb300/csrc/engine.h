@@ -9,6 +9,26 @@
 
 namespace tppsd {
 
+// Kernels of a sampling round are launched with programmatic stream
+// serialization (each calls pdl_wait() before touching global memory), so a
+// kernel's launch overlaps the previous kernel's last CTAs.  g_pdl = 0
+// launches them plainly.
+extern int g_pdl;
+template <typename... P, typename... A>
+inline cudaError_t launch_k(void (*k)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, A... args) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = g_pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, k, args...);
+}
+
 constexpr int MAX_LAYERS = 16;
 constexpr int MAX_MIX = 64;
 constexpr int MAX_MARKS = 256;

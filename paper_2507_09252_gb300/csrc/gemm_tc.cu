@@ -51,6 +51,7 @@ template <int BN>
 __global__ void __launch_bounds__(128, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, TcGemmArgs a) {
     using S = TcShape<BN>;
+    pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     float* bias_s = (float*)(smem + S::STAGES * S::STAGE);
@@ -163,6 +164,7 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
+    pdl_trigger();
 }
 
 // ---------------------------------------------------------------- LayerNorm GEMM
@@ -346,8 +348,7 @@ static cudaError_t launch_bn(const CUtensorMap& A, const CUtensorMap& W, const T
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     const dim3 grid(a.N / BN, (a.R + 127) / 128);
-    k_gemm_tc<BN><<<grid, 128, sm, st>>>(A, W, a);
-    return cudaGetLastError();
+    return launch_k(k_gemm_tc<BN>, grid, dim3(128), sm, st, A, W, a);
 }
 
 template <int BNC>

@@ -30,6 +30,7 @@ __global__ void __launch_bounds__(192, 1)
               Work w, int R) {
     using S = HeadShape;
     constexpr int D = S::D;
+    pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t* bars = (uint64_t*)(smem + S::OFF_BAR);
@@ -157,6 +158,7 @@ __global__ void __launch_bounds__(192, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 128);
+    pdl_trigger();
 }
 
 int head_tc_supported(const DevModel& m) { return m.dtype == 1 && m.d == HeadShape::D; }
@@ -168,8 +170,7 @@ cudaError_t launch_head_tc(const CUtensorMap& hi, const CUtensorMap& lo, const D
     const size_t sm = HeadShape::SMEM;
     cudaError_t e = cudaFuncSetAttribute(k_head_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_head_tc<<<dim3(4, (R + 127) / 128), 192, sm, st>>>(hi, lo, m, w, R);
-    return cudaGetLastError();
+    return launch_k(k_head_tc, dim3(4, (R + 127) / 128), dim3(192), sm, st, hi, lo, m, w, R);
 }
 
 }  // namespace tppsd

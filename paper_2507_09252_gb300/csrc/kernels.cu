@@ -47,6 +47,7 @@ __device__ __forceinline__ void embed_pair(const DevModel& m, double t, int k, i
 // ======================================================================
 template <typename T>
 __global__ void k_embed(DevModel m, SeqState ss, RowSpec rs, Work w) {
+    pdl_wait();
     const int half = m.d / 2;
     const long long total = (long long)rs.count * half;
     T* xb = (T*)w.xb;
@@ -80,6 +81,7 @@ __global__ void k_embed(DevModel m, SeqState ss, RowSpec rs, Work w) {
         St<T>::st(xb + xo, z0);
         St<T>::st(xb + xo + 1, z1);
     }
+    pdl_trigger();
 }
 
 enum { EPI_QKV = 0, EPI_RELU = 1, EPI_RESID = 2, EPI_F32 = 3 };
@@ -703,6 +705,7 @@ __device__ void write_outputs(const SeqState& ss, const CallParams& P, int s, in
 // adds the bonus event from the target head after the last draft (unless
 // NO_BONUS).
 __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
+    pdl_wait();
     // per-component constants of both mixtures for the Theorem-1 loop
     __shared__ float cumT[MAX_MIX], muT[MAX_MIX], sgT[MAX_MIX], isT[MAX_MIX], cT[MAX_MIX];
     __shared__ float muD[MAX_MIX], isD[MAX_MIX], cD[MAX_MIX];
@@ -899,11 +902,13 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         if (iters) atomicAdd(&a.st->resample_iters, iters);
         if (cap) atomicAdd(&a.st->cap_hits, cap);
     }
+    pdl_trigger();
 }
 
 // Autoregressive sample (Sec. 4.2): one thread per sequence, head row s.
 __global__ void k_ar_sample(SeqState ss, const CallParams* Pp, const float* heads, int M, int K,
                             int W, DevStats* st) {
+    pdl_wait();
     const int s = blockIdx.x * blockDim.x + threadIdx.x;
     const CallParams& P = *Pp;
     if (s >= P.B || ss.done[s]) return;
@@ -928,6 +933,7 @@ __global__ void k_ar_sample(SeqState ss, const CallParams* Pp, const float* head
     atomicAdd(&st->rounds, 1ull);
     atomicAdd(&st->emitted, 1ull);
     atomicAdd(&st->target_keys, (unsigned long long)n);  // positions 0..n-1
+    pdl_trigger();
 }
 
 // ======================================================================
@@ -955,6 +961,7 @@ __global__ void k_begin(CallParams p, CallParams* dp, SeqState ss, DevStats* st)
 __global__ void __launch_bounds__(256) k_round_control(SeqState ss, const CallParams* Pp,
                                                        DevStats* st, cudaGraphConditionalHandle h,
                                                        int use_cond, int* active_out) {
+    pdl_wait();
     __shared__ int cnt;
     if (threadIdx.x == 0) cnt = 0;
     __syncthreads();
@@ -1047,7 +1054,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         const long long want = (total + 255) / 256;
         const int blocks = (int)(want < 152 * 16 ? want : 152 * 16);
         PROF_MARK(prof, KC_EMBED, 1, st);
-        k_embed<T><<<blocks, 256, 0, st>>>(m, ss, rs, w);
+        if (const cudaError_t e = launch_k(k_embed<T>, dim3(blocks), dim3(256), 0, st, m, ss, rs, w)) return e;
         PROF_MARK(prof, KC_EMBED, 0, st);
         ++nl;
     }
@@ -1252,23 +1259,21 @@ cudaError_t launch_verify_epilogue(const DevModel& mT, const DevModel& mD, const
     a.ss = ss; a.P = dp; a.th = t_heads; a.dh = d_heads;
     a.MT = mT.M; a.MD = mD.M; a.K = mT.K; a.WT = mT.head_width(); a.WD = mD.head_width();
     a.gamma = gamma; a.gamma_max = gamma_max; a.st = stats;
-    k_verify_epilogue<<<B, 128, 0, st>>>(a);
-    return cudaGetLastError();
+    return launch_k(k_verify_epilogue, dim3(B), dim3(128), 0, st, a);
 }
 
 cudaError_t launch_ar_sample(const DevModel& mT, const SeqState& ss, const CallParams* dp, int B,
                              const float* heads, DevStats* stats, cudaStream_t st) {
-    k_ar_sample<<<(B + 127) / 128, 128, 0, st>>>(ss, dp, heads, mT.M, mT.K, mT.head_width(), stats);
-    return cudaGetLastError();
+    return launch_k(k_ar_sample, dim3((B + 127) / 128), dim3(128), 0, st, ss, dp, heads, mT.M, mT.K,
+                    mT.head_width(), stats);
 }
 
 cudaError_t launch_round_control(const SeqState& ss, const CallParams* dp, int B, DevStats* stats,
                                  unsigned long long cond_handle, int use_cond, int* active_out,
                                  cudaStream_t st) {
     (void)B;
-    k_round_control<<<1, 256, 0, st>>>(ss, dp, stats, (cudaGraphConditionalHandle)cond_handle,
-                                       use_cond, active_out);
-    return cudaGetLastError();
+    return launch_k(k_round_control, dim3(1), dim3(256), 0, st, ss, dp, stats,
+                    (cudaGraphConditionalHandle)cond_handle, use_cond, active_out);
 }
 
 cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work& w, int B, int len,

@@ -73,6 +73,7 @@ __global__ void __launch_bounds__(320, 1)
              const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2, MlpArgs a) {
     using S = MlpShape;
     constexpr int D = S::D;
+    pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* A = smem + S::OFF_A;
@@ -349,6 +350,7 @@ __global__ void __launch_bounds__(320, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 512);
+    pdl_trigger();
 }
 
 int mlp_tc_supported(int d, int F) { return d == MlpShape::D && F % MlpShape::CH == 0 && F <= MlpShape::PF; }
@@ -360,8 +362,7 @@ cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const C
     const size_t sm = MlpShape::SMEM;
     cudaError_t e = cudaFuncSetAttribute(k_mlp_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    k_mlp_tc<<<(a.R + 127) / 128, 320, sm, st>>>(att, wo, w1, w2, a);
-    return cudaGetLastError();
+    return launch_k(k_mlp_tc, dim3((a.R + 127) / 128), dim3(320), sm, st, att, wo, w1, w2, a);
 }
 
 }  // namespace tppsd
