@@ -22,7 +22,8 @@ struct HeadShape {
     static constexpr int TILE = BM * BK * 2;  // 16 KB
     static constexpr int OFF_AH = 0, OFF_AL = KB * TILE, OFF_BH = 2 * KB * TILE, OFF_BL = 3 * KB * TILE;
     static constexpr int OFF_BAR = 4 * KB * TILE;
-    static constexpr size_t SMEM = (size_t)OFF_BAR + 64 + 1024;
+    static constexpr int OFF_W = OFF_BAR + 64;  // small output matrix [D][cnt], its bias, b_k1
+    static constexpr size_t smem_bytes(int cnt) { return (size_t)OFF_W + ((size_t)D * cnt + cnt + D) * 4 + 1024; }
 };
 
 __global__ void __launch_bounds__(192, 1)
@@ -38,6 +39,7 @@ __global__ void __launch_bounds__(192, 1)
     uint64_t* b_full = bars + 1;   // W tiles landed
     uint64_t* done = bars + 2;     // accumulator complete
     uint32_t* tslot = (uint32_t*)(bars + 3);
+    float* ws = (float*)(smem + S::OFF_W);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = blockIdx.x, m0 = blockIdx.y * S::BM, rows = min(S::BM, R - m0);
     if (threadIdx.x == 0) {
@@ -105,35 +107,41 @@ __global__ void __launch_bounds__(192, 1)
         }
         fence_proxy_async_smem();
         mbar_arrive(a_ready);
+        // while the tensor cores run: this block's output matrix (columns
+        // col0.. of the [d][3M+K] head map), its bias and b_k1 into shared memory
+        const int M = m.M, K = m.K, WO = 3 * M + K;
+        const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M;
+        for (int i = t; i < D * cnt; i += 128) ws[i] = m.head_out_t[(size_t)(i / cnt) * WO + col0 + i % cnt];
+        for (int i = t; i < cnt; i += 128) ws[D * cnt + i] = m.head_out_b[col0 + i];
+        for (int i = t; i < D; i += 128) ws[D * cnt + cnt + i] = m.head_ek_b[3 * D + i];
+        asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
         // row t of the tile: its 128 columns of block nb, then its outputs
         const bool live = t < rows && w.row_seq[m0 + t] >= 0;
         mbar_wait(done, 0, w.err, 53);
         tc_fence_after();
         const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
-        const int M = m.M, K = m.K, WO = 3 * M + K;
-        const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M;
-        const float* bk1 = m.head_ek_b + 3 * D;
+        const float* bk1 = ws + D * cnt + cnt;
         float* dst = w.heads + (size_t)(m0 + t) * WO + col0;
-        const float* Wt = m.head_out_t + col0;  // [d][WO]: column col0 + o holds output o's weights
+        const float* Wt = ws;  // [d][cnt]
         float mx = -INFINITY, sum = 0.f;         // online log-sum-exp of the logits
         for (int o0 = 0; o0 < cnt; o0 += 8) {
             float acc[8];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[j] = o0 + j < cnt ? __ldg(m.head_out_b + col0 + o0 + j) : 0.f;
+            for (int j = 0; j < 8; ++j) acc[j] = o0 + j < cnt ? ws[D * cnt + o0 + j] : 0.f;
             // the row's 128 columns, 64 at a time from TMEM (block 3: tanh(. + b_k1))
             for (int hf = 0; hf < 2; ++hf) {
                 float v[64];
                 tmem_ld64(tl + 64 * hf, v);
                 if (nb == 3) {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) v[i] = tanhf(v[i] + __ldg(bk1 + 64 * hf + i));
+                    for (int i = 0; i < 64; ++i) v[i] = tanhf(v[i] + bk1[64 * hf + i]);
                 }
 #pragma unroll
                 for (int i = 0; i < 64; ++i) {
-                    const float* wr = Wt + (size_t)(64 * hf + i) * WO + o0;
+                    const float* wr = Wt + (64 * hf + i) * cnt + o0;
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
-                        if (o0 + j < cnt) acc[j] = fmaf(__ldg(wr + j), v[i], acc[j]);
+                        if (o0 + j < cnt) acc[j] = fmaf(wr[j], v[i], acc[j]);
                 }
             }
             if (!live) continue;
@@ -161,13 +169,16 @@ __global__ void __launch_bounds__(192, 1)
     pdl_trigger();
 }
 
-int head_tc_supported(const DevModel& m) { return m.dtype == 1 && m.d == HeadShape::D; }
+int head_tc_supported(const DevModel& m) {
+    const int cnt = m.M > m.K ? m.M : m.K;
+    return m.dtype == 1 && m.d == HeadShape::D && HeadShape::smem_bytes(cnt) <= 227 * 1024;
+}
 
 cudaError_t launch_head_tc(const CUtensorMap& hi, const CUtensorMap& lo, const DevModel& m, const Work& w, int R,
                            cudaStream_t st) {
     if (R <= 0) return cudaSuccess;
     if (!head_tc_supported(m)) return cudaErrorInvalidValue;
-    const size_t sm = HeadShape::SMEM;
+    const size_t sm = HeadShape::smem_bytes(m.M > m.K ? m.M : m.K);
     cudaError_t e = cudaFuncSetAttribute(k_head_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     return launch_k(k_head_tc, dim3(4, (R + 127) / 128), dim3(192), sm, st, hi, lo, m, w, R);
