@@ -198,11 +198,28 @@ def roofline(kt, stats, wl, peaks):
         peak = peaks.get("bf16_tflops_sustained", 1700.0)
     share = ms / sum(v[0] for v in kt.values())
     return {"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": round(peak, 1),
-            "unit": unit, "frac": round(achieved / peak, 4), "traffic": None,
+            "unit": unit, "frac": round(achieved / peak, 4), "traffic": ncu_traffic(name),
             "per_launch_ms": round(per_launch_s * 1e3, 4), "launches": launches,
             "share_of_device_time": round(share, 3),
             "algorithmic_per_launch": per_launch,
             "peak_source": "MEASURED_PEAKS.json" if peaks else "fallback"}
+
+
+def ncu_traffic(kernel_class):
+    """DRAM bytes per launch of a kernel class from the committed ncu capture
+    (profiles/dram_traffic_c2.json), or None once any source file the
+    capture was taken on has changed since."""
+    import hashlib
+    try:
+        t = json.load(open(os.path.join(ROOT, "profiles", "dram_traffic_c2.json")))
+        e = t["kernels"][kernel_class]
+        for f, digest in e["sources"].items():
+            with open(os.path.join(ROOT, f), "rb") as fh:
+                if hashlib.sha256(fh.read()).hexdigest() != digest:
+                    return None
+        return e["dram_bytes_per_launch"]
+    except (OSError, ValueError, KeyError):
+        return None
 
 
 def load_peaks():

@@ -68,3 +68,23 @@ def test_single_rank_identity():
     a = bench.rank_histories(CF.C1, 0)
     b = bench.rank_histories(CF.C1, 0)
     assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def test_traffic_record_is_dropped_when_a_source_changes(tmp_path, monkeypatch):
+    """bench.py reports an ncu DRAM figure only while every source file the
+    capture was taken on is byte-identical."""
+    import hashlib
+    import json
+    sys.path.insert(0, ROOT)
+    import bench
+    (tmp_path / "profiles").mkdir()
+    src = tmp_path / "k.cu"
+    src.write_text("kernel v1")
+    rec = {"kernels": {"draft": {"dram_bytes_per_launch": 123,
+                                 "sources": {"k.cu": hashlib.sha256(b"kernel v1").hexdigest()}}}}
+    (tmp_path / "profiles" / "dram_traffic_c2.json").write_text(json.dumps(rec))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.ncu_traffic("draft") == 123
+    assert bench.ncu_traffic("attention") is None
+    src.write_text("kernel v2")
+    assert bench.ncu_traffic("draft") is None
