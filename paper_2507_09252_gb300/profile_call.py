@@ -1,15 +1,25 @@
-"""Per-kernel-class timing of one sampling call.
+"""Per-kernel-class timing of sampling calls, and a throughput mode for every
+workload shape.
 
     python -m paper_2507_09252_gb300.profile_call [--workload c2] [--calls 2]
                                                   [--mode sd|ar] [--host-loop]
+    python -m paper_2507_09252_gb300.profile_call --time --workload c3 [--gamma 4]
+                                                  [--batch 16] [--draft 0]
 
-Builds the workload's models and histories (seeded, synthetic), prefills,
-and runs `--calls` sampling calls.  By default each call runs with
-TPPSD_FLAG_PROFILE (every launch bracketed by CUDA events) and the
-per-class totals are printed; with --host-loop the calls run the rounds
-from a host loop without events, which is the form a per-launch profiler
-(ncu) can attribute, since kernels inside a CUDA graph's conditional loop
+Builds the workload's models and histories (seeded, synthetic) and prefills.
+
+Default: runs `--calls` sampling calls with TPPSD_FLAG_PROFILE (every launch
+bracketed by CUDA events) and prints the per-class totals of the last one
+(the first call also pays one-time kernel loading).  With --host-loop the
+calls run the rounds from a host loop without events, the form a per-launch
+profiler (ncu) can attribute: kernels inside a CUDA graph's conditional loop
 are not visible to it.
+
+--time: TPP-SD and target-only AR events/s of the graph-launched calls
+(CUDA events, inputs resident, 2 warm-up + 3 timed calls each, L2 flushed
+before each timed call), mean accepted drafts per verify and acceptance
+rate, as one JSON line.  --gamma / --batch / --draft override the workload's
+gamma, batch and draft model (an index into the workload's draft sweep).
 """
 import argparse
 import json
@@ -20,7 +30,28 @@ from . import inputs as IN
 from . import tppsd as T
 from .sampler import Sampler
 
-WORKLOADS = {"c1": CF.C1, "c2": CF.C2}
+WORKLOADS = {"c1": CF.C1, "c2": CF.C2, "c3": CF.C3, "c4": CF.C4, "c5": CF.C5}
+
+
+def _time_calls(torch, fn, flush, reps=3, warm=2):
+    st = torch.cuda.current_stream()
+    for _ in range(warm):
+        fn()
+    torch.cuda.synchronize()
+    tot = 0.0
+    for _ in range(reps):
+        flush.fill_(1.0)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        fn()
+        e1.record(st)
+        torch.cuda.synchronize()
+        tot += e0.elapsed_time(e1)
+    return tot / reps
+
+
+def _shape(cfg, fields):
+    return " ".join(f"{n}{getattr(cfg, f)}" for n, f in fields)
 
 
 def main(argv=None):
@@ -31,9 +62,19 @@ def main(argv=None):
                          "(the first call also pays one-time kernel loading)")
     ap.add_argument("--mode", default="sd", choices=["sd", "ar"])
     ap.add_argument("--host-loop", action="store_true")
+    ap.add_argument("--time", action="store_true")
+    ap.add_argument("--gamma", type=int, default=None)
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--draft", type=int, default=None)
     a = ap.parse_args(argv)
     import torch
     wl = WORKLOADS[a.workload]
+    if a.gamma is not None:
+        wl = wl.with_(gamma=a.gamma)
+    if a.batch is not None:
+        wl = wl.with_(batch=a.batch)
+    if a.draft is not None:
+        wl = wl.with_(draft=wl.drafts[a.draft])
     B, H, N, g = wl.batch, wl.hist_len, wl.n_events, wl.gamma
     bt, bd = IN.model_blob(wl.target, wl.seed, 0), IN.model_blob(wl.draft, wl.seed, 1)
     tau_np, mk_np = IN.histories(wl, seed=wl.seed)
@@ -41,6 +82,33 @@ def main(argv=None):
     tau, mk = torch.from_numpy(tau_np).cuda(), torch.from_numpy(mk_np).cuda()
     outs = s._outputs(B, N)
     st = torch.cuda.current_stream()
+    if a.time:
+        flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+
+        def sd():
+            T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
+            T.tppsd_sample(s.ctx, B, N, g, 1234, 0, *outs, st)
+
+        def ar():
+            T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
+            T.tppsd_sample_autoregressive(s.ctx, B, N, 1234, 0, *outs, st)
+
+        ms_sd = _time_calls(torch, sd, flush)
+        _, st_sd = T.tppsd_get_stats(s.ctx)
+        ms_ar = _time_calls(torch, ar, flush, reps=2, warm=1)
+        layer = (("L", "layers"), ("d", "d_model"), ("h", "heads"), ("F", "d_ffn"))
+        print(json.dumps({
+            "workload": wl.name, "batch": B, "gamma": g, "n_events": N, "hist_len": H,
+            "target": _shape(wl.target, layer + (("M", "n_mix"), ("K", "n_marks"))),
+            "draft": _shape(wl.draft, layer),
+            "sd_events_per_s": round(B * N / (ms_sd / 1e3), 1), "sd_ms_per_call": round(ms_sd, 3),
+            "ar_events_per_s": round(B * N / (ms_ar / 1e3), 1), "ar_ms_per_call": round(ms_ar, 3),
+            "speedup_vs_ar": round(ms_ar / ms_sd, 3),
+            "mean_accepted_per_verify": round(st_sd["accepted"] / max(st_sd["rounds"], 1), 3),
+            "alpha": round(st_sd["accepted"] / max(st_sd["drafted"], 1), 4),
+            "rounds": st_sd["loop_iters"], "note": "prefill included in both timed calls"}), flush=True)
+        s.close()
+        return 0
     flags = T.TPPSD_FLAG_HOST_LOOP if a.host_loop else T.TPPSD_FLAG_PROFILE
     for _ in range(a.calls):
         T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
