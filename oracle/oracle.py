@@ -63,8 +63,20 @@ def lib():
                                     C.c_int32, C.c_uint64, C.c_uint32, _f64p, _i32p, _i64p]
         L.oracle_toy_ar.argtypes = [C.c_int32, C.c_int32, _f64p, C.c_int32, C.c_int32,
                                     C.c_uint64, _f64p, _i32p]
+        L.oracle_sample_ar_until.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p,
+                                             _i32p, C.c_int32, C.c_double, C.c_uint64, C.c_int32,
+                                             _opt(_i32p), _f64p, _f64p, _i32p, _f64p, _i32p, C.c_int32]
+        L.oracle_sample_sd_until.argtypes = [_i32p, _f32p, C.c_int64, _i32p, _f32p, C.c_int64,
+                                             C.c_int32, C.c_int32, _f32p, _i32p, C.c_int32, C.c_double,
+                                             C.c_int32, C.c_uint64, C.c_uint32, C.c_int32, _opt(_i32p),
+                                             _f64p, _f64p, _i32p, _f64p, _i32p, _i64p, C.c_int32]
+        L.oracle_score_survival.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p,
+                                            _i32p, C.c_double, _f64p, C.c_int32, C.c_int32]
+        L.oracle_log_survival.argtypes = [C.c_int32, _f64p, C.c_double]
+        L.oracle_log_survival.restype = C.c_double
         for f in ("oracle_score", "oracle_sample_ar", "oracle_sample_sd", "oracle_toy_sd",
-                  "oracle_toy_ar"):
+                  "oracle_toy_ar", "oracle_sample_ar_until", "oracle_sample_sd_until",
+                  "oracle_score_survival"):
             getattr(L, f).restype = C.c_int
         _lib = L
     return _lib
@@ -159,6 +171,58 @@ def sample_sd(cfg_t, blob_t, cfg_d, blob_d, hist_tau, hist_marks, n_events, gamm
                                   int(recompute), _ids(seq_ids, B), tau, t, k, mg, st, nthreads),
            "oracle_sample_sd")
     return dict(tau=tau, t=t, k=k, margin=mg, stats=st)
+
+
+def sample_ar_until(cfg_t, blob_t, hist_tau, hist_marks, max_events, t_end, seed, recompute=False,
+                    nthreads=0, seq_ids=None):
+    """AR sampling until the end time t_end (Alg. 1's stop rule) or
+    max_events; count[b] events with t <= t_end fill the first slots."""
+    hist_tau = _c(hist_tau, np.float32)
+    hist_marks = _c(hist_marks, np.int32)
+    B, H = hist_tau.shape
+    N = max_events
+    tau = np.zeros((B, N)); t = np.zeros((B, N))
+    k = np.zeros((B, N), np.int32); mg = np.zeros((B, N)); cnt = np.zeros(B, np.int32)
+    _check(lib().oracle_sample_ar_until(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size, B, H,
+                                        hist_tau, hist_marks, N, float(t_end), seed, int(recompute),
+                                        _ids(seq_ids, B), tau, t, k, mg, cnt, nthreads),
+           "oracle_sample_ar_until")
+    return dict(tau=tau, t=t, k=k, margin=mg, count=cnt)
+
+
+def sample_sd_until(cfg_t, blob_t, cfg_d, blob_d, hist_tau, hist_marks, max_events, t_end, gamma,
+                    seed, flags=0, recompute=False, nthreads=0, seq_ids=None):
+    """TPP-SD until the end time t_end (Alg. 1's stop rule) or max_events."""
+    hist_tau = _c(hist_tau, np.float32)
+    hist_marks = _c(hist_marks, np.int32)
+    B, H = hist_tau.shape
+    N = max_events
+    tau = np.zeros((B, N)); t = np.zeros((B, N))
+    k = np.zeros((B, N), np.int32); mg = np.zeros((B, N)); cnt = np.zeros(B, np.int32)
+    st = np.zeros((B, 5), np.int64)
+    _check(lib().oracle_sample_sd_until(_cfg(cfg_t), _c(blob_t, np.float32), blob_t.size,
+                                        _cfg(cfg_d), _c(blob_d, np.float32), blob_d.size, B, H,
+                                        hist_tau, hist_marks, N, float(t_end), gamma, seed, flags,
+                                        int(recompute), _ids(seq_ids, B), tau, t, k, mg, cnt, st,
+                                        nthreads), "oracle_sample_sd_until")
+    return dict(tau=tau, t=t, k=k, margin=mg, count=cnt, stats=st)
+
+
+def score_survival(cfg, blob, tau, marks, t_end, recompute=False, nthreads=0):
+    """log S(t_end - t_last) per sequence (survival term of Eq. 2)."""
+    tau = _c(tau, np.float32)
+    marks = _c(marks, np.int32)
+    B, n = tau.shape
+    out = np.zeros(B)
+    _check(lib().oracle_score_survival(_cfg(cfg), _c(blob, np.float32), blob.size, B, n, tau, marks,
+                                       float(t_end), out, int(recompute), nthreads),
+           "oracle_score_survival")
+    return out
+
+
+def log_survival(M, head, u):
+    """log(1 - G(u)) of one head's log-normal mixture."""
+    return lib().oracle_log_survival(M, _c(head, np.float64), float(u))
 
 
 def log_g(M, head, tau):

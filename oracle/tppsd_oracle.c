@@ -199,6 +199,28 @@ double oracle_log_g(int32_t M, const double *hd, double tau)
 
 double oracle_log_f(int32_t M, const double *hd, int32_t k) { return hd[3 * M + k]; }
 
+/* log(1 - Phi(z)) = log(erfc(z / sqrt 2) / 2); for z beyond the range where
+ * erfc underflows, the leading term of its asymptotic expansion,
+ * erfc(x) ~ exp(-x^2) / (x sqrt(pi)). */
+static double log_normal_tail(double z)
+{
+    double x = z / sqrt(2.0);
+    if (x < 25.0) return log(0.5 * erfc(x));
+    return -x * x - log(x * 1.7724538509055160273) - log(2.0);  /* sqrt(pi) */
+}
+
+/* log S(u) = log(1 - G(u)), G the log-normal mixture CDF of Sec. 4.2:
+ * 1 - G(u) = sum_m w_m (1 - Phi((log u - mu_m) / sigma_m)).  This is the
+ * survival term of the log-likelihood on [0, T] (Sec. 3.1, Eq. 2): no event
+ * in the u = T - t_last after the last one.  u <= 0 gives 0 (log 1). */
+double oracle_log_survival(int32_t M, const double *hd, double u)
+{
+    if (!(u > 0.0)) return 0.0;
+    double lu = log(u), c[MAXM];
+    for (int m = 0; m < M; ++m) c[m] = hd[m] + log_normal_tail((lu - hd[M + m]) / exp(hd[2 * M + m]));
+    return logsumexp(c, M);
+}
+
 /* Categorical choice: smallest index whose running sum of p reaches u * sum(p).
  * *margin gets the distance of u * sum to the nearest boundary, / sum. */
 static int categorical(const double *p, int n, double u, double *margin)
@@ -421,18 +443,33 @@ static const model_ops TOY_OPS = {toy_len, toy_step, toy_truncate};
 typedef struct { double *tau, *t; int *k; double *mg; } evbuf;
 
 /* Naive autoregressive sampling, Sec. 4.2: sample, append, repeat. */
-static void ar_sequence(const model_ops *T, void *ts, evbuf *ev, int H, int N,
-                        uint64_t seed, uint32_t seq)
+/* Stop rule (Alg. 1): a sequence ends once its last event lies beyond the
+ * end time t_end, or after N generated events; the result is the events
+ * with t <= t_end (a prefix, since times increase).  t_end = +inf gives the
+ * fixed-count form.  Returns the number of generated events kept. */
+static int kept_events(const evbuf *ev, int H, int n, int N, double t_end)
+{
+    int c = n - H < N ? n - H : N;
+    while (c > 0 && ev->t[H + c - 1] > t_end) --c;
+    return c;
+}
+
+/* Naive autoregressive sampling, Sec. 4.2: sample, append, repeat. */
+static int ar_sequence(const model_ops *T, void *ts, evbuf *ev, int H, int N, double t_end,
+                       uint64_t seed, uint32_t seq)
 {
     head_t hd;
     for (int p = 0; p < H - 1; ++p) T->step(ts, ev->t[p], ev->k[p], &hd);
-    for (int p = H; p < H + N; ++p) {
+    int n = H;
+    for (int p = H; p < H + N && ev->t[p - 1] <= t_end; ++p) {
         T->step(ts, ev->t[p - 1], ev->k[p - 1], &hd);   /* head after event p-1 */
         double tau;
         int k;
         draw_event(&hd, seed, seq, (uint32_t)p, &tau, &k, &ev->mg[p]);
         ev->tau[p] = tau; ev->t[p] = ev->t[p - 1] + tau; ev->k[p] = k;
+        n = p + 1;
     }
+    return kept_events(ev, H, n, N, t_end);
 }
 
 /* TPP-SD, Sec. 4.3 and Alg. 1, with these readings:
@@ -446,19 +483,20 @@ static void ar_sequence(const model_ops *T, void *ts, evbuf *ev, int H, int N,
  *  - after a fully accepted draft one bonus event is drawn from the target
  *    head that follows the last draft (the LLM rule of Sec. 2.3), unless
  *    FLAG_NO_BONUS.
- *  - stop after N generated events (truncation, as Alg. 1 truncates at T).
+ *  - stop once the last emitted event lies beyond t_end (Alg. 1's end
+ *    time) or after N generated events; keep the events with t <= t_end.
  * Cache invariant at round start: T has encoded all events but the last;
- * D has encoded all but the last one or two. */
-static void sd_sequence(const model_ops *T, void *ts, const model_ops *D, void *ds,
-                        evbuf *ev, int H, int N, int gamma, uint64_t seed, uint32_t seq,
-                        uint32_t flags, int64_t *st)
+ * D has encoded all but the last one or two.  Returns the kept count. */
+static int sd_sequence(const model_ops *T, void *ts, const model_ops *D, void *ds,
+                       evbuf *ev, int H, int N, double t_end, int gamma, uint64_t seed, uint32_t seq,
+                       uint32_t flags, int64_t *st)
 {
     head_t hd, dhead[64 + 1], thead[64 + 1];
     double tau_hat[64 + 1];
     int k_hat[64 + 1];
     for (int p = 0; p < H - 1; ++p) { T->step(ts, ev->t[p], ev->k[p], &hd); D->step(ds, ev->t[p], ev->k[p], &hd); }
     int n = H;                                      /* events so far */
-    while (n < H + N) {
+    while (n < H + N && ev->t[n - 1] <= t_end) {
         /* Drafting: gamma events from M_D, recording their heads. */
         for (int p = D->len(ds); p <= n - 1; ++p) D->step(ds, ev->t[p], ev->k[p], &hd);
         for (int l = 1; l <= gamma; ++l) {
@@ -521,6 +559,7 @@ static void sd_sequence(const model_ops *T, void *ts, const model_ops *D, void *
         if (D->len(ds) > keepD) D->truncate(ds, keepD);
         n = n_new;
     }
+    return kept_events(ev, H, n, N, t_end);
 }
 
 /* ------------------------------------------------------------------ */
@@ -556,22 +595,24 @@ static void evbuf_alloc(evbuf *ev, int cap)
 
 static void evbuf_free(evbuf *ev) { free(ev->tau); free(ev->t); free(ev->k); free(ev->mg); }
 
-static void store_out(const evbuf *ev, int H, int N, int64_t b, double *o_tau, double *o_t,
+/* The first c generated events of sequence b; slots c..N-1 get NaN / -1. */
+static void store_out(const evbuf *ev, int H, int N, int c, int64_t b, double *o_tau, double *o_t,
                       int32_t *o_k, double *o_mg)
 {
     for (int i = 0; i < N; ++i) {
-        if (o_tau) o_tau[b * N + i] = ev->tau[H + i];
-        if (o_t) o_t[b * N + i] = ev->t[H + i];
-        if (o_k) o_k[b * N + i] = ev->k[H + i];
-        if (o_mg) o_mg[b * N + i] = ev->mg[H + i];
+        const int in = i < c;
+        if (o_tau) o_tau[b * N + i] = in ? ev->tau[H + i] : NAN;
+        if (o_t) o_t[b * N + i] = in ? ev->t[H + i] : NAN;
+        if (o_k) o_k[b * N + i] = in ? ev->k[H + i] : -1;
+        if (o_mg) o_mg[b * N + i] = in ? ev->mg[H + i] : NAN;
     }
 }
 
-int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                     int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
-                     int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
-                     double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
-                     int32_t nthreads)
+int oracle_sample_ar_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                           int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                           int32_t N, double t_end, uint64_t seed, int32_t recompute,
+                           const int32_t *seq_ids, double *out_tau, double *out_t, int32_t *out_k,
+                           double *out_margin, int32_t *out_count, int32_t nthreads)
 {
     model_t mT;
     if (model_init(&mT, cfgT, blobT, nT)) return -1;
@@ -584,21 +625,23 @@ int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
         evbuf_alloc(&ev, cap);
         tstate_init(&ts, &mT, cap, recompute);
         load_history(&ev, hist_tau + (int64_t)b * H, hist_marks + (int64_t)b * H, H);
-        ar_sequence(&TRANSFORMER_OPS, &ts, &ev, H, N, seed, (uint32_t)(seq_ids ? seq_ids[b] : b));
-        store_out(&ev, H, N, b, out_tau, out_t, out_k, out_margin);
+        const int c = ar_sequence(&TRANSFORMER_OPS, &ts, &ev, H, N, t_end, seed,
+                                  (uint32_t)(seq_ids ? seq_ids[b] : b));
+        store_out(&ev, H, N, c, b, out_tau, out_t, out_k, out_margin);
+        if (out_count) out_count[b] = c;
         tstate_free(&ts);
         evbuf_free(&ev);
     }
     return 0;
 }
 
-int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                     const int32_t cfgD[7], const float *blobD, int64_t nD,
-                     int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
-                     int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
-                     const int32_t *seq_ids,
-                     double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
-                     int64_t *stats, int32_t nthreads)
+int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                           const int32_t cfgD[7], const float *blobD, int64_t nD,
+                           int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                           int32_t N, double t_end, int32_t gamma, uint64_t seed, uint32_t flags,
+                           int32_t recompute, const int32_t *seq_ids,
+                           double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
+                           int32_t *out_count, int64_t *stats, int32_t nthreads)
 {
     model_t mT, mD;
     if (model_init(&mT, cfgT, blobT, nT) || model_init(&mD, cfgD, blobD, nD)) return -1;
@@ -613,12 +656,62 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
         tstate_init(&ts, &mT, cap, recompute);
         tstate_init(&ds, &mD, cap, recompute);
         load_history(&ev, hist_tau + (int64_t)b * H, hist_marks + (int64_t)b * H, H);
-        sd_sequence(&TRANSFORMER_OPS, &ts, &TRANSFORMER_OPS, &ds, &ev, H, N, gamma, seed,
-                    (uint32_t)(seq_ids ? seq_ids[b] : b), flags, st);
-        store_out(&ev, H, N, b, out_tau, out_t, out_k, out_margin);
+        const int c = sd_sequence(&TRANSFORMER_OPS, &ts, &TRANSFORMER_OPS, &ds, &ev, H, N, t_end, gamma,
+                                  seed, (uint32_t)(seq_ids ? seq_ids[b] : b), flags, st);
+        store_out(&ev, H, N, c, b, out_tau, out_t, out_k, out_margin);
+        if (out_count) out_count[b] = c;
         if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
         tstate_free(&ts);
         tstate_free(&ds);
+        evbuf_free(&ev);
+    }
+    return 0;
+}
+
+int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                     int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                     int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
+                     double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
+                     int32_t nthreads)
+{
+    return oracle_sample_ar_until(cfgT, blobT, nT, B, H, hist_tau, hist_marks, N, INFINITY, seed,
+                                  recompute, seq_ids, out_tau, out_t, out_k, out_margin, NULL, nthreads);
+}
+
+int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                     const int32_t cfgD[7], const float *blobD, int64_t nD,
+                     int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                     int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
+                     const int32_t *seq_ids,
+                     double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
+                     int64_t *stats, int32_t nthreads)
+{
+    return oracle_sample_sd_until(cfgT, blobT, nT, cfgD, blobD, nD, B, H, hist_tau, hist_marks, N,
+                                  INFINITY, gamma, seed, flags, recompute, seq_ids, out_tau, out_t,
+                                  out_k, out_margin, NULL, stats, nthreads);
+}
+
+/* Survival term of the log-likelihood on [0, t_end] (Sec. 3.1, Eq. 2) of
+ * each sequence's len events: log S(t_end - t_{len-1} | h_{len-1}) from the
+ * head after the last event. */
+int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+                          int32_t B, int32_t len, const float *tau, const int32_t *marks,
+                          double t_end, double *out_logS, int32_t recompute, int32_t nthreads)
+{
+    model_t m;
+    if (model_init(&m, cfg, blob, blob_floats)) return -1;
+    if (B < 0 || len < 1) return -1;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads_or_default(nthreads))
+    for (int b = 0; b < B; ++b) {
+        tstate ts;
+        head_t hd;
+        evbuf ev;
+        evbuf_alloc(&ev, len);
+        tstate_init(&ts, &m, len, recompute);
+        load_history(&ev, tau + (int64_t)b * len, marks + (int64_t)b * len, len);
+        for (int i = 0; i < len; ++i) t_step(&ts, ev.t[i], ev.k[i], &hd);
+        out_logS[b] = oracle_log_survival(m.M, hd.v, t_end - ev.t[len - 1]);
+        tstate_free(&ts);
         evbuf_free(&ev);
     }
     return 0;
@@ -703,8 +796,8 @@ int oracle_toy_sd(int32_t M, int32_t K, const double *tableT, const double *tabl
         int64_t st[5] = {0, 0, 0, 0, 0};
         evbuf_alloc(&ev, cap);
         ev.tau[0] = 1.0; ev.t[0] = 1.0; ev.k[0] = 0;
-        sd_sequence(&TOY_OPS, &ts, &TOY_OPS, &ds, &ev, 1, N, gamma, seed, (uint32_t)b, flags, st);
-        store_out(&ev, 1, N, b, out_tau, NULL, out_k, NULL);
+        sd_sequence(&TOY_OPS, &ts, &TOY_OPS, &ds, &ev, 1, N, INFINITY, gamma, seed, (uint32_t)b, flags, st);
+        store_out(&ev, 1, N, N, b, out_tau, NULL, out_k, NULL);
         if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
         evbuf_free(&ev);
     }
@@ -720,8 +813,8 @@ int oracle_toy_ar(int32_t M, int32_t K, const double *tableT, int32_t B, int32_t
         evbuf ev;
         evbuf_alloc(&ev, 1 + N + 1);
         ev.tau[0] = 1.0; ev.t[0] = 1.0; ev.k[0] = 0;
-        ar_sequence(&TOY_OPS, &ts, &ev, 1, N, seed, (uint32_t)b);
-        store_out(&ev, 1, N, b, out_tau, NULL, out_k, NULL);
+        ar_sequence(&TOY_OPS, &ts, &ev, 1, N, INFINITY, seed, (uint32_t)b);
+        store_out(&ev, 1, N, N, b, out_tau, NULL, out_k, NULL);
         evbuf_free(&ev);
     }
     return 0;

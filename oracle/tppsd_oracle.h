@@ -60,6 +60,31 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                      int64_t *stats, int32_t nthreads);
 
+/* End-time forms (Alg. 1's stop rule): a sequence ends once its last event
+ * lies beyond t_end or after N generated events; out_count[b] (may be NULL)
+ * gets the number of generated events with t <= t_end, which fill the first
+ * out_count[b] slots of the [B][N] outputs (later slots: NaN / -1).  The
+ * forms above are these with t_end = +inf. */
+int oracle_sample_ar_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                           int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                           int32_t N, double t_end, uint64_t seed, int32_t recompute,
+                           const int32_t *seq_ids, double *out_tau, double *out_t, int32_t *out_k,
+                           double *out_margin, int32_t *out_count, int32_t nthreads);
+int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                           const int32_t cfgD[7], const float *blobD, int64_t nD,
+                           int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
+                           int32_t N, double t_end, int32_t gamma, uint64_t seed, uint32_t flags,
+                           int32_t recompute, const int32_t *seq_ids,
+                           double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
+                           int32_t *out_count, int64_t *stats, int32_t nthreads);
+/* Survival term log S(t_end - t_{len-1}) of each sequence's len events, from
+ * the head after the last event (Sec. 3.1, Eq. 2). */
+int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+                          int32_t B, int32_t len, const float *tau, const int32_t *marks,
+                          double t_end, double *out_logS, int32_t recompute, int32_t nthreads);
+/* log(1 - G(u)) for the log-normal mixture of one head; 0 for u <= 0. */
+double oracle_log_survival(int32_t M, const double *hd, double u);
+
 /* Pieces on fixed heads (same row layout as oracle_score; M, K given). */
 double oracle_log_g(int32_t M, const double *head, double tau);
 double oracle_log_f(int32_t M, const double *head, int32_t k);
