@@ -131,6 +131,28 @@ tppsd_status_t tppsd_sample_autoregressive(tppsd_ctx* ctx, int32_t batch, int32_
                                            uint64_t seed, uint32_t flags, float* out_tau,
                                            double* out_t, int32_t* out_marks, void* stream);
 
+/* TPP-SD with the end-time stop rule of Alg. 1: each of the first `batch`
+ * sequences is extended until its last event lies beyond t_end (absolute
+ * time, same clock as the history) or max_events events are drawn, in
+ * rounds of gamma drafts.  Random slots as tppsd_sample, so the events kept
+ * are the prefix with t <= t_end of the tppsd_sample run with the same seed
+ * and n_events = max_events.  Outputs [batch][max_events]: the first
+ * out_count[b] slots hold the kept events; the rest are NaN (out_tau,
+ * out_t) and -1 (out_marks).  out_count [batch] (host or device) is
+ * required; a history already ending beyond t_end gives count 0.  t_end =
+ * +inf is tppsd_sample; NaN is TPPSD_ERR_INVALID_ARG. */
+tppsd_status_t tppsd_sample_until(tppsd_ctx* ctx, int32_t batch, double t_end, int32_t max_events,
+                                  int32_t gamma, uint64_t seed, uint32_t flags, float* out_tau,
+                                  double* out_t, int32_t* out_marks, int32_t* out_count,
+                                  void* stream);
+
+/* Target-only autoregressive sampling (Sec. 4.2) with the same stop rule,
+ * slots and outputs as tppsd_sample_until. */
+tppsd_status_t tppsd_sample_autoregressive_until(tppsd_ctx* ctx, int32_t batch, double t_end,
+                                                 int32_t max_events, uint64_t seed, uint32_t flags,
+                                                 float* out_tau, double* out_t, int32_t* out_marks,
+                                                 int32_t* out_count, void* stream);
+
 /* Teacher-forced scoring with one model (which 0 = target, 1 = draft): for
  * sequences tau/marks [batch][len], out_heads [batch][len][3M+K] (may be
  * NULL) gets the head after events 0..i at row i (row len-1 untouched):
@@ -141,6 +163,19 @@ tppsd_status_t tppsd_sample_autoregressive(tppsd_ctx* ctx, int32_t batch, int32_
 tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
                            const float* tau, const int32_t* marks, float* out_heads,
                            float* out_logg, float* out_logf, void* stream);
+
+/* Log-likelihood on the observation window [0, t_end] (Eq. 2): the outputs
+ * of tppsd_score, and in out_logS [batch] (fp64, host or device, required)
+ * the survival term log(1 - G(t_end - t_last)) of each sequence, G the
+ * inter-event CDF of the head after its last event (the log-normal mixture
+ * of Sec. 4.2; computed in fp64 from the fp32 head), 0 when t_end <= t_last.
+ * One pass over all len positions, so out_heads (may be NULL) also gets row
+ * len-1.  len >= 1; at len = 1 out_logg / out_logf are NaN.  Overwrites the
+ * caches like tppsd_score. */
+tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
+                                 const float* tau, const int32_t* marks, double t_end,
+                                 float* out_heads, float* out_logg, float* out_logf,
+                                 double* out_logS, void* stream);
 
 /* Scoring that allocates nothing (the paper has no counterpart; this is a
  * library convenience).  Same outputs as tppsd_score's out_logg and

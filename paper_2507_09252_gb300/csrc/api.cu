@@ -669,9 +669,11 @@ static tppsd_status_t ensure_stage(tppsd_ctx* ctx, size_t bytes) {
 
 static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int gamma, uint64_t seed,
                                   uint32_t flags, float* out_tau, double* out_t, int32_t* out_k,
-                                  void* stream) {
+                                  void* stream, double t_end = INFINITY, int32_t* out_count = nullptr,
+                                  bool until = false) {
     if (!ctx) return TPPSD_ERR_INVALID_ARG;
     if (N > 0 && (!out_tau || !out_t || !out_k)) return TPPSD_ERR_INVALID_ARG;
+    if (until && (!out_count || t_end != t_end)) return TPPSD_ERR_INVALID_ARG;
     if (!ctx->prefilled || B < 1 || B > ctx->prefill_batch || N < 0) return TPPSD_ERR_INVALID_ARG;
     if (mode == 0 && (gamma < 1 || gamma > ctx->max_gamma)) return TPPSD_ERR_INVALID_ARG;
     const int H = ctx->hist_len;
@@ -685,8 +687,9 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     const size_t nb = (size_t)B * (N > 0 ? N : 1);
     const bool host_out[3] = {N > 0 && !is_device_ptr(out_tau), N > 0 && !is_device_ptr(out_t),
                               N > 0 && !is_device_ptr(out_k)};
-    const bool any_host = host_out[0] || host_out[1] || host_out[2];
-    if (any_host) TRY(ensure_stage(ctx, nb * (4 + 8 + 4) + 64));
+    const bool host_count = until && !is_device_ptr(out_count);
+    const bool any_host = host_out[0] || host_out[1] || host_out[2] || host_count;
+    if (any_host) TRY(ensure_stage(ctx, nb * (4 + 8 + 4) + (size_t)B * 4 + 64));
     char* sb = (char*)ctx->stage;
     CallParams p{};
     p.B = B; p.H = H; p.N = N; p.gamma = mode == 0 ? gamma : 0; p.n_max = ctx->n_max;
@@ -695,6 +698,15 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     p.out_tau = host_out[0] ? (float*)(sb + nb * 8) : out_tau;
     p.out_k = host_out[2] ? (int*)(sb + nb * 12) : out_k;
     p.max_loops = N + 2;
+    p.t_end = t_end;
+    p.out_count = until ? (host_count ? (int*)(sb + nb * 16) : out_count) : nullptr;
+    // stop rule: the slots after each sequence's kept events read NaN / -1
+    // (all-ones bytes are a NaN in fp32 and fp64 and -1 in int32)
+    if (until && N > 0) {
+        CK(cudaMemsetAsync(p.out_t, 0xFF, (size_t)B * N * 8, st));
+        CK(cudaMemsetAsync(p.out_tau, 0xFF, (size_t)B * N * 4, st));
+        CK(cudaMemsetAsync(p.out_k, 0xFF, (size_t)B * N * 4, st));
+    }
     const bool profile = (flags & TPPSD_FLAG_PROFILE) != 0;
     Prof prof{&Profiler::mark, &ctx->prof};
     const Prof* pp = profile ? &prof : nullptr;
@@ -724,6 +736,7 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     if (host_out[1]) CK(cudaMemcpyAsync(out_t, p.out_t, (size_t)B * N * 8, cudaMemcpyDeviceToHost, st));
     if (host_out[0]) CK(cudaMemcpyAsync(out_tau, p.out_tau, (size_t)B * N * 4, cudaMemcpyDeviceToHost, st));
     if (host_out[2]) CK(cudaMemcpyAsync(out_k, p.out_k, (size_t)B * N * 4, cudaMemcpyDeviceToHost, st));
+    if (host_count) CK(cudaMemcpyAsync(out_count, p.out_count, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
     CK(cudaEventRecord(ctx->done_event, st));
     ctx->last_stream = st;
     ctx->last_launches = launches;
@@ -746,11 +759,33 @@ extern "C" tppsd_status_t tppsd_sample_autoregressive(tppsd_ctx* ctx, int32_t ba
     return run_sampler(ctx, 1, batch, n_events, 0, seed, flags, out_tau, out_t, out_marks, stream);
 }
 
-extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
-                                      const float* tau, const int32_t* marks, float* out_heads,
-                                      float* out_logg, float* out_logf, void* stream) {
+extern "C" tppsd_status_t tppsd_sample_until(tppsd_ctx* ctx, int32_t batch, double t_end,
+                                             int32_t max_events, int32_t gamma, uint64_t seed,
+                                             uint32_t flags, float* out_tau, double* out_t,
+                                             int32_t* out_marks, int32_t* out_count, void* stream) {
+    return run_sampler(ctx, 0, batch, max_events, gamma, seed, flags, out_tau, out_t, out_marks,
+                       stream, t_end, out_count, true);
+}
+
+extern "C" tppsd_status_t tppsd_sample_autoregressive_until(tppsd_ctx* ctx, int32_t batch,
+                                                            double t_end, int32_t max_events,
+                                                            uint64_t seed, uint32_t flags,
+                                                            float* out_tau, double* out_t,
+                                                            int32_t* out_marks, int32_t* out_count,
+                                                            void* stream) {
+    return run_sampler(ctx, 1, batch, max_events, 0, seed, flags, out_tau, out_t, out_marks, stream,
+                       t_end, out_count, true);
+}
+
+// Teacher-forced scoring; with logS set the pass also covers the last event
+// (q = len positions) and writes the survival term at t_end.
+static tppsd_status_t run_score(tppsd_ctx* ctx, int which, int batch, int len, const float* tau,
+                                const int32_t* marks, float* out_heads, float* out_logg,
+                                float* out_logf, double t_end, double* out_logS, void* stream) {
     if (!ctx || !tau || !marks || (which != 0 && which != 1)) return TPPSD_ERR_INVALID_ARG;
-    if (batch < 1 || batch > ctx->max_batch || len < 2 || len > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    const int min_len = out_logS ? 1 : 2;
+    if (batch < 1 || batch > ctx->max_batch || len < min_len || len > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    if (out_logS && t_end != t_end) return TPPSD_ERR_INVALID_ARG;
     CK(cudaSetDevice(ctx->device));
     cudaStream_t st = (cudaStream_t)stream;
     HostModel& hm = which == 0 ? ctx->T : ctx->D;
@@ -767,23 +802,46 @@ extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t bat
     const bool hh = out_heads && !is_device_ptr(out_heads);
     const bool hg = out_logg && !is_device_ptr(out_logg);
     const bool hf = out_logf && !is_device_ptr(out_logf);
-    if (hh || hg || hf) TRY(ensure_stage(ctx, (nh + 2 * nl) * sizeof(float) + 64));
+    const bool hs = out_logS && !is_device_ptr(out_logS);
+    if (hh || hg || hf || hs) TRY(ensure_stage(ctx, (nh + 2 * nl) * sizeof(float) + (size_t)batch * 8 + 64));
     float* sb = (float*)ctx->stage;
     float* d_heads = hh ? sb : out_heads;
     float* d_logg = hg ? sb + nh : out_logg;
     float* d_logf = hf ? sb + nh + nl : out_logf;
+    double* d_logS = hs ? (double*)(((uintptr_t)(sb + nh + 2 * nl) + 7) & ~(uintptr_t)7) : out_logS;
+    const int q = out_logS ? len : len - 1;
     auto after = [&](int g0, int rows) -> tppsd_status_t {
-        CK(launch_score_logs(hm.dm, ss, ctx->work, batch, len, g0, rows, d_heads, d_logg, d_logf, st));
+        CK(launch_score_logs(hm.dm, ss, ctx->work, batch, len, q, g0, rows, d_heads, d_logg, d_logf, st));
+        if (out_logS) CK(launch_score_survival(hm.dm, ss, ctx->work, batch, len, g0, rows, t_end, d_logS, st));
         return TPPSD_OK;
     };
     int launches = 0;
-    TRY(span_forward(ctx, hm, kv, batch, len - 1, true, st, after, &launches));
+    if (len == 1 && out_logg) CK(cudaMemsetAsync(d_logg, 0xFF, nl * 4, st));  // NaN at i = 0
+    if (len == 1 && out_logf) CK(cudaMemsetAsync(d_logf, 0xFF, nl * 4, st));
+    TRY(span_forward(ctx, hm, kv, batch, q, true, st, after, &launches));
     if (hh) CK(cudaMemcpyAsync(out_heads, d_heads, nh * 4, cudaMemcpyDeviceToHost, st));
     if (hg) CK(cudaMemcpyAsync(out_logg, d_logg, nl * 4, cudaMemcpyDeviceToHost, st));
     if (hf) CK(cudaMemcpyAsync(out_logf, d_logf, nl * 4, cudaMemcpyDeviceToHost, st));
+    if (hs) CK(cudaMemcpyAsync(out_logS, d_logS, (size_t)batch * 8, cudaMemcpyDeviceToHost, st));
     CK(cudaEventRecord(ctx->done_event, st));
     ctx->last_stream = st;
     return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
+                                      const float* tau, const int32_t* marks, float* out_heads,
+                                      float* out_logg, float* out_logf, void* stream) {
+    return run_score(ctx, which, batch, len, tau, marks, out_heads, out_logg, out_logf, 0.0, nullptr,
+                     stream);
+}
+
+extern "C" tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32_t batch,
+                                            int32_t len, const float* tau, const int32_t* marks,
+                                            double t_end, float* out_heads, float* out_logg,
+                                            float* out_logf, double* out_logS, void* stream) {
+    if (!out_logS) return TPPSD_ERR_INVALID_ARG;
+    return run_score(ctx, which, batch, len, tau, marks, out_heads, out_logg, out_logf, t_end,
+                     out_logS, stream);
 }
 
 extern "C" tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms) {
@@ -1019,7 +1077,7 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     for (long long g0 = 0; g0 < total; g0 += chunk) {
         RowSpec rs{ROWS_SPAN, (int)q, (int)(total - g0 < chunk ? total - g0 : chunk), (int)g0};
         CK(launch_forward(hm.dm, kv, ss, w, rs, true, st, nullptr, nullptr));
-        CK(launch_score_logs(hm.dm, ss, w, batch, len, (int)g0, rs.count, nullptr, out_logg,
+        CK(launch_score_logs(hm.dm, ss, w, batch, len, len - 1, (int)g0, rs.count, nullptr, out_logg,
                              out_logf, st));
     }
     CK(cudaEventRecord(ctx->done_event, st));

@@ -97,6 +97,11 @@ struct CallParams {
     double* out_t;
     int* out_k;
     int max_loops;
+    // End-time stop rule (Alg. 1): with out_count set, a sequence stops once
+    // its last event lies beyond t_end (or after N events); only events with
+    // t <= t_end are written and out_count[s] receives their number.
+    double t_end;
+    int* out_count;
 };
 
 // Device counters of the current call (mirrors tppsd_stats + status).
@@ -258,8 +263,10 @@ cudaError_t launch_ar_sample(const DevModel& mT, const SeqState& ss, const CallP
 cudaError_t launch_round_control(const SeqState& ss, const CallParams* dp, int B,
                                  DevStats* stats, unsigned long long cond_handle, int use_cond,
                                  int* active_out, cudaStream_t st);
+cudaError_t launch_score_survival(const DevModel& m, const SeqState& ss, const Work& w, int B, int len,
+                                  int g0, int rows, double t_end, double* out_logS, cudaStream_t st);
 cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work& w, int B,
-                              int len, int s0, int rows, float* out_heads, float* out_logg,
+                              int len, int q, int s0, int rows, float* out_heads, float* out_logg,
                               float* out_logf, cudaStream_t st);
 size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
 // One-CTA-per-sequence draft (draft.cu) for the shapes it is compiled for.

@@ -683,11 +683,27 @@ struct EpiArgs {
     DevStats* st;
 };
 
+// End-time stop rule (Alg. 1): a sequence with nn events is finished once
+// N events are drawn or its last event lies beyond t_end.  Times increase
+// along a sequence, so the events with t <= t_end are a prefix.
+__device__ __forceinline__ bool seq_finished(const SeqState& ss, const CallParams& P, int s, int nn) {
+    return nn >= P.H + P.N || (P.out_count && ss.t[(size_t)s * ss.n_max + nn - 1] > P.t_end);
+}
+
+// Number of generated events kept (t <= t_end, at most N) of a finished
+// sequence; only the events of its last round can lie beyond t_end.
+__device__ __forceinline__ int kept_count(const SeqState& ss, const CallParams& P, int s, int nn) {
+    int c = min(nn - P.H, P.N);
+    const double* t = ss.t + (size_t)s * ss.n_max + P.H;
+    while (c > 0 && t[c - 1] > P.t_end) --c;
+    return c;
+}
+
 __device__ void write_outputs(const SeqState& ss, const CallParams& P, int s, int n, int emitted) {
     const int lane = threadIdx.x & 31;
     for (int i = lane; i < emitted; i += 32) {
         const int p = n + i, j = p - P.H;
-        if (j < P.N) {
+        if (j < P.N && (!P.out_count || ss.t[(size_t)s * ss.n_max + p] <= P.t_end)) {
             const size_t o = (size_t)s * ss.n_max + p, oo = (size_t)s * P.N + j;
             P.out_tau[oo] = ss.tau[o];
             P.out_t[oo] = ss.t[o];
@@ -893,7 +909,9 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         const int nn = n + emitted;
         ss.n_emit[s] = nn;
         ss.n_draft[s] = n + min(g - 1, A);
-        ss.done[s] = nn >= P.H + P.N;
+        const bool fin = seq_finished(ss, P, s, nn);
+        ss.done[s] = fin;
+        if (fin && P.out_count) P.out_count[s] = kept_count(ss, P, s, nn);
         atomicAdd(&a.st->rounds, 1ull);
         atomicAdd(&a.st->target_keys, (unsigned long long)(n + g));  // positions 0..n+g-1
         atomicAdd(&a.st->drafted, (unsigned long long)g);
@@ -922,14 +940,16 @@ __global__ void k_ar_sample(SeqState ss, const CallParams* Pp, const float* head
     ss.t[o] = ss.t[o - 1] + (double)tau;
     ss.k[o] = k;
     const int j = n - P.H;
-    if (j < P.N) {
+    if (j < P.N && (!P.out_count || ss.t[o] <= P.t_end)) {
         const size_t oo = (size_t)s * P.N + j;
         P.out_tau[oo] = tau;
         P.out_t[oo] = ss.t[o];
         P.out_k[oo] = k;
     }
     ss.n_emit[s] = n + 1;
-    ss.done[s] = n + 1 >= P.H + P.N;
+    const bool fin = seq_finished(ss, P, s, n + 1);
+    ss.done[s] = fin;
+    if (fin && P.out_count) P.out_count[s] = kept_count(ss, P, s, n + 1);
     atomicAdd(&st->rounds, 1ull);
     atomicAdd(&st->emitted, 1ull);
     atomicAdd(&st->target_keys, (unsigned long long)n);  // positions 0..n-1
@@ -951,7 +971,9 @@ __global__ void k_begin(CallParams p, CallParams* dp, SeqState ss, DevStats* st)
     if (s < p.B) {
         ss.n_emit[s] = p.H;
         ss.n_draft[s] = p.H - 1;
-        ss.done[s] = p.N <= 0;
+        // a history that already ends beyond t_end generates nothing
+        ss.done[s] = p.N <= 0 || (p.out_count && ss.t[(size_t)s * ss.n_max + p.H - 1] > p.t_end);
+        if (p.out_count) p.out_count[s] = 0;
     }
 }
 
@@ -992,18 +1014,21 @@ __global__ void k_history_times(SeqState ss, int B, int H) {
     }
 }
 
-// Teacher-forced outputs of a span pass: row r <-> (s, l), head predicts
-// event l+1 (Eq. 2 terms log g(tau_{l+1}), log f(k_{l+1})).
-__global__ void k_score_logs(SeqState ss, Work w, int M, int K, int len, int g0, int rows,
+// Teacher-forced outputs of a span pass over q positions per sequence (q =
+// len-1, or len when the head after the last event is wanted too): row r
+// <-> (s, l), head predicts event l+1 (Eq. 2 terms log g(tau_{l+1}),
+// log f(k_{l+1})).
+__global__ void k_score_logs(SeqState ss, Work w, int M, int K, int len, int q, int g0, int rows,
                              float* out_heads, float* out_logg, float* out_logf) {
     const int r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= rows) return;
     const int W = 3 * M + K;
     const long long g = g0 + (long long)r;
-    const int s = (int)(g / (len - 1)), l = (int)(g % (len - 1));
+    const int s = (int)(g / q), l = (int)(g % q);
     const float* hd = w.heads + (size_t)r * W;
     if (out_heads)
         for (int i = 0; i < W; ++i) out_heads[((size_t)s * len + l) * W + i] = hd[i];
+    if (l + 1 >= len) return;
     const size_t o = (size_t)s * ss.n_max + l + 1;
     if (out_logg) out_logg[(size_t)s * len + l + 1] = head_log_g(hd, M, ss.tau[o]);
     if (out_logf) out_logf[(size_t)s * len + l + 1] = hd[3 * M + ss.k[o]];
@@ -1011,6 +1036,45 @@ __global__ void k_score_logs(SeqState ss, Work w, int M, int K, int len, int g0,
         if (out_logg) out_logg[(size_t)s * len] = NAN;
         if (out_logf) out_logf[(size_t)s * len] = NAN;
     }
+}
+
+// log of the upper tail of the standard normal, 1 - Phi(z): for z > 0 from
+// the scaled complementary error function, erfc(x) = erfcx(x) exp(-x^2),
+// which stays finite far into the tail; for z <= 0 erfc itself (in [1, 2]).
+__device__ __forceinline__ double log_normal_upper(double z) {
+    const double x = z * 0.70710678118654752440;  // z / sqrt(2)
+    return z > 0.0 ? log(0.5 * erfcx(x)) - x * x : log(0.5 * erfc(x));
+}
+
+// Survival term of the log-likelihood on [0, t_end] (Eq. 2): with the head
+// after the last event (row of position len-1), log S(u) = log sum_m w_m
+// (1 - Phi((log u - mu_m) / sigma_m)) at u = t_end - t_last, in fp64; 0 for
+// u <= 0 (the window ends at or before the last event).
+__global__ void k_score_survival(SeqState ss, Work w, int M, int K, int len, int g0, int rows, double t_end,
+                                 double* out_logS) {
+    const int r = blockIdx.x * blockDim.x + threadIdx.x;
+    if (r >= rows) return;
+    const long long g = g0 + (long long)r;
+    const int s = (int)(g / len), l = (int)(g % len);
+    if (l != len - 1) return;
+    const double u = t_end - ss.t[(size_t)s * ss.n_max + l];
+    if (!(u > 0.0)) {
+        out_logS[s] = 0.0;
+        return;
+    }
+    const float* hd = w.heads + (size_t)r * (3 * M + K);
+    const double lu = log(u);
+    double mx = -INFINITY, acc = 0.0;
+    for (int m = 0; m < M; ++m) {  // online log-sum-exp over the components
+        const double v = (double)hd[m] + log_normal_upper((lu - (double)hd[M + m]) * exp(-(double)hd[2 * M + m]));
+        if (v > mx) {
+            acc = acc * exp(mx - v) + 1.0;
+            mx = v;
+        } else {
+            acc += exp(v - mx);
+        }
+    }
+    out_logS[s] = mx + log(acc);
 }
 
 // ======================================================================
@@ -1276,11 +1340,20 @@ cudaError_t launch_round_control(const SeqState& ss, const CallParams* dp, int B
                     (cudaGraphConditionalHandle)cond_handle, use_cond, active_out);
 }
 
+cudaError_t launch_score_survival(const DevModel& m, const SeqState& ss, const Work& w, int B, int len,
+                                  int g0, int rows, double t_end, double* out_logS, cudaStream_t st) {
+    (void)B;
+    if (rows <= 0) return cudaSuccess;
+    k_score_survival<<<(rows + 127) / 128, 128, 0, st>>>(ss, w, m.M, m.K, len, g0, rows, t_end, out_logS);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work& w, int B, int len,
-                              int g0, int rows, float* out_heads, float* out_logg, float* out_logf,
+                              int q, int g0, int rows, float* out_heads, float* out_logg, float* out_logf,
                               cudaStream_t st) {
     (void)B;
-    k_score_logs<<<(rows + 127) / 128, 128, 0, st>>>(ss, w, m.M, m.K, len, g0, rows, out_heads,
+    if (rows <= 0) return cudaSuccess;
+    k_score_logs<<<(rows + 127) / 128, 128, 0, st>>>(ss, w, m.M, m.K, len, q, g0, rows, out_heads,
                                                      out_logg, out_logf);
     return cudaGetLastError();
 }

@@ -63,6 +63,42 @@ class Sampler:
         T.tppsd_sample_autoregressive(self.ctx, B, n_events, seed, flags, tau, t, k, stream)
         return dict(tau=tau, t=t, k=k)
 
+    def sample_until(self, t_end, max_events, gamma, seed, flags=0, batch=None, stream=None):
+        """TPP-SD until the end time t_end (Alg. 1's stop rule) or max_events;
+        count[b] kept events (t <= t_end) fill the first slots."""
+        torch = self.torch
+        B = self.batch if batch is None else batch
+        tau, t, k = self._outputs(B, max_events)
+        cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+        T.tppsd_sample_until(self.ctx, B, t_end, max_events, gamma, seed, flags, tau, t, k, cnt, stream)
+        return dict(tau=tau, t=t, k=k, count=cnt)
+
+    def sample_ar_until(self, t_end, max_events, seed, flags=0, batch=None, stream=None):
+        torch = self.torch
+        B = self.batch if batch is None else batch
+        tau, t, k = self._outputs(B, max_events)
+        cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+        T.tppsd_sample_autoregressive_until(self.ctx, B, t_end, max_events, seed, flags, tau, t, k,
+                                            cnt, stream)
+        return dict(tau=tau, t=t, k=k, count=cnt)
+
+    def score_until(self, which, tau, marks, t_end, heads=True, stream=None):
+        """Eq. 2 on the window [0, t_end]: per-event terms as score() plus the
+        survival term log S(t_end - t_last) per sequence (fp64)."""
+        torch = self.torch
+        tau = self._dev(tau, torch.float32)
+        mk = self._dev(marks, torch.int32)
+        B, n = tau.shape
+        cfg = self.target if which == 0 else self.draft
+        W = 3 * cfg.n_mix + cfg.n_marks
+        hd = torch.full((B, n, W), float("nan"), device="cuda") if heads else None
+        lg = torch.empty((B, n), device="cuda")
+        lf = torch.empty((B, n), device="cuda")
+        ls = torch.empty(B, dtype=torch.float64, device="cuda")
+        T.tppsd_score_until(self.ctx, which, B, n, tau, mk, t_end, hd, lg, lf, ls, stream)
+        self.batch = 0
+        return hd, lg, lf, ls
+
     def score(self, which, tau, marks, heads=True, stream=None):
         torch = self.torch
         tau = self._dev(tau, torch.float32)

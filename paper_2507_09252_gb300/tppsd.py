@@ -76,7 +76,13 @@ def load(build_if_missing: bool = True):
                                _vp, _vp, _vp, _vp]
     L.tppsd_sample_autoregressive.argtypes = [_vp, C.c_int32, C.c_int32, C.c_uint64, C.c_uint32,
                                               _vp, _vp, _vp, _vp]
+    L.tppsd_sample_until.argtypes = [_vp, C.c_int32, C.c_double, C.c_int32, C.c_int32, C.c_uint64,
+                                     C.c_uint32, _vp, _vp, _vp, _vp, _vp]
+    L.tppsd_sample_autoregressive_until.argtypes = [_vp, C.c_int32, C.c_double, C.c_int32, C.c_uint64,
+                                                    C.c_uint32, _vp, _vp, _vp, _vp, _vp]
     L.tppsd_score.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp, _vp]
+    L.tppsd_score_until.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, C.c_double,
+                                    _vp, _vp, _vp, _vp, _vp]
     L.tppsd_score_noalloc.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp]
     L.tppsd_score_noalloc.restype = C.c_int
     L.tppsd_get_stats.argtypes = [_vp, C.POINTER(tppsd_stats)]
@@ -92,7 +98,8 @@ def load(build_if_missing: bool = True):
     L.tppsd_destroy.argtypes = [_vp]
     L.tppsd_destroy.restype = None
     for f in ("tppsd_create_models", "tppsd_prefill", "tppsd_sample",
-              "tppsd_sample_autoregressive", "tppsd_score", "tppsd_get_stats", "tppsd_wait"):
+              "tppsd_sample_autoregressive", "tppsd_sample_until", "tppsd_sample_autoregressive_until",
+              "tppsd_score", "tppsd_score_until", "tppsd_get_stats", "tppsd_wait"):
         getattr(L, f).restype = C.c_int
     _lib = L
     return L
@@ -202,6 +209,41 @@ def tppsd_sample_autoregressive(ctx, batch, n_events, seed, flags, out_tau, out_
                                             _ptr(out_marks, np.int32, n, "out_marks"),
                                             _stream(stream))
     return _check("tppsd_sample_autoregressive", st, ctx)
+
+
+def tppsd_sample_until(ctx, batch, t_end, max_events, gamma, seed, flags, out_tau, out_t, out_marks,
+                       out_count, stream=None):
+    n = batch * max_events
+    st = load().tppsd_sample_until(ctx, batch, float(t_end), max_events, gamma, seed, flags,
+                                   _ptr(out_tau, np.float32, n, "out_tau"),
+                                   _ptr(out_t, np.float64, n, "out_t"),
+                                   _ptr(out_marks, np.int32, n, "out_marks"),
+                                   _ptr(out_count, np.int32, batch, "out_count"), _stream(stream))
+    return _check("tppsd_sample_until", st, ctx)
+
+
+def tppsd_sample_autoregressive_until(ctx, batch, t_end, max_events, seed, flags, out_tau, out_t,
+                                      out_marks, out_count, stream=None):
+    n = batch * max_events
+    st = load().tppsd_sample_autoregressive_until(ctx, batch, float(t_end), max_events, seed, flags,
+                                                  _ptr(out_tau, np.float32, n, "out_tau"),
+                                                  _ptr(out_t, np.float64, n, "out_t"),
+                                                  _ptr(out_marks, np.int32, n, "out_marks"),
+                                                  _ptr(out_count, np.int32, batch, "out_count"),
+                                                  _stream(stream))
+    return _check("tppsd_sample_autoregressive_until", st, ctx)
+
+
+def tppsd_score_until(ctx, which, batch, length, tau, marks, t_end, out_heads, out_logg, out_logf,
+                      out_logS, stream=None):
+    n = batch * length
+    st = load().tppsd_score_until(ctx, which, batch, length, _ptr(tau, np.float32, n, "tau"),
+                                  _ptr(marks, np.int32, n, "marks"), float(t_end),
+                                  _ptr(out_heads, np.float32, None, "out_heads"),
+                                  _ptr(out_logg, np.float32, n, "out_logg"),
+                                  _ptr(out_logf, np.float32, n, "out_logf"),
+                                  _ptr(out_logS, np.float64, batch, "out_logS"), _stream(stream))
+    return _check("tppsd_score_until", st, ctx)
 
 
 def tppsd_score(ctx, which, batch, length, tau, marks, out_heads, out_logg, out_logf, stream=None):
