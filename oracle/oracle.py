@@ -74,9 +74,21 @@ def lib():
                                             _i32p, C.c_double, _f64p, C.c_int32, C.c_int32]
         L.oracle_log_survival.argtypes = [C.c_int32, _f64p, C.c_double]
         L.oracle_log_survival.restype = C.c_double
+        L.oracle_sample_sd_poisson_until.argtypes = [
+            _i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p, _i32p, C.c_int32, C.c_double,
+            C.c_int32, C.c_double, _f64p, C.c_uint64, C.c_uint32, C.c_int32, _opt(_i32p),
+            _f64p, _f64p, _i32p, _f64p, _i32p, _i64p, C.c_int32]
+        L.oracle_sample_poisson.argtypes = [C.c_double, C.c_int32, _f64p, C.c_int32, C.c_uint64,
+                                            _f64p, _i32p]
+        L.oracle_resample_time_poisson.argtypes = [C.c_int32, _f64p, C.c_double, C.c_int32,
+                                                   C.c_uint64, _f64p, _i32p]
+        L.oracle_toy_sd_poisson.argtypes = [C.c_int32, C.c_int32, _f64p, C.c_double, _f64p,
+                                            C.c_int32, C.c_int32, C.c_int32, C.c_uint64, C.c_uint32,
+                                            _f64p, _i32p, _i64p]
         for f in ("oracle_score", "oracle_sample_ar", "oracle_sample_sd", "oracle_toy_sd",
                   "oracle_toy_ar", "oracle_sample_ar_until", "oracle_sample_sd_until",
-                  "oracle_score_survival"):
+                  "oracle_score_survival", "oracle_sample_sd_poisson_until", "oracle_sample_poisson",
+                  "oracle_resample_time_poisson", "oracle_toy_sd_poisson"):
             getattr(L, f).restype = C.c_int
         _lib = L
     return _lib
@@ -252,6 +264,52 @@ def toy_sd(M, K, table_t, table_d, B, N, gamma, seed, flags=0):
     tau = np.zeros((B, N)); k = np.zeros((B, N), np.int32); st = np.zeros((B, 5), np.int64)
     _check(lib().oracle_toy_sd(M, K, _c(table_t, np.float64), _c(table_d, np.float64), B, N,
                                gamma, seed, flags, tau, k, st), "oracle_toy_sd")
+    return tau, k, st
+
+
+def sample_sd_poisson_until(cfg_t, blob_t, hist_tau, hist_marks, max_events, t_end, gamma, lam,
+                            p_marks, seed, flags=0, recompute=False, nthreads=0, seq_ids=None):
+    """TPP-SD with the Poisson draft of App. D.3 (rate lam, mark
+    probabilities p_marks) until t_end or max_events."""
+    hist_tau = _c(hist_tau, np.float32)
+    hist_marks = _c(hist_marks, np.int32)
+    B, H = hist_tau.shape
+    N = max_events
+    tau = np.zeros((B, N)); t = np.zeros((B, N))
+    k = np.zeros((B, N), np.int32); mg = np.zeros((B, N)); cnt = np.zeros(B, np.int32)
+    st = np.zeros((B, 5), np.int64)
+    _check(lib().oracle_sample_sd_poisson_until(
+        _cfg(cfg_t), _c(blob_t, np.float32), blob_t.size, B, H, hist_tau, hist_marks, N,
+        float(t_end), gamma, float(lam), _c(p_marks, np.float64), seed, flags, int(recompute),
+        _ids(seq_ids, B), tau, t, k, mg, cnt, st, nthreads), "oracle_sample_sd_poisson_until")
+    return dict(tau=tau, t=t, k=k, margin=mg, count=cnt, stats=st)
+
+
+def sample_sd_poisson(cfg_t, blob_t, hist_tau, hist_marks, n_events, gamma, lam, p_marks, seed,
+                      **kw):
+    """Fixed-count form (t_end = +inf)."""
+    return sample_sd_poisson_until(cfg_t, blob_t, hist_tau, hist_marks, n_events, np.inf, gamma,
+                                   lam, p_marks, seed, **kw)
+
+
+def sample_poisson(lam, p, n, seed):
+    tau = np.zeros(n); k = np.zeros(n, np.int32)
+    p = _c(p, np.float64)
+    _check(lib().oracle_sample_poisson(float(lam), p.size, p, n, seed, tau, k), "oracle_sample_poisson")
+    return tau, k
+
+
+def resample_time_poisson(M, head_t, lam, n, seed):
+    tau = np.zeros(n); it = np.zeros(n, np.int32)
+    _check(lib().oracle_resample_time_poisson(M, _c(head_t, np.float64), float(lam), n, seed, tau, it),
+           "oracle_resample_time_poisson")
+    return tau, it
+
+
+def toy_sd_poisson(M, K, table_t, lam, p, B, N, gamma, seed, flags=0):
+    tau = np.zeros((B, N)); k = np.zeros((B, N), np.int32); st = np.zeros((B, 5), np.int64)
+    _check(lib().oracle_toy_sd_poisson(M, K, _c(table_t, np.float64), float(lam), _c(p, np.float64),
+                                       B, N, gamma, seed, flags, tau, k, st), "oracle_toy_sd_poisson")
     return tau, k, st
 
 

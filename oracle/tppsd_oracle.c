@@ -165,13 +165,16 @@ void oracle_temporal_encoding(int32_t d, double t, double *out)
 /* ------------------------------------------------------------------ */
 /* Head of Sec. 4.2.  Row layout [log w | mu | s | log f].               */
 /* ------------------------------------------------------------------ */
-typedef struct { int M, K; double v[3 * MAXM + MAXK]; } head_t;
+/* A head of the Poisson draft (App. D.3, history-independent) has
+ * poisson = 1, M = 1, v[0] = log lambda and v[3 + k] = log p_k: the
+ * inter-event density lambda exp(-lambda tau) and iid marks from p. */
+typedef struct { int M, K, poisson; double v[3 * MAXM + MAXK]; } head_t;
 
 static void model_head(const model_t *m, const double *h, head_t *out)
 {
     int d = m->d, M = m->M, K = m->K;
     double e[3 * 512], a[512], lw[MAXM], lk[MAXK];
-    out->M = M; out->K = K;
+    out->M = M; out->K = K; out->poisson = 0;
     linear(m->E, NULL, h, d, 3 * d, e);                     /* e = E h, split e1|e2|e3 */
     linear(m->v_w, m->b_w, e, d, M, lw);                    /* w = softmax(V_w e1 + b_w) */
     double z = logsumexp(lw, M);
@@ -198,6 +201,14 @@ double oracle_log_g(int32_t M, const double *hd, double tau)
 }
 
 double oracle_log_f(int32_t M, const double *hd, int32_t k) { return hd[3 * M + k]; }
+
+/* log g of either kind of head: the mixture above, or for the Poisson
+ * draft the exponential density, log lambda - lambda tau. */
+static double head_log_g(const head_t *h, double tau)
+{
+    if (h->poisson) return h->v[0] - exp(h->v[0]) * tau;
+    return oracle_log_g(h->M, h->v, tau);
+}
 
 /* log(1 - Phi(z)) = log(erfc(z / sqrt 2) / 2); for z beyond the range where
  * erfc underflows, the leading term of its asymptotic expansion,
@@ -263,13 +274,16 @@ static int draw_mark(const double *hd, int M, int K, double u, double *mg)
 }
 
 /* Direct sample of the next event from one head with slot block 0:
- * {u_comp, u_bm1, u_bm2, u_mark}. */
+ * {u_comp, u_bm1, u_bm2, u_mark}.  Reading for the Poisson draft: the
+ * time by inversion of the exponential CDF from the first word,
+ * tau = -log(u_comp) / lambda; the mark from p with u_mark. */
 static void draw_event(const head_t *hd, uint64_t seed, uint32_t seq, uint32_t pos,
                        double *tau, int *k, double *mg)
 {
     double u[4];
     oracle_uniforms(seed, seq, pos, 0, u);
-    *tau = draw_time(hd->v, hd->M, u[0], u[1], u[2], mg);
+    if (hd->poisson) *tau = -log(u[0]) / exp(hd->v[0]);
+    else *tau = draw_time(hd->v, hd->M, u[0], u[1], u[2], mg);
     *k = draw_mark(hd->v, hd->M, hd->K, u[3], mg);
 }
 
@@ -277,15 +291,15 @@ static void draw_event(const head_t *hd, uint64_t seed, uint32_t seq, uint32_t p
  * Iteration i uses slot block 2 + i: {u_comp, u_bm1, u_bm2, u_acc}.
  * Reading: capped at RESAMPLE_CAP iterations; on the cap the last proposal
  * is returned and *cap_hit set. */
-static double resample_time(int MT, const double *hT, int MD, const double *hD, uint64_t seed,
+static double resample_time(const head_t *hT, const head_t *hD, uint64_t seed,
                             uint32_t seq, uint32_t pos, int *iters, int *cap_hit, double *mg)
 {
     double tau = 1.0;
     for (int i = 0; i < RESAMPLE_CAP; ++i) {
         double u[4];
         oracle_uniforms(seed, seq, pos, 2u + (uint32_t)i, u);
-        tau = draw_time(hT, MT, u[0], u[1], u[2], mg);
-        double lgT = oracle_log_g(MT, hT, tau), lgD = oracle_log_g(MD, hD, tau);
+        tau = draw_time(hT->v, hT->M, u[0], u[1], u[2], mg);
+        double lgT = oracle_log_g(hT->M, hT->v, tau), lgD = head_log_g(hD, tau);
         double alpha = 1.0 - exp(lgD - lgT);       /* (g_T - g_D) / g_T */
         if (alpha < 0.0) alpha = 0.0;
         upd(mg, fabs(u[3] - alpha));
@@ -429,12 +443,42 @@ static void toy_step(void *st, double t, int k, head_t *out)
 {
     toystate *s = (toystate *)st;
     (void)t;
-    out->M = s->M; out->K = s->K;
+    out->M = s->M; out->K = s->K; out->poisson = 0;
     memcpy(out->v, s->table + (size_t)k * (3 * s->M + s->K), sizeof(double) * (3 * s->M + s->K));
     s->n++;
 }
 static void toy_truncate(void *st, int n) { toystate *s = (toystate *)st; if (n < s->n) s->n = n; }
 static const model_ops TOY_OPS = {toy_len, toy_step, toy_truncate};
+
+/* Poisson draft (App. D.3): the same head after every event. */
+typedef struct { int n; head_t head; } poisstate;
+static int pois_len(void *st) { return ((poisstate *)st)->n; }
+static void pois_step(void *st, double t, int k, head_t *out)
+{
+    poisstate *s = (poisstate *)st;
+    (void)t; (void)k;
+    *out = s->head;
+    s->n++;
+}
+static void pois_truncate(void *st, int n) { poisstate *s = (poisstate *)st; if (n < s->n) s->n = n; }
+static const model_ops POISSON_OPS = {pois_len, pois_step, pois_truncate};
+
+/* Head of the Poisson draft from the rate and the mark probabilities
+ * (normalised here).  Returns -1 unless lambda > 0, p_k >= 0, sum p > 0. */
+static int poisson_head(double lambda, const double *p, int K, head_t *h)
+{
+    if (!(lambda > 0.0) || !isfinite(lambda) || K < 1 || K > MAXK) return -1;
+    double tot = 0.0;
+    for (int k = 0; k < K; ++k) {
+        if (!(p[k] >= 0.0) || !isfinite(p[k])) return -1;
+        tot += p[k];
+    }
+    if (!(tot > 0.0)) return -1;
+    h->M = 1; h->K = K; h->poisson = 1;
+    h->v[0] = log(lambda); h->v[1] = 0.0; h->v[2] = 0.0;
+    for (int k = 0; k < K; ++k) h->v[3 + k] = log(p[k] / tot);
+    return 0;
+}
 
 /* ------------------------------------------------------------------ */
 /* Samplers over one sequence.  ev_* hold history + generated events at  */
@@ -516,7 +560,7 @@ static int sd_sequence(const model_ops *T, void *ts, const model_ops *D, void *d
             const double *hT = thead[l - 1].v, *hD = dhead[l].v;
             int M_T = thead[l - 1].M, M_D = dhead[l].M;
             oracle_uniforms(seed, seq, (uint32_t)p, 1, u);
-            double rt = exp(oracle_log_g(M_T, hT, tau_hat[l]) - oracle_log_g(M_D, hD, tau_hat[l]));
+            double rt = exp(oracle_log_g(M_T, hT, tau_hat[l]) - head_log_g(&dhead[l], tau_hat[l]));
             double rk = exp(oracle_log_f(M_T, hT, k_hat[l]) - oracle_log_f(M_D, hD, k_hat[l]));
             if (rt > 1.0) rt = 1.0;
             if (rk > 1.0) rk = 1.0;
@@ -535,7 +579,7 @@ static int sd_sequence(const model_ops *T, void *ts, const model_ops *D, void *d
             const head_t *hT = &thead[L - 1], *hD = &dhead[L];
             if (!acc_tau) {
                 int it = 0, cap = 0;
-                tau = resample_time(hT->M, hT->v, hD->M, hD->v, seed, seq, (uint32_t)p, &it, &cap, &ev->mg[p]);
+                tau = resample_time(hT, hD, seed, seq, (uint32_t)p, &it, &cap, &ev->mg[p]);
                 st[3] += it; st[4] += cap;
             }
             if (!acc_k) k = resample_mark(hT->M, hT->v, hD->M, hD->v, hT->K, u[2], &ev->mg[p]);
@@ -668,6 +712,43 @@ int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT
     return 0;
 }
 
+/* TPP-SD with the Poisson draft of App. D.3 (rate lambda, mark
+ * probabilities p[K]) in place of the draft Transformer. */
+int oracle_sample_sd_poisson_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                                   int32_t B, int32_t H, const float *hist_tau,
+                                   const int32_t *hist_marks, int32_t N, double t_end,
+                                   int32_t gamma, double lambda, const double *p_marks,
+                                   uint64_t seed, uint32_t flags, int32_t recompute,
+                                   const int32_t *seq_ids, double *out_tau, double *out_t,
+                                   int32_t *out_k, double *out_margin, int32_t *out_count,
+                                   int64_t *stats, int32_t nthreads)
+{
+    model_t mT;
+    head_t hp;
+    if (model_init(&mT, cfgT, blobT, nT)) return -1;
+    if (poisson_head(lambda, p_marks, mT.K, &hp)) return -1;
+    if (gamma < 1 || gamma > 64 || B < 0 || H < 1 || N < 0) return -1;
+    int cap = H + N + gamma + 2;
+#pragma omp parallel for schedule(dynamic, 1) num_threads(nthreads_or_default(nthreads))
+    for (int b = 0; b < B; ++b) {
+        evbuf ev;
+        tstate ts;
+        poisstate ds = {0, hp};
+        int64_t st[5] = {0, 0, 0, 0, 0};
+        evbuf_alloc(&ev, cap);
+        tstate_init(&ts, &mT, cap, recompute);
+        load_history(&ev, hist_tau + (int64_t)b * H, hist_marks + (int64_t)b * H, H);
+        const int c = sd_sequence(&TRANSFORMER_OPS, &ts, &POISSON_OPS, &ds, &ev, H, N, t_end, gamma,
+                                  seed, (uint32_t)(seq_ids ? seq_ids[b] : b), flags, st);
+        store_out(&ev, H, N, c, b, out_tau, out_t, out_k, out_margin);
+        if (out_count) out_count[b] = c;
+        if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
+        tstate_free(&ts);
+        evbuf_free(&ev);
+    }
+    return 0;
+}
+
 int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
@@ -755,7 +836,7 @@ void oracle_sample_head(int32_t M, int32_t K, const double *head, int32_t n, uin
                         double *out_tau, int32_t *out_k)
 {
     head_t hd;
-    hd.M = M; hd.K = K;
+    hd.M = M; hd.K = K; hd.poisson = 0;
     memcpy(hd.v, head, sizeof(double) * (3 * M + K));
     for (int i = 0; i < n; ++i) {
         int k;
@@ -767,11 +848,44 @@ void oracle_sample_head(int32_t M, int32_t K, const double *head, int32_t n, uin
 void oracle_resample_time(int32_t M, const double *headT, const double *headD, int32_t n,
                           uint64_t seed, double *out_tau, int32_t *iters)
 {
+    head_t hT, hD;
+    hT.M = hD.M = M; hT.K = hD.K = 0; hT.poisson = hD.poisson = 0;
+    memcpy(hT.v, headT, sizeof(double) * 3 * M);
+    memcpy(hD.v, headD, sizeof(double) * 3 * M);
     for (int i = 0; i < n; ++i) {
         int it = 0, cap = 0;
-        out_tau[i] = resample_time(M, headT, M, headD, seed, 0, (uint32_t)i, &it, &cap, NULL);
+        out_tau[i] = resample_time(&hT, &hD, seed, 0, (uint32_t)i, &it, &cap, NULL);
         if (iters) iters[i] = it;
     }
+}
+
+int oracle_resample_time_poisson(int32_t M, const double *headT, double lambda, int32_t n,
+                                 uint64_t seed, double *out_tau, int32_t *iters)
+{
+    head_t hT, hD;
+    double one = 1.0;
+    if (M < 1 || M > MAXM || poisson_head(lambda, &one, 1, &hD)) return -1;
+    hT.M = M; hT.K = 0; hT.poisson = 0;
+    memcpy(hT.v, headT, sizeof(double) * 3 * M);
+    for (int i = 0; i < n; ++i) {
+        int it = 0, cap = 0;
+        out_tau[i] = resample_time(&hT, &hD, seed, 0, (uint32_t)i, &it, &cap, NULL);
+        if (iters) iters[i] = it;
+    }
+    return 0;
+}
+
+int oracle_sample_poisson(double lambda, int32_t K, const double *p, int32_t n, uint64_t seed,
+                          double *out_tau, int32_t *out_k)
+{
+    head_t hd;
+    if (poisson_head(lambda, p, K, &hd)) return -1;
+    for (int i = 0; i < n; ++i) {
+        int k;
+        draw_event(&hd, seed, 0, (uint32_t)i, &out_tau[i], &k, NULL);
+        if (out_k) out_k[i] = k;
+    }
+    return 0;
 }
 
 void oracle_resample_mark(int32_t M, int32_t K, const double *headT, const double *headD,
@@ -797,6 +911,28 @@ int oracle_toy_sd(int32_t M, int32_t K, const double *tableT, const double *tabl
         evbuf_alloc(&ev, cap);
         ev.tau[0] = 1.0; ev.t[0] = 1.0; ev.k[0] = 0;
         sd_sequence(&TOY_OPS, &ts, &TOY_OPS, &ds, &ev, 1, N, INFINITY, gamma, seed, (uint32_t)b, flags, st);
+        store_out(&ev, 1, N, N, b, out_tau, NULL, out_k, NULL);
+        if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
+        evbuf_free(&ev);
+    }
+    return 0;
+}
+
+int oracle_toy_sd_poisson(int32_t M, int32_t K, const double *tableT, double lambda,
+                          const double *p_marks, int32_t B, int32_t N, int32_t gamma, uint64_t seed,
+                          uint32_t flags, double *out_tau, int32_t *out_k, int64_t *stats)
+{
+    head_t hp;
+    if (M < 1 || M > MAXM || gamma < 1 || gamma > 64 || poisson_head(lambda, p_marks, K, &hp)) return -1;
+    int cap = 1 + N + gamma + 2;
+    for (int b = 0; b < B; ++b) {
+        toystate ts = {M, K, 0, tableT};
+        poisstate ds = {0, hp};
+        evbuf ev;
+        int64_t st[5] = {0, 0, 0, 0, 0};
+        evbuf_alloc(&ev, cap);
+        ev.tau[0] = 1.0; ev.t[0] = 1.0; ev.k[0] = 0;
+        sd_sequence(&TOY_OPS, &ts, &POISSON_OPS, &ds, &ev, 1, N, INFINITY, gamma, seed, (uint32_t)b, flags, st);
         store_out(&ev, 1, N, N, b, out_tau, NULL, out_k, NULL);
         if (stats) for (int i = 0; i < 5; ++i) stats[(int64_t)b * 5 + i] = st[i];
         evbuf_free(&ev);

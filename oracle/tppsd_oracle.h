@@ -77,6 +77,35 @@ int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT
                            int32_t recompute, const int32_t *seq_ids,
                            double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
                            int32_t *out_count, int64_t *stats, int32_t nthreads);
+/* TPP-SD with the Poisson draft of App. D.3: a homogeneous Poisson process
+ * of rate lambda > 0 proposes the inter-event times (density
+ * lambda exp(-lambda tau)) and marks are drafted iid from p_marks[K]
+ * (normalised here; entries >= 0); the target's verification, resampling
+ * (Theorem 1 against the exponential density, Eq. 4 against p) and bonus
+ * are those of oracle_sample_sd.  Draft slot: block 0 at the event's
+ * position, tau = -log(u_comp) / lambda, mark from p with u_mark.  Outputs
+ * and stop rule as oracle_sample_sd_until.  Returns -1 on a bad lambda or
+ * p. */
+int oracle_sample_sd_poisson_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+                                   int32_t B, int32_t H, const float *hist_tau,
+                                   const int32_t *hist_marks, int32_t N, double t_end,
+                                   int32_t gamma, double lambda, const double *p_marks,
+                                   uint64_t seed, uint32_t flags, int32_t recompute,
+                                   const int32_t *seq_ids, double *out_tau, double *out_t,
+                                   int32_t *out_k, double *out_margin, int32_t *out_count,
+                                   int64_t *stats, int32_t nthreads);
+/* The Poisson draft's own draws (slot block 0 of positions 0..n-1 of
+ * sequence 0), and Theorem 1 against it for a fixed target head (M
+ * components, no marks). */
+int oracle_sample_poisson(double lambda, int32_t K, const double *p, int32_t n, uint64_t seed,
+                          double *out_tau, int32_t *out_k);
+int oracle_resample_time_poisson(int32_t M, const double *headT, double lambda, int32_t n,
+                                 uint64_t seed, double *out_tau, int32_t *iters);
+/* Toy target (head = tableT[previous mark]) with the Poisson draft. */
+int oracle_toy_sd_poisson(int32_t M, int32_t K, const double *tableT, double lambda,
+                          const double *p_marks, int32_t B, int32_t N, int32_t gamma, uint64_t seed,
+                          uint32_t flags, double *out_tau, int32_t *out_k, int64_t *stats);
+
 /* Survival term log S(t_end - t_{len-1}) of each sequence's len events, from
  * the head after the last event (Sec. 3.1, Eq. 2). */
 int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_floats,
