@@ -153,6 +153,30 @@ tppsd_status_t tppsd_sample_autoregressive_until(tppsd_ctx* ctx, int32_t batch, 
                                                  float* out_tau, double* out_t, int32_t* out_marks,
                                                  int32_t* out_count, void* stream);
 
+/* TPP-SD with the Poisson draft of App. D.3 in place of the draft model: a
+ * homogeneous Poisson process of rate `rate` (> 0) proposes the gamma
+ * inter-event times of a round (density rate exp(-rate tau)) and the marks
+ * are proposed iid from mark_probs, a HOST array of K doubles (the target's
+ * n_marks; entries >= 0 with a positive sum, normalised by the library).
+ * The paper fits both by maximum likelihood on the data (rate = events per
+ * unit time, mark_probs = mark frequencies).  Draft slot: block 0 at the
+ * event's position, tau = -log(u_comp) / rate, mark with u_mark.  The
+ * target's verification, resampling (Theorem 1 against the exponential
+ * density, Eq. 4 against mark_probs) and bonus are those of tppsd_sample,
+ * and so are the outputs; the draft model of the context is not used.  A
+ * bad rate or mark_probs is TPPSD_ERR_INVALID_ARG. */
+tppsd_status_t tppsd_sample_poisson(tppsd_ctx* ctx, int32_t batch, int32_t n_events, int32_t gamma,
+                                    double rate, const double* mark_probs, uint64_t seed,
+                                    uint32_t flags, float* out_tau, double* out_t,
+                                    int32_t* out_marks, void* stream);
+
+/* The same with the end-time stop rule, outputs as tppsd_sample_until. */
+tppsd_status_t tppsd_sample_poisson_until(tppsd_ctx* ctx, int32_t batch, double t_end,
+                                          int32_t max_events, int32_t gamma, double rate,
+                                          const double* mark_probs, uint64_t seed, uint32_t flags,
+                                          float* out_tau, double* out_t, int32_t* out_marks,
+                                          int32_t* out_count, void* stream);
+
 /* Teacher-forced scoring with one model (which 0 = target, 1 = draft): for
  * sequences tau/marks [batch][len], out_heads [batch][len][3M+K] (may be
  * NULL) gets the head after events 0..i at row i (row len-1 untouched):

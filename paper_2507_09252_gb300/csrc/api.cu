@@ -14,6 +14,7 @@
 #include <string.h>
 
 #include <chrono>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <new>
@@ -80,6 +81,7 @@ struct tppsd_ctx {
     Work work{};
     float* draft_heads = nullptr;
     CallParams* d_params = nullptr;
+    float* d_pois_logp = nullptr;  // [MAX_MARKS] log p of the Poisson draft
     DevStats* d_stats = nullptr;
     int* d_active = nullptr;
     int* h_active = nullptr;  // pinned
@@ -486,6 +488,7 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &w.hd4, sizeof(float) * R * 4 * dmax));
     TRY(dalloc(ctx, &ctx->draft_heads, sizeof(float) * (size_t)B * ctx->max_gamma * hwD));
     TRY(dalloc(ctx, &ctx->d_params, sizeof(CallParams)));
+    TRY(dalloc(ctx, &ctx->d_pois_logp, sizeof(float) * MAX_MARKS));
     TRY(dalloc(ctx, &ctx->d_stats, sizeof(DevStats)));
     TRY(dalloc(ctx, &ctx->d_active, sizeof(int)));
     CK(cudaMemset(ctx->d_stats, 0, sizeof(DevStats)));
@@ -589,7 +592,19 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
                                    const Prof* prof) {
     int n = 0;
     Work& w = ctx->work;
-    if (mode == 0) {
+    if (mode == 2) {
+        PROF_MARK(prof, KC_DRAFT, 1, st);
+        CK(launch_poisson_draft(ctx->ss, ctx->d_params, B, gamma, ctx->T.cfg.n_marks, st));
+        PROF_MARK(prof, KC_DRAFT, 0, st);
+        ++n;
+        RowSpec rs{ROWS_STEP, gamma + 1, B * (gamma + 1), 0};
+        CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof, &ctx->tc));
+        PROF_MARK(prof, KC_EPILOGUE, 1, st);
+        CK(launch_verify_epilogue(ctx->T.dm, ctx->D.dm, ctx->ss, ctx->d_params, B, gamma, w.heads,
+                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, st, true));
+        PROF_MARK(prof, KC_EPILOGUE, 0, st);
+        ++n;
+    } else if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
         if (draft_team_supported(ctx->D.dm) && !getenv("TPPSD_DRAFT_CTA"))
             CK(launch_draft_team(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
@@ -667,17 +682,35 @@ static tppsd_status_t ensure_stage(tppsd_ctx* ctx, size_t bytes) {
     return TPPSD_OK;
 }
 
+struct PoissonDraft {
+    double rate;
+    const double* probs;  // [K], host
+};
+
 static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int gamma, uint64_t seed,
                                   uint32_t flags, float* out_tau, double* out_t, int32_t* out_k,
                                   void* stream, double t_end = INFINITY, int32_t* out_count = nullptr,
-                                  bool until = false) {
+                                  bool until = false, const PoissonDraft* pois = nullptr) {
     if (!ctx) return TPPSD_ERR_INVALID_ARG;
     if (N > 0 && (!out_tau || !out_t || !out_k)) return TPPSD_ERR_INVALID_ARG;
     if (until && (!out_count || t_end != t_end)) return TPPSD_ERR_INVALID_ARG;
     if (!ctx->prefilled || B < 1 || B > ctx->prefill_batch || N < 0) return TPPSD_ERR_INVALID_ARG;
-    if (mode == 0 && (gamma < 1 || gamma > ctx->max_gamma)) return TPPSD_ERR_INVALID_ARG;
+    const bool sd = mode != 1;  // 0: draft model, 2: Poisson draft
+    if (sd && (gamma < 1 || gamma > ctx->max_gamma)) return TPPSD_ERR_INVALID_ARG;
     const int H = ctx->hist_len;
-    if ((long long)H + N + (mode == 0 ? gamma : 0) + 2 > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    if ((long long)H + N + (sd ? gamma : 0) + 2 > ctx->n_max) return TPPSD_ERR_INVALID_ARG;
+    float logp[MAX_MARKS];
+    const int K = ctx->T.cfg.n_marks;
+    if (mode == 2) {  // Poisson draft: rate > 0, p >= 0 with a positive sum
+        if (!pois || !pois->probs || !(pois->rate > 0.0) || !std::isfinite(pois->rate)) return TPPSD_ERR_INVALID_ARG;
+        double tot = 0.0;
+        for (int k = 0; k < K; ++k) {
+            if (!(pois->probs[k] >= 0.0) || !std::isfinite(pois->probs[k])) return TPPSD_ERR_INVALID_ARG;
+            tot += pois->probs[k];
+        }
+        if (!(tot > 0.0)) return TPPSD_ERR_INVALID_ARG;
+        for (int k = 0; k < K; ++k) logp[k] = (float)log(pois->probs[k] / tot);
+    }
     CK(cudaSetDevice(ctx->device));
     if (!strcmp(fault_mode(), "launch")) {
         ctx->err = "injected launch failure (TPPSD_FAULT=launch)";
@@ -692,7 +725,13 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     if (any_host) TRY(ensure_stage(ctx, nb * (4 + 8 + 4) + (size_t)B * 4 + 64));
     char* sb = (char*)ctx->stage;
     CallParams p{};
-    p.B = B; p.H = H; p.N = N; p.gamma = mode == 0 ? gamma : 0; p.n_max = ctx->n_max;
+    p.B = B; p.H = H; p.N = N; p.gamma = sd ? gamma : 0; p.n_max = ctx->n_max;
+    if (mode == 2) {
+        CK(cudaMemcpyAsync(ctx->d_pois_logp, logp, sizeof(float) * K, cudaMemcpyHostToDevice, st));
+        p.pois_rate = (float)pois->rate;
+        p.pois_log_rate = (float)log(pois->rate);
+        p.pois_logp = ctx->d_pois_logp;
+    }
     p.flags = flags; p.seed = seed;
     p.out_t = host_out[1] ? (double*)sb : out_t;
     p.out_tau = host_out[0] ? (float*)(sb + nb * 8) : out_tau;
@@ -728,7 +767,7 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
             }
         } else {
             GraphEntry* ge = nullptr;
-            TRY(get_graph(ctx, mode, B, mode == 0 ? gamma : 0, flags & TPPSD_FLAG_NO_BONUS, &ge));
+            TRY(get_graph(ctx, mode, B, sd ? gamma : 0, flags & TPPSD_FLAG_NO_BONUS, &ge));
             CK(cudaGraphLaunch(ge->exec, st));
             launches = -ge->launches_per_round;  // resolved from loop_iters in get_stats
         }
@@ -826,6 +865,26 @@ static tppsd_status_t run_score(tppsd_ctx* ctx, int which, int batch, int len, c
     CK(cudaEventRecord(ctx->done_event, st));
     ctx->last_stream = st;
     return TPPSD_OK;
+}
+
+extern "C" tppsd_status_t tppsd_sample_poisson(tppsd_ctx* ctx, int32_t batch, int32_t n_events,
+                                               int32_t gamma, double rate, const double* mark_probs,
+                                               uint64_t seed, uint32_t flags, float* out_tau,
+                                               double* out_t, int32_t* out_marks, void* stream) {
+    const PoissonDraft pd{rate, mark_probs};
+    return run_sampler(ctx, 2, batch, n_events, gamma, seed, flags, out_tau, out_t, out_marks,
+                       stream, INFINITY, nullptr, false, &pd);
+}
+
+extern "C" tppsd_status_t tppsd_sample_poisson_until(tppsd_ctx* ctx, int32_t batch, double t_end,
+                                                     int32_t max_events, int32_t gamma, double rate,
+                                                     const double* mark_probs, uint64_t seed,
+                                                     uint32_t flags, float* out_tau, double* out_t,
+                                                     int32_t* out_marks, int32_t* out_count,
+                                                     void* stream) {
+    const PoissonDraft pd{rate, mark_probs};
+    return run_sampler(ctx, 2, batch, max_events, gamma, seed, flags, out_tau, out_t, out_marks,
+                       stream, t_end, out_count, true, &pd);
 }
 
 extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,

@@ -102,6 +102,9 @@ struct CallParams {
     // t <= t_end are written and out_count[s] receives their number.
     double t_end;
     int* out_count;
+    // Poisson draft (App. D.3): rate, its log, and log p of the marks [K]
+    float pois_rate, pois_log_rate;
+    const float* pois_logp;
 };
 
 // Device counters of the current call (mirrors tppsd_stats + status).
@@ -257,7 +260,9 @@ cudaError_t launch_draft(const DevModel& m, const KVCache& kv, const SeqState& s
 cudaError_t launch_verify_epilogue(const DevModel& mT, const DevModel& mD, const SeqState& ss,
                                    const CallParams* dp, int B, int gamma, const float* t_heads,
                                    const float* d_heads, int gamma_max, DevStats* stats,
-                                   cudaStream_t st);
+                                   cudaStream_t st, bool poisson = false);
+cudaError_t launch_poisson_draft(const SeqState& ss, const CallParams* dp, int B, int gamma, int K,
+                                 cudaStream_t st);
 cudaError_t launch_ar_sample(const DevModel& mT, const SeqState& ss, const CallParams* dp,
                              int B, const float* heads, DevStats* stats, cudaStream_t st);
 cudaError_t launch_round_control(const SeqState& ss, const CallParams* dp, int B,

@@ -680,6 +680,7 @@ struct EpiArgs {
     const float* th;  // target heads, row s*(gamma+1)+l
     const float* dh;  // draft heads [Bmax][gamma_max][WD]
     int MT, MD, K, WT, WD, gamma, gamma_max;
+    int poisson;  // draft = homogeneous Poisson process (App. D.3), parameters in *P
     DevStats* st;
 };
 
@@ -745,9 +746,17 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
             tau_hat = ss.tau[sb + p];
             k_hat = ss.k[sb + p];
             const float* hT = a.th + ((size_t)s * (g + 1) + lane) * a.WT;
-            const float* hD = a.dh + ((size_t)s * a.gamma_max + lane) * a.WD;
-            const float rt = fminf(1.f, expf(head_log_g(hT, a.MT, tau_hat) - head_log_g(hD, a.MD, tau_hat)));
-            const float rk = fminf(1.f, expf(hT[3 * a.MT + k_hat] - hD[3 * a.MD + k_hat]));
+            float lgD, lfD;
+            if (a.poisson) {  // g_D = lambda exp(-lambda tau), f_D = p
+                lgD = P.pois_log_rate - P.pois_rate * tau_hat;
+                lfD = P.pois_logp[k_hat];
+            } else {
+                const float* hD = a.dh + ((size_t)s * a.gamma_max + lane) * a.WD;
+                lgD = head_log_g(hD, a.MD, tau_hat);
+                lfD = hD[3 * a.MD + k_hat];
+            }
+            const float rt = fminf(1.f, expf(head_log_g(hT, a.MT, tau_hat) - lgD));
+            const float rk = fminf(1.f, expf(hT[3 * a.MT + k_hat] - lfD));
             const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 1u);
             acc_t = u.x < rt;
             acc_k = u.y < rk;
@@ -767,7 +776,6 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
             // log tau and log(2 pi)/2 terms of log g_T and log g_D cancel in
             // their difference.
             const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
-            const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
             const int MT = a.MT, MD = a.MD;
             for (int m = lane; m < MT; m += 32) {
                 muT[m] = hT[MT + m];
@@ -775,10 +783,13 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
                 isT[m] = expf(-hT[2 * MT + m]);
                 cT[m] = hT[m] - hT[2 * MT + m];
             }
-            for (int m = lane; m < MD; m += 32) {
-                muD[m] = hD[MD + m];
-                isD[m] = expf(-hD[2 * MD + m]);
-                cD[m] = hD[m] - hD[2 * MD + m];
+            if (!a.poisson) {
+                const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
+                for (int m = lane; m < MD; m += 32) {
+                    muD[m] = hD[MD + m];
+                    isD[m] = expf(-hD[2 * MD + m]);
+                    cD[m] = hD[m] - hD[2 * MD + m];
+                }
             }
             if (lane == 0) {
                 float run = 0.f;
@@ -813,26 +824,35 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
                 if (cumT[m] >= target) { z = m; break; }
             const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
             const float lt = fmaf(sgT[z], eps, muT[z]);
-            float mT = -INFINITY, mD = -INFINITY;
+            float mT = -INFINITY;
             for (int m = 0; m < MT; ++m) {
                 const float q = (lt - muT[m]) * isT[m];
                 mT = fmaxf(mT, cT[m] - 0.5f * q * q);
             }
-            for (int m = 0; m < MD; ++m) {
-                const float q = (lt - muD[m]) * isD[m];
-                mD = fmaxf(mD, cD[m] - 0.5f * q * q);
-            }
-            float sT = 0.f, sD = 0.f;
+            float sT = 0.f;
             for (int m = 0; m < MT; ++m) {
                 const float q = (lt - muT[m]) * isT[m];
                 sT += expf(cT[m] - 0.5f * q * q - mT);
             }
-            for (int m = 0; m < MD; ++m) {
-                const float q = (lt - muD[m]) * isD[m];
-                sD += expf(cD[m] - 0.5f * q * q - mD);
-            }
-            const float al = fmaxf(0.f, 1.f - expf((mD + logf(sD)) - (mT + logf(sT))));
             const float tp = expf(lt);
+            float ldiff;  // log g_D - log g_T at the proposal
+            if (a.poisson) {
+                const float HALF_LOG_2PI = 0.91893853320467274178f;
+                ldiff = (P.pois_log_rate - P.pois_rate * tp) - (mT + logf(sT) - lt - HALF_LOG_2PI);
+            } else {
+                float mD = -INFINITY;
+                for (int m = 0; m < MD; ++m) {
+                    const float q = (lt - muD[m]) * isD[m];
+                    mD = fmaxf(mD, cD[m] - 0.5f * q * q);
+                }
+                float sD = 0.f;
+                for (int m = 0; m < MD; ++m) {
+                    const float q = (lt - muD[m]) * isD[m];
+                    sD += expf(cD[m] - 0.5f * q * q - mD);
+                }
+                ldiff = (mD + logf(sD)) - (mT + logf(sT));
+            }
+            const float al = fmaxf(0.f, 1.f - expf(ldiff));
             const unsigned okb = __ballot_sync(0xffffffffu, u.w < al);
             if (lane == 0) {
                 win_idx[warp] = okb ? 32 * warp + __ffs(okb) - 1 : 1 << 30;
@@ -864,12 +884,13 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         const int p = n + L - 1, src = L - 1;
         int k = sh_k;
         const float* hT = a.th + ((size_t)s * (g + 1) + src) * a.WT;
-        const float* hD = a.dh + ((size_t)s * a.gamma_max + src) * a.WD;
+        // log f_D: the draft head's mark block, or log p of the Poisson draft
+        const float* lfD = a.poisson ? P.pois_logp : a.dh + ((size_t)s * a.gamma_max + src) * a.WD + 3 * a.MD;
         if (!sh_ak && lane == 0) {
             // f' = norm(max(0, f_T - f_D)); zero mass -> draw from f_T
             const float umr = sh_umr;
             float tot = 0.f;
-            for (int kk = 0; kk < a.K; ++kk) tot += fmaxf(0.f, expf(hT[3 * a.MT + kk]) - expf(hD[3 * a.MD + kk]));
+            for (int kk = 0; kk < a.K; ++kk) tot += fmaxf(0.f, expf(hT[3 * a.MT + kk]) - expf(lfD[kk]));
             if (tot < 1e-12f) {
                 k = pick_categorical_log(hT + 3 * a.MT, a.K, umr);
             } else {
@@ -877,7 +898,7 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
                 float run = 0.f;
                 k = a.K - 1;
                 for (int kk = 0; kk < a.K; ++kk) {
-                    run += fmaxf(0.f, expf(hT[3 * a.MT + kk]) - expf(hD[3 * a.MD + kk]));
+                    run += fmaxf(0.f, expf(hT[3 * a.MT + kk]) - expf(lfD[kk]));
                     if (run >= target) { k = kk; break; }
                 }
             }
@@ -919,6 +940,32 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         atomicAdd(&a.st->emitted, (unsigned long long)emitted);
         if (iters) atomicAdd(&a.st->resample_iters, iters);
         if (cap) atomicAdd(&a.st->cap_hits, cap);
+    }
+    pdl_trigger();
+}
+
+// Poisson draft (App. D.3): the gamma drafts of an active sequence, all at
+// once since the draft ignores the history.  Position p = n + l uses its
+// block-0 slot: tau = -log(u_comp) / lambda (inversion of the exponential
+// CDF), mark from p with u_mark.  One thread per sequence keeps the
+// absolute times a sequential fp64 sum.
+__global__ void k_poisson_draft(SeqState ss, const CallParams* Pp, int gamma, int K) {
+    pdl_wait();
+    const int s = blockIdx.x * blockDim.x + threadIdx.x;
+    const CallParams& P = *Pp;
+    if (s < P.B && !ss.done[s]) {
+        const int n = ss.n_emit[s];
+        const size_t sb = (size_t)s * ss.n_max;
+        double t = ss.t[sb + n - 1];
+        for (int l = 0; l < gamma; ++l) {
+            const int p = n + l;
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
+            const float tau = -logf(u.x) / P.pois_rate;
+            t += (double)tau;
+            ss.tau[sb + p] = tau;
+            ss.t[sb + p] = t;
+            ss.k[sb + p] = pick_categorical_log(P.pois_logp, K, u.w);
+        }
     }
     pdl_trigger();
 }
@@ -1318,12 +1365,18 @@ cudaError_t launch_draft(const DevModel& m, const KVCache& kv, const SeqState& s
 cudaError_t launch_verify_epilogue(const DevModel& mT, const DevModel& mD, const SeqState& ss,
                                    const CallParams* dp, int B, int gamma, const float* t_heads,
                                    const float* d_heads, int gamma_max, DevStats* stats,
-                                   cudaStream_t st) {
+                                   cudaStream_t st, bool poisson) {
     EpiArgs a{};
     a.ss = ss; a.P = dp; a.th = t_heads; a.dh = d_heads;
     a.MT = mT.M; a.MD = mD.M; a.K = mT.K; a.WT = mT.head_width(); a.WD = mD.head_width();
     a.gamma = gamma; a.gamma_max = gamma_max; a.st = stats;
+    a.poisson = poisson ? 1 : 0;
     return launch_k(k_verify_epilogue, dim3(B), dim3(128), 0, st, a);
+}
+
+cudaError_t launch_poisson_draft(const SeqState& ss, const CallParams* dp, int B, int gamma, int K,
+                                 cudaStream_t st) {
+    return launch_k(k_poisson_draft, dim3((B + 127) / 128), dim3(128), 0, st, ss, dp, gamma, K);
 }
 
 cudaError_t launch_ar_sample(const DevModel& mT, const SeqState& ss, const CallParams* dp, int B,

@@ -20,6 +20,8 @@ are not visible to it.
 before each timed call), mean accepted drafts per verify and acceptance
 rate, as one JSON line.  --gamma / --batch / --draft override the workload's
 gamma, batch and draft model (an index into the workload's draft sweep).
+--poisson: the draft is the Poisson process of App. D.3, fitted by maximum
+likelihood on a pilot AR sample of the target (64 events per sequence).
 """
 import argparse
 import json
@@ -66,6 +68,7 @@ def main(argv=None):
     ap.add_argument("--gamma", type=int, default=None)
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--draft", type=int, default=None)
+    ap.add_argument("--poisson", action="store_true")
     a = ap.parse_args(argv)
     import torch
     wl = WORKLOADS[a.workload]
@@ -82,12 +85,26 @@ def main(argv=None):
     tau, mk = torch.from_numpy(tau_np).cuda(), torch.from_numpy(mk_np).cuda()
     outs = s._outputs(B, N)
     st = torch.cuda.current_stream()
+    from .sampler import fit_poisson_draft
+    rate, probs = 1.0, None
+    if a.poisson:  # MLE on a pilot AR sample of the target (the data it models)
+        T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
+        pilot = s._outputs(B, min(N, 64))
+        T.tppsd_sample_autoregressive(s.ctx, B, min(N, 64), 99, 0, *pilot, st)
+        rate, probs = fit_poisson_draft(pilot[0].cpu().numpy(), pilot[2].cpu().numpy(),
+                                        wl.target.n_marks)
+
+    def sample_call(flags):
+        if a.poisson:
+            T.tppsd_sample_poisson(s.ctx, B, N, g, rate, probs, 1234, flags, *outs, st)
+        else:
+            T.tppsd_sample(s.ctx, B, N, g, 1234, flags, *outs, st)
     if a.time:
         flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
 
         def sd():
             T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
-            T.tppsd_sample(s.ctx, B, N, g, 1234, 0, *outs, st)
+            sample_call(0)
 
         def ar():
             T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
@@ -100,7 +117,7 @@ def main(argv=None):
         print(json.dumps({
             "workload": wl.name, "batch": B, "gamma": g, "n_events": N, "hist_len": H,
             "target": _shape(wl.target, layer + (("M", "n_mix"), ("K", "n_marks"))),
-            "draft": _shape(wl.draft, layer),
+            "draft": f"Poisson rate {rate:.4g}" if a.poisson else _shape(wl.draft, layer),
             "sd_events_per_s": round(B * N / (ms_sd / 1e3), 1), "sd_ms_per_call": round(ms_sd, 3),
             "ar_events_per_s": round(B * N / (ms_ar / 1e3), 1), "ar_ms_per_call": round(ms_ar, 3),
             "speedup_vs_ar": round(ms_ar / ms_sd, 3),
@@ -113,7 +130,7 @@ def main(argv=None):
     for _ in range(a.calls):
         T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
         if a.mode == "sd":
-            T.tppsd_sample(s.ctx, B, N, g, 1234, flags, *outs, st)
+            sample_call(flags)
         else:
             T.tppsd_sample_autoregressive(s.ctx, B, N, 1234, flags, *outs, st)
     torch.cuda.synchronize()

@@ -82,6 +82,25 @@ class Sampler:
                                             cnt, stream)
         return dict(tau=tau, t=t, k=k, count=cnt)
 
+    def sample_poisson(self, n_events, gamma, rate, mark_probs, seed, flags=0, batch=None,
+                       stream=None):
+        """TPP-SD with the Poisson draft of App. D.3 (rate, mark_probs)."""
+        B = self.batch if batch is None else batch
+        tau, t, k = self._outputs(B, n_events)
+        T.tppsd_sample_poisson(self.ctx, B, n_events, gamma, rate, mark_probs, seed, flags, tau, t, k,
+                               stream)
+        return dict(tau=tau, t=t, k=k)
+
+    def sample_poisson_until(self, t_end, max_events, gamma, rate, mark_probs, seed, flags=0,
+                             batch=None, stream=None):
+        torch = self.torch
+        B = self.batch if batch is None else batch
+        tau, t, k = self._outputs(B, max_events)
+        cnt = torch.empty(B, dtype=torch.int32, device="cuda")
+        T.tppsd_sample_poisson_until(self.ctx, B, t_end, max_events, gamma, rate, mark_probs, seed,
+                                     flags, tau, t, k, cnt, stream)
+        return dict(tau=tau, t=t, k=k, count=cnt)
+
     def score_until(self, which, tau, marks, t_end, heads=True, stream=None):
         """Eq. 2 on the window [0, t_end]: per-event terms as score() plus the
         survival term log S(t_end - t_last) per sequence (fp64)."""
@@ -115,3 +134,15 @@ class Sampler:
 
     def stats(self):
         return T.tppsd_get_stats(self.ctx)
+
+
+def fit_poisson_draft(hist_tau, hist_marks, n_marks):
+    """Maximum-likelihood Poisson draft of App. D.3 from observed sequences:
+    rate = events / total observed time (sum over sequences of the time of
+    their last event), mark probabilities = mark frequencies.  Fitting the
+    draft is set-up, like loading weights; it is not part of sampling."""
+    tau = np.asarray(hist_tau, dtype=np.float64)
+    marks = np.asarray(hist_marks).ravel()
+    rate = tau.size / tau.sum()
+    probs = np.bincount(marks, minlength=n_marks)[:n_marks].astype(np.float64)
+    return float(rate), probs / probs.sum()

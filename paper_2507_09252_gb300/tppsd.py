@@ -80,6 +80,11 @@ def load(build_if_missing: bool = True):
                                      C.c_uint32, _vp, _vp, _vp, _vp, _vp]
     L.tppsd_sample_autoregressive_until.argtypes = [_vp, C.c_int32, C.c_double, C.c_int32, C.c_uint64,
                                                     C.c_uint32, _vp, _vp, _vp, _vp, _vp]
+    L.tppsd_sample_poisson.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, C.c_double, _vp,
+                                       C.c_uint64, C.c_uint32, _vp, _vp, _vp, _vp]
+    L.tppsd_sample_poisson_until.argtypes = [_vp, C.c_int32, C.c_double, C.c_int32, C.c_int32,
+                                             C.c_double, _vp, C.c_uint64, C.c_uint32, _vp, _vp, _vp,
+                                             _vp, _vp]
     L.tppsd_score.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, _vp, _vp, _vp, _vp]
     L.tppsd_score_until.argtypes = [_vp, C.c_int32, C.c_int32, C.c_int32, _vp, _vp, C.c_double,
                                     _vp, _vp, _vp, _vp, _vp]
@@ -99,6 +104,7 @@ def load(build_if_missing: bool = True):
     L.tppsd_destroy.restype = None
     for f in ("tppsd_create_models", "tppsd_prefill", "tppsd_sample",
               "tppsd_sample_autoregressive", "tppsd_sample_until", "tppsd_sample_autoregressive_until",
+              "tppsd_sample_poisson", "tppsd_sample_poisson_until",
               "tppsd_score", "tppsd_score_until", "tppsd_get_stats", "tppsd_wait"):
         getattr(L, f).restype = C.c_int
     _lib = L
@@ -232,6 +238,40 @@ def tppsd_sample_autoregressive_until(ctx, batch, t_end, max_events, seed, flags
                                                   _ptr(out_count, np.int32, batch, "out_count"),
                                                   _stream(stream))
     return _check("tppsd_sample_autoregressive_until", st, ctx)
+
+
+def _host_f64(a, name):
+    a = np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+    if a.ndim != 1:
+        raise ValueError(f"{name}: expected a 1-D host array")
+    return a, a.ctypes.data_as(_vp)
+
+
+def tppsd_sample_poisson(ctx, batch, n_events, gamma, rate, mark_probs, seed, flags, out_tau, out_t,
+                         out_marks, stream=None):
+    n = batch * n_events
+    probs, pp = _host_f64(mark_probs, "mark_probs")
+    st = load().tppsd_sample_poisson(ctx, batch, n_events, gamma, float(rate), pp, seed, flags,
+                                     _ptr(out_tau, np.float32, n, "out_tau"),
+                                     _ptr(out_t, np.float64, n, "out_t"),
+                                     _ptr(out_marks, np.int32, n, "out_marks"), _stream(stream))
+    del probs
+    return _check("tppsd_sample_poisson", st, ctx)
+
+
+def tppsd_sample_poisson_until(ctx, batch, t_end, max_events, gamma, rate, mark_probs, seed, flags,
+                               out_tau, out_t, out_marks, out_count, stream=None):
+    n = batch * max_events
+    probs, pp = _host_f64(mark_probs, "mark_probs")
+    st = load().tppsd_sample_poisson_until(ctx, batch, float(t_end), max_events, gamma, float(rate),
+                                           pp, seed, flags,
+                                           _ptr(out_tau, np.float32, n, "out_tau"),
+                                           _ptr(out_t, np.float64, n, "out_t"),
+                                           _ptr(out_marks, np.int32, n, "out_marks"),
+                                           _ptr(out_count, np.int32, batch, "out_count"),
+                                           _stream(stream))
+    del probs
+    return _check("tppsd_sample_poisson_until", st, ctx)
 
 
 def tppsd_score_until(ctx, which, batch, length, tau, marks, t_end, out_heads, out_logg, out_logf,

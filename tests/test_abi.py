@@ -91,3 +91,16 @@ def test_no_device_is_reported_not_crashed():
     with pytest.raises(T.TppsdError) as e:
         _try_create()
     assert e.value.status == T.TPPSD_ERR_NO_DEVICE
+
+
+def test_poisson_draft_fit_is_the_mle():
+    """Rate = events / observed time, mark probabilities = frequencies; on a
+    homogeneous Poisson sample the fitted rate recovers the true one."""
+    from paper_2507_09252_gb300.sampler import fit_poisson_draft
+    rng = np.random.default_rng(0)
+    tau = rng.exponential(1 / 2.5, (200, 50))
+    mk = rng.choice(3, size=(200, 50), p=[0.6, 0.3, 0.1])
+    rate, p = fit_poisson_draft(tau, mk, 4)
+    assert rate == pytest.approx(tau.size / tau.sum())
+    assert abs(rate - 2.5) < 0.1
+    assert np.allclose(p[:3], np.bincount(mk.ravel(), minlength=3) / mk.size) and p[3] == 0.0
