@@ -290,7 +290,7 @@ def main():
     import torch.distributed as dist
 
     from paper_2507_09252_gb300 import tppsd as T
-    from paper_2507_09252_gb300.sampler import Sampler
+    from paper_2507_09252_gb300.sampler import Sampler, fit_poisson_draft
 
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
@@ -342,6 +342,20 @@ def main():
     ms_ar = timed(step_ar, max(1, min(args.steps, 3)), 1)
     _, st_ar = T.tppsd_get_stats(s.ctx)
 
+    # Poisson draft (App. D.3) in place of the draft model, fitted by maximum
+    # likelihood on a pilot AR sample of the target (64 events per sequence)
+    pilot = s._outputs(B, 64)
+    T.tppsd_prefill(s.ctx, B, tau, mk, H, stream)
+    T.tppsd_sample_autoregressive(s.ctx, B, 64, 99, 0, *pilot, stream)
+    rate, probs = fit_poisson_draft(pilot[0].cpu().numpy(), pilot[2].cpu().numpy(), wl.target.n_marks)
+
+    def step_pois():
+        T.tppsd_prefill(s.ctx, B, tau, mk, H, stream)
+        T.tppsd_sample_poisson(s.ctx, B, N, g, rate, probs, 1234, fl, *outs, stream)
+
+    ms_pois = timed(step_pois, max(1, min(args.steps, 3)), 1)
+    _, st_pois = T.tppsd_get_stats(s.ctx)
+
     # end to end through the C ABI with pinned host buffers
     h_tau = torch.from_numpy(tau_np).pin_memory()
     h_mk = torch.from_numpy(mk_np).pin_memory()
@@ -379,6 +393,12 @@ def main():
         "ar": {"value": round(events / (ms_ar / 1e3), 1), "unit": UNIT, "ms_per_step": round(ms_ar, 3),
                "rounds": st_ar["loop_iters"]},
         "speedup_vs_ar": round(ms_ar / ms_sd, 3),
+        "poisson_draft": {"value": round(events / (ms_pois / 1e3), 1), "unit": UNIT,
+                          "ms_per_step": round(ms_pois, 3), "gamma": g, "rate": round(rate, 5),
+                          "mean_accepted_per_verify": round(st_pois["accepted"] / max(st_pois["rounds"], 1), 3),
+                          "alpha": round(st_pois["accepted"] / max(st_pois["drafted"], 1), 4),
+                          "speedup_vs_ar": round(ms_ar / ms_pois, 3),
+                          "fit": "MLE on a pilot AR sample of the target, 64 events per sequence"},
         "e2e": {"value": round(events / (ms_e2e / 1e3), 1), "unit": UNIT, "ms_per_step": round(ms_e2e, 3),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": args.steps * (st_sd["kernel_launches"] + st_sd["prefill_launches"]),

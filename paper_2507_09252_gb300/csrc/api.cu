@@ -428,6 +428,7 @@ static void build_tc_plan(tppsd_ctx* ctx) {
              make_tmap_bf16(&p.layer[l].w2, L.w_2, F, d, bo);
     }
     p.mlp = ok && mlp_tc_supported(d, F) && !getenv("TPPSD_NO_MLP_FUSION");
+    p.mlp_cl = p.mlp && mlp_cl_supported(d, F) && !getenv("TPPSD_MLP_SERIAL");
     for (int l = 0; l < m.L && p.mlp; ++l) {
         const LayerW& L = m.layer[l];
         p.mlp = make_tmap_bf16(&p.layer[l].wo_m, L.w_o, d, d, 128) &&

@@ -209,6 +209,7 @@ struct TcPlan {
     int enabled;
     int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
     int mlp;                    // post-attention block by the fused kernel
+    int mlp_cl;                 // ... in its cluster form (FFN split over F / 128 CTAs)
     int head;                   // heads by the tensor-core head kernel
     CUtensorMap head_hi, head_lo;
     int* err;
@@ -228,6 +229,9 @@ struct MlpArgs {
     int* err;
 };
 int mlp_tc_supported(int d, int F);
+int mlp_cl_supported(int d, int F);
+cudaError_t launch_mlp_cl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
+                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st);
 // att: tensor map of the attention output rows (box 64 x 128); wo / w1 / w2:
 // weight maps with boxes of 64 x 128.
 cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,

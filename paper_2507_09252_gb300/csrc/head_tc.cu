@@ -85,11 +85,24 @@ __global__ void __launch_bounds__(192, 1)
     } else {
         const int t = threadIdx.x;
         // A operands: h rows split into hi / lo bf16, written in the swizzled
-        // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7))
-        for (int f = t; f < S::BM * D / 4; f += 128) {
-            const int r = f >> 5, c4 = f & 31;
-            const float4 x = r < rows ? *reinterpret_cast<const float4*>(w.x + (size_t)(m0 + r) * D + 4 * c4)
-                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+        // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7)).
+        // Loads are issued in batches of 16 float4 per thread so that their
+        // latencies overlap (a load-convert-store loop would pay one global
+        // round trip per float4).
+        constexpr int NV = S::BM * D / 4 / 128, NB = 16;
+#pragma unroll 1
+        for (int b0 = 0; b0 < NV; b0 += NB) {
+            float4 xv[NB];
+#pragma unroll
+            for (int j = 0; j < NB; ++j) {
+                const int f = t + (b0 + j) * 128, r = f >> 5, c4 = f & 31;
+                xv[j] = r < rows ? *reinterpret_cast<const float4*>(w.x + (size_t)(m0 + r) * D + 4 * c4)
+                                 : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int j = 0; j < NB; ++j) {
+            const int f = t + (b0 + j) * 128, r = f >> 5, c4 = f & 31;
+            const float4 x = xv[j];
             const float xs[4] = {x.x, x.y, x.z, x.w};
             uint32_t hi[2], lo[2];
 #pragma unroll
@@ -104,6 +117,7 @@ __global__ void __launch_bounds__(192, 1)
             const int off = kb * S::TILE + r * 128 + ((ch ^ (r & 7)) << 4) + half * 8;
             *reinterpret_cast<uint2*>(smem + S::OFF_AH + off) = make_uint2(hi[0], hi[1]);
             *reinterpret_cast<uint2*>(smem + S::OFF_AL + off) = make_uint2(lo[0], lo[1]);
+            }
         }
         fence_proxy_async_smem();
         mbar_arrive(a_ready);
@@ -111,7 +125,17 @@ __global__ void __launch_bounds__(192, 1)
         // col0.. of the [d][3M+K] head map), its bias and b_k1 into shared memory
         const int M = m.M, K = m.K, WO = 3 * M + K;
         const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M;
-        for (int i = t; i < D * cnt; i += 128) ws[i] = m.head_out_t[(size_t)(i / cnt) * WO + col0 + i % cnt];
+        for (int i0 = t; i0 < D * cnt; i0 += 8 * 128) {  // batches of 8 loads per thread
+            float v[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int i = i0 + j * 128;
+                v[j] = i < D * cnt ? m.head_out_t[(size_t)(i / cnt) * WO + col0 + i % cnt] : 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (i0 + j * 128 < D * cnt) ws[i0 + j * 128] = v[j];
+        }
         for (int i = t; i < cnt; i += 128) ws[D * cnt + i] = m.head_out_b[col0 + i];
         for (int i = t; i < D; i += 128) ws[D * cnt + cnt + i] = m.head_ek_b[3 * D + i];
         asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps

@@ -1204,7 +1204,8 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
                 ma.b_1 = L.b_1; ma.b_2 = L.b_2; ma.ln2_g = L.ln2_g; ma.ln2_b = L.ln2_b;
                 ma.x = w.x; ma.xb = (bf16*)xb; ma.err = tc->err;
                 PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
-                e = launch_mlp_tc(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st);
+                e = tc->mlp_cl ? launch_mlp_cl(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st)
+                               : launch_mlp_tc(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st);
                 if (e != cudaSuccess) return e;
                 PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
                 nl += 3;

@@ -353,6 +353,361 @@ __global__ void __launch_bounds__(320, 1)
     pdl_trigger();
 }
 
+// ---------------------------------------------------------------------------
+// Cluster form of the same block: the F hidden columns are split over a
+// cluster of F / 128 CTAs (at most 8) that share one 128-row tile.  CTA c
+// of the cluster computes the output projection and LN1 of the tile (every
+// CTA the same values, the same instructions on the same inputs), FFN1
+// chunk c with its ReLU, and the partial FFN2 product of that chunk; CTA 0
+// adds x1 + b_2 to its partial.  The partials meet through distributed
+// shared memory: each CTA pushes row slice p of its partial to CTA p with
+// one bulk copy (into the weight region, free once every CTA's FFN2 is
+// done); CTA c sums rows 128c/n .. of all n partials (in CTA order),
+// applies LN2 and writes them.  The dependent chain of one CTA is
+// thus one FFN1 chunk and one FFN2 chunk instead of F / 128 of each, and
+// the weights a CTA streams drop to W_o plus 1/n of W_1 and W_2 (six tiles,
+// all in flight at once).  TMEM: 0-127 the output projection, then the
+// FFN2 partial; 128-255 the FFN1 chunk; 256-383 x1 in fp32.
+struct MlpClShape {
+    static constexpr int D = 128, BM = 128, BK = 64, CH = 128;
+    static constexpr int TILE = BM * BK * 2;
+    static constexpr int NT = 6;                           // W_o, W_1 chunk, W_2 chunk: 2 tiles each
+    static constexpr int RLD = D + 4;
+    static constexpr int OFF_A = 0;                        // attention tile, then x1 (bf16)
+    static constexpr int OFF_R = OFF_A + 2 * TILE;         // residual, then activations, then partial
+    static constexpr int R_BYTES = ((BM * RLD * 4 + 1023) / 1024) * 1024;
+    static constexpr int OFF_W = OFF_R + R_BYTES;
+    static constexpr int OFF_P = OFF_W + NT * TILE;        // b_o g1 be1 b_2 g2 be2 (D each), b_1 chunk
+    static constexpr int OFF_RED = OFF_P + (6 * D + CH) * 4;
+    static constexpr int OFF_B = OFF_RED + 4 * BM * 4;
+    static constexpr int NBAR = 14;
+    __host__ __device__ static constexpr int SLICE_BYTES(int ncl) { return (BM / ncl) * RLD * 4; }
+    static_assert(NT * TILE >= BM * RLD * 4, "the partial slices fit in the weight region");
+    static constexpr size_t SMEM = (size_t)OFF_B + NBAR * 8 + 16 + 1024;
+    static_assert(R_BYTES >= 2 * TILE, "the activation tile fits in the residual region");
+    static_assert(SMEM <= 227 * 1024, "shared memory");
+};
+
+template <int NCL>
+__global__ void __launch_bounds__(320, 1)
+    k_mlp_cl(const __grid_constant__ CUtensorMap mapAtt, const __grid_constant__ CUtensorMap mapWo,
+             const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2, MlpArgs a) {
+    using S = MlpClShape;
+    constexpr int D = S::D;
+    pdl_wait();
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    unsigned char* A = smem + S::OFF_A;
+    unsigned char* Rg = smem + S::OFF_R;
+    float* res = (float*)Rg;     // residual tile, later this CTA's FFN2 partial [BM][RLD]
+    unsigned char* Wt = smem + S::OFF_W;
+    float* prm = (float*)(smem + S::OFF_P);
+    float* red = (float*)(smem + S::OFF_RED);
+    uint64_t* bars = (uint64_t*)(smem + S::OFF_B);
+    uint64_t* full = bars;            // [NT] weight tile i landed
+    uint64_t* abar = bars + 6;        // attention tile landed
+    uint64_t* o_done = bars + 7;      // output projection in TMEM
+    uint64_t* x1_ready = bars + 8;    // x1 operand written (256 arrivals)
+    uint64_t* h_done = bars + 9;      // FFN1 chunk in TMEM
+    uint64_t* e2_done = bars + 10;    // chunk activations written (256 arrivals)
+    uint64_t* y_done = bars + 11;     // FFN2 partial in TMEM
+    uint64_t* rbar = bars + 12;       // the other CTAs' partial slices landed
+    uint32_t* tslot = (uint32_t*)(bars + 13);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int c = (int)cluster_ctarank();
+    const int m0 = blockIdx.y * S::BM, rows = min(S::BM, a.R - m0);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < S::NT; ++i) mbar_init(&full[i], 1);
+        mbar_init(abar, 1);
+        mbar_init(o_done, 1);
+        mbar_init(x1_ready, 256);
+        mbar_init(h_done, 1);
+        mbar_init(e2_done, 256);
+        mbar_init(y_done, 1);
+        mbar_init(rbar, 1);
+        mbar_fence_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, 512);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0) {  // every tile of this CTA at once: nothing is reused
+            mbar_arrive_expect_tx(abar, 2 * S::TILE);
+            tma_load_2d(A, &mapAtt, abar, 0, m0);
+            tma_load_2d(A + S::TILE, &mapAtt, abar, 64, m0);
+            const CUtensorMap* maps[S::NT] = {&mapWo, &mapWo, &mapW1, &mapW1, &mapW2, &mapW2};
+            const int xs[S::NT] = {0, 64, 0, 64, c * S::CH, c * S::CH + 64};
+            const int ys[S::NT] = {0, 0, c * S::CH, c * S::CH, 0, 0};
+            for (int i = 0; i < S::NT; ++i) {
+                mbar_arrive_expect_tx(&full[i], S::TILE);
+                tma_load_2d(Wt + i * S::TILE, maps[i], &full[i], xs[i], ys[i]);
+            }
+            if (NCL > 1) mbar_arrive_expect_tx(rbar, (uint32_t)(NCL - 1) * S::SLICE_BYTES(NCL));
+        }
+        __syncwarp();
+    } else if (warp == 9) {
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16(128, 128);
+            bool ok = true;
+            // D (+)= A (two 64-column k-blocks at a_addr) x W tiles i0, i0 + 1
+            auto mma_pair = [&](uint32_t a_addr, int i0, uint32_t d_tmem) {
+                for (int kb = 0; kb < 2; ++kb) {
+                    ok = ok && mbar_wait(&full[i0 + kb], 0, a.err, 61);
+                    if (!ok) return;
+                    tc_fence_after();
+                    const uint32_t b_addr = smem_u32(Wt + (i0 + kb) * S::TILE);
+#pragma unroll
+                    for (int kk = 0; kk < S::BK / 16; ++kk)
+                        tc_mma_bf16(d_tmem, sw128_desc(a_addr + kb * S::TILE + kk * 32),
+                                    sw128_desc(b_addr + kk * 32), idesc, (kb | kk) ? 1u : 0u);
+                }
+            };
+            const uint32_t a0 = smem_u32(A), r0 = smem_u32(Rg);
+            ok = mbar_wait(abar, 0, a.err, 62);
+            tc_fence_after();
+            mma_pair(a0, 0, tmem);
+            tc_commit(o_done);
+            ok = ok && mbar_wait(x1_ready, 0, a.err, 63);
+            tc_fence_after();
+            mma_pair(a0, 2, tmem + 128);
+            tc_commit(h_done);
+            ok = ok && mbar_wait(e2_done, 0, a.err, 64);
+            tc_fence_after();
+            mma_pair(r0, 4, tmem);
+            tc_commit(y_done);
+        }
+        __syncwarp();
+    } else {
+        // epilogue warps 0-7: row t = 32 (warp % 4) + lane, columns cb..cb+63
+        const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * 64;
+        const bool live = t < rows;
+        {   // residual tile and parameters; all loads issued before any store
+            constexpr int NV = S::BM * D / 4 / 256;
+            float4 v[NV];
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                v[k] = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            const float* src[6] = {a.b_o, a.ln1_g, a.ln1_b, a.b_2, a.ln2_g, a.ln2_b};
+            float pv[3];
+#pragma unroll
+            for (int k = 0; k < 3; ++k) {
+                const int i = tid + 256 * k;
+                pv[k] = src[i / D][i % D];
+            }
+            const float b1v = tid < S::CH ? a.b_1[c * S::CH + tid] : 0.f;
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                *reinterpret_cast<float4*>(res + r * S::RLD + 4 * c4) = v[k];
+            }
+#pragma unroll
+            for (int k = 0; k < 3; ++k) prm[tid + 256 * k] = pv[k];
+            if (tid < S::CH) prm[6 * D + tid] = b1v;
+        }
+        epi_sync();
+        const float *p_bo = prm + cb, *p_g1 = prm + D + cb, *p_be1 = prm + 2 * D + cb, *p_b2 = prm + 3 * D + cb;
+        const float* p_b1 = prm + 6 * D + cb;
+        const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
+        float* xr = res + t * S::RLD + cb;
+        float y[64];
+        mbar_wait(o_done, 0, a.err, 65);
+        tc_fence_after();
+        tmem_ld64(tl + cb, y);
+#pragma unroll
+        for (int cc = 0; cc < 64; cc += 4) {
+            const float4 r4 = *reinterpret_cast<const float4*>(xr + cc);
+            y[cc] += p_bo[cc] + r4.x;
+            y[cc + 1] += p_bo[cc + 1] + r4.y;
+            y[cc + 2] += p_bo[cc + 2] + r4.z;
+            y[cc + 3] += p_bo[cc + 3] + r4.w;
+        }
+        {   // LN1 (row halves held by the thread pairs hh = 0 / 1)
+            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+            for (int cc = 0; cc < 64; cc += 4) {
+                s0 += y[cc];
+                s1 += y[cc + 1];
+                s2 += y[cc + 2];
+                s3 += y[cc + 3];
+            }
+            red[hh * S::BM + t] = (s0 + s1) + (s2 + s3);
+            epi_sync();
+            const float mean = (red[t] + red[S::BM + t]) / D;
+            s0 = s1 = s2 = s3 = 0.f;
+#pragma unroll
+            for (int cc = 0; cc < 64; cc += 4) {
+                s0 = fmaf(y[cc] - mean, y[cc] - mean, s0);
+                s1 = fmaf(y[cc + 1] - mean, y[cc + 1] - mean, s1);
+                s2 = fmaf(y[cc + 2] - mean, y[cc + 2] - mean, s2);
+                s3 = fmaf(y[cc + 3] - mean, y[cc + 3] - mean, s3);
+            }
+            red[(2 + hh) * S::BM + t] = (s0 + s1) + (s2 + s3);
+            epi_sync();  // also ends every read of the residual tile
+            const float inv = 1.0f / sqrtf((red[2 * S::BM + t] + red[3 * S::BM + t]) / D + LN_EPS);
+#pragma unroll
+            for (int cc = 0; cc < 64; ++cc) y[cc] = live ? (y[cc] - mean) * inv * p_g1[cc] + p_be1[cc] : 0.f;
+        }
+        tmem_st64(tl + 256 + cb, y);
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(A, t, cb + c0, y + c0);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(x1_ready);
+        // FFN1 chunk c: ReLU(H + b_1) -> bf16 operand of FFN2 (residual region)
+        mbar_wait(h_done, 0, a.err, 66);
+        tc_fence_after();
+        tmem_ld64(tl + 128 + cb, y);
+#pragma unroll
+        for (int cc = 0; cc < 64; ++cc) y[cc] = fmaxf(y[cc] + p_b1[cc], 0.f);
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(Rg, t, cb + c0, y + c0);
+        fence_proxy_async_smem();
+        tc_fence_before();
+        mbar_arrive(e2_done);
+        // this CTA's FFN2 partial (CTA 0: + b_2 + x1) into the residual region
+        mbar_wait(y_done, 0, a.err, 67);
+        tc_fence_after();
+        tmem_ld64(tl + cb, y);
+        if (c == 0) {
+            float x1[64];
+            tmem_ld64(tl + 256 + cb, x1);
+#pragma unroll
+            for (int cc = 0; cc < 64; ++cc) y[cc] += p_b2[cc] + x1[cc];
+        }
+#pragma unroll
+        for (int cc = 0; cc < 64; cc += 4)
+            *reinterpret_cast<float4*>(xr + cc) = make_float4(y[cc], y[cc + 1], y[cc + 2], y[cc + 3]);
+        fence_proxy_async_smem();  // the bulk copies below read these writes
+    }
+    // every partial of the cluster is in shared memory and every CTA's
+    // weight region is free
+    cluster_sync();
+    if (threadIdx.x == 0 && NCL > 1) {  // slice p of this partial -> slot c of CTA p's weight region
+        for (int p = 0; p < NCL; ++p)
+            if (p != c)
+                bulk_s2peer(Wt + (size_t)c * S::SLICE_BYTES(NCL), res + p * (S::BM / NCL) * S::RLD,
+                            (uint32_t)S::SLICE_BYTES(NCL), rbar, (uint32_t)p);
+        bulk_commit();
+    }
+    if (warp < 8) {
+        // rows c RW .. c RW + RW - 1 of the tile: TPR threads per row, CPT columns each
+        constexpr int RW = S::BM / NCL, TPR = 256 / RW, CPT = D / TPR;
+        const int tid = threadIdx.x, rr = tid / TPR, col = (tid % TPR) * CPT, r = c * RW + rr;
+        const float *p_g2 = prm + 4 * D, *p_be2 = prm + 5 * D;
+        // slice of CTA pr: this CTA's own partial for pr = c, else slot pr
+        // of the weight region (all loads before the first sum)
+        if (NCL > 1) mbar_wait(rbar, 0, a.err, 68);
+        const float* wslots = reinterpret_cast<const float*>(Wt);
+        float4 ld[NCL][CPT / 4];
+#pragma unroll
+        for (int pr = 0; pr < NCL; ++pr) {
+            const float* src = pr == c ? res + r * S::RLD + col : wslots + (pr * RW + rr) * S::RLD + col;
+#pragma unroll
+            for (int j = 0; j < CPT / 4; ++j) ld[pr][j] = *reinterpret_cast<const float4*>(src + 4 * j);
+        }
+        float v[CPT];
+#pragma unroll
+        for (int j = 0; j < CPT / 4; ++j) {
+            v[4 * j] = ld[0][j].x; v[4 * j + 1] = ld[0][j].y; v[4 * j + 2] = ld[0][j].z; v[4 * j + 3] = ld[0][j].w;
+        }
+#pragma unroll
+        for (int pr = 1; pr < NCL; ++pr)
+#pragma unroll
+            for (int j = 0; j < CPT / 4; ++j) {
+                v[4 * j] += ld[pr][j].x; v[4 * j + 1] += ld[pr][j].y;
+                v[4 * j + 2] += ld[pr][j].z; v[4 * j + 3] += ld[pr][j].w;
+            }
+        // LN2: row sums over the TPR consecutive lanes of the row
+        float sm = 0.f;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) sm += v[j];
+#pragma unroll
+        for (int o = TPR >> 1; o > 0; o >>= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+        const float mean = sm / D;
+        float sq = 0.f;
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) sq = fmaf(v[j] - mean, v[j] - mean, sq);
+#pragma unroll
+        for (int o = TPR >> 1; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+        const float inv = 1.0f / sqrtf(sq / D + LN_EPS);
+        if (r < rows) {
+            float* xo = a.x + (size_t)(m0 + r) * D + col;
+            bf16* xbo = a.xb + (size_t)(m0 + r) * D + col;
+#pragma unroll
+            for (int j = 0; j < CPT; j += 4) {
+                float4 o;
+                o.x = (v[j] - mean) * inv * p_g2[col + j] + p_be2[col + j];
+                o.y = (v[j + 1] - mean) * inv * p_g2[col + j + 1] + p_be2[col + j + 1];
+                o.z = (v[j + 2] - mean) * inv * p_g2[col + j + 2] + p_be2[col + j + 2];
+                o.w = (v[j + 3] - mean) * inv * p_g2[col + j + 3] + p_be2[col + j + 3];
+                *reinterpret_cast<float4*>(xo + j) = o;
+                const __nv_bfloat162 p0 = __floats2bfloat162_rn(o.x, o.y);
+                const __nv_bfloat162 p1 = __floats2bfloat162_rn(o.z, o.w);
+                uint2 w;
+                w.x = *reinterpret_cast<const uint32_t*>(&p0);
+                w.y = *reinterpret_cast<const uint32_t*>(&p1);
+                *reinterpret_cast<uint2*>(xbo + j) = w;
+            }
+        }
+    }
+    // the sources of this CTA's bulk copies have been read before it exits;
+    // its own slots were all filled (rbar) before the sums above
+    if (threadIdx.x == 0 && NCL > 1) bulk_wait_read_all();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tmem, 512);
+    pdl_trigger();
+}
+
+int mlp_cl_supported(int d, int F) {
+    const int n = F / MlpClShape::CH;
+    return d == MlpClShape::D && F % MlpClShape::CH == 0 && (n == 1 || n == 2 || n == 4 || n == 8);
+}
+
+template <int NCL>
+static cudaError_t launch_mlp_ncl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
+                                  const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st) {
+    const size_t sm = MlpClShape::SMEM;
+    cudaError_t e = cudaFuncSetAttribute(k_mlp_cl<NCL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+    if (e != cudaSuccess) return e;
+    const int ncl = NCL;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(ncl, (a.R + 127) / 128, 1);
+    cfg.blockDim = dim3(320, 1, 1);
+    cfg.dynamicSmemBytes = sm;
+    cfg.stream = st;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = ncl;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = g_pdl ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, k_mlp_cl<NCL>, att, wo, w1, w2, a);
+}
+
+cudaError_t launch_mlp_cl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
+                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st) {
+    if (a.R <= 0) return cudaSuccess;
+    if (!mlp_cl_supported(MlpClShape::D, a.F)) return cudaErrorInvalidValue;
+    switch (a.F / MlpClShape::CH) {
+        case 1: return launch_mlp_ncl<1>(att, wo, w1, w2, a, st);
+        case 2: return launch_mlp_ncl<2>(att, wo, w1, w2, a, st);
+        case 4: return launch_mlp_ncl<4>(att, wo, w1, w2, a, st);
+        case 8: return launch_mlp_ncl<8>(att, wo, w1, w2, a, st);
+    }
+    return cudaErrorInvalidValue;
+}
+
 int mlp_tc_supported(int d, int F) { return d == MlpShape::D && F % MlpShape::CH == 0 && F <= MlpShape::PF; }
 
 cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,

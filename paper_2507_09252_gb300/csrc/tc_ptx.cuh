@@ -203,6 +203,35 @@ __device__ __forceinline__ float ld_dsmem_f32(const float* local, uint32_t rank)
     return v;
 }
 
+// 16-byte load from the same shared-memory offset in CTA `rank` of the
+// cluster (address 16-byte aligned).
+__device__ __forceinline__ float4 ld_dsmem_f32x4(const float* local, uint32_t rank) {
+    uint32_t ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(smem_u32(local)), "r"(rank));
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(ra) : "memory");
+    return v;
+}
+
+// Bulk copy of `bytes` (16-byte aligned, multiple of 16) from this CTA's
+// shared memory to CTA `rank` of the cluster: dst_local and bar_local are
+// offsets in this CTA's shared window, mapped to the same offsets in the
+// peer; the copy completes transaction bytes on the peer's mbarrier.
+__device__ __forceinline__ void bulk_s2peer(void* dst_local, const void* src, uint32_t bytes, uint64_t* bar_local,
+                                            uint32_t rank) {
+    uint32_t d, b;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(d) : "r"(smem_u32(dst_local)), "r"(rank));
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(b) : "r"(smem_u32(bar_local)), "r"(rank));
+    asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+                 ::"r"(d), "r"(smem_u32(src)), "r"(bytes), "r"(b)
+                 : "memory");
+}
+// Groups of this thread's bulk copies: commit, then wait until their
+// sources have been read (the shared memory may then be reused or freed).
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+
 // Shared-memory matrix descriptor of a K-major operand tile laid out by TMA
 // with 128-byte swizzling: rows of 128 B (64 bf16), 8-row groups 1024 B
 // apart (stride byte offset), tile base 1024-byte aligned.

@@ -81,6 +81,17 @@ def test_score_parity_fp32_large_shapes(idx, B, n):
     _score_case(tcfg, dcfg, bt, bd, B, n, tcfg.n_marks, G.TOL_FP32, rel_logg=True)
 
 
+@pytest.mark.parametrize("F", [128, 256, 1024])
+def test_score_parity_bf16_d128_ffn_widths(F):
+    """d = 128 bf16 targets whose FFN width gives 1, 2 and 8 FFN chunks (the
+    cluster sizes of the fused post-attention block; the headline width 512
+    is covered above), over 5 row tiles with a ragged last one."""
+    tcfg = CF.ModelCfg(2, 128, 4, F, 8, 5, CF.BF16)
+    dcfg = CF.ModelCfg(1, 32, 2, 128, 8, 5, CF.BF16)
+    bt, bd = IN.model_blob(tcfg, 3, 0, head_gain=2.0), IN.model_blob(dcfg, 3, 1)
+    _score_case(tcfg, dcfg, bt, bd, 2, 300, 5, G.TOL_BF16)
+
+
 def test_score_parity_sweep_drafts():
     wl = CF.C5
     bt = IN.model_blob(wl.target, 0, 0)
