@@ -150,17 +150,20 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- roofline
-def roofline(kt, stats, wl, peaks):
-    """Dominant kernel class of a profiled SD call, with its algorithmic
-    bytes (or FLOPs) per launch.
+def class_roofline(name, ms, launches, stats, wl, peaks, fused):
+    """Algorithmic bytes (or FLOPs) per launch of one kernel class of a
+    profiled SD call ÷ its mean CUDA-event time, against the measured peak.
 
     attention:  K and V of every cached position read once per (sequence,
                 layer) + Q read + output write:  target_keys * 2 d eb + 2 R d eb
     draft:      draft K/V of each sequence loaded once per round (the kernel
                 keeps it in shared memory for the round) + draft heads
                 written + the draft model once per launch (L2-resident)
-    gemm_*:     2 R N K FLOPs per layer (tcgen05 bf16 path for bf16 models)
-    others:     bytes of their inputs and outputs
+    gemm_*:     2 R N K FLOPs per layer (tcgen05 bf16 path for bf16 models);
+                the fused post-attention block (timed as gemm_ffn2) does
+                2 R (d^2 + 2 d F)
+    head:       h rows read + head rows written + head weights
+    others:     bytes of the rows they read and write (latency-bound)
     """
     T, D = wl.target, wl.draft
     eb = 2 if T.dtype == CF.BF16 else 4
@@ -168,7 +171,6 @@ def roofline(kt, stats, wl, peaks):
     rows = rounds * (wl.gamma + 1)                   # verify rows over the call
     d, F, L = T.d_model, T.d_ffn, T.layers
     W = 3 * T.n_mix + T.n_marks
-    name, (ms, launches) = max(((k, v) for k, v in kt.items() if v[1] > 0), key=lambda kv: kv[1][0])
     per_launch_s = ms / 1e3 / max(launches, 1)
     bound, unit = "hbm", "GB/s"
     if name == "attention":
@@ -185,24 +187,42 @@ def roofline(kt, stats, wl, peaks):
     elif name.startswith("gemm"):
         nk = {"gemm_qkv": (3 * d, d), "gemm_o": (d, d), "gemm_ffn1": (F, d), "gemm_ffn2": (d, F)}[name]
         total = 2.0 * rows * nk[0] * nk[1] * L
+        if name == "gemm_ffn2" and fused:
+            total = 2.0 * rows * (d * d + 2 * d * F) * L
         bound, unit = "tensor", "TFLOP/s"
     else:
         total = rows * d * 4 * 2
+        bound = "latency"
     per_launch = total / max(launches, 1)
-    if bound == "hbm":
-        achieved = per_launch / per_launch_s / 1e9
-        peak = peaks.get("hbm_gbs", 6800.0)
-    else:
+    if bound == "tensor":
         achieved = per_launch / per_launch_s / 1e12
         # dense bf16 tensor peak, sustained (the kernel runs inside a long step)
         peak = peaks.get("bf16_tflops_sustained", 1700.0)
-    share = ms / sum(v[0] for v in kt.values())
-    return {"kernel": name, "bound": bound, "achieved": round(achieved, 2), "peak": round(peak, 1),
-            "unit": unit, "frac": round(achieved / peak, 4), "traffic": ncu_traffic(name),
-            "per_launch_ms": round(per_launch_s * 1e3, 4), "launches": launches,
-            "share_of_device_time": round(share, 3),
-            "algorithmic_per_launch": per_launch,
-            "peak_source": "MEASURED_PEAKS.json" if peaks else "fallback"}
+    else:
+        achieved = per_launch / per_launch_s / 1e9
+        peak = peaks.get("hbm_gbs", 6800.0)
+    return {"bound": bound, "achieved": round(achieved, 2), "peak": round(peak, 1), "unit": unit,
+            "frac": round(achieved / peak, 4), "per_launch_ms": round(per_launch_s * 1e3, 4),
+            "launches": launches, "algorithmic_per_launch": per_launch}
+
+
+def roofline(kt, stats, wl, peaks):
+    """The dominant kernel class of a profiled SD call (largest share of the
+    device time) with its roofline, plus every class's own figures."""
+    fused = kt.get("gemm_o", (0.0, 0))[1] == 0 and kt.get("gemm_ffn2", (0.0, 0))[1] > 0
+    live = {k: v for k, v in kt.items() if v[1] > 0}
+    tot = sum(v[0] for v in live.values())
+    per = {k: {**class_roofline(k, ms, n, stats, wl, peaks, fused), "share_of_device_time": round(ms / tot, 3)}
+           for k, (ms, n) in live.items()}
+    name = max(live, key=lambda k: live[k][0])
+    top = per[name]
+    dom = {"kernel": name, "bound": "hbm" if top["bound"] == "latency" else top["bound"],
+           "achieved": top["achieved"], "peak": top["peak"], "unit": top["unit"], "frac": top["frac"],
+           "traffic": ncu_traffic(name), "per_launch_ms": top["per_launch_ms"], "launches": top["launches"],
+           "share_of_device_time": top["share_of_device_time"],
+           "algorithmic_per_launch": top["algorithmic_per_launch"],
+           "peak_source": "MEASURED_PEAKS.json" if peaks else "fallback"}
+    return dom, per
 
 
 def ncu_traffic(kernel_class):
@@ -377,7 +397,7 @@ def main():
     kt = T.tppsd_kernel_times(s.ctx)
     _, st_prof = T.tppsd_get_stats(s.ctx)
     peaks = load_peaks()
-    roof = roofline(kt, st_prof, wl, peaks)
+    roof, per_class = roofline(kt, st_prof, wl, peaks)
 
     events = world * B * N
     value = job_rate(world, B, N, ms_sd)
@@ -404,6 +424,9 @@ def main():
         "gpu_launches": args.steps * (st_sd["kernel_launches"] + st_sd["prefill_launches"]),
         "clocks": clk.summary(),
         "roofline": roof,
+        "kernel_roofline": {k: {kk: v[kk] for kk in ("bound", "achieved", "peak", "unit", "frac",
+                                                     "per_launch_ms", "share_of_device_time")}
+                            for k, v in sorted(per_class.items(), key=lambda kv: -kv[1]["share_of_device_time"])},
         "kernel_ms": {k: round(v[0], 3) for k, v in kt.items() if v[1]},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

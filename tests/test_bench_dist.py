@@ -88,3 +88,26 @@ def test_traffic_record_is_dropped_when_a_source_changes(tmp_path, monkeypatch):
     assert bench.ncu_traffic("attention") is None
     src.write_text("kernel v2")
     assert bench.ncu_traffic("draft") is None
+
+
+def test_roofline_reports_every_class():
+    """bench.py's roofline: the dominant class (largest device time) with
+    its algorithmic figure, and every class's own fraction; the fused
+    post-attention block counts O-proj + FFN1 + FFN2 FLOPs."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2507_09252_gb300 import configs as CF
+    kt = {"draft": (7.0, 70), "attention": (5.5, 280), "gemm_ffn2": (4.7, 280), "gemm_qkv": (2.8, 280),
+          "head": (1.4, 70), "epilogue": (1.1, 70), "control": (0.4, 70), "gemm_o": (0.0, 0)}
+    stats = {"rounds": 16376, "drafted": 131008, "accepted": 115668, "target_keys": 5340083}
+    peaks = {"hbm_gbs": 6682.5, "bf16_tflops_sustained": 1772.7}
+    dom, per = bench.roofline(kt, stats, CF.C2, peaks)
+    assert dom["kernel"] == "draft" and dom["unit"] == "GB/s" and 0 < dom["frac"] < 1
+    assert set(per) == {k for k, v in kt.items() if v[1]}
+    T = CF.C2.target
+    rows = stats["rounds"] * (CF.C2.gamma + 1)
+    flops = 2.0 * rows * (T.d_model ** 2 + 2 * T.d_model * T.d_ffn) * T.layers / 280
+    assert per["gemm_ffn2"]["bound"] == "tensor"
+    assert per["gemm_ffn2"]["achieved"] == pytest.approx(flops / (4.7e-3 / 280) / 1e12, rel=1e-3)
+    assert per["control"]["bound"] == "latency"
+    assert abs(sum(v["share_of_device_time"] for v in per.values()) - 1.0) < 0.01
