@@ -72,6 +72,8 @@ def lib():
                                              _f64p, _f64p, _i32p, _f64p, _i32p, _i64p, C.c_int32]
         L.oracle_score_survival.argtypes = [_i32p, _f32p, C.c_int64, C.c_int32, C.c_int32, _f32p,
                                             _i32p, C.c_double, _f64p, C.c_int32, C.c_int32]
+        L.oracle_model_temporal_encoding.argtypes = [_i32p, _f32p, C.c_int64, C.c_double, _f64p]
+        L.oracle_model_temporal_encoding.restype = C.c_int
         L.oracle_log_survival.argtypes = [C.c_int32, _f64p, C.c_double]
         L.oracle_log_survival.restype = C.c_double
         L.oracle_sample_sd_poisson_until.argtypes = [
@@ -96,7 +98,7 @@ def lib():
 
 def _cfg(cfg):
     return np.array([cfg.layers, cfg.d_model, cfg.heads, cfg.d_ffn, cfg.n_mix, cfg.n_marks,
-                     cfg.dtype], np.int32)
+                     cfg.dtype, getattr(cfg, "encoder", 0)], np.int32)
 
 
 def _c(a, dt):
@@ -235,6 +237,14 @@ def score_survival(cfg, blob, tau, marks, t_end, recompute=False, nthreads=0):
 def log_survival(M, head, u):
     """log(1 - G(u)) of one head's log-normal mixture."""
     return lib().oracle_log_survival(M, _c(head, np.float64), float(u))
+
+
+def model_temporal_encoding(cfg, blob, t):
+    """z(t) of a model's encoder (THP, SAHP or AttNHP form)."""
+    out = np.zeros(cfg.d_model)
+    _check(lib().oracle_model_temporal_encoding(_cfg(cfg), _c(blob, np.float32), blob.size, float(t), out),
+           "oracle_model_temporal_encoding")
+    return out
 
 
 def log_g(M, head, tau):

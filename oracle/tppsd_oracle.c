@@ -78,31 +78,47 @@ typedef struct {
 
 typedef struct {
     int L, d, nh, F, M, K, bf16;
+    int enc;                       /* 0 THP, 1 SAHP, 2 AttNHP (App. D.4) */
     const float *type_emb;
+    const float *tenc_w;           /* SAHP: per-dimension frequencies w_j [d] */
+    double scale_m, scale_M;       /* AttNHP: time scales m, M */
     layer_p layer[64];
     const float *E, *v_w, *b_w, *v_mu, *b_mu, *v_s, *b_s, *v_k1, *b_k1, *v_k2, *b_k2;
 } model_t;
 
-static int64_t model_floats(const int32_t c[7])
+/* Blob size of a model: THP and SAHP layers carry QKV, the output
+ * projection, two LayerNorms and the FFN; AttNHP layers only QKV over the
+ * 2d inputs [z(t); h].  SAHP appends w_j [d], AttNHP its scales (m, M). */
+static int64_t model_floats(const int32_t c[8])
 {
-    int64_t L = c[0], d = c[1], F = c[3], M = c[4], K = c[5];
-    int64_t per_layer = 3 * d * d + 3 * d + d * d + d + 2 * d + F * d + F + d * F + d + 2 * d;
-    return K * d + L * per_layer + 3 * d * d + 3 * (M * d + M) + d * d + d + K * d + K;
+    int64_t L = c[0], d = c[1], F = c[3], M = c[4], K = c[5], enc = c[7];
+    int64_t per_layer = enc == 2 ? 3 * d * 2 * d + 3 * d
+                                 : 3 * d * d + 3 * d + d * d + d + 2 * d + F * d + F + d * F + d + 2 * d;
+    int64_t tail = enc == 1 ? d : enc == 2 ? 2 : 0;
+    return K * d + L * per_layer + 3 * d * d + 3 * (M * d + M) + d * d + d + K * d + K + tail;
 }
 
-static int model_init(model_t *m, const int32_t c[7], const float *blob, int64_t n)
+static int model_init(model_t *m, const int32_t c[8], const float *blob, int64_t n)
 {
     if (c[0] < 1 || c[0] > 64 || c[1] < 2 || c[1] > 512 || c[1] % 2 || c[2] < 1 || c[1] % c[2] ||
-        c[3] < 1 || c[4] < 1 || c[4] > MAXM || c[5] < 1 || c[5] > MAXK)
+        c[3] < 1 || c[4] < 1 || c[4] > MAXM || c[5] < 1 || c[5] > MAXK || c[7] < 0 || c[7] > 2)
         return -1;
     if (model_floats(c) != n) return -2;
     m->L = c[0]; m->d = c[1]; m->nh = c[2]; m->F = c[3]; m->M = c[4]; m->K = c[5];
     m->bf16 = c[6] == 1;
+    m->enc = c[7];
+    m->tenc_w = NULL;
+    m->scale_m = m->scale_M = 0.0;
     int d = m->d, F = m->F, M = m->M, K = m->K;
     const float *p = blob;
     m->type_emb = p; p += (int64_t)K * d;
     for (int l = 0; l < m->L; ++l) {
         layer_p *q = &m->layer[l];
+        memset(q, 0, sizeof(*q));
+        if (m->enc == 2) {
+            q->w_qkv = p; p += 3 * d * 2 * d;  q->b_qkv = p; p += 3 * d;
+            continue;
+        }
         q->w_qkv = p; p += 3 * d * d;  q->b_qkv = p; p += 3 * d;
         q->w_o = p; p += d * d;        q->b_o = p; p += d;
         q->ln1_g = p; p += d;          q->ln1_b = p; p += d;
@@ -116,6 +132,11 @@ static int model_init(model_t *m, const int32_t c[7], const float *blob, int64_t
     m->v_s = p; p += M * d;  m->b_s = p; p += M;
     m->v_k1 = p; p += d * d; m->b_k1 = p; p += d;
     m->v_k2 = p; p += K * d; m->b_k2 = p; p += K;
+    if (m->enc == 1) { m->tenc_w = p; p += d; }
+    if (m->enc == 2) {
+        m->scale_m = p[0]; m->scale_M = p[1]; p += 2;
+        if (!(m->scale_m > 0.0) || !(m->scale_M > 0.0)) return -1;
+    }
     return (p - blob) == n ? 0 : -2;
 }
 
@@ -160,6 +181,39 @@ void oracle_temporal_encoding(int32_t d, double t, double *out)
         double arg = t / pow(10000.0, (double)je / (double)d);
         out[j] = (j & 1) ? cos(arg) : sin(arg);
     }
+}
+
+/* Temporal encoding of a model (App. D.4), j 0-based, je = j - (j mod 2):
+ *   THP:    sin / cos (t / 10000^{je/D})                 (even / odd j)
+ *   SAHP:   sin / cos (j / 10000^{je/D} + w_j t)
+ *   AttNHP: sin / cos (t / (m (5M/m)^{je/D}))
+ * Readings: the AttNHP formula's "t/m * (5M/m)^{j/D}" is taken as t divided
+ * by the wavelength m (5M/m)^{j/D} (wavelengths from m to 5M), and its odd
+ * dimensions as cos (the printed sin on both lines would duplicate every
+ * pair). */
+static void model_temporal_encoding(const model_t *m, double t, double *out)
+{
+    int d = m->d;
+    for (int j = 0; j < d; ++j) {
+        int je = j - (j & 1);
+        double arg;
+        if (m->enc == 1)
+            arg = (double)j / pow(10000.0, (double)je / (double)d) + (double)m->tenc_w[j] * t;
+        else if (m->enc == 2)
+            arg = t / (m->scale_m * pow(5.0 * m->scale_M / m->scale_m, (double)je / (double)d));
+        else
+            arg = t / pow(10000.0, (double)je / (double)d);
+        out[j] = (j & 1) ? cos(arg) : sin(arg);
+    }
+}
+
+int oracle_model_temporal_encoding(const int32_t cfg[8], const float *blob, int64_t blob_floats,
+                                   double t, double *out)
+{
+    model_t m;
+    if (model_init(&m, cfg, blob, blob_floats)) return -1;
+    model_temporal_encoding(&m, t, out);
+    return 0;
 }
 
 /* ------------------------------------------------------------------ */
@@ -370,10 +424,49 @@ static void encode_position(tstate *s, int pos, double t, int k, double *h)
     double xin[512], qkv[3 * 512], att[512], tmp[512], *hid;
     hid = (double *)malloc(sizeof(double) * F * 2);
     double *hin = hid + F;
-    oracle_temporal_encoding(d, t, h);
-    for (int i = 0; i < d; ++i) h[i] += (double)m->type_emb[(int64_t)k * d + i];
+    double z[512], u[1024];
+    model_temporal_encoding(m, t, z);
+    for (int i = 0; i < d; ++i) h[i] = z[i] + (double)m->type_emb[(int64_t)k * d + i];
     double scale = 1.0 / sqrt((double)dh);
     double *sc = (double *)malloc(sizeof(double) * (pos + 1));
+    if (m->enc == 2) {
+        /* AttNHP layer (App. D.4): q, k, v = W [1; z(t); h] (the 1 is the
+         * bias), per head a = sum_j f_j v_j / (1 + sum_j f_j) with
+         * f_j = exp(q k_j / sqrt(d_head)) over keys j <= pos, then
+         * h <- h + tanh(a) (heads concatenated; no output projection,
+         * LayerNorm or FFN).  bf16 rounding at the GEMM input [z; h] and of
+         * q, k, v. */
+        for (int l = 0; l < m->L; ++l) {
+            const layer_p *P = &m->layer[l];
+            double *Kl = s->K + (size_t)l * s->cap * d, *Vl = s->V + (size_t)l * s->cap * d;
+            for (int i = 0; i < d; ++i) { u[i] = rnd(m, z[i]); u[d + i] = rnd(m, h[i]); }
+            linear(P->w_qkv, P->b_qkv, u, 2 * d, 3 * d, qkv);
+            for (int i = 0; i < 3 * d; ++i) qkv[i] = rnd(m, qkv[i]);
+            memcpy(Kl + (size_t)pos * d, qkv + d, sizeof(double) * d);
+            memcpy(Vl + (size_t)pos * d, qkv + 2 * d, sizeof(double) * d);
+            for (int hh = 0; hh < nh; ++hh) {
+                const double *q = qkv + hh * dh;
+                double mx = 0.0;                    /* the "1" term: exp(0) */
+                for (int j = 0; j <= pos; ++j) {
+                    double a = 0.0;
+                    for (int c = 0; c < dh; ++c) a += q[c] * Kl[(size_t)j * d + hh * dh + c];
+                    sc[j] = a * scale;
+                    if (sc[j] > mx) mx = sc[j];
+                }
+                double den = exp(-mx);
+                for (int j = 0; j <= pos; ++j) { sc[j] = exp(sc[j] - mx); den += sc[j]; }
+                for (int c = 0; c < dh; ++c) {
+                    double a = 0.0;
+                    for (int j = 0; j <= pos; ++j) a += sc[j] * Vl[(size_t)j * d + hh * dh + c];
+                    att[hh * dh + c] = a / den;
+                }
+            }
+            for (int i = 0; i < d; ++i) h[i] += tanh(att[i]);
+        }
+        free(sc);
+        free(hid);
+        return;
+    }
     for (int l = 0; l < m->L; ++l) {
         const layer_p *P = &m->layer[l];
         double *Kl = s->K + (size_t)l * s->cap * d, *Vl = s->V + (size_t)l * s->cap * d;
@@ -652,7 +745,7 @@ static void store_out(const evbuf *ev, int H, int N, int c, int64_t b, double *o
     }
 }
 
-int oracle_sample_ar_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_ar_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
                            int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                            int32_t N, double t_end, uint64_t seed, int32_t recompute,
                            const int32_t *seq_ids, double *out_tau, double *out_t, int32_t *out_k,
@@ -679,8 +772,8 @@ int oracle_sample_ar_until(const int32_t cfgT[7], const float *blobT, int64_t nT
     return 0;
 }
 
-int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                           const int32_t cfgD[7], const float *blobD, int64_t nD,
+int oracle_sample_sd_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
+                           const int32_t cfgD[8], const float *blobD, int64_t nD,
                            int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                            int32_t N, double t_end, int32_t gamma, uint64_t seed, uint32_t flags,
                            int32_t recompute, const int32_t *seq_ids,
@@ -714,7 +807,7 @@ int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT
 
 /* TPP-SD with the Poisson draft of App. D.3 (rate lambda, mark
  * probabilities p[K]) in place of the draft Transformer. */
-int oracle_sample_sd_poisson_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_sd_poisson_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
                                    int32_t B, int32_t H, const float *hist_tau,
                                    const int32_t *hist_marks, int32_t N, double t_end,
                                    int32_t gamma, double lambda, const double *p_marks,
@@ -749,7 +842,7 @@ int oracle_sample_sd_poisson_until(const int32_t cfgT[7], const float *blobT, in
     return 0;
 }
 
-int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_ar(const int32_t cfgT[8], const float *blobT, int64_t nT,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
@@ -759,8 +852,8 @@ int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
                                   recompute, seq_ids, out_tau, out_t, out_k, out_margin, NULL, nthreads);
 }
 
-int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                     const int32_t cfgD[7], const float *blobD, int64_t nD,
+int oracle_sample_sd(const int32_t cfgT[8], const float *blobT, int64_t nT,
+                     const int32_t cfgD[8], const float *blobD, int64_t nD,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
                      const int32_t *seq_ids,
@@ -775,7 +868,7 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
 /* Survival term of the log-likelihood on [0, t_end] (Sec. 3.1, Eq. 2) of
  * each sequence's len events: log S(t_end - t_{len-1} | h_{len-1}) from the
  * head after the last event. */
-int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+int oracle_score_survival(const int32_t cfg[8], const float *blob, int64_t blob_floats,
                           int32_t B, int32_t len, const float *tau, const int32_t *marks,
                           double t_end, double *out_logS, int32_t recompute, int32_t nthreads)
 {
@@ -798,7 +891,7 @@ int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_
     return 0;
 }
 
-int oracle_score(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+int oracle_score(const int32_t cfg[8], const float *blob, int64_t blob_floats,
                  int32_t B, int32_t len, const float *tau, const int32_t *marks,
                  double *out_heads, double *out_logg, double *out_logf,
                  int32_t recompute, int32_t nthreads)

@@ -18,14 +18,19 @@
 extern "C" {
 #endif
 
-/* cfg[7] = {layers, d_model, heads, d_ffn, n_mix, n_marks, dtype}; dtype 0 =
- * fp64 everywhere, 1 = bf16 rounding emulated at the GEMM inputs and of
- * Q/K/V (the points the CUDA path rounds at), all else fp64. */
+/* cfg[8] = {layers, d_model, heads, d_ffn, n_mix, n_marks, dtype, encoder};
+ * dtype 0 = fp64 everywhere, 1 = bf16 rounding emulated at the GEMM inputs
+ * and of Q/K/V (the points the CUDA path rounds at), all else fp64;
+ * encoder 0 = THP, 1 = SAHP, 2 = AttNHP (App. D.4). */
 
 /* Philox4x32-10 (Salmon et al., SC'11): one block of four 32-bit words. */
 void oracle_philox4x32(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
 /* The four uniforms in (0,1) of slot (seed, seq, pos, block). */
 void oracle_uniforms(uint64_t seed, uint32_t seq, uint32_t pos, uint32_t block, double u[4]);
+
+/* The model's temporal encoding z(t) (THP, SAHP or AttNHP form), d values. */
+int oracle_model_temporal_encoding(const int32_t cfg[8], const float *blob, int64_t blob_floats,
+                                   double t, double *out);
 
 /* Teacher-forced heads: for every sequence b and position i in 0..len-2 the
  * head computed after encoding events 0..i (it predicts event i+1).  Head
@@ -33,7 +38,7 @@ void oracle_uniforms(uint64_t seed, uint32_t seq, uint32_t pos, uint32_t block, 
  * out_heads has B*len*(3M+K) doubles; row i = len-1 is left untouched.
  * out_logg / out_logf (B*len, may be NULL) get log g(tau_i | h_{i-1}) and
  * log f(k_i | h_{i-1}) for i >= 1 and NaN at i = 0. */
-int oracle_score(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+int oracle_score(const int32_t cfg[8], const float *blob, int64_t blob_floats,
                  int32_t B, int32_t len, const float *tau, const int32_t *marks,
                  double *out_heads, double *out_logg, double *out_logf,
                  int32_t recompute, int32_t nthreads);
@@ -43,7 +48,7 @@ int oracle_score(const int32_t cfg[7], const float *blob, int64_t blob_floats,
  * mark, and the smallest decision margin taken at that event.  seq_ids
  * (may be NULL = 0..B-1) gives each row's sequence index, which keys its
  * random slots. */
-int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_ar(const int32_t cfgT[8], const float *blobT, int64_t nT,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, uint64_t seed, int32_t recompute, const int32_t *seq_ids,
                      double *out_tau, double *out_t, int32_t *out_k, double *out_margin,
@@ -52,8 +57,8 @@ int oracle_sample_ar(const int32_t cfgT[7], const float *blobT, int64_t nT,
 /* TPP-SD (Sec. 4.3, Alg. 1).  flags bit 0 = no bonus event after a fully
  * accepted draft.  stats[B][5] = rounds, drafted, accepted, resample
  * iterations, resample-cap hits. */
-int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                     const int32_t cfgD[7], const float *blobD, int64_t nD,
+int oracle_sample_sd(const int32_t cfgT[8], const float *blobT, int64_t nT,
+                     const int32_t cfgD[8], const float *blobD, int64_t nD,
                      int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                      int32_t N, int32_t gamma, uint64_t seed, uint32_t flags, int32_t recompute,
                      const int32_t *seq_ids,
@@ -65,13 +70,13 @@ int oracle_sample_sd(const int32_t cfgT[7], const float *blobT, int64_t nT,
  * gets the number of generated events with t <= t_end, which fill the first
  * out_count[b] slots of the [B][N] outputs (later slots: NaN / -1).  The
  * forms above are these with t_end = +inf. */
-int oracle_sample_ar_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_ar_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
                            int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                            int32_t N, double t_end, uint64_t seed, int32_t recompute,
                            const int32_t *seq_ids, double *out_tau, double *out_t, int32_t *out_k,
                            double *out_margin, int32_t *out_count, int32_t nthreads);
-int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
-                           const int32_t cfgD[7], const float *blobD, int64_t nD,
+int oracle_sample_sd_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
+                           const int32_t cfgD[8], const float *blobD, int64_t nD,
                            int32_t B, int32_t H, const float *hist_tau, const int32_t *hist_marks,
                            int32_t N, double t_end, int32_t gamma, uint64_t seed, uint32_t flags,
                            int32_t recompute, const int32_t *seq_ids,
@@ -86,7 +91,7 @@ int oracle_sample_sd_until(const int32_t cfgT[7], const float *blobT, int64_t nT
  * position, tau = -log(u_comp) / lambda, mark from p with u_mark.  Outputs
  * and stop rule as oracle_sample_sd_until.  Returns -1 on a bad lambda or
  * p. */
-int oracle_sample_sd_poisson_until(const int32_t cfgT[7], const float *blobT, int64_t nT,
+int oracle_sample_sd_poisson_until(const int32_t cfgT[8], const float *blobT, int64_t nT,
                                    int32_t B, int32_t H, const float *hist_tau,
                                    const int32_t *hist_marks, int32_t N, double t_end,
                                    int32_t gamma, double lambda, const double *p_marks,
@@ -108,7 +113,7 @@ int oracle_toy_sd_poisson(int32_t M, int32_t K, const double *tableT, double lam
 
 /* Survival term log S(t_end - t_{len-1}) of each sequence's len events, from
  * the head after the last event (Sec. 3.1, Eq. 2). */
-int oracle_score_survival(const int32_t cfg[7], const float *blob, int64_t blob_floats,
+int oracle_score_survival(const int32_t cfg[8], const float *blob, int64_t blob_floats,
                           int32_t B, int32_t len, const float *tau, const int32_t *marks,
                           double t_end, double *out_logS, int32_t recompute, int32_t nthreads);
 /* log(1 - G(u)) for the log-normal mixture of one head; 0 for u <= 0. */

@@ -18,6 +18,7 @@ from typing import Tuple
 
 FP32 = 0
 BF16 = 1
+THP, SAHP, ATTNHP = 0, 1, 2  # history encoders of App. D.4
 
 
 @dataclass(frozen=True)
@@ -29,6 +30,7 @@ class ModelCfg:
     n_mix: int
     n_marks: int
     dtype: int  # FP32 or BF16
+    encoder: int = 0  # THP, SAHP or ATTNHP (App. D.4)
 
     @property
     def d_head(self) -> int:

@@ -30,16 +30,28 @@ INIT_STD = 0.02
 TAU_MIN = 1e-12
 
 
+# AttNHP temporal-encoding time scales (m, M) written into its blobs: the
+# wavelengths of the encoding run from m to 5M.
+ATTNHP_SCALES = (0.1, 1000.0)
+
+
 def blob_layout(cfg: ModelCfg):
     """Ordered (name, shape, init) triples of the weight blob.
 
-    init: "w" = N(0, 0.02), "0" = zeros, "1" = ones.  Matrices are row-major
-    [out][in] (y = W x + b).
+    init: "w" = N(0, 0.02), "0" = zeros, "1" = ones, "scales" = the AttNHP
+    time scales above.  Matrices are row-major [out][in] (y = W x + b).
+    THP and SAHP layers: QKV, output projection, two LayerNorms, FFN.
+    AttNHP layers: QKV from [z(t); h] (2d inputs) only.  SAHP appends its
+    per-dimension temporal frequencies, AttNHP its two time scales.
     """
     d, F, M, K = cfg.d_model, cfg.d_ffn, cfg.n_mix, cfg.n_marks
+    enc = getattr(cfg, "encoder", 0)
     out = [("type_emb", (K, d), "w")]
     for l in range(cfg.layers):
         p = f"layer{l}."
+        if enc == 2:
+            out += [(p + "w_qkv", (3 * d, 2 * d), "w"), (p + "b_qkv", (3 * d,), "0")]
+            continue
         out += [
             (p + "w_qkv", (3 * d, d), "w"), (p + "b_qkv", (3 * d,), "0"),
             (p + "w_o", (d, d), "w"), (p + "b_o", (d,), "0"),
@@ -56,6 +68,10 @@ def blob_layout(cfg: ModelCfg):
         ("head.v_k1", (d, d), "w"), ("head.b_k1", (d,), "0"),
         ("head.v_k2", (K, d), "w"), ("head.b_k2", (K,), "0"),
     ]
+    if enc == 1:
+        out += [("tenc_w", (d,), "w")]
+    elif enc == 2:
+        out += [("tenc_scales", (2,), "scales")]
     return out
 
 
@@ -95,6 +111,8 @@ def model_blob(cfg: ModelCfg, seed: int, role: int, head_gain: float = 1.0) -> n
             parts.append(rng.normal(0.0, std, n).astype(np.float32))
         elif init == "1":
             parts.append(np.ones(n, np.float32))
+        elif init == "scales":
+            parts.append(np.array(ATTNHP_SCALES, np.float32))
         else:
             parts.append(np.zeros(n, np.float32))
     blob = np.concatenate(parts)

@@ -52,13 +52,40 @@ def chi2_pvalue(observed, expected):
     return stats.chi2.sf(stat, dof)
 
 
-def torch_reference_heads(cfg, blob, tau, marks):
+def torch_heads(cfg, blob, x):
+    """Heads of Sec. 4.2 on hidden states x [..., d] with F.linear and
+    log_softmax in float64: [..., 3M+K] = [log w | mu | log sigma | log f]."""
+    import torch
+    import torch.nn.functional as Fn
+    from paper_2507_09252_gb300.inputs import blob_offsets
+
+    offs = blob_offsets(cfg)
+    bt = torch.from_numpy(np.asarray(blob, np.float64))
+
+    def P(name):
+        o, shape = offs[name]
+        return bt[o:o + int(np.prod(shape))].reshape(shape)
+
+    d = cfg.d_model
+    x = torch.as_tensor(np.asarray(x, np.float64))
+    with torch.no_grad():
+        e = Fn.linear(x, P("head.E"))
+        lw = torch.log_softmax(Fn.linear(e[..., :d], P("head.v_w"), P("head.b_w")), -1)
+        mu = Fn.linear(e[..., d:2 * d], P("head.v_mu"), P("head.b_mu"))
+        s = Fn.linear(e[..., 2 * d:], P("head.v_s"), P("head.b_s"))
+        a = torch.tanh(Fn.linear(x, P("head.v_k1"), P("head.b_k1")))
+        lf = torch.log_softmax(Fn.linear(a, P("head.v_k2"), P("head.b_k2")), -1)
+    return torch.cat([lw, mu, s, lf], -1).numpy()
+
+
+def torch_reference_heads(cfg, blob, tau, marks, z=None):
     """Heads of one model built from torch library modules in float64.
 
     The encoder is torch.nn.TransformerEncoderLayer (post-LN, ReLU, eps 1e-5,
     causal mask); the temporal encoding and heads use torch.sin/cos,
     F.linear and log_softmax.  Returns [B][n][3M+K] (row i = head after
-    events 0..i).
+    events 0..i).  z [B][n][d], if given, replaces the THP temporal
+    encoding (for encoders whose encoding is pinned separately).
     """
     import torch
     import torch.nn.functional as Fn
@@ -97,7 +124,10 @@ def torch_reference_heads(cfg, blob, tau, marks):
     j = torch.arange(d, dtype=torch.float64)
     je = j - (j.long() % 2).double()
     arg = t[..., None] / torch.pow(torch.tensor(10000.0, dtype=torch.float64), je / d)
-    z = torch.where((j.long() % 2) == 1, torch.cos(arg), torch.sin(arg))
+    if z is None:
+        z = torch.where((j.long() % 2) == 1, torch.cos(arg), torch.sin(arg))
+    else:
+        z = torch.as_tensor(np.asarray(z, np.float64))
     x = z + P("type_emb")[torch.from_numpy(np.asarray(marks, np.int64))]
     mask = torch.triu(torch.full((n, n), float("-inf"), dtype=torch.float64), diagonal=1)
     with torch.no_grad():
