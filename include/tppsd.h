@@ -49,18 +49,27 @@ typedef enum {
 /* Model shape.  Weight blob layout (float32 values, row-major [out][in],
  * y = W x + b), in this order:
  *   type_emb [K][d]                                  (W of Sec. 4.2)
- *   for each layer: w_qkv [3d][d], b_qkv [3d], w_o [d][d], b_o [d],
+ *   for each layer, THP and SAHP:
+ *                   w_qkv [3d][d], b_qkv [3d], w_o [d][d], b_o [d],
  *                   ln1_g [d], ln1_b [d], w_1 [F][d], b_1 [F],
  *                   w_2 [d][F], b_2 [d], ln2_g [d], ln2_b [d]
+ *                 AttNHP: w_qkv [3d][2d] (inputs [z(t); h]), b_qkv [3d]
  *   E [3d][d]                                        (e = E h, no bias)
  *   v_w [M][d], b_w [M], v_mu [M][d], b_mu [M], v_s [M][d], b_s [M]
  *   v_k1 [d][d], b_k1 [d], v_k2 [K][d], b_k2 [K]
- * Model (Sec. 4.2): x_i = z(t_i) + W[k_i] with the THP temporal encoding
- * z_2j = sin(t w_j), z_2j+1 = cos(t w_j), w_j = 10000^(-2j/d), t absolute
- * (App. D.4); post-LN layers h <- LN(h + MHA(h)), h <- LN(h + W2 ReLU(W1 h
- * + b1) + b2) with causal softmax attention (scale 1/sqrt(d/heads)),
- * LayerNorm eps 1e-5; heads: w = softmax(v_w e1 + b_w), mu = v_mu e2 + b_mu,
- * sigma = exp(v_s e3 + b_s), f = softmax(v_k2 tanh(v_k1 h + b_k1) + b_k2).
+ *   SAHP only: w [d] (temporal frequencies); AttNHP only: m, M (time scales)
+ * Model (Sec. 4.2): x_i = z(t_i) + W[k_i]; heads w = softmax(v_w e1 + b_w),
+ * mu = v_mu e2 + b_mu, sigma = exp(v_s e3 + b_s), f = softmax(v_k2
+ * tanh(v_k1 h + b_k1) + b_k2).  Encoders (App. D.4), t absolute, j 0-based,
+ * je = j - j mod 2, sin for even j and cos for odd j of:
+ *   THP     t / 10000^(je/d)
+ *   SAHP    j / 10000^(je/d) + w_j t
+ *   AttNHP  t / (m (5M/m)^(je/d))
+ * THP and SAHP layers: post-LN h <- LN(h + MHA(h)), h <- LN(h + W2 ReLU(W1
+ * h + b1) + b2), causal softmax attention (scale 1/sqrt(d/heads)), LayerNorm
+ * eps 1e-5.  AttNHP layers: q, k, v = w_qkv [z; h] + b_qkv; per head
+ * a = sum_j f_j v_j / (1 + sum_j f_j), f_j = exp(q k_j / sqrt(d/heads)) over
+ * keys j <= i; h <- h + tanh(a) (heads concatenated).
  * dtype 0 = fp32 throughout.  dtype 1 = bf16: the blob's values must be
  * bf16-representable; GEMM inputs and Q/K/V are rounded to bf16 (nearest
  * even), accumulation, LayerNorm, softmax, heads and sampling are fp32. */
@@ -68,10 +77,13 @@ typedef struct {
     int32_t layers;   /* 1..16 */
     int32_t d_model;  /* multiple of 16, <= 512 */
     int32_t heads;    /* 1..8 (draft: 1, 2 or 4); d_model / heads in {8, 16, 32, 64} */
-    int32_t d_ffn;    /* multiple of 16, <= 4096 */
+    int32_t d_ffn;    /* multiple of 16, <= 4096 (unused by AttNHP) */
     int32_t n_mix;    /* M, 1..64 */
     int32_t n_marks;  /* K, 1..256; equal for target and draft */
     int32_t dtype;    /* 0 fp32, 1 bf16 */
+    int32_t encoder;  /* 0 THP, 1 SAHP, 2 AttNHP (an AttNHP draft model must
+                         fit the one-CTA draft kernel: heads 1, 2 or 4 and
+                         d/heads 16 or 32, else TPPSD_ERR_UNSUPPORTED) */
 } tppsd_model_cfg;
 
 /* Counters of the last tppsd_sample / tppsd_sample_autoregressive call. */

@@ -144,14 +144,17 @@ static bool cfg_ok(const tppsd_model_cfg* c) {
     if (c->d_ffn < 16 || c->d_ffn > 4096 || c->d_ffn % 16) return false;
     if (c->n_mix < 1 || c->n_mix > MAX_MIX) return false;
     if (c->n_marks < 1 || c->n_marks > MAX_MARKS) return false;
+    if (c->encoder < 0 || c->encoder > 2) return false;
     return c->dtype == 0 || c->dtype == 1;
 }
 
 extern "C" size_t tppsd_blob_floats(const tppsd_model_cfg* c) {
     if (!cfg_ok(c)) return 0;
     const size_t L = c->layers, d = c->d_model, F = c->d_ffn, M = c->n_mix, K = c->n_marks;
-    const size_t layer = 3 * d * d + 3 * d + d * d + d + 2 * d + F * d + F + d * F + d + 2 * d;
-    return K * d + L * layer + 3 * d * d + 3 * (M * d + M) + d * d + d + K * d + K;
+    const size_t layer = c->encoder == 2 ? 3 * d * 2 * d + 3 * d
+                                         : 3 * d * d + 3 * d + d * d + d + 2 * d + F * d + F + d * F + d + 2 * d;
+    const size_t tail = c->encoder == 1 ? d : c->encoder == 2 ? 2 : 0;
+    return K * d + L * layer + 3 * d * d + 3 * (M * d + M) + d * d + d + K * d + K + tail;
 }
 
 static uint16_t f32_to_bf16_bits(float f) {
@@ -168,6 +171,9 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
                                    const float* blob_any, size_t nfloats) {
     hm.cfg = *cfg;
     const int L = cfg->layers, d = cfg->d_model, F = cfg->d_ffn, M = cfg->n_mix, K = cfg->n_marks;
+    const int enc = cfg->encoder;
+    const bool att = enc == 2;             // AttNHP: QKV over [z; h] only
+    const size_t din = att ? 2 * (size_t)d : (size_t)d;
     std::vector<float> blob(nfloats);
     if (is_device_ptr(blob_any)) {
         CK(cudaMemcpy(blob.data(), blob_any, nfloats * sizeof(float), cudaMemcpyDeviceToHost));
@@ -181,7 +187,8 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     struct LO { size_t wqkv, bqkv, wo, bo, g1, b1n, w1, b1, w2, b2, g2, b2n; };
     std::vector<LO> lo(L);
     for (int l = 0; l < L; ++l) {
-        lo[l].wqkv = take(3 * (size_t)d * d); lo[l].bqkv = take(3 * d);
+        lo[l].wqkv = take(3 * (size_t)d * din); lo[l].bqkv = take(3 * d);
+        if (att) continue;
         lo[l].wo = take((size_t)d * d); lo[l].bo = take(d);
         lo[l].g1 = take(d); lo[l].b1n = take(d);
         lo[l].w1 = take((size_t)F * d); lo[l].b1 = take(F);
@@ -192,6 +199,7 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const size_t ovw = take((size_t)M * d), obw = take(M), ovm = take((size_t)M * d), obm = take(M);
     const size_t ovs = take((size_t)M * d), obs = take(M);
     const size_t ok1 = take((size_t)d * d), obk1 = take(d), ok2 = take((size_t)K * d), obk2 = take(K);
+    const size_t o_tail = take(enc == 1 ? d : att ? 2 : 0);
     if (o != nfloats) {
         ctx->err = "blob size does not match the model shape";
         return TPPSD_ERR_INVALID_ARG;
@@ -214,13 +222,16 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     struct LB { size_t wqkv, bqkv, wo, bo, g1, b1n, w1, b1, w2, b2, g2, b2n; };
     std::vector<LB> lb(L);
     for (int l = 0; l < L; ++l) {
-        lb[l].wqkv = add_mat(lo[l].wqkv, 3 * (size_t)d * d);
+        lb[l].wqkv = add_mat(lo[l].wqkv, 3 * (size_t)d * din);
+        if (att) continue;
         lb[l].wo = add_mat(lo[l].wo, (size_t)d * d);
         lb[l].w1 = add_mat(lo[l].w1, (size_t)F * d);
         lb[l].w2 = add_mat(lo[l].w2, (size_t)d * F);
     }
     for (int l = 0; l < L; ++l) {
-        lb[l].bqkv = add_vec(lo[l].bqkv, 3 * d); lb[l].bo = add_vec(lo[l].bo, d);
+        lb[l].bqkv = add_vec(lo[l].bqkv, 3 * d);
+        if (att) continue;
+        lb[l].bo = add_vec(lo[l].bo, d);
         lb[l].g1 = add_vec(lo[l].g1, d); lb[l].b1n = add_vec(lo[l].b1n, d);
         lb[l].b1 = add_vec(lo[l].b1, F); lb[l].b2 = add_vec(lo[l].b2, d);
         lb[l].g2 = add_vec(lo[l].g2, d); lb[l].b2n = add_vec(lo[l].b2n, d);
@@ -232,9 +243,25 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const size_t bvs = add_vec(ovs, (size_t)M * d), bbs = add_vec(obs, M);
     const size_t bk1 = add_vec(ok1, (size_t)d * d), bbk1 = add_vec(obk1, d);
     const size_t bk2 = add_vec(ok2, (size_t)K * d), bbk2 = add_vec(obk2, K);
-    std::vector<double> omega(d / 2);
-    for (int i = 0; i < d / 2; ++i) omega[i] = pow(10000.0, -2.0 * i / (double)d);
-    const size_t b_om = add(omega.data(), omega.size() * sizeof(double));
+    // temporal encoding (App. D.4): z_j = sin / cos (a_j + b_j t), je = j - j mod 2
+    std::vector<double> tenc(2 * (size_t)d, 0.0);
+    if (att && !(blob[o_tail] > 0.f && blob[o_tail + 1] > 0.f)) {
+        ctx->err = "AttNHP time scales must be positive";
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    for (int j = 0; j < d; ++j) {
+        const double je = (double)(j - (j & 1)), e = je / (double)d;
+        if (enc == 1) {          // SAHP: phase j / 10000^(je/d), learned frequency w_j
+            tenc[j] = (double)j / pow(10000.0, e);
+            tenc[d + j] = (double)blob[o_tail + j];
+        } else if (att) {        // AttNHP: wavelength m (5M/m)^(je/d)
+            const double sm = blob[o_tail], sM = blob[o_tail + 1];
+            tenc[d + j] = 1.0 / (sm * pow(5.0 * sM / sm, e));
+        } else {                 // THP: frequency 10000^(-je/d)
+            tenc[d + j] = pow(10000.0, -e);
+        }
+    }
+    const size_t b_om = add(tenc.data(), tenc.size() * sizeof(double));
     // head matrices regrouped for the batched head: [E; v_k1] (4d x d) with
     // bias [0; b_k1], and the output maps transposed side by side (d x (3M+K))
     std::vector<float> ek((size_t)4 * d * d), ekb((size_t)4 * d, 0.f);
@@ -270,11 +297,15 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     DevModel& m = hm.dm;
     m.L = L; m.d = d; m.nh = cfg->heads; m.dh = d / cfg->heads; m.F = F; m.M = M; m.K = K;
     m.dtype = cfg->dtype;
+    m.enc = enc;
+    m.tenc_paired = enc != 1;
     m.type_emb = (const float*)(b + b_emb);
-    m.omega = (const double*)(b + b_om);
+    m.tenc = (const double*)(b + b_om);
     for (int l = 0; l < L; ++l) {
         LayerW& w = m.layer[l];
+        w = LayerW{};
         w.w_qkv = b + lb[l].wqkv; w.b_qkv = (const float*)(b + lb[l].bqkv);
+        if (att) continue;
         w.w_o = b + lb[l].wo; w.b_o = (const float*)(b + lb[l].bo);
         w.ln1_g = (const float*)(b + lb[l].g1); w.ln1_b = (const float*)(b + lb[l].b1n);
         w.w_1 = b + lb[l].w1; w.b_1 = (const float*)(b + lb[l].b1);
@@ -319,13 +350,16 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     auto tvec = [&](size_t off, size_t n) { return tadd(blob.data() + off, n * sizeof(float)); };
     std::vector<LB> tl(L);
     for (int l = 0; l < L; ++l) {
-        tl[l].wqkv = tmat(lo[l].wqkv, 3 * (size_t)d, d, true);
+        tl[l].wqkv = tmat(lo[l].wqkv, 3 * (size_t)d, din, true);
+        if (att) continue;
         tl[l].wo = tmat(lo[l].wo, d, d, true);
         tl[l].w1 = tmat(lo[l].w1, F, d, true);
         tl[l].w2 = tmat(lo[l].w2, d, F, true);
     }
     for (int l = 0; l < L; ++l) {
-        tl[l].bqkv = tvec(lo[l].bqkv, 3 * d); tl[l].bo = tvec(lo[l].bo, d);
+        tl[l].bqkv = tvec(lo[l].bqkv, 3 * d);
+        if (att) continue;
+        tl[l].bo = tvec(lo[l].bo, d);
         tl[l].g1 = tvec(lo[l].g1, d); tl[l].b1n = tvec(lo[l].b1n, d);
         tl[l].b1 = tvec(lo[l].b1, F); tl[l].b2 = tvec(lo[l].b2, d);
         tl[l].g2 = tvec(lo[l].g2, d); tl[l].b2n = tvec(lo[l].b2n, d);
@@ -337,7 +371,7 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const size_t tvs = tmat(ovs, M, d, false), tbs = tvec(obs, M);
     const size_t tk1 = tmat(ok1, d, d, false), tbk1 = tvec(obk1, d);
     const size_t tk2 = tmat(ok2, K, d, false), tbk2 = tvec(obk2, K);
-    const size_t t_om = tadd(omega.data(), omega.size() * sizeof(double));
+    const size_t t_om = tadd(tenc.data(), tenc.size() * sizeof(double));
     tb.resize((tb.size() + 15) & ~(size_t)15);
     tb.resize((tb.size() + 15) & ~(size_t)15);  // whole 16-byte chunks: one bulk copy stages it
     CK(cudaMalloc(&hm.tbuf, tb.size()));
@@ -346,10 +380,12 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const char* tbp = (const char*)hm.tbuf;
     DevModelT& mt = m.t;
     mt.type_emb = (const float*)(tbp + t_emb);
-    mt.omega = (const double*)(tbp + t_om);
+    mt.tenc = (const double*)(tbp + t_om);
     for (int l = 0; l < L; ++l) {
         LayerW& w = mt.layer[l];
+        w = LayerW{};
         w.w_qkv = tbp + tl[l].wqkv; w.b_qkv = (const float*)(tbp + tl[l].bqkv);
+        if (att) continue;
         w.w_o = tbp + tl[l].wo; w.b_o = (const float*)(tbp + tl[l].bo);
         w.ln1_g = (const float*)(tbp + tl[l].g1); w.ln1_b = (const float*)(tbp + tl[l].b1n);
         w.w_1 = tbp + tl[l].w1; w.b_1 = (const float*)(tbp + tl[l].b1);
@@ -411,12 +447,27 @@ static void build_tc_plan(tppsd_ctx* ctx) {
     const tppsd_model_cfg& c = ctx->T.cfg;
     if (getenv("TPPSD_NO_TC") || c.dtype != 1) return;
     const int d = c.d_model, F = c.d_ffn;
+    const Work& w = ctx->work;
+    if (c.encoder == 2) {  // AttNHP: only the QKV GEMM over the [z | h] rows
+        if (d % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
+        p.bn_qkv = pick_bn(3 * d);
+        if (!p.bn_qkv) return;
+        bool ok = make_tmap_bf16(&p.a_zh, w.xb, 2 * d, w.R, 128);
+        for (int l = 0; l < m.L && ok; ++l)
+            ok = make_tmap_bf16(&p.layer[l].wqkv, m.layer[l].w_qkv, 2 * d, 3 * d, p.bn_qkv < 256 ? p.bn_qkv : 256);
+        p.mlp = p.mlp_cl = 0;
+        p.head = ok && head_tc_supported(m) &&
+                 make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
+                 make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
+        p.err = ctx->d_err;
+        p.enabled = ok ? 1 : 0;
+        return;
+    }
     if (d % 64 || F % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
     p.bn_qkv = pick_bn(3 * d);
     p.bn_ffn1 = pick_bn(F);
     p.bn_o = ln_cluster_cols(d);
     if (!p.bn_qkv || !p.bn_ffn1 || !p.bn_o) return;
-    const Work& w = ctx->work;
     bool ok = make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128) &&
               make_tmap_bf16(&p.a_hid, w.hid, F, w.R, 128);
     const int bo = p.bn_o < 256 ? p.bn_o : 256;
@@ -454,6 +505,10 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     CK(cudaGetDevice(&ctx->device));
     TRY(upload_model(ctx, ctx->T, target, tb, tn));
     TRY(upload_model(ctx, ctx->D, draft, db, dn));
+    if (draft->encoder == 2 && !draft_team_supported(ctx->D.dm)) {
+        ctx->err = "an AttNHP draft model must fit the one-CTA draft kernel (heads 1, 2 or 4, d/heads 16 or 32)";
+        return TPPSD_ERR_UNSUPPORTED;
+    }
     const int B = ctx->max_batch, nm = ctx->n_max;
     SeqState& ss = ctx->ss;
     ss.n_max = nm;
@@ -481,7 +536,7 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &w.row_pos, sizeof(int) * R));
     TRY(dalloc(ctx, &w.x, sizeof(float) * R * dmax));
     TRY(dalloc(ctx, &w.y, sizeof(float) * R * dmax));
-    TRY(dalloc(ctx, &w.xb, sizeof(float) * R * dmax));
+    TRY(dalloc(ctx, &w.xb, sizeof(float) * R * 2 * dmax));  // [z | h] rows of AttNHP
     TRY(dalloc(ctx, &w.q, sizeof(float) * R * dmax));
     TRY(dalloc(ctx, &w.att, sizeof(float) * R * dmax));
     TRY(dalloc(ctx, &w.hid, sizeof(float) * R * fmax));
@@ -607,7 +662,7 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
         ++n;
     } else if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
-        if (draft_team_supported(ctx->D.dm) && !getenv("TPPSD_DRAFT_CTA"))
+        if (draft_team_supported(ctx->D.dm) && (ctx->D.dm.enc == 2 || !getenv("TPPSD_DRAFT_CTA")))
             CK(launch_draft_team(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
         else
@@ -1115,7 +1170,7 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     w.row_pos = (int*)take(rows * 4);
     w.x = (float*)take(rows * d * 4);
     w.y = (float*)take(rows * d * 4);
-    w.xb = take(rows * d * eb);
+    w.xb = take(rows * 2 * d * eb);  // [z | h] rows of AttNHP
     w.q = take(rows * d * eb);
     w.att = take(rows * d * eb);
     w.hid = take(rows * F * eb);

@@ -244,7 +244,14 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
             L += p[16 + row] * e;
             O += p[32 + row * DH + col] * e;
         }
-        a.out[(size_t)(rb + row) * a.d + h * DH + col] = __float2bfloat16_rn(O / L);
+        if (a.attnhp) {  // a = sum f v / (1 + sum f); h <- h + tanh(a)
+            const size_t xi = (size_t)(rb + row) * a.d + h * DH + col;
+            const float hn = a.x[xi] + tanhf(O / (L + expf(-M)));
+            a.x[xi] = hn;
+            a.hb[(size_t)(rb + row) * 2 * a.d + a.d + h * DH + col] = __float2bfloat16_rn(hn);
+        } else {
+            a.out[(size_t)(rb + row) * a.d + h * DH + col] = __float2bfloat16_rn(O / L);
+        }
     }
     pdl_trigger();
 }

@@ -125,11 +125,14 @@ __device__ __forceinline__ void warp_resid_ln(float yv, float* x, float* xin, in
 // 0..n_keys-1 of K/V blocks [nh][stride][DH] (shared or global): warp w
 // takes head w % nh and key range w / nh of 4 / nh; lane-strided keys with
 // a private online softmax (exp2 units), warp merge by shuffles, then the
-// warps of a head merge through shared memory; the output is rounded to
-// the storage type.  Ends with a barrier.
+// warps of a head merge through shared memory.  Softmax: the output is
+// rounded to the storage type.  attnhp (App. D.4): the normaliser is
+// 1 + sum_j f_j (an extra term exp(0)) and the fp32 output is kept.  Ends
+// with a barrier.
 template <typename T, int DH>
 __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
-                                            int n_keys, int nh, float* out, float* scratch) {
+                                            int n_keys, int nh, float* out, float* scratch,
+                                            bool attnhp = false) {
     const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31;
     const int h = warp % nh, split = warp / nh, S = 4 / nh;
     const int per = (n_keys + S - 1) / S, lo = split * per, hi = min(n_keys, lo + per);
@@ -189,7 +192,7 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
             L += src[1] * e;
             O += src[2 + c] * e;
         }
-        out[t] = St<T>::rnd(O / L);
+        out[t] = attnhp ? O / (L + exp2f(-M)) : St<T>::rnd(O / L);
     }
     team_sync();
 }
@@ -245,9 +248,9 @@ __device__ __forceinline__ int warp_logsoftmax_pick(float* v, int n, float u) {
 // onto a staged copy of its bytes at dst.
 __device__ void rebase_model(DevModelT& m, const DevModelT& src, int L, const char* dst) {
     m = src;
-    auto rb = [&](const void* p) { return dst + ((const char*)p - src.base); };
+    auto rb = [&](const void* p) { return p ? dst + ((const char*)p - src.base) : nullptr; };
     m.type_emb = (const float*)rb(m.type_emb);
-    m.omega = (const double*)rb(m.omega);
+    m.tenc = (const double*)rb(m.tenc);
     for (int l = 0; l < L; ++l) {
         LayerW& w = m.layer[l];
         w.w_qkv = rb(w.w_qkv); w.b_qkv = (const float*)rb(w.b_qkv);
@@ -309,7 +312,8 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     T* kvs = (T*)area;
     uint64_t* bar = (uint64_t*)(area + kvb);
     float* x = (float*)(area + kvb + 16);
-    float* xin = x + d;
+    float* zin = x + d;   // rounded temporal encoding; [zin | xin] is the AttNHP QKV input
+    float* xin = zin + d;
     float* qkv = xin + d;
     float* att = qkv + 3 * d;
     float* hid = att + d;
@@ -382,7 +386,35 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     };
     // Layers of the encode step at position p from x / xin (set and synced
     // by the caller); leaves the final hidden state in x (synced).
+    const bool att_enc = a.m.enc == 2;
     auto layers = [&](int p) {
+        if (att_enc) {
+            // AttNHP (App. D.4): q, k, v = W [z; h] + b, a = sum f v / (1 + sum f),
+            // h <- h + tanh(a)
+            for (int l = 0; l < L; ++l) {
+                const LayerW& Wl = m.layer[l];
+                for (int o = tid; o < 3 * d; o += 128) {
+                    const float v = St<T>::rnd(dot_col<T>((const T*)Wl.w_qkv, 3 * d, o, zin, 2 * d) + Wl.b_qkv[o]);
+                    qkv[o] = v;
+                    if (o >= d) {
+                        const int w = o < 2 * d ? 0 : 1, c = o - d - w * d, hh = c / DH, ee = c - hh * DH;
+                        const size_t off = ((size_t)hh * n_max + p) * DH + ee;
+                        St<T>::st(gk(l, w) + off, v);
+                        if (KVS) St<T>::st(sk(l, w) + off, v);
+                    }
+                }
+                team_sync();
+                const T* kb = KVS ? sk(l, 0) : gk(l, 0);
+                const T* vb = KVS ? sk(l, 1) : gk(l, 1);
+                team_attend<T, DH>(qkv, kb, vb, n_max, p + 1, NH, att, attn, true);
+                for (int i = tid; i < d; i += 128) {
+                    x[i] += tanhf(att[i]);
+                    xin[i] = St<T>::rnd(x[i]);
+                }
+                team_sync();
+            }
+            return;
+        }
         for (int l = 0; l < L; ++l) {
             const LayerW& Wl = m.layer[l];
             // Q, K, V; K and V appended to the cache at position p
@@ -407,15 +439,18 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             proj_resid_ln((const T*)Wl.w_2, Wl.b_2, hid, F, Wl.ln2_g, Wl.ln2_b);
         }
     };
-    // Encoding of event (t, k) into x / xin (App. D.4 THP encoding, angle
-    // reduced mod 2 pi in fp64, plus the mark embedding).  Not synced.
+    // Encoding of event (t, k) into x / xin (App. D.4 temporal encoding
+    // z_i = sin / cos (a_i + b_i t), angle reduced mod 2 pi in fp64, plus the
+    // mark embedding); zin = rounded z.  Not synced.
     auto embed = [&](double t, int k) {
         for (int i = tid; i < d; i += 128) {
-            const double ang = t * m.omega[i >> 1];
+            const double ang = m.tenc[i] + m.tenc[d + i] * t;
             const double red = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
             float sv, cv;
             sincosf((float)red, &sv, &cv);
-            const float v = ((i & 1) ? cv : sv) + m.type_emb[(size_t)k * d + i];
+            const float z = (i & 1) ? cv : sv;
+            const float v = z + m.type_emb[(size_t)k * d + i];
+            zin[i] = St<T>::rnd(z);
             x[i] = v;
             xin[i] = St<T>::rnd(v);
         }

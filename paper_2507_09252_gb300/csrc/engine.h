@@ -53,7 +53,7 @@ struct HeadW {  // all fp32 (exact copies of the blob values)
 // are copied in too, and every pointer lies in [base, base + bytes).
 struct DevModelT {
     const float* type_emb;   // [K][d]
-    const double* omega;     // [d/2]
+    const double* tenc;      // [2d] temporal encoding: phases a_j, then frequencies b_j
     LayerW layer[MAX_LAYERS];  // w_qkv [d][3d], w_o [d][d], w_1 [d][F], w_2 [F][d]
     HeadW head;              // E [d][3d], v_w/v_mu/v_s [d][M], v_k1 [d][d], v_k2 [d][K]
     const char* base;
@@ -64,8 +64,12 @@ struct DevModelT {
 // kernel can copy the whole model to shared memory and rebase the pointers.
 struct DevModel {
     int L, d, nh, dh, F, M, K, dtype;
+    int enc;                 // encoder: 0 THP, 1 SAHP, 2 AttNHP (App. D.4)
+    int tenc_paired;         // dims 2i and 2i+1 share one angle (THP, AttNHP)
     const float* type_emb;   // [K][d] fp32
-    const double* omega;     // [d/2] temporal-encoding frequencies
+    // temporal encoding z_j = sin / cos (a_j + b_j t) for even / odd j:
+    // [2d] phases a_j then frequencies b_j (fp64)
+    const double* tenc;
     LayerW layer[MAX_LAYERS];
     HeadW head;
     const char* base;
@@ -180,6 +184,12 @@ struct AttArgs {
     int count, q_per_seq, g0, d, nh, layer;
     KVCache kv;
     float scale;
+    // AttNHP (App. D.4): normaliser 1 + sum f, and instead of `out` the
+    // residual h <- h + tanh(a) into x (fp32 [R][d]) and its rounded copy
+    // into the h half of the [z | h] rows hb ([R][2d])
+    int attnhp;
+    float* x;
+    T* hb;
 };
 cudaError_t launch_attn_mma(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int nseg, int* err,
                             cudaStream_t st);
@@ -214,6 +224,7 @@ struct TcPlan {
     CUtensorMap head_hi, head_lo;
     int* err;
     CUtensorMap a_xb, a_att, a_hid;
+    CUtensorMap a_zh;           // [R][2d] view of the [z | h] rows (AttNHP QKV input)
     TcLayerMaps layer[MAX_LAYERS];
 };
 bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows);

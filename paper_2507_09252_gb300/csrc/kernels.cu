@@ -28,18 +28,31 @@ __device__ __forceinline__ void load_row(const T* p, float* out, int n) {
     for (int c = 0; c < n; ++c) out[c] = St<T>::ld(p + c);
 }
 
-// Temporal encoding (App. D.4) + type embedding (Sec. 4.2) of pair i:
-// angle t * w_i in fp64, reduced mod 2 pi in fp64, then fp32 sin/cos.
-// Marks outside 0..K-1 are clamped into range (the row gather stays in bounds).
+// Angle a + b t in fp64, reduced mod 2 pi in fp64 (then fp32 sin / cos).
+__device__ __forceinline__ float tenc_angle(const double* tenc, int d, int j, double t) {
+    const double ang = tenc[j] + tenc[d + j] * t;
+    return (float)fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
+}
+
+// Temporal encoding (App. D.4: z_j = sin / cos (a_j + b_j t) for even / odd
+// j) of dimensions 2i, 2i+1.  THP and AttNHP pairs share one angle (one
+// sincos); SAHP's dimensions have their own.
+__device__ __forceinline__ void tenc_pair(const DevModel& m, double t, int i, float* z0, float* z1) {
+    float sv, cv;
+    sincosf(tenc_angle(m.tenc, m.d, 2 * i, t), &sv, &cv);
+    if (!m.tenc_paired) cv = cosf(tenc_angle(m.tenc, m.d, 2 * i + 1, t));
+    *z0 = sv;
+    *z1 = cv;
+}
+
+// Temporal encoding + type embedding (Sec. 4.2) of pair i.  Marks outside
+// 0..K-1 are clamped into range (the row gather stays in bounds).
 __device__ __forceinline__ void embed_pair(const DevModel& m, double t, int k, int i, float* z0,
                                            float* z1) {
     k = min(max(k, 0), m.K - 1);
-    const double ang = t * m.omega[i];
-    const double red = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
-    float sv, cv;
-    sincosf((float)red, &sv, &cv);
-    *z0 = sv + m.type_emb[(size_t)k * m.d + 2 * i];
-    *z1 = cv + m.type_emb[(size_t)k * m.d + 2 * i + 1];
+    tenc_pair(m, t, i, z0, z1);
+    *z0 += m.type_emb[(size_t)k * m.d + 2 * i];
+    *z1 += m.type_emb[(size_t)k * m.d + 2 * i + 1];
 }
 
 // ======================================================================
@@ -70,16 +83,27 @@ __global__ void k_embed(DevModel m, SeqState ss, RowSpec rs, Work w) {
             w.row_seq[r] = active ? s : -1;
             w.row_pos[r] = pos;
         }
-        float z0 = 0.f, z1 = 0.f;
+        float z0 = 0.f, z1 = 0.f, e0 = 0.f, e1 = 0.f;
         if (active) {
             const size_t o = (size_t)s * ss.n_max + pos;
-            embed_pair(m, ss.t[o], ss.k[o], i, &z0, &z1);
+            const int k = min(max(ss.k[o], 0), m.K - 1);
+            tenc_pair(m, ss.t[o], i, &z0, &z1);
+            e0 = m.type_emb[(size_t)k * m.d + 2 * i];
+            e1 = m.type_emb[(size_t)k * m.d + 2 * i + 1];
         }
         const size_t xo = (size_t)r * m.d + 2 * i;
-        w.x[xo] = z0;
-        w.x[xo + 1] = z1;
-        St<T>::st(xb + xo, z0);
-        St<T>::st(xb + xo + 1, z1);
+        w.x[xo] = z0 + e0;
+        w.x[xo + 1] = z1 + e1;
+        if (m.enc == 2) {  // AttNHP: rows [z | h] (the QKV input of every layer)
+            const size_t zo = (size_t)r * 2 * m.d + 2 * i;
+            St<T>::st(xb + zo, z0);
+            St<T>::st(xb + zo + 1, z1);
+            St<T>::st(xb + zo + m.d, z0 + e0);
+            St<T>::st(xb + zo + m.d + 1, z1 + e1);
+        } else {
+            St<T>::st(xb + xo, z0 + e0);
+            St<T>::st(xb + xo + 1, z1 + e1);
+        }
     }
     pdl_trigger();
 }
@@ -284,11 +308,19 @@ __global__ void __launch_bounds__(128) k_attention(AttArgs<T> a) {
     for (int qq = 0; qq < 4; ++qq) {
         const int qi = warp + 4 * qq;
         if (qi >= nq) break;
-        const float inv = 1.0f / l[qq];
+        const float inv = 1.0f / (a.attnhp ? l[qq] + expf(-m[qq]) : l[qq]);
 #pragma unroll
         for (int c = 0; c < OPL; ++c) {
             const int cc = lane + 32 * c;
-            if (cc < DH) St<T>::st(a.out + (size_t)(rb + qi) * a.d + h * DH + cc, o[qq][c] * inv);
+            if (cc >= DH) continue;
+            if (a.attnhp) {  // h <- h + tanh(a) (App. D.4)
+                const size_t xi = (size_t)(rb + qi) * a.d + h * DH + cc;
+                const float hn = a.x[xi] + tanhf(o[qq][c] * inv);
+                a.x[xi] = hn;
+                St<T>::st(a.hb + (size_t)(rb + qi) * 2 * a.d + a.d + h * DH + cc, hn);
+            } else {
+                St<T>::st(a.out + (size_t)(rb + qi) * a.d + h * DH + cc, o[qq][c] * inv);
+            }
         }
     }
 }
@@ -383,7 +415,7 @@ __device__ __forceinline__ void softmax_merge(float& m, float& l, float* o, floa
 // [nh*DH].  scratch: nw * (DH + 2) floats.
 template <typename T, int DH>
 __device__ void cta_attend_one(const float* q, const T* kc, const T* vc, int n_keys, int nh,
-                               int n_max, float scale, float* out, float* scratch) {
+                               int n_max, float scale, float* out, float* scratch, bool attnhp = false) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
     const int h = warp % nh, split = warp / nh, S = nw / nh;
     const int per = (n_keys + S - 1) / S;
@@ -440,7 +472,7 @@ __device__ void cta_attend_one(const float* q, const T* kc, const T* vc, int n_k
             oo = oo * a + src[2 + c] * b;
             mm = mn;
         }
-        out[t] = oo / ll;
+        out[t] = attnhp ? oo / (ll + expf(-mm)) : oo / ll;
     }
     __syncthreads();
 }
@@ -459,8 +491,16 @@ __global__ void __launch_bounds__(256) k_attention_single(AttArgs<T> a) {
     __syncthreads();
     const size_t base = kv_index(a.kv, a.nh, DH, a.layer, s, 0, 0);
     cta_attend_one<T, DH>(qs, a.kc + base, a.vc + base, a.row_pos[r] + 1, a.nh, a.kv.n_max,
-                          a.scale, os, scratch);
-    for (int i = threadIdx.x; i < a.d; i += blockDim.x) St<T>::st(a.out + (size_t)r * a.d + i, os[i]);
+                          a.scale, os, scratch, a.attnhp != 0);
+    for (int i = threadIdx.x; i < a.d; i += blockDim.x) {
+        if (a.attnhp) {  // h <- h + tanh(a) (App. D.4)
+            const float hn = a.x[(size_t)r * a.d + i] + tanhf(os[i]);
+            a.x[(size_t)r * a.d + i] = hn;
+            St<T>::st(a.hb + (size_t)r * 2 * a.d + a.d + i, hn);
+        } else {
+            St<T>::st(a.out + (size_t)r * a.d + i, os[i]);
+        }
+    }
 }
 
 // Head outputs from the batched pre-activations hd4 = [E h | V_k1 h + b_k1]
@@ -611,7 +651,7 @@ __global__ void __launch_bounds__(128) k_draft(DraftArgs a) {
         for (size_t i = threadIdx.x; i < m.bytes / 16; i += blockDim.x) dst[i] = src[i];
         const char* nb = smem;
         m.type_emb = rebase<float>(m.type_emb, m.base, nb);
-        m.omega = rebase<double>(m.omega, m.base, nb);
+        m.tenc = rebase<double>(m.tenc, m.base, nb);
         for (int l = 0; l < m.L; ++l) {
             LayerW& L = m.layer[l];
             L.w_qkv = rebase<char>(L.w_qkv, m.base, nb); L.b_qkv = rebase<float>(L.b_qkv, m.base, nb);
@@ -1177,7 +1217,43 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
     auto grid = [&](int N) { return dim3((N + 63) / 64, (R + 63) / 64); };
     const int nseg = (int)((rs.g0 + (long long)R - 1) / rs.q - rs.g0 / rs.q + 1);
     const bool use_tc = tc && tc->enabled && m.dtype == 1;
-    for (int l = 0; l < m.L; ++l) {
+    for (int l = 0; l < m.L && m.enc == 2; ++l) {
+        // AttNHP layer (App. D.4): q, k, v = W [z; h] + b from the [z | h] rows
+        // (K/V into the cache), then attention with the 1 + sum f normaliser
+        // whose epilogue applies h <- h + tanh(a)
+        const LayerW& L = m.layer[l];
+        cudaError_t e = cudaSuccess;
+        PROF_MARK(prof, KC_GEMM_QKV, 1, st);
+        if (use_tc) {
+            TcGemmArgs g{};
+            g.R = R; g.N = 3 * d; g.K = 2 * d; g.epi = EPI_TC_QKV; g.bias = L.b_qkv;
+            g.q_out = (bf16*)q; g.kc = (bf16*)kv.k; g.vc = (bf16*)kv.v;
+            g.row_seq = w.row_seq; g.row_pos = w.row_pos;
+            g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+            g.err = tc->err;
+            e = launch_gemm_tc(tc->a_zh, tc->layer[l].wqkv, g, tc->bn_qkv, st);
+        } else {
+            GemmArgs<T> g{};
+            g.A = xb; g.W = (const T*)L.w_qkv; g.bias = L.b_qkv; g.R = R; g.N = 3 * d; g.K = 2 * d;
+            g.q_out = q; g.kc = (T*)kv.k; g.vc = (T*)kv.v; g.row_seq = w.row_seq; g.row_pos = w.row_pos;
+            g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+            k_gemm<T, EPI_QKV><<<grid(3 * d), blk, 0, st>>>(g);
+            e = cudaGetLastError();
+        }
+        if (e != cudaSuccess) return e;
+        PROF_MARK(prof, KC_GEMM_QKV, 0, st);
+        AttArgs<T> aa{};
+        aa.q = q; aa.kc = (const T*)kv.k; aa.vc = (const T*)kv.v; aa.out = att;
+        aa.row_seq = w.row_seq; aa.row_pos = w.row_pos; aa.count = R; aa.q_per_seq = rs.q;
+        aa.g0 = rs.g0; aa.d = d; aa.nh = m.nh; aa.layer = l; aa.kv = kv;
+        aa.scale = 1.0f / sqrtf((float)m.dh);
+        aa.attnhp = 1; aa.x = w.x; aa.hb = xb;
+        PROF_MARK(prof, KC_ATTENTION, 1, st);
+        if ((e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st)) != cudaSuccess) return e;
+        PROF_MARK(prof, KC_ATTENTION, 0, st);
+        nl += 2;
+    }
+    for (int l = 0; l < m.L && m.enc != 2; ++l) {
         const LayerW& L = m.layer[l];
         if (use_tc) {
             cudaError_t e;

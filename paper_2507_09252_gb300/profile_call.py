@@ -4,7 +4,7 @@ workload shape.
     python -m paper_2507_09252_gb300.profile_call [--workload c2] [--calls 2]
                                                   [--mode sd|ar] [--host-loop]
     python -m paper_2507_09252_gb300.profile_call --time --workload c3 [--gamma 4]
-                                                  [--batch 16] [--draft 0]
+                                                  [--batch 16] [--draft 0] [--encoder attnhp]
 
 Builds the workload's models and histories (seeded, synthetic) and prefills.
 
@@ -69,6 +69,8 @@ def main(argv=None):
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--draft", type=int, default=None)
     ap.add_argument("--poisson", action="store_true")
+    ap.add_argument("--encoder", default=None, choices=["thp", "sahp", "attnhp"],
+                    help="history encoder of both models (App. D.4); default: the workload's")
     a = ap.parse_args(argv)
     import torch
     wl = WORKLOADS[a.workload]
@@ -78,6 +80,10 @@ def main(argv=None):
         wl = wl.with_(batch=a.batch)
     if a.draft is not None:
         wl = wl.with_(draft=wl.drafts[a.draft])
+    if a.encoder is not None:
+        enc = {"thp": CF.THP, "sahp": CF.SAHP, "attnhp": CF.ATTNHP}[a.encoder]
+        wl = wl.with_(target=CF.ModelCfg(**{**wl.target.__dict__, "encoder": enc}),
+                      draft=CF.ModelCfg(**{**wl.draft.__dict__, "encoder": enc}))
     B, H, N, g = wl.batch, wl.hist_len, wl.n_events, wl.gamma
     bt, bd = IN.model_blob(wl.target, wl.seed, 0), IN.model_blob(wl.draft, wl.seed, 1)
     tau_np, mk_np = IN.histories(wl, seed=wl.seed)
@@ -118,6 +124,7 @@ def main(argv=None):
             "workload": wl.name, "batch": B, "gamma": g, "n_events": N, "hist_len": H,
             "target": _shape(wl.target, layer + (("M", "n_mix"), ("K", "n_marks"))),
             "draft": f"Poisson rate {rate:.4g}" if a.poisson else _shape(wl.draft, layer),
+            "encoder": ["THP", "SAHP", "AttNHP"][wl.target.encoder],
             "sd_events_per_s": round(B * N / (ms_sd / 1e3), 1), "sd_ms_per_call": round(ms_sd, 3),
             "ar_events_per_s": round(B * N / (ms_ar / 1e3), 1), "ar_ms_per_call": round(ms_ar, 3),
             "speedup_vs_ar": round(ms_ar / ms_sd, 3),

@@ -30,7 +30,7 @@ TPPSD_KERNEL_CLASSES = 13
 class tppsd_model_cfg(C.Structure):
     _fields_ = [("layers", C.c_int32), ("d_model", C.c_int32), ("heads", C.c_int32),
                 ("d_ffn", C.c_int32), ("n_mix", C.c_int32), ("n_marks", C.c_int32),
-                ("dtype", C.c_int32)]
+                ("dtype", C.c_int32), ("encoder", C.c_int32)]
 
 
 class tppsd_stats(C.Structure):
@@ -118,7 +118,8 @@ def status_str(s: int) -> str:
 def _cfg(c):
     if isinstance(c, tppsd_model_cfg):
         return c
-    return tppsd_model_cfg(c.layers, c.d_model, c.heads, c.d_ffn, c.n_mix, c.n_marks, c.dtype)
+    return tppsd_model_cfg(c.layers, c.d_model, c.heads, c.d_ffn, c.n_mix, c.n_marks, c.dtype,
+                           getattr(c, "encoder", 0))
 
 
 def _ptr(a, dtype=None, n=None, name="array"):

@@ -35,6 +35,15 @@ def test_library_exports_every_declared_symbol():
 def test_blob_size_agrees_with_generator(wl):
     for cfg in (wl.target, wl.draft) + tuple(wl.drafts):
         assert T.tppsd_blob_floats(cfg) == IN.blob_size(cfg) == IN.model_blob(cfg, 0, 0).size
+        for enc in (CF.SAHP, CF.ATTNHP):
+            c = CF.ModelCfg(**{**cfg.__dict__, "encoder": enc})
+            assert T.tppsd_blob_floats(c) == IN.blob_size(c)
+    small = CF.ModelCfg(2, 32, 2, 64, 4, 3, CF.BF16)
+    for enc in (CF.SAHP, CF.ATTNHP):
+        c = CF.ModelCfg(**{**small.__dict__, "encoder": enc})
+        assert T.tppsd_blob_floats(c) == IN.model_blob(c, 0, 0).size
+    bad = CF.ModelCfg(**{**wl.target.__dict__, "encoder": 3})
+    assert T.tppsd_blob_floats(bad) == 0
 
 
 def test_invalid_shapes_rejected():
