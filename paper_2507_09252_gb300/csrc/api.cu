@@ -450,7 +450,7 @@ static void build_tc_plan(tppsd_ctx* ctx) {
     const Work& w = ctx->work;
     if (c.encoder == 2) {  // AttNHP: only the QKV GEMM over the [z | h] rows
         if (d % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
-        p.bn_qkv = pick_bn(3 * d);
+        p.bn_qkv = d <= 128 ? 64 : pick_bn(3 * d);
         if (!p.bn_qkv) return;
         bool ok = make_tmap_bf16(&p.a_zh, w.xb, 2 * d, w.R, 128);
         for (int l = 0; l < m.L && ok; ++l)
@@ -464,7 +464,9 @@ static void build_tc_plan(tppsd_ctx* ctx) {
         return;
     }
     if (d % 64 || F % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
-    p.bn_qkv = pick_bn(3 * d);
+    // QKV: 64-column tiles up to d = 128 (more CTAs, each with a shorter
+    // epilogue; measured 9.6 -> 8.5 us per launch at 2 304 rows, d = 128)
+    p.bn_qkv = d <= 128 ? 64 : pick_bn(3 * d);
     p.bn_ffn1 = pick_bn(F);
     p.bn_o = ln_cluster_cols(d);
     if (!p.bn_qkv || !p.bn_ffn1 || !p.bn_o) return;

@@ -6,9 +6,14 @@
 // CTAs.  The head is fp32 arithmetic: h W^T is formed as
 // h_hi W_hi + h_hi W_lo + h_lo W_hi with both operands split into two bf16
 // parts (x = x_hi + x_lo), fp32 accumulation in TMEM (relative error about
-// 2^-16 of |h| |W|).  Warps 0-3 split the h rows (coalesced reads) into the
-// two swizzled A operands and later own one row each (TMEM lane); warp 4
-// loads the W_hi / W_lo tiles by TMA; one thread of warp 5 issues the MMAs.
+// 2^-16 of |h| |W|).  Ten warps: warps 0-7 split the h rows (coalesced
+// reads) into the two swizzled A operands and later own one row and 64 of
+// its 128 accumulator columns each (warps w and w+4 share TMEM lanes
+// 32 (w % 4)..); warp 8 loads the W_hi / W_lo tiles by TMA; one thread of
+// warp 9 issues the MMAs.  The small output matrix is staged transposed
+// ([output][128], rows padded to a multiple of 8 with zeros) so that a
+// thread reads four weights per shared-memory load; the two column halves
+// of a row meet through shared memory.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -22,11 +27,17 @@ struct HeadShape {
     static constexpr int TILE = BM * BK * 2;  // 16 KB
     static constexpr int OFF_AH = 0, OFF_AL = KB * TILE, OFF_BH = 2 * KB * TILE, OFF_BL = 3 * KB * TILE;
     static constexpr int OFF_BAR = 4 * KB * TILE;
-    static constexpr int OFF_W = OFF_BAR + 64;  // small output matrix [D][cnt], its bias, b_k1
-    static constexpr size_t smem_bytes(int cnt) { return (size_t)OFF_W + ((size_t)D * cnt + cnt + D) * 4 + 1024; }
+    static constexpr int OFF_PART = OFF_BAR + 64;               // [BM][8] partial sums of column half 1
+    static constexpr int OFF_W = OFF_PART + BM * 8 * 4;         // [cntp][D] outputs, bias [cntp], b_k1 [D]
+    __host__ __device__ static constexpr int cntp(int cnt) { return (cnt + 7) & ~7; }
+    __host__ __device__ static constexpr size_t smem_bytes(int cnt) {
+        return (size_t)OFF_W + ((size_t)cntp(cnt) * D + cntp(cnt) + D) * 4 + 1024;
+    }
 };
 
-__global__ void __launch_bounds__(192, 1)
+__device__ __forceinline__ void head_epi_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+__global__ void __launch_bounds__(320, 1)
     k_head_tc(const __grid_constant__ CUtensorMap mapHi, const __grid_constant__ CUtensorMap mapLo, DevModel m,
               Work w, int R) {
     using S = HeadShape;
@@ -35,15 +46,16 @@ __global__ void __launch_bounds__(192, 1)
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t* bars = (uint64_t*)(smem + S::OFF_BAR);
-    uint64_t* a_ready = bars;      // both A operands written (128 arrivals)
+    uint64_t* a_ready = bars;      // both A operands written (256 arrivals)
     uint64_t* b_full = bars + 1;   // W tiles landed
     uint64_t* done = bars + 2;     // accumulator complete
     uint32_t* tslot = (uint32_t*)(bars + 3);
+    float* part = (float*)(smem + S::OFF_PART);
     float* ws = (float*)(smem + S::OFF_W);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = blockIdx.x, m0 = blockIdx.y * S::BM, rows = min(S::BM, R - m0);
     if (threadIdx.x == 0) {
-        mbar_init(a_ready, 128);
+        mbar_init(a_ready, 256);
         mbar_init(b_full, 1);
         mbar_init(done, 1);
         mbar_fence_init();
@@ -54,7 +66,7 @@ __global__ void __launch_bounds__(192, 1)
     tc_fence_after();
     const uint32_t tmem = *tslot;
 
-    if (warp == 4) {
+    if (warp == 8) {
         if (lane == 0) {
             mbar_arrive_expect_tx(b_full, 2 * S::KB * S::TILE);
             for (int kb = 0; kb < S::KB; ++kb) {
@@ -62,7 +74,7 @@ __global__ void __launch_bounds__(192, 1)
                 tma_load_2d(smem + S::OFF_BL + kb * S::TILE, &mapLo, b_full, kb * S::BK, nb * 128);
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == 9) {
         if (lane == 0) {
             bool ok = mbar_wait(a_ready, 0, w.err, 51);
             ok = ok && mbar_wait(b_full, 0, w.err, 52);
@@ -83,108 +95,124 @@ __global__ void __launch_bounds__(192, 1)
             tc_commit(done);
         }
     } else {
-        const int t = threadIdx.x;
+        const int tid = threadIdx.x;
         // A operands: h rows split into hi / lo bf16, written in the swizzled
-        // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7)).
-        // Loads are issued in batches of 16 float4 per thread so that their
-        // latencies overlap (a load-convert-store loop would pay one global
-        // round trip per float4).
-        constexpr int NV = S::BM * D / 4 / 128, NB = 16;
-#pragma unroll 1
-        for (int b0 = 0; b0 < NV; b0 += NB) {
-            float4 xv[NB];
+        // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7)); all
+        // 16 global loads of a thread are issued before the first store
+        constexpr int NV = S::BM * D / 4 / 256;
+        {
+            float4 xv[NV];
 #pragma unroll
-            for (int j = 0; j < NB; ++j) {
-                const int f = t + (b0 + j) * 128, r = f >> 5, c4 = f & 31;
+            for (int j = 0; j < NV; ++j) {
+                const int f = tid + j * 256, r = f >> 5, c4 = f & 31;
                 xv[j] = r < rows ? *reinterpret_cast<const float4*>(w.x + (size_t)(m0 + r) * D + 4 * c4)
                                  : make_float4(0.f, 0.f, 0.f, 0.f);
             }
 #pragma unroll
-            for (int j = 0; j < NB; ++j) {
-            const int f = t + (b0 + j) * 128, r = f >> 5, c4 = f & 31;
-            const float4 x = xv[j];
-            const float xs[4] = {x.x, x.y, x.z, x.w};
-            uint32_t hi[2], lo[2];
+            for (int j = 0; j < NV; ++j) {
+                const int f = tid + j * 256, r = f >> 5, c4 = f & 31;
+                const float xs[4] = {xv[j].x, xv[j].y, xv[j].z, xv[j].w};
+                uint32_t hi[2], lo[2];
 #pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                const __nv_bfloat162 h2 = __floats2bfloat162_rn(xs[2 * i], xs[2 * i + 1]);
-                const float2 hf = __bfloat1622float2(h2);
-                const __nv_bfloat162 l2 = __floats2bfloat162_rn(xs[2 * i] - hf.x, xs[2 * i + 1] - hf.y);
-                hi[i] = *reinterpret_cast<const uint32_t*>(&h2);
-                lo[i] = *reinterpret_cast<const uint32_t*>(&l2);
-            }
-            const int kb = c4 >> 4, ch = (c4 & 15) >> 1, half = c4 & 1;
-            const int off = kb * S::TILE + r * 128 + ((ch ^ (r & 7)) << 4) + half * 8;
-            *reinterpret_cast<uint2*>(smem + S::OFF_AH + off) = make_uint2(hi[0], hi[1]);
-            *reinterpret_cast<uint2*>(smem + S::OFF_AL + off) = make_uint2(lo[0], lo[1]);
+                for (int i = 0; i < 2; ++i) {
+                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(xs[2 * i], xs[2 * i + 1]);
+                    const float2 hf = __bfloat1622float2(h2);
+                    const __nv_bfloat162 l2 = __floats2bfloat162_rn(xs[2 * i] - hf.x, xs[2 * i + 1] - hf.y);
+                    hi[i] = *reinterpret_cast<const uint32_t*>(&h2);
+                    lo[i] = *reinterpret_cast<const uint32_t*>(&l2);
+                }
+                const int kb = c4 >> 4, ch = (c4 & 15) >> 1, half = c4 & 1;
+                const int off = kb * S::TILE + r * 128 + ((ch ^ (r & 7)) << 4) + half * 8;
+                *reinterpret_cast<uint2*>(smem + S::OFF_AH + off) = make_uint2(hi[0], hi[1]);
+                *reinterpret_cast<uint2*>(smem + S::OFF_AL + off) = make_uint2(lo[0], lo[1]);
             }
         }
         fence_proxy_async_smem();
         mbar_arrive(a_ready);
         // while the tensor cores run: this block's output matrix (columns
-        // col0.. of the [d][3M+K] head map), its bias and b_k1 into shared memory
+        // col0.. of the [d][3M+K] head map) transposed into [cntp][D], its
+        // bias and b_k1
         const int M = m.M, K = m.K, WO = 3 * M + K;
-        const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M;
-        for (int i0 = t; i0 < D * cnt; i0 += 8 * 128) {  // batches of 8 loads per thread
+        const int cnt = nb < 3 ? M : K, col0 = nb < 3 ? nb * M : 3 * M, cp = S::cntp(cnt);
+        float* wb = ws + cp * D;
+        float* bk1 = wb + cp;
+        for (int i0 = tid; i0 < cp * D; i0 += 8 * 256) {  // batches of 8 loads per thread
             float v[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-                const int i = i0 + j * 128;
-                v[j] = i < D * cnt ? m.head_out_t[(size_t)(i / cnt) * WO + col0 + i % cnt] : 0.f;
+                const int i = i0 + j * 256, o = i / D, c = i % D;
+                v[j] = i < cp * D && o < cnt ? m.head_out_t[(size_t)c * WO + col0 + o] : 0.f;
             }
 #pragma unroll
             for (int j = 0; j < 8; ++j)
-                if (i0 + j * 128 < D * cnt) ws[i0 + j * 128] = v[j];
+                if (i0 + j * 256 < cp * D) ws[i0 + j * 256] = v[j];
         }
-        for (int i = t; i < cnt; i += 128) ws[D * cnt + i] = m.head_out_b[col0 + i];
-        for (int i = t; i < D; i += 128) ws[D * cnt + cnt + i] = m.head_ek_b[3 * D + i];
-        asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
-        // row t of the tile: its 128 columns of block nb, then its outputs
+        for (int i = tid; i < cp; i += 256) wb[i] = i < cnt ? m.head_out_b[col0 + i] : 0.f;
+        for (int i = tid; i < D; i += 256) bk1[i] = m.head_ek_b[3 * D + i];
+        head_epi_sync();
+        // row t of the tile, accumulator columns 64 hf .. 64 hf + 63
+        const int q = warp & 3, hf = warp >> 2, t = q * 32 + lane;
         const bool live = t < rows && w.row_seq[m0 + t] >= 0;
         mbar_wait(done, 0, w.err, 53);
         tc_fence_after();
-        const uint32_t tl = tmem + ((uint32_t)(warp * 32) << 16);
-        const float* bk1 = ws + D * cnt + cnt;
+        float v[64];
+        tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + 64 * hf, v);
+        if (nb == 3) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) v[i] = tanhf(v[i] + bk1[64 * hf + i]);
+        }
         float* dst = w.heads + (size_t)(m0 + t) * WO + col0;
-        const float* Wt = ws;  // [d][cnt]
-        float mx = -INFINITY, sum = 0.f;         // online log-sum-exp of the logits
-        for (int o0 = 0; o0 < cnt; o0 += 8) {
+        const bool norm = nb == 0 || nb == 3;  // log w, log f: subtract log sum exp
+        float mx = -INFINITY, sum = 0.f;
+        for (int o0 = 0; o0 < cp; o0 += 8) {
             float acc[8];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[j] = o0 + j < cnt ? ws[D * cnt + o0 + j] : 0.f;
-            // the row's 128 columns, 64 at a time from TMEM (block 3: tanh(. + b_k1))
-            for (int hf = 0; hf < 2; ++hf) {
-                float v[64];
-                tmem_ld64(tl + 64 * hf, v);
-                if (nb == 3) {
+            for (int j = 0; j < 8; ++j) {
+                const float4* wr = reinterpret_cast<const float4*>(ws + (o0 + j) * D + 64 * hf);
+                float a0 = 0.f, a1 = 0.f;
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) v[i] = tanhf(v[i] + bk1[64 * hf + i]);
+                for (int i = 0; i < 16; i += 2) {
+                    const float4 w0 = wr[i], w1 = wr[i + 1];
+                    a0 = fmaf(w0.x, v[4 * i], a0);
+                    a0 = fmaf(w0.y, v[4 * i + 1], a0);
+                    a0 = fmaf(w0.z, v[4 * i + 2], a0);
+                    a0 = fmaf(w0.w, v[4 * i + 3], a0);
+                    a1 = fmaf(w1.x, v[4 * i + 4], a1);
+                    a1 = fmaf(w1.y, v[4 * i + 5], a1);
+                    a1 = fmaf(w1.z, v[4 * i + 6], a1);
+                    a1 = fmaf(w1.w, v[4 * i + 7], a1);
                 }
+                acc[j] = a0 + a1;
+            }
+            if (hf == 1) {
 #pragma unroll
-                for (int i = 0; i < 64; ++i) {
-                    const float* wr = Wt + (64 * hf + i) * cnt + o0;
+                for (int j = 0; j < 8; ++j) part[t * 8 + j] = acc[j];
+            }
+            head_epi_sync();
+            if (hf == 0) {
+#pragma unroll
+                for (int j = 0; j < 8; ++j) acc[j] = wb[o0 + j] + (acc[j] + part[t * 8 + j]);
+                if (norm) {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        if (o0 + j >= cnt) continue;
+                        const float mn = fmaxf(mx, acc[j]);
+                        sum = sum * expf(mx - mn) + expf(acc[j] - mn);
+                        mx = mn;
+                    }
+                }
+                if (live) {
+                    const float sub = norm && cp == 8 ? mx + logf(sum) : 0.f;  // one chunk: final here
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
-                        if (o0 + j < cnt) acc[j] = fmaf(wr[j], v[i], acc[j]);
+                        if (o0 + j < cnt) dst[o0 + j] = acc[j] - sub;
                 }
             }
-            if (!live) continue;
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                if (o0 + j >= cnt) continue;
-                dst[o0 + j] = acc[j];
-                if (nb == 0 || nb == 3) {
-                    const float mn = fmaxf(mx, acc[j]);
-                    sum = sum * expf(mx - mn) + expf(acc[j] - mn);
-                    mx = mn;
-                }
-            }
+            head_epi_sync();  // part is rewritten by the next chunk
         }
-        if (live) {
-            if (nb == 0 || nb == 3) {  // log w, log f: subtract log sum exp
-                const float lz = mx + logf(sum);
-                for (int o = 0; o < cnt; ++o) dst[o] -= lz;
-            }
+        if (hf == 0 && live && norm && cp > 8) {  // several chunks: normalise what was written
+            const float lz = mx + logf(sum);
+            for (int o = 0; o < cnt; ++o) dst[o] -= lz;
         }
     }
     tc_fence_before();
@@ -205,7 +233,7 @@ cudaError_t launch_head_tc(const CUtensorMap& hi, const CUtensorMap& lo, const D
     const size_t sm = HeadShape::smem_bytes(m.M > m.K ? m.M : m.K);
     cudaError_t e = cudaFuncSetAttribute(k_head_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    return launch_k(k_head_tc, dim3(4, (R + 127) / 128), dim3(192), sm, st, hi, lo, m, w, R);
+    return launch_k(k_head_tc, dim3(4, (R + 127) / 128), dim3(320), sm, st, hi, lo, m, w, R);
 }
 
 }  // namespace tppsd
