@@ -35,6 +35,7 @@ struct HostModel {
     DevModel dm{};
     void* dbuf = nullptr;
     void* tbuf = nullptr;
+    void* pbuf = nullptr;
 };
 
 struct GraphEntry {
@@ -401,6 +402,83 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     th.v_k2 = (const float*)(tbp + tk2); th.b_k2 = (const float*)(tbp + tbk2);
     mt.base = tbp;
     mt.bytes = tb.size();
+    // lane-packed, self-contained copy: chunk c (CH consecutive inputs) of
+    // output j at element (c * rows + j) * CH, CH = 16 bytes / element
+    std::vector<char> pb;
+    auto padd = [&](const void* src, size_t bytes) {
+        size_t off = (pb.size() + 15) & ~(size_t)15;
+        pb.resize(off + bytes);
+        memcpy(pb.data() + off, src, bytes);
+        return off;
+    };
+    auto pmat = [&](size_t off, size_t rows, size_t cols, bool storage) {  // blob [rows][cols]
+        const bool b16 = storage && bf;
+        const size_t CH = b16 ? 8 : 4, nch = (cols + CH - 1) / CH;
+        if (b16) {
+            std::vector<uint16_t> t(nch * rows * CH, 0);
+            for (size_t r = 0; r < rows; ++r)
+                for (size_t c2 = 0; c2 < cols; ++c2)
+                    t[((c2 / CH) * rows + r) * CH + c2 % CH] = f32_to_bf16_bits(blob[off + r * cols + c2]);
+            return padd(t.data(), t.size() * 2);
+        }
+        std::vector<float> t(nch * rows * CH, 0.f);
+        for (size_t r = 0; r < rows; ++r)
+            for (size_t c2 = 0; c2 < cols; ++c2) t[((c2 / CH) * rows + r) * CH + c2 % CH] = blob[off + r * cols + c2];
+        return padd(t.data(), t.size() * 4);
+    };
+    auto pvec = [&](size_t off, size_t n) { return padd(blob.data() + off, n * sizeof(float)); };
+    std::vector<LB> pl(L);
+    for (int l = 0; l < L; ++l) {
+        pl[l].wqkv = pmat(lo[l].wqkv, 3 * (size_t)d, din, true);
+        if (att) continue;
+        pl[l].wo = pmat(lo[l].wo, d, d, true);
+        pl[l].w1 = pmat(lo[l].w1, F, d, true);
+        pl[l].w2 = pmat(lo[l].w2, d, F, true);
+    }
+    for (int l = 0; l < L; ++l) {
+        pl[l].bqkv = pvec(lo[l].bqkv, 3 * d);
+        if (att) continue;
+        pl[l].bo = pvec(lo[l].bo, d);
+        pl[l].g1 = pvec(lo[l].g1, d); pl[l].b1n = pvec(lo[l].b1n, d);
+        pl[l].b1 = pvec(lo[l].b1, F); pl[l].b2 = pvec(lo[l].b2, d);
+        pl[l].g2 = pvec(lo[l].g2, d); pl[l].b2n = pvec(lo[l].b2n, d);
+    }
+    const size_t p_emb = pvec(o_emb, (size_t)K * d);
+    const size_t pE = pmat(oE, 3 * (size_t)d, d, false);
+    const size_t pvw = pmat(ovw, M, d, false), pbw = pvec(obw, M);
+    const size_t pvm = pmat(ovm, M, d, false), pbm = pvec(obm, M);
+    const size_t pvs = pmat(ovs, M, d, false), pbs = pvec(obs, M);
+    const size_t pk1 = pmat(ok1, d, d, false), pbk1 = pvec(obk1, d);
+    const size_t pk2 = pmat(ok2, K, d, false), pbk2 = pvec(obk2, K);
+    const size_t p_om = padd(tenc.data(), tenc.size() * sizeof(double));
+    pb.resize((pb.size() + 15) & ~(size_t)15);  // whole 16-byte chunks: one bulk copy stages it
+    CK(cudaMalloc(&hm.pbuf, pb.size()));
+    ctx->allocs.push_back(hm.pbuf);
+    CK(cudaMemcpy(hm.pbuf, pb.data(), pb.size(), cudaMemcpyHostToDevice));
+    const char* pbp = (const char*)hm.pbuf;
+    DevModelT& mp = m.p;
+    mp.type_emb = (const float*)(pbp + p_emb);
+    mp.tenc = (const double*)(pbp + p_om);
+    for (int l = 0; l < L; ++l) {
+        LayerW& w = mp.layer[l];
+        w = LayerW{};
+        w.w_qkv = pbp + pl[l].wqkv; w.b_qkv = (const float*)(pbp + pl[l].bqkv);
+        if (att) continue;
+        w.w_o = pbp + pl[l].wo; w.b_o = (const float*)(pbp + pl[l].bo);
+        w.ln1_g = (const float*)(pbp + pl[l].g1); w.ln1_b = (const float*)(pbp + pl[l].b1n);
+        w.w_1 = pbp + pl[l].w1; w.b_1 = (const float*)(pbp + pl[l].b1);
+        w.w_2 = pbp + pl[l].w2; w.b_2 = (const float*)(pbp + pl[l].b2);
+        w.ln2_g = (const float*)(pbp + pl[l].g2); w.ln2_b = (const float*)(pbp + pl[l].b2n);
+    }
+    HeadW& ph = mp.head;
+    ph.E = (const float*)(pbp + pE);
+    ph.v_w = (const float*)(pbp + pvw); ph.b_w = (const float*)(pbp + pbw);
+    ph.v_mu = (const float*)(pbp + pvm); ph.b_mu = (const float*)(pbp + pbm);
+    ph.v_s = (const float*)(pbp + pvs); ph.b_s = (const float*)(pbp + pbs);
+    ph.v_k1 = (const float*)(pbp + pk1); ph.b_k1 = (const float*)(pbp + pbk1);
+    ph.v_k2 = (const float*)(pbp + pk2); ph.b_k2 = (const float*)(pbp + pbk2);
+    mp.base = pbp;
+    mp.bytes = pb.size();
     return TPPSD_OK;
 }
 
@@ -664,7 +742,11 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
         ++n;
     } else if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
-        if (draft_team_supported(ctx->D.dm) && (ctx->D.dm.enc == 2 || !getenv("TPPSD_DRAFT_CTA")))
+        const bool team = draft_team_supported(ctx->D.dm) && (ctx->D.dm.enc == 2 || !getenv("TPPSD_DRAFT_CTA"));
+        if (team && draft_lane_supported(ctx->D.dm, ctx->kvD.n_max) && !getenv("TPPSD_DRAFT_TEAM"))
+            CK(launch_draft_lane(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
+                                 ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
+        else if (team)
             CK(launch_draft_team(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
         else

@@ -586,4 +586,424 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     return launch_team<bf16, 32>(a, B, kvs, ws, area, wb, st);
 }
 
+
+// ---------------------------------------------------------------- lane form
+// Draft models with d <= 32 and one or two heads.  Lane i of every warp of
+// a sequence's team holds component i of the hidden state, so residual adds,
+// LayerNorms and activations run in registers, and each warp computes the
+// matrix-vector products it needs itself from the lane-packed model copy
+// (chunk c of output j at (c * out + j) * CH: the lanes of a warp read 512
+// consecutive bytes per load, CH weights each).  Per layer warp w attends
+// with head w % nh over key range w / nh of its key positions (scores kept
+// in shared memory, one max and one exponential per key, no rescaling),
+// reduces its numerator by a scatter-reduce across lanes and publishes it;
+// after one team barrier every warp merges the ranges of every head itself.
+// The FFN hidden units are split in quarters (warp w computes quarter w and
+// its FFN2 partial; a second barrier sums them).  The draw: warp 0 computes
+// the time head [E_1; E_2; E_3] h and (w, mu, s) and draws tau, warp 3 the
+// mark head and the mark, then a third barrier hands (t, k) to every warp.
+
+__device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
+
+// sum over chunks c < nch of the CH products of output j's chunk c with
+// in[c * CH ..] (in: shared, 16-byte aligned; P: lane-packed with OUT outputs)
+template <typename TW>
+__device__ __forceinline__ float pdot(const TW* __restrict__ P, int OUT, int j, const float* __restrict__ in,
+                                      int nch) {
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+    const uint4* w = reinterpret_cast<const uint4*>(P) + j;
+    const float4* x = reinterpret_cast<const float4*>(in);
+#pragma unroll 4
+    for (int c = 0; c < nch; ++c) {
+        const uint4 u = w[(size_t)c * OUT];
+        if constexpr (sizeof(TW) == 2) {
+            const float4 x0 = x[2 * c], x1 = x[2 * c + 1];
+            a0 = fmaf(bf_lo(u.x), x0.x, a0);
+            a1 = fmaf(bf_hi(u.x), x0.y, a1);
+            a2 = fmaf(bf_lo(u.y), x0.z, a2);
+            a3 = fmaf(bf_hi(u.y), x0.w, a3);
+            a0 = fmaf(bf_lo(u.z), x1.x, a0);
+            a1 = fmaf(bf_hi(u.z), x1.y, a1);
+            a2 = fmaf(bf_lo(u.w), x1.z, a2);
+            a3 = fmaf(bf_hi(u.w), x1.w, a3);
+        } else {
+            const float4 x0 = x[c];
+            a0 = fmaf(__uint_as_float(u.x), x0.x, a0);
+            a1 = fmaf(__uint_as_float(u.y), x0.y, a1);
+            a2 = fmaf(__uint_as_float(u.z), x0.z, a2);
+            a3 = fmaf(__uint_as_float(u.w), x0.w, a3);
+        }
+    }
+    return (a0 + a1) + (a2 + a3);
+}
+
+// One halving step of a scatter-reduce over lane pairs (lane, lane ^ OFF):
+// the lane with bit OFF set keeps the upper CNT / 2 entries (moved down),
+// the other the lower ones, each adding its partner's copy.
+template <int CNT, int OFF, int N>
+__device__ __forceinline__ void rs_step(float (&v)[N], int lane) {
+    const bool up = (lane & OFF) != 0;
+#pragma unroll
+    for (int i = 0; i < CNT / 2; ++i) {
+        const float send = up ? v[i] : v[CNT / 2 + i];
+        const float keep = up ? v[CNT / 2 + i] : v[i];
+        v[i] = keep + __shfl_xor_sync(FULL, send, OFF);
+    }
+}
+// Sum of v[c] over the 32 lanes; lane receives the total of entry
+// (N == 16 ? lane >> 1 : lane).
+template <int N>
+__device__ __forceinline__ float warp_scatter_sum(float (&v)[N], int lane) {
+    static_assert(N == 16 || N == 32, "16 or 32 entries");
+    if constexpr (N == 32) rs_step<32, 16>(v, lane);
+    rs_step<N == 32 ? 16 : 16, N == 32 ? 8 : 16>(v, lane);
+    rs_step<8, N == 32 ? 4 : 8>(v, lane);
+    rs_step<4, N == 32 ? 2 : 4>(v, lane);
+    rs_step<2, N == 32 ? 1 : 2>(v, lane);
+    if constexpr (N == 16) v[0] += __shfl_xor_sync(FULL, v[0], 1);
+    return v[0];
+}
+
+// LayerNorm of the d values held by lanes < d (v; others ignored).
+__device__ __forceinline__ float lane_ln(float v, int lane, int d, const float* g, const float* b) {
+    const bool live = lane < d;
+    const float mean = warp_sum(live ? v : 0.f) / d;
+    const float c = live ? v - mean : 0.f;
+    const float inv = 1.0f / sqrtf(warp_sum(c * c) / d + LN_EPS);
+    return live ? c * inv * g[lane] + b[lane] : 0.f;
+}
+
+// Shared-memory floats of one team besides its KV: head row, attention
+// partials (two sets of 4 warps x (max, sum, -, -, 32 numerators)), FFN2
+// partials (4 x 32), the drawn event (16 bytes), then per warp: input
+// vector (64), attention output / fp32 hidden state (32), FFN quarter (64),
+// head activations (96), query (32) and the key scores (sc).
+__host__ __device__ inline int lane_team_floats(int W, int sc) {
+    return ((W + 3) & ~3) + 2 * 4 * 36 + 128 + 4 + 4 * (288 + sc);
+}
+
+template <typename T, int DH>
+__global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_bytes, int sc_stride) {
+    pdl_wait();
+    extern __shared__ __align__(16) char smem[];
+    __shared__ uint64_t wbar;
+    const DevModelT& mp = a.m.p;
+    const char* gb = mp.base;
+    const uint32_t wb = (uint32_t)mp.bytes;
+    if (threadIdx.x == 0) {  // stage the packed model once per CTA
+        mbar_init(&wbar, 1);
+        mbar_fence_init();
+        mbar_arrive_expect_tx(&wbar, wb);
+        bulk_load(smem, gb, wb, &wbar);
+    }
+    __syncthreads();
+    mbar_wait(&wbar, 0, a.err, 14);
+    // shared-memory address of a piece of the packed model
+    auto sm = [&](const void* g) -> const char* { return smem + ((const char*)g - gb); };
+    const int team = threadIdx.x >> 7;
+    const int s = blockIdx.x * 2 + team;
+    const CallParams& P = *a.P;
+    if (s >= P.B || a.ss.done[s]) return;  // the rest synchronises within the team only
+    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
+    const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
+    const int n_max = a.kv.n_max;
+    const int S = 4 / NH, hw = warp % NH, spw = warp / NH;  // this warp's head and key range
+    constexpr int CH = 16 / sizeof(T);
+    const bool att_enc = a.m.enc == 2;
+    char* area = smem + wb + (size_t)team * area_bytes;
+    const size_t kvb = ((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15;
+    T* kvs = (T*)area;
+    uint64_t* bar = (uint64_t*)(area + kvb);
+    float* hd = (float*)(area + kvb + 16);
+    float* red = hd + ((W + 3) & ~3);  // [2][4][36]
+    float* part = red + 2 * 4 * 36;    // [4][32]
+    double* ev_t = (double*)(part + 128);
+    int* ev_k = (int*)(ev_t + 1);
+    float* mine = part + 128 + 4 + warp * (288 + sc_stride);
+    float* v_in = mine;        // [zin | xin] (AttNHP) or xin
+    float* v_att = mine + 64;  // attention output; fp32 hidden state for the head
+    float* v_hid = mine + 96;  // this warp's FFN quarter
+    float* v_e = mine + 160;   // head activations
+    float* v_q = mine + 256;   // query of this warp's head
+    float* sc = mine + 288;    // scores of this warp's keys
+    const SeqState& ss = a.ss;
+    const int n = ss.n_emit[s], nd = ss.n_draft[s];
+    auto gk = [&](int l, int w) -> T* {
+        return (T*)(w ? a.kv.v : a.kv.k) + (((size_t)l * a.kv.Bmax + s) * NH) * (size_t)n_max * DH;
+    };
+    auto sk = [&](int l, int w) -> T* { return kvs + (((size_t)l * 2 + w) * NH) * (size_t)n_max * DH; };
+    if (nd > 0) {  // each (layer, K/V, head) block of positions 0..nd-1 is contiguous in HBM
+        if (tid == 0) {
+            const uint32_t bytes = (uint32_t)nd * DH * sizeof(T);
+            mbar_init(bar, 1);
+            mbar_fence_init();
+            mbar_arrive_expect_tx(bar, bytes * (uint32_t)(L * 2 * NH));
+            for (int l = 0; l < L; ++l)
+                for (int w = 0; w < 2; ++w)
+                    for (int h = 0; h < NH; ++h)
+                        bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
+        }
+        team_sync();
+        mbar_wait(bar, 0, a.err, 12);
+    }
+    const float* type_emb = (const float*)sm(mp.type_emb);
+    const double* tenc = (const double*)sm(mp.tenc);
+    // Encoding of event (t, k) (App. D.4 temporal encoding z_i = sin / cos
+    // (a_i + b_i t), angle reduced mod 2 pi in fp64, plus the mark
+    // embedding): returns x_lane and writes the rounded GEMM input.
+    auto embed = [&](double t, int k) -> float {
+        float xv = 0.f;
+        if (lane < d) {
+            const double ang = tenc[lane] + tenc[d + lane] * t;
+            const double rd = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
+            float sv, cv;
+            sincosf((float)rd, &sv, &cv);
+            const float z = (lane & 1) ? cv : sv;
+            xv = z + type_emb[(size_t)k * d + lane];
+            if (att_enc) {
+                v_in[lane] = St<T>::rnd(z);
+                v_in[d + lane] = St<T>::rnd(xv);
+            } else {
+                v_in[lane] = St<T>::rnd(xv);
+            }
+        }
+        __syncwarp();
+        return xv;
+    };
+    const float scale = 1.4426950408889634f / sqrtf((float)DH);
+    // Layers of the encode step at position p; x holds the embedding on entry
+    // and the final hidden state on exit (lanes < d, every warp).
+    auto layers = [&](int p, float x) -> float {
+        const int nk = p + 1, per = (nk + S - 1) / S, lo = spw * per, hi = min(nk, lo + per);
+        const bool writer = spw == p / per;  // the warp of this head whose range holds key p
+        for (int l = 0; l < L; ++l) {
+            const LayerW& Wl = mp.layer[l];
+            const T* wqkv = (const T*)sm(Wl.w_qkv);
+            const float* bqkv = (const float*)sm(Wl.b_qkv);
+            const int nin = (att_enc ? 2 * d : d) / CH;
+            // q of head hw; the writer also appends k and v at position p
+            for (int o = lane; o < (writer ? 3 * DH : DH); o += 32) {
+                const int part3 = o / DH, c = o - part3 * DH, row = part3 * d + hw * DH + c;
+                const float v = St<T>::rnd(pdot<T>(wqkv, 3 * d, row, v_in, nin) + bqkv[row]);
+                if (part3 == 0) {
+                    v_q[c] = v * scale;
+                } else {
+                    const size_t off = ((size_t)hw * n_max + p) * DH + c;
+                    St<T>::st(gk(l, part3 - 1) + off, v);
+                    St<T>::st(sk(l, part3 - 1) + off, v);
+                }
+            }
+            __syncwarp();
+            // attention of head hw over keys lo..hi-1 (exp2 units)
+            float q[DH];
+#pragma unroll
+            for (int c = 0; c < DH; ++c) q[c] = v_q[c];
+            const T* kb = sk(l, 0) + (size_t)hw * n_max * DH;
+            const T* vb = sk(l, 1) + (size_t)hw * n_max * DH;
+            float mx = -INFINITY;
+#pragma unroll 2
+            for (int j = lo + lane; j < hi; j += 32) {
+                float kr[DH];
+                load_row16<T, DH>(kb + (size_t)j * DH, kr);
+                float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+                for (int c = 0; c < DH; c += 2) {
+                    s0 = fmaf(q[c], kr[c], s0);
+                    s1 = fmaf(q[c + 1], kr[c + 1], s1);
+                }
+                const float sv = s0 + s1;
+                sc[j - lo] = sv;
+                mx = fmaxf(mx, sv);
+            }
+            mx = warp_max(mx);
+            float ll = 0.f, o[DH];
+#pragma unroll
+            for (int c = 0; c < DH; ++c) o[c] = 0.f;
+#pragma unroll 2
+            for (int j = lo + lane; j < hi; j += 32) {
+                const float pj = exp2f(sc[j - lo] - mx);
+                float vr[DH];
+                load_row16<T, DH>(vb + (size_t)j * DH, vr);
+                ll += pj;
+#pragma unroll
+                for (int c = 0; c < DH; ++c) o[c] = fmaf(pj, vr[c], o[c]);
+            }
+            ll = warp_sum(ll);
+            const float oc = warp_scatter_sum<DH>(o, lane);
+            float* rw = red + ((l & 1) * 4 + warp) * 36;
+            if (lane == 0) {
+                rw[0] = mx;
+                rw[1] = ll;
+            }
+            if (DH == 32 || !(lane & 1)) rw[4 + (DH == 16 ? lane >> 1 : lane)] = oc;
+            team_sync();
+            // merge the key ranges of head lane / DH for output component lane
+            float at = 0.f;
+            if (lane < d) {
+                const int hj = lane / DH, c = lane - hj * DH;
+                const float* rb = red + (l & 1) * 4 * 36;
+                float Mx = -INFINITY;
+                for (int sp = 0; sp < S; ++sp) Mx = fmaxf(Mx, rb[(sp * NH + hj) * 36]);
+                float Lx = 0.f, Ox = 0.f;
+                for (int sp = 0; sp < S; ++sp) {
+                    const float* src = rb + (sp * NH + hj) * 36;
+                    if (src[0] == -INFINITY) continue;
+                    const float e = exp2f(src[0] - Mx);
+                    Lx += src[1] * e;
+                    Ox += src[4 + c] * e;
+                }
+                at = att_enc ? Ox / (Lx + exp2f(-Mx)) : St<T>::rnd(Ox / Lx);
+            }
+            if (att_enc) {  // AttNHP (App. D.4): h <- h + tanh(a), no projection or FFN
+                if (lane < d) {
+                    x += tanhf(at);
+                    v_in[d + lane] = St<T>::rnd(x);
+                }
+                __syncwarp();
+                continue;
+            }
+            // x = LN1(x + W_o a + b_o)
+            if (lane < d) v_att[lane] = at;
+            __syncwarp();
+            float y = 0.f;
+            if (lane < d) y = pdot<T>((const T*)sm(Wl.w_o), d, lane, v_att, d / CH) + ((const float*)sm(Wl.b_o))[lane];
+            x = lane_ln(x + y, lane, d, (const float*)sm(Wl.ln1_g), (const float*)sm(Wl.ln1_b));
+            if (lane < d) v_in[lane] = St<T>::rnd(x);
+            __syncwarp();
+            // FFN quarter of this warp: hidden units f0 .. f0 + F/4 - 1
+            const int Fq = F >> 2, f0 = warp * Fq;
+            const T* w1 = (const T*)sm(Wl.w_1);
+            const float* b1 = (const float*)sm(Wl.b_1);
+            for (int jj = lane; jj < Fq; jj += 32)
+                v_hid[jj] = St<T>::rnd(fmaxf(pdot<T>(w1, F, f0 + jj, v_in, d / CH) + b1[f0 + jj], 0.f));
+            __syncwarp();
+            if (lane < d)
+                part[warp * 32 + lane] =
+                    pdot<T>((const T*)sm(Wl.w_2) + (size_t)(f0 / CH) * d * CH, d, lane, v_hid, Fq / CH);
+            team_sync();
+            // x = LN2(x + W_2 relu(.) + b_2)
+            float y2 = 0.f;
+            if (lane < d)
+                y2 = ((const float*)sm(Wl.b_2))[lane] +
+                     ((part[lane] + part[32 + lane]) + (part[64 + lane] + part[96 + lane]));
+            x = lane_ln(x + y2, lane, d, (const float*)sm(Wl.ln2_g), (const float*)sm(Wl.ln2_b));
+            if (lane < d) v_in[lane] = St<T>::rnd(x);
+            __syncwarp();
+        }
+        return x;
+    };
+    float x = 0.f;
+    for (int p = nd; p < n; ++p) {  // catch-up over events already emitted
+        const size_t so = (size_t)s * ss.n_max + p;
+        x = embed(ss.t[so], min(max(ss.k[so], 0), K - 1));
+        x = layers(p, x);
+    }
+    if (tid == 0) {
+        const long long last = n + a.gamma - 2;  // last position the round encodes
+        atomicAdd(&a.st->draft_keys, (unsigned long long)((last + 1) * (last + 2) / 2 - (long long)nd * (nd + 1) / 2));
+    }
+    const HeadW& H = mp.head;
+    double t_prev = ss.t[(size_t)s * ss.n_max + n - 1];
+    for (int l = 1; l <= a.gamma; ++l) {
+        const int p = n + l - 1;  // index of the drafted event
+        const size_t so = (size_t)s * ss.n_max + p;
+        if (warp == 0) {
+            // time head (Sec. 4.2): e_r = E_r h, then log w, mu, s; tau by
+            // z ~ Cat(w), eps by Box-Muller, tau = exp(mu_z + sigma_z eps)
+            if (lane < d) v_att[lane] = x;
+            __syncwarp();
+            const float* E = (const float*)sm(H.E);
+            if (lane < d) {
+#pragma unroll
+                for (int r = 0; r < 3; ++r) v_e[r * d + lane] = pdot<float>(E, 3 * d, r * d + lane, v_att, d / 4);
+            }
+            __syncwarp();
+            for (int o = lane; o < 3 * M; o += 32) {
+                const int seg = o / M, jj = o - seg * M;
+                const float* V = (const float*)sm(seg == 0 ? H.v_w : seg == 1 ? H.v_mu : H.v_s);
+                const float* bb = (const float*)sm(seg == 0 ? H.b_w : seg == 1 ? H.b_mu : H.b_s);
+                hd[o] = pdot<float>(V, M, jj, v_e + seg * d, d / 4) + bb[jj];
+            }
+            __syncwarp();
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
+            const int z = warp_logsoftmax_pick<2>(hd, M, u.x);
+            if (lane == 0) {
+                const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
+                const float tau = expf(hd[M + z] + expf(hd[2 * M + z]) * eps);
+                const double t = t_prev + (double)tau;
+                ss.tau[so] = tau;
+                ss.t[so] = t;
+                *ev_t = t;
+            }
+        } else if (warp == 3) {
+            // mark head: a = tanh(V_k1 h + b_k1), log f = log_softmax(V_k2 a + b_k2)
+            if (lane < d) v_att[lane] = x;
+            __syncwarp();
+            if (lane < d)
+                v_e[lane] = tanhf(pdot<float>((const float*)sm(H.v_k1), d, lane, v_att, d / 4) +
+                                  ((const float*)sm(H.b_k1))[lane]);
+            __syncwarp();
+            const float* V2 = (const float*)sm(H.v_k2);
+            const float* b2 = (const float*)sm(H.b_k2);
+            for (int o = lane; o < K; o += 32) hd[3 * M + o] = pdot<float>(V2, K, o, v_e, d / 4) + b2[o];
+            __syncwarp();
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
+            const int k = warp_logsoftmax_pick<8>(hd + 3 * M, K, u.w);
+            if (lane == 0) {
+                ss.k[so] = k;
+                *ev_k = k;
+            }
+        }
+        team_sync();
+        const double t_new = *ev_t;
+        const int k_new = *ev_k;
+        t_prev = t_new;
+        if (warp == 1) {
+            float* rec = a.heads + ((size_t)s * a.gamma_max + (l - 1)) * W;
+            for (int i = lane; i < W; i += 32) rec[i] = hd[i];
+        }
+        if (l < a.gamma) x = layers(p, embed(t_new, k_new));
+    }
+    pdl_trigger();
+}
+
+// Shared-memory bytes of one team of the lane form (0: the shape is not covered).
+static size_t lane_area(const DevModel& m, int n_max, int* sc_out) {
+    const int CH = m.dtype == 1 ? 8 : 4;
+    const bool shape = (m.nh == 1 && (m.dh == 16 || m.dh == 32)) || (m.nh == 2 && m.dh == 16);
+    if (!shape || m.d % CH || m.M > 64 || m.K > 256 || m.L < 1) return 0;
+    if (m.enc != 2 && (m.F % (4 * CH) || m.F > 256)) return 0;
+    const size_t eb = m.dtype == 1 ? 2 : 4;
+    const int S = 4 / m.nh;
+    const int sc = (((n_max + S - 1) / S) + 3) & ~3;
+    const size_t kvb = ((size_t)m.L * 2 * n_max * m.d * eb + 15) & ~(size_t)15;
+    if (sc_out) *sc_out = sc;
+    return kvb + 16 + sizeof(float) * (size_t)lane_team_floats(3 * m.M + m.K, sc);
+}
+
+int draft_lane_supported(const DevModel& m, int n_max) {
+    const size_t area = lane_area(m, n_max, nullptr);
+    if (!area || m.p.bytes % 16) return 0;
+    return m.p.bytes + 2 * area <= 224 * 1024;
+}
+
+cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqState& ss,
+                              const CallParams* dp, int B, int gamma, float* draft_heads,
+                              int gamma_max, DevStats* stats, int* err, cudaStream_t st) {
+    DraftTeamArgs a{};
+    a.m = m; a.kv = kv; a.ss = ss; a.P = dp; a.st = stats; a.heads = draft_heads;
+    a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
+    int sc = 0;
+    const size_t area = lane_area(m, kv.n_max, &sc);
+    const size_t sm = m.p.bytes + 2 * area;
+    auto go = [&](auto kern) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+        if (e != cudaSuccess) return e;
+        return launch_k(kern, dim3((B + 1) / 2), dim3(256), sm, st, a, (int)area, sc);
+    };
+    if (m.dtype == 0) return m.dh == 16 ? go(k_draft_lane<float, 16>) : go(k_draft_lane<float, 32>);
+    return m.dh == 16 ? go(k_draft_lane<bf16, 16>) : go(k_draft_lane<bf16, 32>);
+}
+
 }  // namespace tppsd

@@ -81,6 +81,12 @@ struct DevModel {
     const void* head_ek_hi;  // [4d][d] bf16: head_ek_w = hi + lo (split of each fp32 value)
     const void* head_ek_lo;
     DevModelT t;             // transposed copy (read by the per-sequence draft kernel)
+    // Lane-packed copy (same struct, read by the lane form of the draft
+    // kernel): a matrix W [out][in] is stored as chunks of CH = 16 / sizeof
+    // (element) consecutive inputs, chunk c of output j at element
+    // (c * out + j) * CH, so the lanes of a warp that own consecutive outputs
+    // read consecutive 16-byte words.  Vectors as in the other copies.
+    DevModelT p;
     __host__ __device__ int head_width() const { return 3 * M + K; }
 };
 
@@ -291,6 +297,12 @@ cudaError_t launch_score_logs(const DevModel& m, const SeqState& ss, const Work&
 size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
 // One-CTA-per-sequence draft (draft.cu) for the shapes it is compiled for.
 int draft_team_supported(const DevModel& m);
+// Lane form of the draft kernel (draft.cu) for d <= 32 models whose packed
+// copy and two sequences' draft KV fit in shared memory.
+int draft_lane_supported(const DevModel& m, int n_max);
+cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqState& ss,
+                              const CallParams* dp, int B, int gamma, float* draft_heads,
+                              int gamma_max, DevStats* stats, int* err, cudaStream_t st);
 cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st);
