@@ -451,6 +451,34 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     const size_t pk1 = pmat(ok1, d, d, false), pbk1 = pvec(obk1, d);
     const size_t pk2 = pmat(ok2, K, d, false), pbk2 = pvec(obk2, K);
     const size_t p_om = padd(tenc.data(), tenc.size() * sizeof(double));
+    // the encoding table as fp32 pairs (hi + lo = the fp64 value to ~48 bits)
+    std::vector<float> tff(4 * (size_t)d);
+    for (int j = 0; j < d; ++j)
+        for (int w = 0; w < 2; ++w) {
+            const double v = tenc[(size_t)w * d + j];
+            const float hi = (float)v;
+            tff[(size_t)(2 * w) * d + j] = hi;
+            tff[(size_t)(2 * w + 1) * d + j] = (float)(v - (double)hi);
+        }
+    const size_t p_tff = padd(tff.data(), tff.size() * 4);
+    // time head folded into one map: rows V_w E_1, V_mu E_2, V_s E_3 (fp64
+    // products rounded once), bias b_w, b_mu, b_s
+    std::vector<float> ht((size_t)3 * M * d), htb((size_t)3 * M);
+    const size_t vsrc[3] = {ovw, ovm, ovs}, vb[3] = {obw, obm, obs};
+    for (int seg = 0; seg < 3; ++seg)
+        for (int j = 0; j < M; ++j) {
+            htb[(size_t)seg * M + j] = blob[vb[seg] + j];
+            for (int i = 0; i < d; ++i) {
+                double acc = 0.0;
+                for (int r = 0; r < d; ++r)
+                    acc += (double)blob[vsrc[seg] + (size_t)j * d + r] * (double)blob[oE + ((size_t)seg * d + r) * d + i];
+                ht[((size_t)seg * M + j) * d + i] = (float)acc;
+            }
+        }
+    std::vector<float> htp(ht.size());
+    for (int j = 0; j < 3 * M; ++j)
+        for (int i = 0; i < d; ++i) htp[((size_t)(i / 4) * 3 * M + j) * 4 + i % 4] = ht[(size_t)j * d + i];
+    const size_t p_ht = padd(htp.data(), htp.size() * 4), p_htb = padd(htb.data(), htb.size() * 4);
     pb.resize((pb.size() + 15) & ~(size_t)15);  // whole 16-byte chunks: one bulk copy stages it
     CK(cudaMalloc(&hm.pbuf, pb.size()));
     ctx->allocs.push_back(hm.pbuf);
@@ -477,6 +505,9 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     ph.v_s = (const float*)(pbp + pvs); ph.b_s = (const float*)(pbp + pbs);
     ph.v_k1 = (const float*)(pbp + pk1); ph.b_k1 = (const float*)(pbp + pbk1);
     ph.v_k2 = (const float*)(pbp + pk2); ph.b_k2 = (const float*)(pbp + pbk2);
+    mp.tenc_ff = (const float*)(pbp + p_tff);
+    mp.head_t = (const float*)(pbp + p_ht);
+    mp.head_tb = (const float*)(pbp + p_htb);
     mp.base = pbp;
     mp.bytes = pb.size();
     return TPPSD_OK;
@@ -743,7 +774,7 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
     } else if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
         const bool team = draft_team_supported(ctx->D.dm) && (ctx->D.dm.enc == 2 || !getenv("TPPSD_DRAFT_CTA"));
-        if (team && draft_lane_supported(ctx->D.dm, ctx->kvD.n_max) && !getenv("TPPSD_DRAFT_TEAM"))
+        if (team && draft_lane_supported(ctx->D.dm, ctx->kvD.n_max, ctx->max_gamma) && !getenv("TPPSD_DRAFT_TEAM"))
             CK(launch_draft_lane(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
         else if (team)

@@ -600,8 +600,22 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
 // after one team barrier every warp merges the ranges of every head itself.
 // The FFN hidden units are split in quarters (warp w computes quarter w and
 // its FFN2 partial; a second barrier sums them).  The draw: warp 0 computes
-// the time head [E_1; E_2; E_3] h and (w, mu, s) and draws tau, warp 3 the
-// mark head and the mark, then a third barrier hands (t, k) to every warp.
+// the time head and tau, warp 3 the mark head and the mark, then a third
+// barrier hands the event to every warp.
+//
+// Catch-up encodes and drafted events run through one loop body, so the
+// code of a drafted event is already in the instruction cache when the
+// first draft is drawn.  The uniforms of all gamma draws (and the
+// Box-Muller normals) are computed up front, lanes in parallel.  Absolute
+// time is carried as a pair of fp32 values (hi + lo, ~48 bits) for the
+// temporal encoding, whose angle a_j + b_j t is formed and reduced mod 2 pi
+// in that pair arithmetic (FMA-exact products, 2 pi as an fp32 pair); the
+// fp64 times written for the target are summed by warp 1 off the critical
+// path (fp64 arithmetic is slow on this GPU).  bf16 models also take the
+// time head as one folded map [V_w E_1; V_mu E_2; V_s E_3] h (products
+// formed in fp64 on the host), a reciprocal square root in the LayerNorms
+// and a fast divide in the attention merge; fp32 models keep the unfolded
+// head and IEEE operations.
 
 __device__ __forceinline__ float bf_lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t u) { return __uint_as_float(u & 0xffff0000u); }
@@ -657,7 +671,7 @@ template <int N>
 __device__ __forceinline__ float warp_scatter_sum(float (&v)[N], int lane) {
     static_assert(N == 16 || N == 32, "16 or 32 entries");
     if constexpr (N == 32) rs_step<32, 16>(v, lane);
-    rs_step<N == 32 ? 16 : 16, N == 32 ? 8 : 16>(v, lane);
+    rs_step<16, N == 32 ? 8 : 16>(v, lane);
     rs_step<8, N == 32 ? 4 : 8>(v, lane);
     rs_step<4, N == 32 ? 2 : 4>(v, lane);
     rs_step<2, N == 32 ? 1 : 2>(v, lane);
@@ -665,116 +679,324 @@ __device__ __forceinline__ float warp_scatter_sum(float (&v)[N], int lane) {
     return v[0];
 }
 
-// LayerNorm of the d values held by lanes < d (v; others ignored).
-__device__ __forceinline__ float lane_ln(float v, int lane, int d, const float* g, const float* b) {
+// LayerNorm of the d values held by lanes < d (v; others ignored); FAST
+// takes the reciprocal square root instruction instead of 1 / sqrt.
+template <bool FAST>
+__device__ __forceinline__ float lane_ln(float v, int lane, float inv_d, int d, const float* g, const float* b) {
     const bool live = lane < d;
-    const float mean = warp_sum(live ? v : 0.f) / d;
+    const float mean = warp_sum(live ? v : 0.f) * inv_d;
     const float c = live ? v - mean : 0.f;
-    const float inv = 1.0f / sqrtf(warp_sum(c * c) / d + LN_EPS);
+    const float var = warp_sum(c * c) * inv_d + LN_EPS;
+    const float inv = FAST ? rsqrtf(var) : 1.0f / sqrtf(var);
     return live ? c * inv * g[lane] + b[lane] : 0.f;
+}
+
+// Log-softmax of v[0..n) (shared, n <= NMAX) in place by one thread, and
+// the smallest index whose running sum of probabilities reaches u * total
+// (the same rule as warp_logsoftmax_pick, summed in index order).
+template <int NMAX>
+__device__ __forceinline__ int serial_logsoftmax_pick(float* v, int n, float u) {
+    float x[NMAX], p[NMAX];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i) {
+        x[i] = i < n ? v[i] : -INFINITY;
+        mx = fmaxf(mx, x[i]);
+    }
+    float sm = 0.f;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i) sm += i < n ? expf(x[i] - mx) : 0.f;
+    const float lz = mx + logf(sm);
+    float tot = 0.f;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i) {
+        p[i] = 0.f;
+        if (i < n) {
+            x[i] -= lz;
+            v[i] = x[i];
+            p[i] = expf(x[i]);
+        }
+        tot += p[i];
+    }
+    const float target = u * tot;
+    float run = 0.f;
+    int pick = n - 1;
+    bool found = false;
+#pragma unroll
+    for (int i = 0; i < NMAX; ++i) {
+        run += p[i];
+        if (!found && i < n && run >= target) {
+            pick = i;
+            found = true;
+        }
+    }
+    return pick;
+}
+
+// fp32 pair arithmetic (hi + lo): exact sum of two floats, and sum of a
+// pair and a float (Knuth's two-sum; Dekker's fast two-sum for |a| >= |b|).
+struct F2 { float h, l; };
+__device__ __forceinline__ F2 two_sum(float a, float b) {
+    const float s = a + b, bb = s - a;
+    return {s, (a - (s - bb)) + (b - bb)};
+}
+__device__ __forceinline__ F2 fast_two_sum(float a, float b) {
+    const float s = a + b;
+    return {s, b - (s - a)};
+}
+__device__ __forceinline__ F2 f2_add(F2 a, float b) {
+    const F2 s = two_sum(a.h, b);
+    return fast_two_sum(s.h, s.l + a.l);
+}
+__device__ __forceinline__ F2 f2_from_double(double t) {
+    const float h = __double2float_rn(t);
+    return {h, __double2float_rn(t - (double)h)};
+}
+// (a + b t) mod 2 pi in [-pi, pi] as fp32, from fp32 pairs a, b, t: the
+// product and sums in pair arithmetic, then k = rint(angle / 2 pi) removed
+// with 2 pi = P_HI + P_LO (k * P_HI split exactly by an FMA; the angle minus
+// k * P_HI is exact because both lie within a factor of two).
+__device__ __forceinline__ float reduced_angle(F2 a, F2 b, F2 t) {
+    const float P_HI = 6.28318548202514648f, P_LO = -1.74845553e-7f, INV = 0.159154943091895336f;
+    const float p = b.h * t.h;
+    float e = fmaf(b.h, t.h, -p);
+    e = fmaf(b.h, t.l, e);
+    e = fmaf(b.l, t.h, e);
+    const F2 s = two_sum(a.h, p);
+    const F2 ang = fast_two_sum(s.h, s.l + (e + a.l));
+    const float k = rintf(ang.h * INV);
+    const float q = k * P_HI, qe = fmaf(k, P_HI, -q);
+    float r = ang.h - q;
+    r = r - qe;
+    r = r + ang.l;
+    return fmaf(-k, P_LO, r);
 }
 
 // Shared-memory floats of one team besides its KV: head row, attention
 // partials (two sets of 4 warps x (max, sum, -, -, 32 numerators)), FFN2
-// partials (4 x 32), the drawn event (16 bytes), then per warp: input
-// vector (64), attention output / fp32 hidden state (32), FFN quarter (64),
-// head activations (96), query (32) and the key scores (sc).
-__host__ __device__ inline int lane_team_floats(int W, int sc) {
-    return ((W + 3) & ~3) + 2 * 4 * 36 + 128 + 4 + 4 * (288 + sc);
+// partials (4 x 32), the drawn event (t hi, t lo, tau, k), then per warp:
+// input vector (64), attention output / fp32 hidden state (32), FFN quarter
+// (64), head activations (96), query (32), draw constants (2 G) and the key
+// scores (sc).
+__host__ __device__ inline int lane_warp_floats(int G, int sc) { return 288 + 2 * G + sc; }
+__host__ __device__ inline int lane_team_floats(int W, int G, int sc) {
+    return ((W + 3) & ~3) + 2 * 4 * 36 + 128 + 4 + 4 * lane_warp_floats(G, sc);
 }
 
 template <typename T, int DH>
-__global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_bytes, int sc_stride) {
+__global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_bytes, int sc_stride, int g_stride) {
     pdl_wait();
     extern __shared__ __align__(16) char smem[];
     __shared__ uint64_t wbar;
+    constexpr bool BF = sizeof(T) == 2;
+    constexpr int CH = 16 / sizeof(T);
     const DevModelT& mp = a.m.p;
     const char* gb = mp.base;
     const uint32_t wb = (uint32_t)mp.bytes;
+    const int team = threadIdx.x >> 7;
+    const int s = blockIdx.x * 2 + team;
+    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
+    const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
+    const int n_max = a.kv.n_max;
+    const CallParams& P = *a.P;
+    const SeqState& ss = a.ss;
+    const bool live = s < P.B && !ss.done[s];
+    char* area = smem + wb + (size_t)team * area_bytes;
+    const size_t kvb = ((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15;
+    T* kvs = (T*)area;
+    uint64_t* bar = (uint64_t*)(area + kvb);
+    int n = 0, nd = 0;
+    if (live) {
+        n = ss.n_emit[s];
+        nd = ss.n_draft[s];
+    }
+    auto gk = [&](int l, int w) -> T* {
+        return (T*)(w ? a.kv.v : a.kv.k) + (((size_t)l * a.kv.Bmax + s) * NH) * (size_t)n_max * DH;
+    };
+    auto sk = [&](int l, int w) -> T* { return kvs + (((size_t)l * 2 + w) * NH) * (size_t)n_max * DH; };
     if (threadIdx.x == 0) {  // stage the packed model once per CTA
         mbar_init(&wbar, 1);
         mbar_fence_init();
         mbar_arrive_expect_tx(&wbar, wb);
         bulk_load(smem, gb, wb, &wbar);
     }
+    if (tid == 0 && live && nd > 0) {
+        // the sequence's draft KV: each (layer, K/V, head) block of positions
+        // 0..nd-1 is contiguous in HBM
+        const uint32_t bytes = (uint32_t)nd * DH * sizeof(T);
+        mbar_init(bar, 1);
+        mbar_fence_init();
+        mbar_arrive_expect_tx(bar, bytes * (uint32_t)(L * 2 * NH));
+        for (int l = 0; l < L; ++l)
+            for (int w = 0; w < 2; ++w)
+                for (int h = 0; h < NH; ++h)
+                    bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
+    }
     __syncthreads();
-    mbar_wait(&wbar, 0, a.err, 14);
-    // shared-memory address of a piece of the packed model
-    auto sm = [&](const void* g) -> const char* { return smem + ((const char*)g - gb); };
-    const int team = threadIdx.x >> 7;
-    const int s = blockIdx.x * 2 + team;
-    const CallParams& P = *a.P;
-    if (s >= P.B || a.ss.done[s]) return;  // the rest synchronises within the team only
-    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
-    const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
-    const int n_max = a.kv.n_max;
+    if (!live) return;  // the rest synchronises within the team only
     const int S = 4 / NH, hw = warp % NH, spw = warp / NH;  // this warp's head and key range
-    constexpr int CH = 16 / sizeof(T);
     const bool att_enc = a.m.enc == 2;
-    char* area = smem + wb + (size_t)team * area_bytes;
-    const size_t kvb = ((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15;
-    T* kvs = (T*)area;
-    uint64_t* bar = (uint64_t*)(area + kvb);
+    const float inv_d = 1.0f / (float)d;
     float* hd = (float*)(area + kvb + 16);
     float* red = hd + ((W + 3) & ~3);  // [2][4][36]
     float* part = red + 2 * 4 * 36;    // [4][32]
-    double* ev_t = (double*)(part + 128);
-    int* ev_k = (int*)(ev_t + 1);
-    float* mine = part + 128 + 4 + warp * (288 + sc_stride);
+    float* ev = part + 128;            // t hi, t lo, tau, k (int bits)
+    float* mine = ev + 4 + warp * lane_warp_floats(g_stride, sc_stride);
     float* v_in = mine;        // [zin | xin] (AttNHP) or xin
     float* v_att = mine + 64;  // attention output; fp32 hidden state for the head
     float* v_hid = mine + 96;  // this warp's FFN quarter
     float* v_e = mine + 160;   // head activations
     float* v_q = mine + 256;   // query of this warp's head
-    float* sc = mine + 288;    // scores of this warp's keys
-    const SeqState& ss = a.ss;
-    const int n = ss.n_emit[s], nd = ss.n_draft[s];
-    auto gk = [&](int l, int w) -> T* {
-        return (T*)(w ? a.kv.v : a.kv.k) + (((size_t)l * a.kv.Bmax + s) * NH) * (size_t)n_max * DH;
-    };
-    auto sk = [&](int l, int w) -> T* { return kvs + (((size_t)l * 2 + w) * NH) * (size_t)n_max * DH; };
-    if (nd > 0) {  // each (layer, K/V, head) block of positions 0..nd-1 is contiguous in HBM
-        if (tid == 0) {
-            const uint32_t bytes = (uint32_t)nd * DH * sizeof(T);
-            mbar_init(bar, 1);
-            mbar_fence_init();
-            mbar_arrive_expect_tx(bar, bytes * (uint32_t)(L * 2 * NH));
-            for (int l = 0; l < L; ++l)
-                for (int w = 0; w < 2; ++w)
-                    for (int h = 0; h < NH; ++h)
-                        bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
+    float* v_rng = mine + 288; // draw constants of the gamma events
+    float* sc = v_rng + 2 * g_stride;  // scores of this warp's keys
+    auto sm = [&](const void* g) -> const char* { return smem + ((const char*)g - gb); };
+    const int gamma = a.gamma, p_last = n + gamma - 1;
+    // draw constants: warp 0 (u_comp, eps) and warp 3 (u_mark) of draft l at
+    // position n + l, from the block-0 slot of that position
+    if (warp == 0 || warp == 3)
+        for (int l = lane; l < gamma; l += 32) {
+            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)(n + l), 0u);
+            if (warp == 0) {
+                v_rng[2 * l] = u.x;
+                v_rng[2 * l + 1] = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
+            } else {
+                v_rng[2 * l] = u.w;
+            }
         }
-        team_sync();
-        mbar_wait(bar, 0, a.err, 12);
+    // catch-up events (t, k) read before the waits
+    double t_cu[2] = {0.0, 0.0};
+    int k_cu[2] = {0, 0};
+    for (int i = 0; i < 2 && nd + i < n; ++i) {
+        const size_t so = (size_t)s * ss.n_max + nd + i;
+        t_cu[i] = ss.t[so];
+        k_cu[i] = min(max(ss.k[so], 0), K - 1);
     }
+    double t64 = ss.t[(size_t)s * ss.n_max + n - 1];  // fp64 time of the last event (warp 1)
+    if (tid == 0) {  // its pair form, which the first draft adds to
+        const F2 t2 = f2_from_double(t64);
+        ev[0] = t2.h;
+        ev[1] = t2.l;
+    }
+    mbar_wait(&wbar, 0, a.err, 14);
+    if (nd > 0) mbar_wait(bar, 0, a.err, 12);
     const float* type_emb = (const float*)sm(mp.type_emb);
-    const double* tenc = (const double*)sm(mp.tenc);
-    // Encoding of event (t, k) (App. D.4 temporal encoding z_i = sin / cos
-    // (a_i + b_i t), angle reduced mod 2 pi in fp64, plus the mark
-    // embedding): returns x_lane and writes the rounded GEMM input.
-    auto embed = [&](double t, int k) -> float {
-        float xv = 0.f;
+    const float* tff = (const float*)sm(mp.tenc_ff);
+    F2 ta{0.f, 0.f}, tb{0.f, 0.f};  // a_lane, b_lane of the encoding
+    if (lane < d) {
+        ta = {tff[lane], tff[d + lane]};
+        tb = {tff[2 * d + lane], tff[3 * d + lane]};
+    }
+    const float scale = 1.4426950408889634f / sqrtf((float)DH);
+    float x = 0.f;
+    __syncwarp();
+    for (int p = nd;; ++p) {
+        F2 tp;
+        int kp;
+        if (p >= n) {
+            // draw event p from the head of the hidden state x of p - 1
+            // (Sec. 4.2): z ~ Cat(w), tau = exp(mu_z + sigma_z eps); k ~ f
+            const int l = p - n;
+            const size_t so = (size_t)s * ss.n_max + p;
+            const HeadW& H = mp.head;
+            if (warp == 0) {
+                if (lane < d) v_att[lane] = x;
+                __syncwarp();
+                if constexpr (BF) {
+                    const float* ht = (const float*)sm(mp.head_t);
+                    const float* htb = (const float*)sm(mp.head_tb);
+                    for (int o = lane; o < 3 * M; o += 32) hd[o] = pdot<float>(ht, 3 * M, o, v_att, d / 4) + htb[o];
+                } else {
+                    const float* E = (const float*)sm(H.E);
+                    if (lane < d) {
+#pragma unroll
+                        for (int r = 0; r < 3; ++r)
+                            v_e[r * d + lane] = pdot<float>(E, 3 * d, r * d + lane, v_att, d / 4);
+                    }
+                    __syncwarp();
+                    for (int o = lane; o < 3 * M; o += 32) {
+                        const int seg = o / M, jj = o - seg * M;
+                        const float* V = (const float*)sm(seg == 0 ? H.v_w : seg == 1 ? H.v_mu : H.v_s);
+                        const float* bb = (const float*)sm(seg == 0 ? H.b_w : seg == 1 ? H.b_mu : H.b_s);
+                        hd[o] = pdot<float>(V, M, jj, v_e + seg * d, d / 4) + bb[jj];
+                    }
+                }
+                __syncwarp();
+                int z;
+                if (M <= 8) {
+                    z = lane == 0 ? serial_logsoftmax_pick<8>(hd, M, v_rng[2 * l]) : 0;
+                } else {
+                    z = warp_logsoftmax_pick<2>(hd, M, v_rng[2 * l]);
+                }
+                if (lane == 0) {
+                    const float tau = expf(hd[M + z] + expf(hd[2 * M + z]) * v_rng[2 * l + 1]);
+                    const F2 tn = f2_add(F2{ev[0], ev[1]}, tau);
+                    ev[0] = tn.h;
+                    ev[1] = tn.l;
+                    ev[2] = tau;
+                    ss.tau[so] = tau;
+                }
+            } else if (warp == 3) {
+                if (lane < d) v_att[lane] = x;
+                __syncwarp();
+                if (lane < d)
+                    v_e[lane] = tanhf(pdot<float>((const float*)sm(H.v_k1), d, lane, v_att, d / 4) +
+                                      ((const float*)sm(H.b_k1))[lane]);
+                __syncwarp();
+                const float* V2 = (const float*)sm(H.v_k2);
+                const float* b2 = (const float*)sm(H.b_k2);
+                for (int o = lane; o < K; o += 32) hd[3 * M + o] = pdot<float>(V2, K, o, v_e, d / 4) + b2[o];
+                __syncwarp();
+                int k;
+                if (K <= 8) {
+                    k = lane == 0 ? serial_logsoftmax_pick<8>(hd + 3 * M, K, v_rng[2 * l]) : 0;
+                } else {
+                    k = warp_logsoftmax_pick<8>(hd + 3 * M, K, v_rng[2 * l]);
+                }
+                if (lane == 0) {
+                    ss.k[so] = k;
+                    ev[3] = __int_as_float(k);
+                }
+            }
+            team_sync();
+            tp = {ev[0], ev[1]};
+            kp = __float_as_int(ev[3]);
+            if (warp == 1) {
+                float* rec = a.heads + ((size_t)s * a.gamma_max + l) * W;
+                for (int i = lane; i < W; i += 32) rec[i] = hd[i];
+                if (lane == 0) {  // the fp64 time of the event, as the target reads it
+                    t64 += (double)ev[2];
+                    ss.t[so] = t64;
+                }
+            }
+            if (p == p_last) break;
+        } else {
+            const int i = p - nd;
+            double t;
+            if (i < 2) {
+                t = i == 0 ? t_cu[0] : t_cu[1];
+                kp = i == 0 ? k_cu[0] : k_cu[1];
+            } else {
+                const size_t so = (size_t)s * ss.n_max + p;
+                t = ss.t[so];
+                kp = min(max(ss.k[so], 0), K - 1);
+            }
+            tp = f2_from_double(t);
+        }
+        // ---- encode event p: temporal encoding z_i = sin / cos (a_i + b_i t)
+        // (App. D.4) plus the mark embedding
         if (lane < d) {
-            const double ang = tenc[lane] + tenc[d + lane] * t;
-            const double rd = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
             float sv, cv;
-            sincosf((float)rd, &sv, &cv);
+            sincosf(reduced_angle(ta, tb, tp), &sv, &cv);
             const float z = (lane & 1) ? cv : sv;
-            xv = z + type_emb[(size_t)k * d + lane];
+            x = z + type_emb[(size_t)kp * d + lane];
             if (att_enc) {
                 v_in[lane] = St<T>::rnd(z);
-                v_in[d + lane] = St<T>::rnd(xv);
+                v_in[d + lane] = St<T>::rnd(x);
             } else {
-                v_in[lane] = St<T>::rnd(xv);
+                v_in[lane] = St<T>::rnd(x);
             }
         }
         __syncwarp();
-        return xv;
-    };
-    const float scale = 1.4426950408889634f / sqrtf((float)DH);
-    // Layers of the encode step at position p; x holds the embedding on entry
-    // and the final hidden state on exit (lanes < d, every warp).
-    auto layers = [&](int p, float x) -> float {
         const int nk = p + 1, per = (nk + S - 1) / S, lo = spw * per, hi = min(nk, lo + per);
         const bool writer = spw == p / per;  // the warp of this head whose range holds key p
         for (int l = 0; l < L; ++l) {
@@ -802,7 +1024,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             const T* kb = sk(l, 0) + (size_t)hw * n_max * DH;
             const T* vb = sk(l, 1) + (size_t)hw * n_max * DH;
             float mx = -INFINITY;
-#pragma unroll 2
+#pragma unroll 1
             for (int j = lo + lane; j < hi; j += 32) {
                 float kr[DH];
                 load_row16<T, DH>(kb + (size_t)j * DH, kr);
@@ -820,7 +1042,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             float ll = 0.f, o[DH];
 #pragma unroll
             for (int c = 0; c < DH; ++c) o[c] = 0.f;
-#pragma unroll 2
+#pragma unroll 1
             for (int j = lo + lane; j < hi; j += 32) {
                 const float pj = exp2f(sc[j - lo] - mx);
                 float vr[DH];
@@ -853,7 +1075,8 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                     Lx += src[1] * e;
                     Ox += src[4 + c] * e;
                 }
-                at = att_enc ? Ox / (Lx + exp2f(-Mx)) : St<T>::rnd(Ox / Lx);
+                if (att_enc) at = Ox / (Lx + exp2f(-Mx));
+                else at = St<T>::rnd(BF ? __fdividef(Ox, Lx) : Ox / Lx);
             }
             if (att_enc) {  // AttNHP (App. D.4): h <- h + tanh(a), no projection or FFN
                 if (lane < d) {
@@ -868,7 +1091,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             __syncwarp();
             float y = 0.f;
             if (lane < d) y = pdot<T>((const T*)sm(Wl.w_o), d, lane, v_att, d / CH) + ((const float*)sm(Wl.b_o))[lane];
-            x = lane_ln(x + y, lane, d, (const float*)sm(Wl.ln1_g), (const float*)sm(Wl.ln1_b));
+            x = lane_ln<BF>(x + y, lane, inv_d, d, (const float*)sm(Wl.ln1_g), (const float*)sm(Wl.ln1_b));
             if (lane < d) v_in[lane] = St<T>::rnd(x);
             __syncwarp();
             // FFN quarter of this warp: hidden units f0 .. f0 + F/4 - 1
@@ -887,104 +1110,37 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             if (lane < d)
                 y2 = ((const float*)sm(Wl.b_2))[lane] +
                      ((part[lane] + part[32 + lane]) + (part[64 + lane] + part[96 + lane]));
-            x = lane_ln(x + y2, lane, d, (const float*)sm(Wl.ln2_g), (const float*)sm(Wl.ln2_b));
+            x = lane_ln<BF>(x + y2, lane, inv_d, d, (const float*)sm(Wl.ln2_g), (const float*)sm(Wl.ln2_b));
             if (lane < d) v_in[lane] = St<T>::rnd(x);
             __syncwarp();
         }
-        return x;
-    };
-    float x = 0.f;
-    for (int p = nd; p < n; ++p) {  // catch-up over events already emitted
-        const size_t so = (size_t)s * ss.n_max + p;
-        x = embed(ss.t[so], min(max(ss.k[so], 0), K - 1));
-        x = layers(p, x);
     }
     if (tid == 0) {
-        const long long last = n + a.gamma - 2;  // last position the round encodes
+        const long long last = n + gamma - 2;  // last position the round encodes
         atomicAdd(&a.st->draft_keys, (unsigned long long)((last + 1) * (last + 2) / 2 - (long long)nd * (nd + 1) / 2));
-    }
-    const HeadW& H = mp.head;
-    double t_prev = ss.t[(size_t)s * ss.n_max + n - 1];
-    for (int l = 1; l <= a.gamma; ++l) {
-        const int p = n + l - 1;  // index of the drafted event
-        const size_t so = (size_t)s * ss.n_max + p;
-        if (warp == 0) {
-            // time head (Sec. 4.2): e_r = E_r h, then log w, mu, s; tau by
-            // z ~ Cat(w), eps by Box-Muller, tau = exp(mu_z + sigma_z eps)
-            if (lane < d) v_att[lane] = x;
-            __syncwarp();
-            const float* E = (const float*)sm(H.E);
-            if (lane < d) {
-#pragma unroll
-                for (int r = 0; r < 3; ++r) v_e[r * d + lane] = pdot<float>(E, 3 * d, r * d + lane, v_att, d / 4);
-            }
-            __syncwarp();
-            for (int o = lane; o < 3 * M; o += 32) {
-                const int seg = o / M, jj = o - seg * M;
-                const float* V = (const float*)sm(seg == 0 ? H.v_w : seg == 1 ? H.v_mu : H.v_s);
-                const float* bb = (const float*)sm(seg == 0 ? H.b_w : seg == 1 ? H.b_mu : H.b_s);
-                hd[o] = pdot<float>(V, M, jj, v_e + seg * d, d / 4) + bb[jj];
-            }
-            __syncwarp();
-            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
-            const int z = warp_logsoftmax_pick<2>(hd, M, u.x);
-            if (lane == 0) {
-                const float eps = sqrtf(-2.0f * logf(u.y)) * cospif(2.0f * u.z);
-                const float tau = expf(hd[M + z] + expf(hd[2 * M + z]) * eps);
-                const double t = t_prev + (double)tau;
-                ss.tau[so] = tau;
-                ss.t[so] = t;
-                *ev_t = t;
-            }
-        } else if (warp == 3) {
-            // mark head: a = tanh(V_k1 h + b_k1), log f = log_softmax(V_k2 a + b_k2)
-            if (lane < d) v_att[lane] = x;
-            __syncwarp();
-            if (lane < d)
-                v_e[lane] = tanhf(pdot<float>((const float*)sm(H.v_k1), d, lane, v_att, d / 4) +
-                                  ((const float*)sm(H.b_k1))[lane]);
-            __syncwarp();
-            const float* V2 = (const float*)sm(H.v_k2);
-            const float* b2 = (const float*)sm(H.b_k2);
-            for (int o = lane; o < K; o += 32) hd[3 * M + o] = pdot<float>(V2, K, o, v_e, d / 4) + b2[o];
-            __syncwarp();
-            const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
-            const int k = warp_logsoftmax_pick<8>(hd + 3 * M, K, u.w);
-            if (lane == 0) {
-                ss.k[so] = k;
-                *ev_k = k;
-            }
-        }
-        team_sync();
-        const double t_new = *ev_t;
-        const int k_new = *ev_k;
-        t_prev = t_new;
-        if (warp == 1) {
-            float* rec = a.heads + ((size_t)s * a.gamma_max + (l - 1)) * W;
-            for (int i = lane; i < W; i += 32) rec[i] = hd[i];
-        }
-        if (l < a.gamma) x = layers(p, embed(t_new, k_new));
     }
     pdl_trigger();
 }
 
-// Shared-memory bytes of one team of the lane form (0: the shape is not covered).
-static size_t lane_area(const DevModel& m, int n_max, int* sc_out) {
+// Shared-memory bytes of one team of the lane form (0: the shape is not
+// covered).
+static size_t lane_area(const DevModel& m, int n_max, int gamma_max, int* sc_out, int* g_out) {
     const int CH = m.dtype == 1 ? 8 : 4;
     const bool shape = (m.nh == 1 && (m.dh == 16 || m.dh == 32)) || (m.nh == 2 && m.dh == 16);
     if (!shape || m.d % CH || m.M > 64 || m.K > 256 || m.L < 1) return 0;
     if (m.enc != 2 && (m.F % (4 * CH) || m.F > 256)) return 0;
     const size_t eb = m.dtype == 1 ? 2 : 4;
     const int S = 4 / m.nh;
-    const int sc = (((n_max + S - 1) / S) + 3) & ~3;
+    const int sc = (((n_max + S - 1) / S) + 3) & ~3, G = (gamma_max + 3) & ~3;
     const size_t kvb = ((size_t)m.L * 2 * n_max * m.d * eb + 15) & ~(size_t)15;
     if (sc_out) *sc_out = sc;
-    return kvb + 16 + sizeof(float) * (size_t)lane_team_floats(3 * m.M + m.K, sc);
+    if (g_out) *g_out = G;
+    return kvb + 16 + sizeof(float) * (size_t)lane_team_floats(3 * m.M + m.K, G, sc);
 }
 
-int draft_lane_supported(const DevModel& m, int n_max) {
-    const size_t area = lane_area(m, n_max, nullptr);
-    if (!area || m.p.bytes % 16) return 0;
+int draft_lane_supported(const DevModel& m, int n_max, int gamma_max) {
+    const size_t area = lane_area(m, n_max, gamma_max, nullptr, nullptr);
+    if (!area || m.p.bytes % 16 || !m.p.tenc_ff) return 0;
     return m.p.bytes + 2 * area <= 224 * 1024;
 }
 
@@ -994,13 +1150,13 @@ cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqSta
     DraftTeamArgs a{};
     a.m = m; a.kv = kv; a.ss = ss; a.P = dp; a.st = stats; a.heads = draft_heads;
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
-    int sc = 0;
-    const size_t area = lane_area(m, kv.n_max, &sc);
+    int sc = 0, G = 0;
+    const size_t area = lane_area(m, kv.n_max, gamma_max, &sc, &G);
     const size_t sm = m.p.bytes + 2 * area;
     auto go = [&](auto kern) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
         if (e != cudaSuccess) return e;
-        return launch_k(kern, dim3((B + 1) / 2), dim3(256), sm, st, a, (int)area, sc);
+        return launch_k(kern, dim3((B + 1) / 2), dim3(256), sm, st, a, (int)area, sc, G);
     };
     if (m.dtype == 0) return m.dh == 16 ? go(k_draft_lane<float, 16>) : go(k_draft_lane<float, 32>);
     return m.dh == 16 ? go(k_draft_lane<bf16, 16>) : go(k_draft_lane<bf16, 32>);

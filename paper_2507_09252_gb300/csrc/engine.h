@@ -58,6 +58,10 @@ struct DevModelT {
     HeadW head;              // E [d][3d], v_w/v_mu/v_s [d][M], v_k1 [d][d], v_k2 [d][K]
     const char* base;
     size_t bytes;
+    // lane-packed copy only (null in the transposed one):
+    const float* tenc_ff;    // [4][d] fp32 pairs of the encoding table: a_hi, a_lo, b_hi, b_lo
+    const float* head_t;     // [3M][d] lane-packed [V_w E_1; V_mu E_2; V_s E_3] (products in fp64)
+    const float* head_tb;    // [3M] b_w, b_mu, b_s
 };
 
 // One model on the device.  Every pointer lies in [base, base + bytes), so a
@@ -299,7 +303,7 @@ size_t draft_smem_bytes(const DevModel& m, bool stage_weights);
 int draft_team_supported(const DevModel& m);
 // Lane form of the draft kernel (draft.cu) for d <= 32 models whose packed
 // copy and two sequences' draft KV fit in shared memory.
-int draft_lane_supported(const DevModel& m, int n_max);
+int draft_lane_supported(const DevModel& m, int n_max, int gamma_max);
 cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st);
