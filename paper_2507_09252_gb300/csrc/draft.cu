@@ -785,7 +785,6 @@ __host__ __device__ inline int lane_team_floats(int W, int G, int sc) {
 
 template <typename T, int DH>
 __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_bytes, int sc_stride, int g_stride) {
-    pdl_wait();
     extern __shared__ __align__(16) char smem[];
     __shared__ uint64_t wbar;
     constexpr bool BF = sizeof(T) == 2;
@@ -793,6 +792,15 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
     const DevModelT& mp = a.m.p;
     const char* gb = mp.base;
     const uint32_t wb = (uint32_t)mp.bytes;
+    // the model is never written by a sampling kernel: stage it while the
+    // previous kernel of the stream finishes
+    if (threadIdx.x == 0) {
+        mbar_init(&wbar, 1);
+        mbar_fence_init();
+        mbar_arrive_expect_tx(&wbar, wb);
+        bulk_load(smem, gb, wb, &wbar);
+    }
+    pdl_wait();
     const int team = threadIdx.x >> 7;
     const int s = blockIdx.x * 2 + team;
     const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
@@ -814,12 +822,6 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
         return (T*)(w ? a.kv.v : a.kv.k) + (((size_t)l * a.kv.Bmax + s) * NH) * (size_t)n_max * DH;
     };
     auto sk = [&](int l, int w) -> T* { return kvs + (((size_t)l * 2 + w) * NH) * (size_t)n_max * DH; };
-    if (threadIdx.x == 0) {  // stage the packed model once per CTA
-        mbar_init(&wbar, 1);
-        mbar_fence_init();
-        mbar_arrive_expect_tx(&wbar, wb);
-        bulk_load(smem, gb, wb, &wbar);
-    }
     if (tid == 0 && live && nd > 0) {
         // the sequence's draft KV: each (layer, K/V, head) block of positions
         // 0..nd-1 is contiguous in HBM
@@ -997,8 +999,10 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             }
         }
         __syncwarp();
-        const int nk = p + 1, per = (nk + S - 1) / S, lo = spw * per, hi = min(nk, lo + per);
-        const bool writer = spw == p / per;  // the warp of this head whose range holds key p
+        // key ranges of length per, the last one ~32 keys shorter: the warp
+        // whose range holds key p also computes k and v of p
+        const int nk = p + 1, per = (nk + 32 + S - 1) / S, lo = spw * per, hi = min(nk, lo + per);
+        const bool writer = spw == p / per;
         for (int l = 0; l < L; ++l) {
             const LayerW& Wl = mp.layer[l];
             const T* wqkv = (const T*)sm(Wl.w_qkv);
@@ -1131,7 +1135,7 @@ static size_t lane_area(const DevModel& m, int n_max, int gamma_max, int* sc_out
     if (m.enc != 2 && (m.F % (4 * CH) || m.F > 256)) return 0;
     const size_t eb = m.dtype == 1 ? 2 : 4;
     const int S = 4 / m.nh;
-    const int sc = (((n_max + S - 1) / S) + 3) & ~3, G = (gamma_max + 3) & ~3;
+    const int sc = (((n_max + 32 + S - 1) / S) + 3) & ~3, G = (gamma_max + 3) & ~3;
     const size_t kvb = ((size_t)m.L * 2 * n_max * m.d * eb + 15) & ~(size_t)15;
     if (sc_out) *sc_out = sc;
     if (g_out) *g_out = G;

@@ -148,6 +148,28 @@ def test_sequence_parity_fp32_with_rejections(gamma, flags):
         assert stats["resample_iters"] == ostats[:, 3].sum()
 
 
+@pytest.mark.parametrize("form", ["lane", "team"])
+@pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
+def test_draft_kernel_forms_match_oracle(form, dtype, monkeypatch):
+    """Both forms of the per-sequence draft kernel on a d = 32, two-head
+    draft (lane form: one hidden component per lane, the default for
+    d <= 32; team form: TPPSD_DRAFT_TEAM=1) reproduce the oracle's
+    sequences, rejections and resampling included."""
+    if form == "team":
+        monkeypatch.setenv("TPPSD_DRAFT_TEAM", "1")
+    dcfg = CF.ModelCfg(1, 32, 2, 128, 4, 3, dtype)
+    tcfg = None if dtype == CF.FP32 else CF.ModelCfg(2, 128, 4, 512, 4, 3, dtype)
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5, dtype=dtype, tcfg=tcfg, dcfg=dcfg)
+    tau, mk = G.hist(16, 9, 3, 8)
+    g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 50, 5, 31)
+    fp32 = dtype == CF.FP32
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32 if fp32 else G.MARGIN_BF16,
+                                            rtol=1e-4 if fp32 else 2e-2)
+    assert not fails, fails
+    assert ident >= 12
+    assert st == T.TPPSD_OK and stats["accepted"] < stats["drafted"]
+
+
 def test_sequence_parity_bf16_prefix():
     """bf16: teacher-forced parity is the strict check; sampled sequences
     agree until a decision within bf16 noise of its threshold."""
