@@ -163,7 +163,13 @@ def class_roofline(name, ms, launches, stats, wl, peaks, fused):
                 the fused post-attention block (timed as gemm_ffn2) does
                 2 R (d^2 + 2 d F)
     head:       h rows read + head rows written + head weights
-    others:     bytes of the rows they read and write (latency-bound)
+    embed:      per verify row: (t, k) read, fp32 and storage-type rows written
+    epilogue:   per (sequence, round): target heads of gamma+1 rows and draft
+                heads of gamma rows read, up to gamma+1 events written
+    control:    n_emit and done of every sequence read
+    begin:      the output arrays initialised (tau, t, k of B x N events)
+    The last four are latency-bound; their figures say how far they are
+    from moving bytes at all.
     """
     T, D = wl.target, wl.draft
     eb = 2 if T.dtype == CF.BF16 else 4
@@ -191,7 +197,16 @@ def class_roofline(name, ms, launches, stats, wl, peaks, fused):
             total = 2.0 * rows * (d * d + 2 * d * F) * L
         bound, unit = "tensor", "TFLOP/s"
     else:
-        total = rows * d * 4 * 2
+        if name == "embed":
+            total = rows * (12 + d * (4 + eb))
+        elif name == "epilogue":
+            total = rounds * ((2 * wl.gamma + 1) * W * 4 + (wl.gamma + 1) * 16)
+        elif name == "control":
+            total = launches * wl.batch * 8
+        elif name == "begin":
+            total = launches * wl.batch * wl.n_events * 16
+        else:
+            total = rows * d * 4 * 2
         bound = "latency"
     per_launch = total / max(launches, 1)
     if bound == "tensor":
