@@ -12,21 +12,32 @@
 // m16n8k16 with bf16 inputs (exact products, fp32 accumulation); P V splits
 // P into two bf16 parts (P = P_hi + P_lo, 16 significant bits) against the
 // bf16 V tile as copied, with fp32 accumulation.  The four partial results
-// are merged through shared memory.
+// are merged through shared memory, each written over its warp's own stages.
+// Two tile sizes: 1 KB tiles keep a CTA at ~17 KB of shared memory and 72
+// registers per thread (d_head <= 32), so seven CTAs fit an SM and a grid of
+// up to 7 x (SM count) items (the 1 024 (sequence, head) items of a
+// 256-sequence verify pass) runs in one wave; larger grids run in several
+// waves anyway and take 2 KB tiles (half the tiles per key range).
+#include <stdlib.h>
+
 #include "common.cuh"
 #include "engine.h"
 #include "tc_ptx.cuh"
 
 namespace tppsd {
 
-template <int DH>
+template <int DH, int TB>
 struct AttnShape {
-    static constexpr int KT = 1024 / DH;             // keys per tile: 2 KB of K, 2 KB of V
+    // keys per tile: TB bytes of K and TB of V (at least 16 keys, one P V step)
+    static constexpr int KT = TB / (2 * DH) < 16 ? 16 : TB / (2 * DH);
     static constexpr int TILE_BYTES = KT * DH * 2;
     static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
     static constexpr int WARP_BYTES = 2 * STAGE_BYTES + 32;  // two stages + two mbarriers
-    static constexpr int MERGE_BYTES = 4 * (16 * DH + 32) * 4;
-    static constexpr int SMEM = 4 * WARP_BYTES + MERGE_BYTES + 16 * 4 + 64;
+    // a warp's partial result (max, sum, 16 x DH numerators), written over
+    // its own stages once its last tile is consumed
+    static constexpr int MERGE_FLOATS = 16 * DH + 32;
+    static_assert(MERGE_FLOATS * 4 <= 2 * STAGE_BYTES, "partial result must fit the warp's stages");
+    static constexpr int SMEM = 4 * WARP_BYTES + 16 * 4 + 64;
 };
 
 __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
@@ -49,9 +60,11 @@ __device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uin
     lo = *reinterpret_cast<const uint32_t*>(&l);
 }
 
-template <int DH>
-__global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) {
-    using S = AttnShape<DH>;
+// TB = 1024: small footprint, seven CTAs per SM (d_head <= 32); TB = 2048:
+// fewer tiles per key range, four CTAs per SM.
+template <int DH, int TB>
+__global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_mma(AttArgs<bf16> a, int* err) {
+    using S = AttnShape<DH, TB>;
     constexpr int KT = S::KT, NT = KT / 8, KS = DH / 16;
     pdl_wait();
     extern __shared__ __align__(128) unsigned char smem[];
@@ -70,8 +83,7 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
     const int nq = re - rb;
     unsigned char* wbase = smem + warp * S::WARP_BYTES;
     uint64_t* bars = (uint64_t*)(wbase + 2 * S::STAGE_BYTES);
-    float* merge = (float*)(smem + 4 * S::WARP_BYTES);
-    int* qpos = (int*)(smem + 4 * S::WARP_BYTES + S::MERGE_BYTES);
+    int* qpos = (int*)(smem + 4 * S::WARP_BYTES);
     // this warp's key range [klo, khi)
     const int nkeys = maxpos + 1;
     const int share = (((nkeys + 3) / 4) + 7) & ~7;
@@ -215,8 +227,9 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
         }
         __syncwarp();
     }
-    // per-warp partial results -> shared memory
-    float* mw = merge + warp * (16 * DH + 32);
+    // per-warp partial results -> shared memory (over this warp's stages)
+    auto mslot = [&](int w) { return (float*)(smem + w * S::WARP_BYTES); };
+    float* mw = mslot(warp);
     if (t4 == 0) {
         mw[g] = m0; mw[g + 8] = m1;
         mw[16 + g] = l0; mw[16 + g + 8] = l1;
@@ -234,11 +247,11 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
         const int row = i / DH, col = i % DH;
         float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < 4; ++w) M = fmaxf(M, merge[w * (16 * DH + 32) + row]);
+        for (int w = 0; w < 4; ++w) M = fmaxf(M, mslot(w)[row]);
         float L = 0.f, O = 0.f;
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
-            const float* p = merge + w * (16 * DH + 32);
+            const float* p = mslot(w);
             if (p[row] == -INFINITY) continue;
             const float e = expf(p[row] - M);
             L += p[16 + row] * e;
@@ -256,30 +269,33 @@ __global__ void __launch_bounds__(128, 4) k_attn_mma(AttArgs<bf16> a, int* err) 
     pdl_trigger();
 }
 
+template <int DH, int TB>
+static cudaError_t launch_attn_t(const AttArgs<bf16>& a, dim3 grid, int* err, cudaStream_t st) {
+    const int sm = AttnShape<DH, TB>::SMEM;
+    cudaFuncSetAttribute(k_attn_mma<DH, TB>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
+    return launch_k(k_attn_mma<DH, TB>, grid, dim3(128), sm, st, a, err);
+}
+
 cudaError_t launch_attn_mma(const AttArgs<bf16>& a, int dh, int nh, int nseg, int* err, cudaStream_t st) {
     const dim3 grid((a.q_per_seq + 15) / 16, nh, nseg);
-    switch (dh) {
-        case 16: {
-            const int sm = AttnShape<16>::SMEM;
-            cudaFuncSetAttribute(k_attn_mma<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            if (const cudaError_t e = launch_k(k_attn_mma<16>, grid, dim3(128), sm, st, a, err)) return e;
-            break;
-        }
-        case 32: {
-            const int sm = AttnShape<32>::SMEM;
-            cudaFuncSetAttribute(k_attn_mma<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            if (const cudaError_t e = launch_k(k_attn_mma<32>, grid, dim3(128), sm, st, a, err)) return e;
-            break;
-        }
-        case 64: {
-            const int sm = AttnShape<64>::SMEM;
-            cudaFuncSetAttribute(k_attn_mma<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-            if (const cudaError_t e = launch_k(k_attn_mma<64>, grid, dim3(128), sm, st, a, err)) return e;
-            break;
-        }
-        default:
-            return cudaErrorInvalidValue;
+    // small tiles when the grid fits one wave of seven CTAs per SM
+    // (TPPSD_ATTN_TILE=1024 / 2048 forces a size)
+    static int n_sm = 0;
+    if (!n_sm) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n_sm <= 0) n_sm = 148;
     }
+    bool small = (long long)grid.x * grid.y * grid.z <= 7LL * n_sm;
+    if (const char* f = getenv("TPPSD_ATTN_TILE")) small = atoi(f) == 1024;
+    cudaError_t e;
+    switch (dh) {
+        case 16: e = small ? launch_attn_t<16, 1024>(a, grid, err, st) : launch_attn_t<16, 2048>(a, grid, err, st); break;
+        case 32: e = small ? launch_attn_t<32, 1024>(a, grid, err, st) : launch_attn_t<32, 2048>(a, grid, err, st); break;
+        case 64: e = launch_attn_t<64, 2048>(a, grid, err, st); break;
+        default: return cudaErrorInvalidValue;
+    }
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
