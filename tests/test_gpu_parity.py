@@ -170,6 +170,27 @@ def test_draft_kernel_forms_match_oracle(form, dtype, monkeypatch):
     assert st == T.TPPSD_OK and stats["accepted"] < stats["drafted"]
 
 
+@pytest.mark.parametrize("form", ["lane", "team"])
+@pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
+def test_draft_kernel_wide_heads_match_oracle(form, dtype, monkeypatch):
+    """M = 12 mixture components and K = 20 marks: the draft kernels draw
+    the component and the mark with the warp-wide log-softmax (more than
+    eight values), and the sequences still follow the oracle."""
+    if form == "team":
+        monkeypatch.setenv("TPPSD_DRAFT_TEAM", "1")
+    dcfg = CF.ModelCfg(1, 32, 2, 128, 12, 20, dtype)
+    tcfg = CF.ModelCfg(2, 32, 2, 64, 12, 20, dtype) if dtype == CF.FP32 else CF.ModelCfg(2, 128, 4, 512, 12, 20, dtype)
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5, dtype=dtype, tcfg=tcfg, dcfg=dcfg)
+    tau, mk = G.hist(16, 9, 20, 4)
+    g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 50, 5, 17)
+    fp32 = dtype == CF.FP32
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32 if fp32 else G.MARGIN_BF16,
+                                            rtol=1e-4 if fp32 else 2e-2)
+    assert not fails, fails
+    assert ident >= 10
+    assert st == T.TPPSD_OK and len(np.unique(g["k"])) > 8
+
+
 def test_sequence_parity_bf16_prefix():
     """bf16: teacher-forced parity is the strict check; sampled sequences
     agree until a decision within bf16 noise of its threshold."""
