@@ -783,7 +783,9 @@ __host__ __device__ inline int lane_team_floats(int W, int G, int sc) {
     return ((W + 3) & ~3) + 2 * 4 * 36 + 128 + 4 + 4 * lane_warp_floats(G, sc);
 }
 
-template <typename T, int DH>
+// D: the draft width (16 or 32), a compile-time constant so that the
+// product loops, lane predicates and head splits are fixed.
+template <typename T, int DH, int D>
 __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_bytes, int sc_stride, int g_stride) {
     extern __shared__ __align__(16) char smem[];
     __shared__ uint64_t wbar;
@@ -804,7 +806,8 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
     const int team = threadIdx.x >> 7;
     const int s = blockIdx.x * 2 + team;
     const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
-    const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
+    constexpr int d = D, NH = D / DH;
+    const int F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L;
     const int n_max = a.kv.n_max;
     const CallParams& P = *a.P;
     const SeqState& ss = a.ss;
@@ -836,7 +839,8 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
     }
     __syncthreads();
     if (!live) return;  // the rest synchronises within the team only
-    const int S = 4 / NH, hw = warp % NH, spw = warp / NH;  // this warp's head and key range
+    constexpr int S = 4 / NH;
+    const int hw = warp % NH, spw = warp / NH;  // this warp's head and key range
     const bool att_enc = a.m.enc == 2;
     const float inv_d = 1.0f / (float)d;
     float* hd = (float*)(area + kvb + 16);
@@ -1130,7 +1134,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
 // covered).
 static size_t lane_area(const DevModel& m, int n_max, int gamma_max, int* sc_out, int* g_out) {
     const int CH = m.dtype == 1 ? 8 : 4;
-    const bool shape = (m.nh == 1 && (m.dh == 16 || m.dh == 32)) || (m.nh == 2 && m.dh == 16);
+    const bool shape = (m.nh == 1 && (m.dh == 16 || m.dh == 32)) || (m.nh == 2 && m.dh == 16);  // d = 16 or 32
     if (!shape || m.d % CH || m.M > 64 || m.K > 256 || m.L < 1) return 0;
     if (m.enc != 2 && (m.F % (4 * CH) || m.F > 256)) return 0;
     const size_t eb = m.dtype == 1 ? 2 : 4;
@@ -1162,8 +1166,9 @@ cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqSta
         if (e != cudaSuccess) return e;
         return launch_k(kern, dim3((B + 1) / 2), dim3(256), sm, st, a, (int)area, sc, G);
     };
-    if (m.dtype == 0) return m.dh == 16 ? go(k_draft_lane<float, 16>) : go(k_draft_lane<float, 32>);
-    return m.dh == 16 ? go(k_draft_lane<bf16, 16>) : go(k_draft_lane<bf16, 32>);
+    if (m.d == 16) return m.dtype == 0 ? go(k_draft_lane<float, 16, 16>) : go(k_draft_lane<bf16, 16, 16>);
+    if (m.dtype == 0) return m.dh == 16 ? go(k_draft_lane<float, 16, 32>) : go(k_draft_lane<float, 32, 32>);
+    return m.dh == 16 ? go(k_draft_lane<bf16, 16, 32>) : go(k_draft_lane<bf16, 32, 32>);
 }
 
 }  // namespace tppsd
