@@ -838,7 +838,11 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                     bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
     }
     __syncthreads();
-    if (!live) return;  // the rest synchronises within the team only
+    if (!live) {
+        // a CTA may not exit while the model copy still writes its shared memory
+        mbar_wait(&wbar, 0, a.err, 14);
+        return;  // the rest synchronises within the team only
+    }
     constexpr int S = 4 / NH;
     const int hw = warp % NH, spw = warp / NH;  // this warp's head and key range
     const bool att_enc = a.m.enc == 2;
