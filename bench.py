@@ -281,7 +281,8 @@ def cpu_oracle_rate(wl, bt, bd, tau, mk, budget_s=12.0):
     dt = time.perf_counter() - t0
     return {"value": round(S * wl.n_events / dt, 1), "unit": UNIT, "cores": cores, "kind": "oracle",
             "sample": f"first {S} of {wl.batch} sequences, all {wl.n_events} events, gamma "
-                      f"{wl.gamma}, fp64 oracle with bf16 emulation, {dt:.1f} s"}
+                      f"{wl.gamma}, fp64 oracle with bf16 emulation, {dt:.1f} s",
+            "value_1core": round(wl.n_events / max(one, 1e-9), 1)}
 
 
 # ---------------------------------------------------------------- reference arm
