@@ -240,6 +240,20 @@ def roofline(kt, stats, wl, peaks):
     return dom, per
 
 
+def path_roofline(per, ms_step):
+    """The whole path against its roofline: every kernel class's algorithmic
+    bytes over the profiled call at the measured HBM peak (FLOPs at the
+    tensor peak for the tensor-core classes), summed, over the measured step
+    time (whose prefill the profiled call leaves out, so the fraction is a
+    lower bound)."""
+    ideal_s = 0.0
+    for r in per.values():
+        scale = 1e12 if r["unit"] == "TFLOP/s" else 1e9
+        ideal_s += r["algorithmic_per_launch"] * r["launches"] / (r["peak"] * scale)
+    return {"ideal_ms": round(ideal_s * 1e3, 3), "measured_ms": round(ms_step, 3),
+            "frac": round(ideal_s * 1e3 / ms_step, 4)}
+
+
 def ncu_traffic(kernel_class):
     """DRAM bytes per launch of a kernel class from the committed ncu capture
     (profiles/dram_traffic_c2.json), or None once any source file the
@@ -440,6 +454,7 @@ def main():
         "gpu_launches": args.steps * (st_sd["kernel_launches"] + st_sd["prefill_launches"]),
         "clocks": clk.summary(),
         "roofline": roof,
+        "path_roofline": path_roofline(per_class, ms_sd),
         "kernel_roofline": {k: {kk: v[kk] for kk in ("bound", "achieved", "peak", "unit", "frac",
                                                      "per_launch_ms", "share_of_device_time")}
                             for k, v in sorted(per_class.items(), key=lambda kv: -kv[1]["share_of_device_time"])},

@@ -49,3 +49,16 @@ def test_per_launch_units():
     assert per["gemm_ffn2"]["achieved"] == pytest.approx(ffn / (4.693e-3 / 280) / 1e12, rel=1e-3)
     # begin: one launch initialising B x N output events (16 bytes each)
     assert per["begin"]["achieved"] == pytest.approx(wl.batch * wl.n_events * 16 / 4e-6 / 1e9, rel=1e-3)
+
+
+def test_path_roofline():
+    """The whole path's ideal time is the sum of the classes' ideal times
+    and is a small fraction of the recorded 15.30 ms step."""
+    _, per = bench.roofline(KT, STATS, CF.C2, PEAKS)
+    pr = bench.path_roofline(per, 15.30)
+    parts = sum(r["algorithmic_per_launch"] * r["launches"] / (r["peak"] * (1e12 if r["unit"] == "TFLOP/s" else 1e9))
+                for r in per.values())
+    assert pr["ideal_ms"] == pytest.approx(parts * 1e3, abs=1e-3)
+    assert 0.05 < pr["frac"] < 0.3
+    att = per["attention"]
+    assert att["algorithmic_per_launch"] * 280 / (att["peak"] * 1e9) * 1e3 > 0.5 * pr["ideal_ms"]
