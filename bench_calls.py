@@ -1,10 +1,9 @@
 """Per-kernel-class timing of sampling calls, and a throughput mode for every
 workload shape.
 
-    python -m paper_2507_09252_gb300.profile_call [--workload c2] [--calls 2]
-                                                  [--mode sd|ar] [--host-loop]
-    python -m paper_2507_09252_gb300.profile_call --time --workload c3 [--gamma 4]
-                                                  [--batch 16] [--draft 0] [--encoder attnhp]
+    python bench_calls.py [--workload c2] [--calls 2] [--mode sd|ar] [--host-loop]
+    python bench_calls.py --time --workload c3 [--gamma 4] [--batch 16] [--draft 0]
+                          [--encoder attnhp]
 
 Builds the workload's models and histories (seeded, synthetic) and prefills.
 
@@ -25,12 +24,15 @@ likelihood on a pilot AR sample of the target (64 events per sequence).
 """
 import argparse
 import json
+import os
 import sys
 
-from . import configs as CF
-from . import inputs as IN
-from . import tppsd as T
-from .sampler import Sampler
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+
+from paper_2507_09252_gb300 import configs as CF  # noqa: E402
+from paper_2507_09252_gb300 import inputs as IN  # noqa: E402
+from paper_2507_09252_gb300 import tppsd as T  # noqa: E402
+from paper_2507_09252_gb300.sampler import Sampler  # noqa: E402
 
 WORKLOADS = {"c1": CF.C1, "c2": CF.C2, "c3": CF.C3, "c4": CF.C4, "c5": CF.C5}
 
@@ -91,7 +93,7 @@ def main(argv=None):
     tau, mk = torch.from_numpy(tau_np).cuda(), torch.from_numpy(mk_np).cuda()
     outs = s._outputs(B, N)
     st = torch.cuda.current_stream()
-    from .sampler import fit_poisson_draft
+    from paper_2507_09252_gb300.sampler import fit_poisson_draft
     rate, probs = 1.0, None
     if a.poisson:  # MLE on a pilot AR sample of the target (the data it models)
         T.tppsd_prefill(s.ctx, B, tau, mk, H, st)

@@ -182,6 +182,23 @@ tppsd_status_t tppsd_sample_poisson(tppsd_ctx* ctx, int32_t batch, int32_t n_eve
                                     uint32_t flags, float* out_tau, double* out_t,
                                     int32_t* out_marks, void* stream);
 
+/* Maximum-likelihood fit of the Poisson draft of App. D.3 from observed
+ * sequences tau / marks [batch][len] (host or device; inter-event times,
+ * marks in 0..n_marks-1): a homogeneous Poisson process observed on the
+ * windows [0, T_b] has likelihood prod lambda^n_b exp(-lambda T_b), so
+ * rate = (number of events) / (sum of T_b), and iid marks give
+ * mark_probs[k] = (events with mark k) / (number of events).  t_window
+ * [batch] (host, may be NULL) holds each sequence's observation window
+ * T_b, which must reach its last event; NULL takes T_b = time of the last
+ * event (the sum of its tau).  Outputs: *out_rate and out_mark_probs
+ * [n_marks] (host, fp64), ready for tppsd_sample_poisson.  Host work, no
+ * context needed.  TPPSD_ERR_INVALID_ARG for empty input, a negative or
+ * non-finite tau, a mark out of range, a window before the last event or a
+ * total window of zero. */
+tppsd_status_t tppsd_fit_poisson_draft(int32_t batch, int32_t len, const float* tau,
+                                       const int32_t* marks, const double* t_window,
+                                       int32_t n_marks, double* out_rate, double* out_mark_probs);
+
 /* The same with the end-time stop rule, outputs as tppsd_sample_until. */
 tppsd_status_t tppsd_sample_poisson_until(tppsd_ctx* ctx, int32_t batch, double t_end,
                                           int32_t max_events, int32_t gamma, double rate,
@@ -229,10 +246,23 @@ tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32_t batch, i
  * stream capture.  Every call shares the array: calls that overlap on the
  * GPU (other streams, other contexts, other host threads) race and give
  * wrong results; serialise them.  Unlike tppsd_score it leaves the
- * prefilled caches intact. */
+ * prefilled caches intact.  A bounded wait that runs out inside a kernel is
+ * reported by tppsd_wait, as for tppsd_score. */
 tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
                                    const float* tau, const int32_t* marks, float* out_logg,
                                    float* out_logf, void* stream);
+
+/* Safety limits of the sampling calls that follow (diagnostics and tests).
+ * resample_cap: iteration cap of the Theorem-1 resampling loop (Theorem 1
+ * leaves the loop unbounded; the library stops it after resample_cap
+ * proposals, keeps the last proposal and reports TPPSD_WARN_RESAMPLE_CAP,
+ * reading c6 of the sampler); 0 restores the default 65 536.  max_rounds:
+ * cap on the device round loop of Alg. 1 below its natural bound of
+ * n_events + 2 rounds (every round emits at least one event per active
+ * sequence); a call that reaches it stops and tppsd_get_stats returns
+ * TPPSD_ERR_ROUND_LIMIT; 0 removes the extra cap.  Negative values are
+ * TPPSD_ERR_INVALID_ARG.  Host-side only; takes effect at the next call. */
+tppsd_status_t tppsd_set_limits(tppsd_ctx* ctx, int32_t resample_cap, int32_t max_rounds);
 
 /* Synchronises the last stream used and copies the last call's counters.
  * Returns that call's status (OK, WARN_RESAMPLE_CAP or ERR_ROUND_LIMIT). */
@@ -246,7 +276,13 @@ tppsd_status_t tppsd_get_stats(tppsd_ctx* ctx, tppsd_stats* out);
 tppsd_status_t tppsd_kernel_times(tppsd_ctx* ctx, double* ms, int64_t* launches);
 const char* tppsd_kernel_class_name(int32_t cls);
 
-/* Host watchdog: waits at most timeout_ms for the last call's work. */
+/* Host watchdog: waits at most timeout_ms for the last call's work;
+ * TPPSD_ERR_TIMEOUT if it is still running then, or if a bounded wait
+ * inside one of the call's kernels ran out (the kernel recorded it and
+ * returned early; the context stays usable and the next call clears the
+ * record).  Setting TPPSD_FAULT=wait in the environment makes the
+ * tensor-core QKV GEMM of the scoring calls wait on a barrier that nothing
+ * completes, so its bounded wait runs out: a test of that path. */
 tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms);
 
 const char* tppsd_status_str(tppsd_status_t status);

@@ -8,7 +8,8 @@
  * bench.py's cpu_baseline / reference leg may load it.  It shares no code,
  * header, table or helper with the CUDA library.
  *
- * Parity status of each part is stated in oracle/README.md.
+ * Each function cites the passage of the paper it follows; where the paper
+ * is silent the reading taken is stated beside the code.
  */
 #ifndef TPPSD_ORACLE_H
 #define TPPSD_ORACLE_H

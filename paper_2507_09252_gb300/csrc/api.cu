@@ -71,6 +71,11 @@ struct Profiler {
     }
 };
 
+// Iteration cap of the Theorem-1 resampling loop: the paper's loop is
+// unbounded; the cap keeps the kernel's run time bounded (the bias it can
+// introduce is at most the probability of (1 - TV)^cap).
+constexpr int DEFAULT_RESAMPLE_CAP = 65536;
+
 }  // namespace
 
 struct tppsd_ctx {
@@ -101,7 +106,9 @@ struct tppsd_ctx {
     Profiler prof;
     bool profiled = false;
     TcPlan tc{};          // tensor-core GEMM plan of the target model (enabled if supported)
-    int* d_err = nullptr; // sticky device error code (pipeline wait timeouts)
+    int* d_err = nullptr; // device error code of the current call (pipeline wait timeouts)
+    int resample_cap = DEFAULT_RESAMPLE_CAP;  // Theorem-1 loop cap (tppsd_set_limits)
+    int max_rounds = 0;   // round-loop cap below the natural N + 2 (0: none)
     std::string err;
     std::vector<void*> allocs;
 };
@@ -737,6 +744,7 @@ extern "C" tppsd_status_t tppsd_prefill(tppsd_ctx* ctx, int32_t batch, const flo
                          sizeof(float) * hist_len, batch, cudaMemcpyDefault, st));
     CK(cudaMemcpy2DAsync(ss.k, pitch_i, hist_marks, sizeof(int) * hist_len,
                          sizeof(int) * hist_len, batch, cudaMemcpyDefault, st));
+    CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), st));  // the flag reports this call only
     CK(launch_history_times(ss, batch, hist_len, st));
     int nl = 1;
     if (hist_len >= 2) {
@@ -908,6 +916,9 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     p.out_tau = host_out[0] ? (float*)(sb + nb * 8) : out_tau;
     p.out_k = host_out[2] ? (int*)(sb + nb * 12) : out_k;
     p.max_loops = N + 2;
+    if (ctx->max_rounds > 0 && ctx->max_rounds < p.max_loops) p.max_loops = ctx->max_rounds;
+    p.resample_cap = ctx->resample_cap;
+    CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), st));  // the flag reports this call only
     p.t_end = t_end;
     p.out_count = until ? (host_count ? (int*)(sb + nb * 16) : out_count) : nullptr;
     // stop rule: the slots after each sequence's kept events read NaN / -1
@@ -1002,6 +1013,11 @@ static tppsd_status_t run_score(tppsd_ctx* ctx, int which, int batch, int len, c
     KVCache& kv = which == 0 ? ctx->kvT : ctx->kvD;
     SeqState& ss = ctx->ss;
     ctx->prefilled = false;
+    CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), st));  // the flag reports this call only
+    // TPPSD_FAULT=wait: the tensor-core QKV GEMM waits on a barrier nothing
+    // completes, so its bounded wait runs out and the call reports
+    // TPPSD_ERR_TIMEOUT (tests of the timeout path; no GPU fault involved)
+    ctx->tc.stall = !strcmp(fault_mode(), "wait");
     CK(cudaMemcpy2DAsync(ss.tau, sizeof(float) * ss.n_max, tau, sizeof(float) * len,
                          sizeof(float) * len, batch, cudaMemcpyDefault, st));
     CK(cudaMemcpy2DAsync(ss.k, sizeof(int) * ss.n_max, marks, sizeof(int) * len, sizeof(int) * len,
@@ -1033,6 +1049,7 @@ static tppsd_status_t run_score(tppsd_ctx* ctx, int which, int batch, int len, c
     if (hg) CK(cudaMemcpyAsync(out_logg, d_logg, nl * 4, cudaMemcpyDeviceToHost, st));
     if (hf) CK(cudaMemcpyAsync(out_logf, d_logf, nl * 4, cudaMemcpyDeviceToHost, st));
     if (hs) CK(cudaMemcpyAsync(out_logS, d_logS, (size_t)batch * 8, cudaMemcpyDeviceToHost, st));
+    ctx->tc.stall = 0;
     CK(cudaEventRecord(ctx->done_event, st));
     ctx->last_stream = st;
     return TPPSD_OK;
@@ -1058,6 +1075,51 @@ extern "C" tppsd_status_t tppsd_sample_poisson_until(tppsd_ctx* ctx, int32_t bat
                        stream, t_end, out_count, true, &pd);
 }
 
+extern "C" tppsd_status_t tppsd_fit_poisson_draft(int32_t batch, int32_t len, const float* tau,
+                                                  const int32_t* marks, const double* t_window,
+                                                  int32_t n_marks, double* out_rate,
+                                                  double* out_mark_probs) {
+    if (batch < 1 || len < 1 || !tau || !marks || !out_rate || !out_mark_probs || n_marks < 1 ||
+        n_marks > MAX_MARKS)
+        return TPPSD_ERR_INVALID_ARG;
+    const size_t n = (size_t)batch * len;
+    std::vector<float> ht;
+    std::vector<int32_t> hk;
+    const float* pt = tau;
+    const int32_t* pk = marks;
+    if (is_device_ptr(tau)) {
+        ht.resize(n);
+        if (cudaMemcpy(ht.data(), tau, n * 4, cudaMemcpyDeviceToHost) != cudaSuccess) return TPPSD_ERR_CUDA;
+        pt = ht.data();
+    }
+    if (is_device_ptr(marks)) {
+        hk.resize(n);
+        if (cudaMemcpy(hk.data(), marks, n * 4, cudaMemcpyDeviceToHost) != cudaSuccess) return TPPSD_ERR_CUDA;
+        pk = hk.data();
+    }
+    std::vector<double> cnt(n_marks, 0.0);
+    double window = 0.0;
+    for (int32_t b = 0; b < batch; ++b) {
+        double t = 0.0;
+        for (int32_t i = 0; i < len; ++i) {
+            const float v = pt[(size_t)b * len + i];
+            const int32_t k = pk[(size_t)b * len + i];
+            if (!(v >= 0.f) || !std::isfinite(v) || k < 0 || k >= n_marks) return TPPSD_ERR_INVALID_ARG;
+            t += (double)v;
+            cnt[k] += 1.0;
+        }
+        if (t_window) {
+            if (!(t_window[b] >= t) || !std::isfinite(t_window[b])) return TPPSD_ERR_INVALID_ARG;
+            t = t_window[b];
+        }
+        window += t;
+    }
+    if (!(window > 0.0)) return TPPSD_ERR_INVALID_ARG;
+    *out_rate = (double)n / window;
+    for (int32_t k = 0; k < n_marks; ++k) out_mark_probs[k] = cnt[k] / (double)n;
+    return TPPSD_OK;
+}
+
 extern "C" tppsd_status_t tppsd_score(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
                                       const float* tau, const int32_t* marks, float* out_heads,
                                       float* out_logg, float* out_logf, void* stream) {
@@ -1072,6 +1134,13 @@ extern "C" tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32
     if (!out_logS) return TPPSD_ERR_INVALID_ARG;
     return run_score(ctx, which, batch, len, tau, marks, out_heads, out_logg, out_logf, t_end,
                      out_logS, stream);
+}
+
+extern "C" tppsd_status_t tppsd_set_limits(tppsd_ctx* ctx, int32_t resample_cap, int32_t max_rounds) {
+    if (!ctx || resample_cap < 0 || max_rounds < 0) return TPPSD_ERR_INVALID_ARG;
+    ctx->resample_cap = resample_cap > 0 ? resample_cap : DEFAULT_RESAMPLE_CAP;
+    ctx->max_rounds = max_rounds;
+    return TPPSD_OK;
 }
 
 extern "C" tppsd_status_t tppsd_wait(tppsd_ctx* ctx, int32_t timeout_ms) {
@@ -1249,9 +1318,14 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     // fixed part: sequence copy, per-sequence state, K and V of every scored position
     const size_t seq_bytes = up(n * 4) + up(n * 8) + up(n * 4) + 3 * up((size_t)batch * 4);
     const size_t kv_bytes = 2 * up((size_t)c.layers * n * d * eb);
-    // per workspace row: row tables, x and y (fp32), xb/q/att (storage type), hid, head
-    const size_t row_bytes = 2 * 4 + 2 * d * 4 + 3 * d * eb + F * eb + W * 4 + 4 * d * 4;
-    const size_t fixed = seq_bytes + kv_bytes + 13 * 256;
+    // per workspace row, in the order the buffers are carved below: row_seq,
+    // row_pos, x and y (fp32), xb (the [z | h] rows of AttNHP: 2d), q and
+    // att (storage type), hid, heads, head pre-activations (fp32)
+    const size_t per_row[] = {4, 4, d * 4, d * 4, 2 * d * eb, d * eb, d * eb, F * eb, W * 4, 4 * d * 4};
+    constexpr int NROW_BUFS = (int)(sizeof(per_row) / sizeof(per_row[0]));
+    size_t row_bytes = 0;
+    for (size_t b : per_row) row_bytes += b;
+    const size_t fixed = seq_bytes + kv_bytes + NROW_BUFS * 256;  // each row buffer rounds up to 256 B
     const long long q = len - 1, total = (long long)batch * q;
     long long rows = fixed < NOALLOC_SCRATCH_BYTES ? (long long)((NOALLOC_SCRATCH_BYTES - fixed) / row_bytes) : 0;
     if (rows > total) rows = total;
@@ -1280,17 +1354,20 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     kv.Bmax = batch;
     kv.n_max = len;
     Work w{};
+    w.err = ctx->d_err;  // bounded pipeline waits report here, as in tppsd_score
     w.R = (int)rows;
-    w.row_seq = (int*)take(rows * 4);
-    w.row_pos = (int*)take(rows * 4);
-    w.x = (float*)take(rows * d * 4);
-    w.y = (float*)take(rows * d * 4);
-    w.xb = take(rows * 2 * d * eb);  // [z | h] rows of AttNHP
-    w.q = take(rows * d * eb);
-    w.att = take(rows * d * eb);
-    w.hid = take(rows * F * eb);
-    w.heads = (float*)take(rows * W * 4);
-    w.hd4 = (float*)take(rows * 4 * d * 4);
+    void* rb[NROW_BUFS];
+    for (int i = 0; i < NROW_BUFS; ++i) rb[i] = take((size_t)rows * per_row[i]);
+    w.row_seq = (int*)rb[0];
+    w.row_pos = (int*)rb[1];
+    w.x = (float*)rb[2];
+    w.y = (float*)rb[3];
+    w.xb = rb[4];
+    w.q = rb[5];
+    w.att = rb[6];
+    w.hid = rb[7];
+    w.heads = (float*)rb[8];
+    w.hd4 = (float*)rb[9];
     if (off > NOALLOC_SCRATCH_BYTES) {
         ctx->err = "tppsd_score_noalloc: scratch layout overflow";
         return TPPSD_ERR_INVALID_ARG;
@@ -1299,6 +1376,7 @@ extern "C" tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int
     // Every byte read below is written first in this call (sequence copy,
     // times, then K/V of positions 0..i before any query at i), so nothing
     // left by an earlier call is ever read.
+    CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), st));  // the flag reports this call only
     CK(cudaMemcpyAsync(ss.tau, tau, n * 4, cudaMemcpyDeviceToDevice, st));
     CK(cudaMemcpyAsync(ss.k, marks, n * 4, cudaMemcpyDeviceToDevice, st));
     CK(launch_history_times(ss, batch, len, st));

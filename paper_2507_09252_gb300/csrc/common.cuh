@@ -6,7 +6,6 @@
 
 namespace tppsd {
 
-constexpr int RESAMPLE_CAP = 65536;
 constexpr float LN_EPS = 1e-5f;
 constexpr uint32_t FLAG_NO_BONUS = 1u;
 

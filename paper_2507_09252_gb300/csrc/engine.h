@@ -119,6 +119,9 @@ struct CallParams {
     // Poisson draft (App. D.3): rate, its log, and log p of the marks [K]
     float pois_rate, pois_log_rate;
     const float* pois_logp;
+    // iteration cap of the Theorem-1 resampling loop (65 536 unless lowered
+    // by tppsd_set_limits)
+    int resample_cap;
 };
 
 // Device counters of the current call (mirrors tppsd_stats + status).
@@ -218,6 +221,7 @@ struct TcGemmArgs {
     // EPI_TC_RESID_LN
     const float* resid; float* x_out; __nv_bfloat16* xb_out; const float* ln_g; const float* ln_b;
     int* err;  // set (first error wins) if a pipeline wait times out
+    int stall; // diagnostic: wait on a barrier nothing completes, so the bounded wait runs out
 };
 struct TcLayerMaps {
     CUtensorMap wqkv, wo, w1, w2;      // boxes of the separate GEMMs
@@ -233,6 +237,7 @@ struct TcPlan {
     int head;                   // heads by the tensor-core head kernel
     CUtensorMap head_hi, head_lo;
     int* err;
+    int stall;                  // diagnostic stall of the QKV GEMM (TcGemmArgs.stall)
     CUtensorMap a_xb, a_att, a_hid;
     CUtensorMap a_zh;           // [R][2d] view of the [z | h] rows (AttNHP QKV input)
     TcLayerMaps layer[MAX_LAYERS];

@@ -79,6 +79,17 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_after();
     const uint32_t tmem = *tslot;
 
+    if (a.stall) {
+        // Diagnostic requested by the host: wait on the completion barrier
+        // before anything is issued.  Nothing can complete it, so the bounded
+        // wait runs out, records its code in *a.err and the CTA returns with
+        // no copy or MMA in flight.
+        if (threadIdx.x == 0) mbar_wait(done, 0, a.err, 9);
+        __syncthreads();
+        if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
+        return;
+    }
+
     if (warp == 0 && lane == 0) {
         // producer: TMA loads of the A and W tiles of every K block
         for (int kb = 0; kb < KB; ++kb) {

@@ -855,8 +855,10 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         const float totT = cumT[MT - 1];
         bool found = false;
         float last = 0.f;
-        for (int base = 0; base < RESAMPLE_CAP && !found; base += 128) {
+        const int rcap = P.resample_cap;
+        for (int base = 0; base < rcap && !found; base += 128) {
             const int it = base + tid;
+            const bool live_it = it < rcap;
             const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 2u + (uint32_t)it);
             const float target = u.x * totT;
             int z = MT - 1;
@@ -893,12 +895,12 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
                 ldiff = (mD + logf(sD)) - (mT + logf(sT));
             }
             const float al = fmaxf(0.f, 1.f - expf(ldiff));
-            const unsigned okb = __ballot_sync(0xffffffffu, u.w < al);
+            const unsigned okb = __ballot_sync(0xffffffffu, live_it && u.w < al);
             if (lane == 0) {
                 win_idx[warp] = okb ? 32 * warp + __ffs(okb) - 1 : 1 << 30;
             }
             if (okb && lane == __ffs(okb) - 1) win_tau[warp] = tp;
-            if (tid == 127) last = tp;
+            if (it == rcap - 1) last = tp;
             __syncthreads();
             int best = 1 << 30, bw = 0;
             for (int w = 0; w < 4; ++w)
@@ -910,11 +912,11 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
             }
             __syncthreads();  // the winner slots are rewritten by the next step
         }
-        if (!found) {  // the last proposal of the capped loop (thread 127's)
-            if (tid == 127) sh_tau = last;
+        if (!found) {  // the last proposal of the capped loop (iteration rcap - 1)
+            if (tid == (rcap - 1) % 128) sh_tau = last;
             __syncthreads();
             tau = sh_tau;
-            iters = RESAMPLE_CAP;
+            iters = (unsigned long long)rcap;
             cap = 1;
         }
     }
@@ -1263,6 +1265,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             g.row_seq = w.row_seq; g.row_pos = w.row_pos;
             g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
             g.err = tc->err;
+            g.stall = tc->stall;
             PROF_MARK(prof, KC_GEMM_QKV, 1, st);
             if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].wqkv, g, tc->bn_qkv, st)) != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_QKV, 0, st);

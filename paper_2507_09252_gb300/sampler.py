@@ -136,13 +136,10 @@ class Sampler:
         return T.tppsd_get_stats(self.ctx)
 
 
-def fit_poisson_draft(hist_tau, hist_marks, n_marks):
-    """Maximum-likelihood Poisson draft of App. D.3 from observed sequences:
-    rate = events / total observed time (sum over sequences of the time of
-    their last event), mark probabilities = mark frequencies.  Fitting the
-    draft is set-up, like loading weights; it is not part of sampling."""
-    tau = np.asarray(hist_tau, dtype=np.float64)
-    marks = np.asarray(hist_marks).ravel()
-    rate = tau.size / tau.sum()
-    probs = np.bincount(marks, minlength=n_marks)[:n_marks].astype(np.float64)
-    return float(rate), probs / probs.sum()
+def fit_poisson_draft(hist_tau, hist_marks, n_marks, t_window=None):
+    """Maximum-likelihood Poisson draft of App. D.3 from observed sequences
+    (tppsd_fit_poisson_draft): rate = events / total observation window
+    (each sequence's window t_window[b], default the time of its last event),
+    mark probabilities = mark frequencies.  Fitting the draft is set-up, like
+    loading weights; it is not part of sampling."""
+    return T.tppsd_fit_poisson_draft(hist_tau, hist_marks, n_marks, t_window)

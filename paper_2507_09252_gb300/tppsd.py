@@ -92,6 +92,9 @@ def load(build_if_missing: bool = True):
     L.tppsd_score_noalloc.restype = C.c_int
     L.tppsd_get_stats.argtypes = [_vp, C.POINTER(tppsd_stats)]
     L.tppsd_wait.argtypes = [_vp, C.c_int32]
+    L.tppsd_set_limits.argtypes = [_vp, C.c_int32, C.c_int32]
+    L.tppsd_fit_poisson_draft.argtypes = [C.c_int32, C.c_int32, _vp, _vp, _vp, C.c_int32,
+                                          C.POINTER(C.c_double), _vp]
     L.tppsd_kernel_times.argtypes = [_vp, C.POINTER(C.c_double), C.POINTER(C.c_int64)]
     L.tppsd_kernel_times.restype = C.c_int
     L.tppsd_kernel_class_name.argtypes = [C.c_int32]
@@ -105,7 +108,8 @@ def load(build_if_missing: bool = True):
     for f in ("tppsd_create_models", "tppsd_prefill", "tppsd_sample",
               "tppsd_sample_autoregressive", "tppsd_sample_until", "tppsd_sample_autoregressive_until",
               "tppsd_sample_poisson", "tppsd_sample_poisson_until",
-              "tppsd_score", "tppsd_score_until", "tppsd_get_stats", "tppsd_wait"):
+              "tppsd_score", "tppsd_score_until", "tppsd_get_stats", "tppsd_wait",
+              "tppsd_set_limits", "tppsd_fit_poisson_draft"):
         getattr(L, f).restype = C.c_int
     _lib = L
     return L
@@ -275,6 +279,28 @@ def tppsd_sample_poisson_until(ctx, batch, t_end, max_events, gamma, rate, mark_
     return _check("tppsd_sample_poisson_until", st, ctx)
 
 
+def tppsd_fit_poisson_draft(tau, marks, n_marks, t_window=None):
+    """(rate, mark_probs) of the App. D.3 Poisson draft fitted by maximum
+    likelihood on tau / marks [batch][len]; t_window [batch] optional."""
+    if isinstance(tau, np.ndarray):
+        tau = np.ascontiguousarray(tau, np.float32)
+        marks = np.ascontiguousarray(marks, np.int32)
+    B, n = tau.shape
+    win = None
+    if t_window is not None:
+        win, _ = _host_f64(t_window, "t_window")
+        if win.size != B:
+            raise ValueError("t_window must hold one value per sequence")
+    rate = C.c_double()
+    probs = np.zeros(n_marks, np.float64)
+    st = load().tppsd_fit_poisson_draft(B, n, _ptr(tau, np.float32, B * n, "tau"),
+                                        _ptr(marks, np.int32, B * n, "marks"),
+                                        None if win is None else win.ctypes.data, n_marks,
+                                        C.byref(rate), probs.ctypes.data)
+    _check("tppsd_fit_poisson_draft", st)
+    return rate.value, probs
+
+
 def tppsd_score_until(ctx, which, batch, length, tau, marks, t_end, out_heads, out_logg, out_logf,
                       out_logS, stream=None):
     n = batch * length
@@ -327,6 +353,10 @@ def tppsd_kernel_times(ctx):
 
 def tppsd_kernel_class_name(cls):
     return load().tppsd_kernel_class_name(cls).decode()
+
+
+def tppsd_set_limits(ctx, resample_cap, max_rounds):
+    return _check("tppsd_set_limits", load().tppsd_set_limits(ctx, resample_cap, max_rounds), ctx)
 
 
 def tppsd_wait(ctx, timeout_ms):

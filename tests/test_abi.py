@@ -103,13 +103,33 @@ def test_no_device_is_reported_not_crashed():
 
 
 def test_poisson_draft_fit_is_the_mle():
-    """Rate = events / observed time, mark probabilities = frequencies; on a
-    homogeneous Poisson sample the fitted rate recovers the true one."""
+    """tppsd_fit_poisson_draft (App. D.3): rate = events / observed time,
+    mark probabilities = frequencies.  Pinned by the likelihood itself: the
+    Poisson log-likelihood n log(rate) - rate * sum(T_b) is stationary at the
+    fitted rate and lower on both sides of it; on a homogeneous Poisson
+    sample the fit recovers the true rate.  Host arrays, so no GPU is needed."""
     from paper_2507_09252_gb300.sampler import fit_poisson_draft
     rng = np.random.default_rng(0)
-    tau = rng.exponential(1 / 2.5, (200, 50))
-    mk = rng.choice(3, size=(200, 50), p=[0.6, 0.3, 0.1])
+    tau = rng.exponential(1 / 2.5, (200, 50)).astype(np.float32)
+    mk = rng.choice(3, size=(200, 50), p=[0.6, 0.3, 0.1]).astype(np.int32)
     rate, p = fit_poisson_draft(tau, mk, 4)
-    assert rate == pytest.approx(tau.size / tau.sum())
+    T_obs = tau.astype(np.float64).sum()
+    assert rate == pytest.approx(tau.size / T_obs, rel=1e-12)
     assert abs(rate - 2.5) < 0.1
     assert np.allclose(p[:3], np.bincount(mk.ravel(), minlength=3) / mk.size) and p[3] == 0.0
+
+    def loglik(lam, T_tot):
+        return tau.size * np.log(lam) - lam * T_tot
+
+    for T_tot in (T_obs, T_obs + 300.0):
+        win = None if T_tot == T_obs else tau.astype(np.float64).sum(1) + 1.5
+        r, _ = fit_poisson_draft(tau, mk, 4, t_window=win)
+        assert loglik(r, T_tot) > loglik(r * 1.01, T_tot) and loglik(r, T_tot) > loglik(r * 0.99, T_tot)
+        assert abs(tau.size / r - T_tot) < 1e-6 * T_tot          # d/dlam loglik = 0
+    # invalid inputs
+    with pytest.raises(T.TppsdError):
+        fit_poisson_draft(tau, mk, 2)                              # mark 2 out of range
+    with pytest.raises(T.TppsdError):
+        fit_poisson_draft(tau, mk, 4, t_window=np.zeros(200))      # window before the last event
+    with pytest.raises(T.TppsdError):
+        fit_poisson_draft(-tau, mk, 4)                             # negative times

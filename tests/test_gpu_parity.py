@@ -22,7 +22,15 @@ def _cuda():
 
 
 # ------------------------------------------------------------------ scoring
-def _score_case(tcfg, dcfg, bt, bd, B, n, K, tol, seed=0, rel_logg=False):
+def _score_case(tcfg, dcfg, bt, bd, B, n, K, tol, seed=0, all_tau=True):
+    """Teacher-forced heads, log g and log f of both models against the
+    oracle.  log g is compared absolutely at every position for models with
+    the workloads' head scale (all_tau).  The high-gain stress models have
+    components with small sigma, where log g's sensitivity to a head value,
+    |log tau - mu| / sigma^2, multiplies fp32 rounding of the head by up to
+    ~1e3; for them log g is compared absolutely where every component has
+    sigma >= 0.2, and everywhere against the exact log density of the GPU's
+    own heads (which pins the GPU's log g arithmetic itself at 1e-4)."""
     tau, mk = G.hist(B, n, K, seed)
     s = G.make_sampler(tcfg, dcfg, bt, bd, B, n + 4, 2)
     for which, cfg, blob in ((0, tcfg, bt), (1, dcfg, bd)):
@@ -32,15 +40,18 @@ def _score_case(tcfg, dcfg, bt, bd, B, n, K, tol, seed=0, rel_logg=False):
         M = cfg.n_mix
         dh = np.abs(hd[:, :-1] - ohd[:, :-1]).max()
         df = np.abs(lf[:, 1:] - olf[:, 1:]).max()
-        # log g(tau) amplifies head differences by ~|log tau - mu| / sigma^2, so
-        # it is compared absolutely where it is well conditioned, and
-        # everywhere against the exact log density of the GPU's own heads.
-        well = (tau[:, 1:] >= 0.1) & (tau[:, 1:] <= 10.0)
-        scale = np.maximum(1.0, np.abs(olg[:, 1:])) if rel_logg else 1.0
-        dg = (np.abs(lg[:, 1:] - olg[:, 1:]) / scale)[well].max()
+        err_g = np.abs(lg[:, 1:] - olg[:, 1:])
+        if all_tau:
+            cond = np.ones_like(err_g, dtype=bool)
+        else:
+            cond = np.exp(ohd[:, :-1, 2 * M:3 * M].min(-1)) >= 0.2
+            assert cond.mean() > 0.5, cond.mean()
+        dg = err_g[cond].max()
         own = np.array([[O.log_g(M, hd[b, i - 1].astype(np.float64), tau[b, i])[0]
                          for i in range(1, n)] for b in range(B)])
         de = np.abs(lg[:, 1:] - own).max()
+        print(f"[score] which={which} heads {dh:.2e} log g {dg:.2e} (all tau {err_g.max():.2e}) "
+              f"log f {df:.2e} own {de:.2e}")
         assert dh < tol and dg < tol and df < tol and de < 1e-4, (which, dh, dg, df, de)
         assert np.isnan(lg[:, 0]).all()
     s.close()
@@ -54,7 +65,7 @@ def test_score_parity_fp32_tiny_workload():
 
 def test_score_parity_fp32_history_dependent_heads():
     tcfg, dcfg, bt, bd = G.small_models()
-    _score_case(tcfg, dcfg, bt, bd, 5, 150, 3, G.TOL_FP32)
+    _score_case(tcfg, dcfg, bt, bd, 5, 150, 3, G.TOL_FP32, all_tau=False)
 
 
 @pytest.mark.parametrize("idx,B,n", [(1, 3, 130), (2, 2, 140), (3, 1, 530), (4, 2, 80)])
@@ -77,8 +88,7 @@ def test_score_parity_fp32_large_shapes(idx, B, n):
     dcfg = CF.ModelCfg(**{**wl.draft.__dict__, "dtype": CF.FP32})
     bt = IN.model_blob(tcfg, 0, 0, head_gain=4.0)
     bd = IN.model_blob(dcfg, 0, 1, head_gain=4.0)
-    # gain-4 heads have small sigma, so log g is compared relative to |log g|
-    _score_case(tcfg, dcfg, bt, bd, B, n, tcfg.n_marks, G.TOL_FP32, rel_logg=True)
+    _score_case(tcfg, dcfg, bt, bd, B, n, tcfg.n_marks, G.TOL_FP32, all_tau=False)
 
 
 @pytest.mark.parametrize("F", [128, 256, 1024])
@@ -164,7 +174,7 @@ def test_draft_kernel_forms_match_oracle(form, dtype, monkeypatch):
     g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 50, 5, 31)
     fp32 = dtype == CF.FP32
     ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32 if fp32 else G.MARGIN_BF16,
-                                            rtol=1e-4 if fp32 else 2e-2)
+                                            rtol=1e-4 if fp32 else G.RTOL_BF16)
     assert not fails, fails
     assert ident >= 12
     assert st == T.TPPSD_OK and stats["accepted"] < stats["drafted"]
@@ -185,7 +195,7 @@ def test_draft_kernel_wide_heads_match_oracle(form, dtype, monkeypatch):
     g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 50, 5, 17)
     fp32 = dtype == CF.FP32
     ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_FP32 if fp32 else G.MARGIN_BF16,
-                                            rtol=1e-4 if fp32 else 2e-2)
+                                            rtol=1e-4 if fp32 else G.RTOL_BF16)
     assert not fails, fails
     assert ident >= 10
     assert st == T.TPPSD_OK and len(np.unique(g["k"])) > 8
@@ -200,8 +210,10 @@ def test_sequence_parity_bf16_prefix():
     bd = IN.shift_blob(dcfg, IN.model_blob(dcfg, 0, 1, head_gain=4.0), **{"head.b_mu": 0.3})
     tau, mk = IN.histories(wl, batch=6)
     g, o, st, stats = _run_both(tcfg, dcfg, bt, bd, tau, mk, 48, wl.gamma, 9)
-    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_BF16, rtol=2e-2)
+    ident, exc, fails = G.compare_sequences(g, o, G.MARGIN_BF16, rtol=G.RTOL_BF16)
+    print(f"[parity] bf16 prefix: {ident} identical, {exc} excused of 6")
     assert not fails, fails
+    assert ident >= G.MIN_IDENTICAL_FRAC * 6
 
 
 def test_identical_draft_gives_autoregressive_output():
@@ -310,11 +322,20 @@ def test_full_size_headline_workload():
     assert np.allclose(out["t"][:, 0], t_hist + out["tau"][:, 0], rtol=1e-9)
     assert (np.diff(out["t"], axis=1) > 0).all()
     assert stats_["emitted"] >= B * N and stats_["loop_iters"] <= N + 1
-    pick = [0, 97, 255]
-    o = O.sample_sd(wl.target, bt, wl.draft, bd, tau[pick], mk[pick], 40, g, 2024, seq_ids=pick)
-    sub = {k: out[k][pick, :40] for k in ("tau", "k")}
-    _, _, fails = G.compare_sequences(sub, {**o, "margin": o["margin"]}, G.MARGIN_BF16, rtol=2e-2)
+    # 32 sequences spread over the batch, all 512 events, against the oracle
+    pick = list(range(0, B, B // 32))[:32]
+    o = O.sample_sd(wl.target, bt, wl.draft, bd, tau[pick], mk[pick], N, g, 2024, seq_ids=pick)
+    sub = {k: out[k][pick] for k in ("tau", "k")}
+    ident, exc, fails = G.compare_sequences(sub, o, G.MARGIN_BF16, rtol=G.RTOL_BF16)
+    firsts = [G.first_divergence({k: sub[k][i] for k in sub}, {k: o[k][i] for k in ("tau", "k")},
+                                 G.RTOL_BF16) for i in range(len(pick))]
+    same = sum(N if f < 0 else f for f in firsts)
+    print(f"[parity] headline 32x512: {ident} identical, {exc} excused; "
+          f"{same} of {len(pick) * N} events before the first divergence")
     assert not fails, fails
+    # the prefix before each sequence's first (excused) divergence covers
+    # most events: divergences are rare near-ties, not systematic drift
+    assert same >= 0.5 * len(pick) * N, (same, firsts)
     full_tau = np.concatenate([tau[pick], out["tau"][pick]], 1)
     full_k = np.concatenate([mk[pick], out["k"][pick]], 1)
     hd, lg, lf = s.score(0, full_tau, full_k)

@@ -178,22 +178,47 @@ def test_model_heads_match_torch_library_transformer(wl):
 
 
 def test_attention_with_zero_qk_is_causal_mean():
-    """With Q and K weights zeroed every score is equal, so attention is the
-    running mean of V over positions 0..i (closed form)."""
-    import torch
+    """With the Q and K weights zeroed (biases are zero too) every score is
+    equal, so the attention output at position i is the plain mean of the
+    values v_j over positions j = 0..i.  The layer is rebuilt here in numpy
+    with that closed form in place of attention (THP encoding of App. D.4,
+    post-LN layer, heads of Sec. 4.2 by library F.linear); a wrong causal
+    bound, normaliser or head split in the oracle's attention fails it."""
     cfg = CF.ModelCfg(1, 16, 2, 32, 3, 4, CF.FP32)
     blob = IN.model_blob(cfg, 5, 0)
     offs = IN.blob_offsets(cfg)
-    o, shape = offs["layer0.w_qkv"]
     d = cfg.d_model
-    w = blob[o:o + 3 * d * d].reshape(3 * d, d)
-    w[:2 * d] = 0.0
+
+    def P(name):
+        o, shape = offs[name]
+        return blob[o:o + int(np.prod(shape))].reshape(shape).astype(np.float64)
+
+    o, _ = offs["layer0.w_qkv"]
+    blob[o:o + 2 * d * d] = 0.0                       # W_q and W_k rows
+    assert not P("layer0.b_qkv")[:2 * d].any()         # zero biases: every score is 0
     rng = np.random.default_rng(2)
     B, n = 2, 12
     tau = rng.exponential(1.0, (B, n)).astype(np.float32)
     marks = rng.integers(0, cfg.n_marks, (B, n)).astype(np.int32)
     hd, _, _ = O.score(cfg, blob, tau, marks)
-    ref = HP.torch_reference_heads(cfg, blob, tau, marks)
+
+    t = np.cumsum(tau.astype(np.float64), 1)
+    j = np.arange(d)
+    ang = t[..., None] / 10000.0 ** ((j - j % 2) / d)
+    x = np.where(j % 2 == 1, np.cos(ang), np.sin(ang)) + P("type_emb")[marks]
+    wqkv, bqkv = P("layer0.w_qkv"), P("layer0.b_qkv")
+    v = x @ wqkv[2 * d:].T + bqkv[2 * d:]
+    a = np.cumsum(v, 1) / np.arange(1, n + 1)[None, :, None]   # causal mean of V
+
+    def ln(y, g, b):
+        mu = y.mean(-1, keepdims=True)
+        var = ((y - mu) ** 2).mean(-1, keepdims=True)
+        return (y - mu) / np.sqrt(var + 1e-5) * g + b
+
+    h1 = ln(x + a @ P("layer0.w_o").T + P("layer0.b_o"), P("layer0.ln1_g"), P("layer0.ln1_b"))
+    f = np.maximum(h1 @ P("layer0.w_1").T + P("layer0.b_1"), 0.0) @ P("layer0.w_2").T + P("layer0.b_2")
+    h2 = ln(h1 + f, P("layer0.ln2_g"), P("layer0.ln2_b"))
+    ref = HP.torch_heads(cfg, blob, h2)
     assert np.allclose(hd[:, :-1], ref[:, :-1], atol=1e-10)
 
 
