@@ -14,7 +14,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libtppsd.so")
-UNITS = ["kernels.cu", "draft.cu", "gemm_tc.cu", "mlp_tc.cu", "head_tc.cu", "attn.cu", "api.cu"]
+UNITS = ["kernels.cu", "draft.cu", "gemm_tc.cu", "mlp_tc.cu", "head_tc.cu", "attn.cu", "attn_tc.cu", "api.cu"]
 HEADERS = ["common.cuh", "engine.h", "tc_ptx.cuh"]
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -540,6 +540,10 @@ static tppsd_status_t alloc_kv(tppsd_ctx* ctx, KVCache& kv, const tppsd_model_cf
     const size_t n = (size_t)c.layers * ctx->max_batch * ctx->n_max * c.d_model;
     TRY(dalloc(ctx, &kv.k, n * el));
     TRY(dalloc(ctx, &kv.v, n * el));
+    // positions never written read as zeros (the attention kernels load whole
+    // 128-position tiles and multiply the unused rows by P = 0)
+    CK(cudaMemset(kv.k, 0, n * el));
+    CK(cudaMemset(kv.v, 0, n * el));
     kv.Bmax = ctx->max_batch;
     kv.n_max = ctx->n_max;
     return TPPSD_OK;
@@ -623,6 +627,14 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     CK(cudaGetDevice(&ctx->device));
     TRY(upload_model(ctx, ctx->T, target, tb, tn));
     TRY(upload_model(ctx, ctx->D, draft, db, dn));
+    // TPPSD_ATTN_TC=1: the target's attention runs on the tcgen05 tensor
+    // cores where its head width allows (d_head 32 or 64, bf16), with its V
+    // cache kept in fp16.  Default: the mma.sync kernel of attn.cu (bf16 V
+    // cache), measured faster at every workload shape (the decode shapes
+    // leave the 128-row tensor-core products mostly idle).
+    ctx->T.dm.v_f16 = target->dtype == 1 && attn_tc_supported(target->d_model / target->heads) &&
+                      getenv("TPPSD_ATTN_TC") != nullptr;
+    ctx->D.dm.v_f16 = 0;
     if (draft->encoder == 2 && !draft_team_supported(ctx->D.dm)) {
         ctx->err = "an AttNHP draft model must fit the one-CTA draft kernel (heads 1, 2 or 4, d/heads 16 or 32)";
         return TPPSD_ERR_UNSUPPORTED;
@@ -669,6 +681,25 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &ctx->d_err, sizeof(int)));
     CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
     w.err = ctx->d_err;
+    // split-key attention scratch for the target's step passes (verify and
+    // AR): one partial result per (item, split), one counter per item
+    if (target->dtype == 1) {
+        int n_sm = 0;
+        CK(cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, ctx->device));
+        const int dh = target->d_model / target->heads;
+        long long need = 0;
+        const int nq = 32;  // query columns of the tensor-core attention's products
+        const long long items = (long long)B * target->heads;
+        const long long ns = attn_splits(items, ctx->n_max, dh, nq, n_sm);
+        if (ctx->T.dm.v_f16 && ns > 1) need = items * ns * nq * (dh + 2) * 4;
+        if (need > 0) {
+            TRY(dalloc(ctx, &w.attn.part, (size_t)need));
+            TRY(dalloc(ctx, &w.attn.cnt, sizeof(int) * (size_t)B * target->heads));
+            CK(cudaMemset(w.attn.cnt, 0, sizeof(int) * (size_t)B * target->heads));
+            w.attn.part_bytes = (size_t)need;
+            w.attn.cnt_items = (long long)B * target->heads;
+        }
+    }
     build_tc_plan(ctx);
     CK(cudaMallocHost(&ctx->h_active, sizeof(int)));
     CK(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking));

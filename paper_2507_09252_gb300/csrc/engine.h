@@ -2,6 +2,7 @@
 // (kernels.cu): device model descriptors, per-call parameters, launchers.
 #pragma once
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
@@ -69,6 +70,8 @@ struct DevModelT {
 struct DevModel {
     int L, d, nh, dh, F, M, K, dtype;
     int enc;                 // encoder: 0 THP, 1 SAHP, 2 AttNHP (App. D.4)
+    int v_f16;               // V cache stored as fp16 (the bf16-rounded values, for the
+                             // fp16 x fp16 second product of the tensor-core attention)
     int tenc_paired;         // dims 2i and 2i+1 share one angle (THP, AttNHP)
     const float* type_emb;   // [K][d] fp32
     // temporal encoding z_j = sin / cos (a_j + b_j t) for even / odd j:
@@ -159,6 +162,15 @@ struct SeqState {
     int n_max;
 };
 
+// Device memory of the split-key form: partial results and arrival counters
+// (zeroed once; every launch leaves them zero).  Null: no splits.
+struct AttnScratch {
+    float* part;
+    size_t part_bytes;
+    int* cnt;
+    long long cnt_items;
+};
+
 // Row workspace of the batched forward.
 struct Work {
     int* err;            // device error flag for bounded waits (may be null)
@@ -173,6 +185,7 @@ struct Work {
     float* y;            // [R][dmax] pre-LayerNorm sums
     float* heads;        // [R][hw_max]
     float* hd4;          // [R][4 dmax] head pre-activations (e = E h, V_k1 h + b_k1)
+    AttnScratch attn;    // split-key attention scratch (may be empty)
 };
 
 // Row modes of a forward pass.
@@ -207,6 +220,31 @@ struct AttArgs {
 cudaError_t launch_attn_mma(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int nseg, int* err,
                             cudaStream_t st);
 
+// Attention on the tcgen05 tensor cores (attn_tc.cu).  Device arguments of
+// one launch; the K / V / Q tensor maps are passed beside them.
+struct AttTcArgs {
+    const int* row_seq;
+    const int* row_pos;
+    __nv_bfloat16* out;   // [R][d] attention output (softmax layers)
+    float* x;             // AttNHP: residual h (fp32 [R][d]) ...
+    __nv_bfloat16* hb;    // ... and its rounded copy in the [z | h] rows ([R][2d])
+    int count, q_per_seq, g0, d, nh, layer, Bmax, n_max, attnhp;
+    float c2;             // 1/sqrt(d_head) * log2(e): scores in base-2 units
+    float slack;          // a tile whose scores exceed the reference by more starts a new one
+    int nsplit;           // key splits per item (flash-decoding)
+    float* part;          // [items * nsplit][NQ * (d_head + 2)] partial results
+    int* cnt;             // [items] arrival counters, zero between launches
+    int* err;
+};
+int attn_tc_supported(int dh);
+// Key splits per item of a step pass of `items` (query block, head,
+// sequence) items over a cache of n_max positions.
+long long attn_splits(long long items, int n_max, int dh, int nq, int n_sm);
+// step_rows: one pass of gamma+1 (or 1) rows per sequence, where key splits
+// are allowed; prefill and scoring passes use one CTA per query block.
+cudaError_t launch_attn_tc(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int nseg, bool step_rows,
+                           const AttnScratch& sc, int* err, cudaStream_t st);
+
 // ---------------------------------------------------------------- tensor-core GEMM
 enum { EPI_TC_QKV = 0, EPI_TC_RELU = 1, EPI_TC_RESID_LN = 2 };
 struct TcGemmArgs {
@@ -222,6 +260,7 @@ struct TcGemmArgs {
     const float* resid; float* x_out; __nv_bfloat16* xb_out; const float* ln_g; const float* ln_b;
     int* err;  // set (first error wins) if a pipeline wait times out
     int stall; // diagnostic: wait on a barrier nothing completes, so the bounded wait runs out
+    int v_f16; // EPI_TC_QKV: V stored as fp16 (of the bf16-rounded value)
 };
 struct TcLayerMaps {
     CUtensorMap wqkv, wo, w1, w2;      // boxes of the separate GEMMs
@@ -243,6 +282,8 @@ struct TcPlan {
     TcLayerMaps layer[MAX_LAYERS];
 };
 bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_rows);
+// The driver's cuTensorMapEncodeTiled (null if unavailable).
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder();
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
                            cudaStream_t st);
 // Fused post-attention block of a layer (mlp_tc.cu): x1 = LN1(x + att W_o^T

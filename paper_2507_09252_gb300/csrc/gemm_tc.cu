@@ -16,6 +16,8 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 #include "engine.h"
 #include "tc_ptx.cuh"
@@ -165,9 +167,22 @@ __global__ void __launch_bounds__(128, 1)
                     st_bf16x16(a.q_out + (size_t)r * a.d + cc, v);
                 } else if (s >= 0) {
                     const int h = cc / a.dh, e = cc - h * a.dh;
-                    bf16* dst = (which == 1 ? a.kc : a.vc) +
-                                ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
-                    st_bf16x16(dst, v);
+                    const size_t o = ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
+                    if (which == 2 && a.v_f16) {
+                        // fp16 of the bf16-rounded value (exact in the fp16 range)
+                        uint32_t w[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const __half2 p2 = __floats2half2_rn(__bfloat162float(__float2bfloat16_rn(v[2 * i])),
+                                                                 __bfloat162float(__float2bfloat16_rn(v[2 * i + 1])));
+                            w[i] = *reinterpret_cast<const uint32_t*>(&p2);
+                        }
+                        uint4* d4 = reinterpret_cast<uint4*>(a.vc + o);
+                        d4[0] = make_uint4(w[0], w[1], w[2], w[3]);
+                        d4[1] = make_uint4(w[4], w[5], w[6], w[7]);
+                    } else {
+                        st_bf16x16((which == 1 ? a.kc : a.vc) + o, v);
+                    }
                 }
             }
         }
@@ -328,7 +343,7 @@ __global__ void __launch_bounds__(128, 1)
 }
 
 // ---------------------------------------------------------------- host side
-static PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
+PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
         void* p = nullptr;

@@ -9,6 +9,9 @@
 // Theorem-1 / Eq. 4 resampling, commit and cache rollback) ->
 // k_round_control.
 #include <math.h>
+#include <stdlib.h>
+
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 #include "engine.h"
@@ -116,9 +119,9 @@ struct GemmArgs {
     const T* W;          // [N][K]
     const float* bias;   // [N]
     int R, N, K;
-    // EPI_QKV
+    // EPI_QKV (v_f16: V stored as fp16 of the storage-type value)
     T* q_out; T* kc; T* vc; const int* row_seq; const int* row_pos;
-    int d, nh, dh, layer, Bmax, n_max;
+    int d, nh, dh, layer, Bmax, n_max, v_f16;
     // EPI_RELU: T out [R][N]; EPI_RESID: float out [R][N] = acc + b + resid
     T* out_t; float* out_f; const float* resid;
 };
@@ -178,7 +181,10 @@ __global__ void __launch_bounds__(256) k_gemm(GemmArgs<T> a) {
                     const int h = cc / a.dh, e = cc - h * a.dh;
                     const size_t o = ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max +
                                       a.row_pos[r]) * a.dh + e;
-                    St<T>::st((which == 1 ? a.kc : a.vc) + o, v);
+                    if (which == 2 && a.v_f16)  // exact: a bf16 value in the fp16 range
+                        reinterpret_cast<__half*>(a.vc)[o] = __float2half_rn(St<T>::rnd(v));
+                    else
+                        St<T>::st((which == 1 ? a.kc : a.vc) + o, v);
                 }
             } else if (EPI == EPI_RELU) {
                 St<T>::st(a.out_t + (size_t)r * a.N + c, fmaxf(v, 0.f));
@@ -1182,9 +1188,11 @@ __global__ void k_score_survival(SeqState ss, Work w, int M, int K, int len, int
 // attn.cu; fp32 caches (the fp32 models) use the SIMT kernels above.
 template <typename T>
 static cudaError_t attention_launch(const AttArgs<T>& aa, const DevModel& m, const RowSpec& rs, int R,
-                                    int nseg, int* err, cudaStream_t st) {
+                                    int nseg, const Work& w, cudaStream_t st) {
     if constexpr (sizeof(T) == 2) {
-        if (m.dh >= 16) return launch_attn_mma(aa, m.dh, m.nh, nseg, err, st);
+        // tcgen05 form (attn_tc.cu); TPPSD_ATTN_MMA=1 selects the mma.sync form
+        if (m.v_f16) return launch_attn_tc(aa, m.dh, m.nh, nseg, rs.mode == ROWS_STEP, w.attn, w.err, st);
+        if (m.dh >= 16) return launch_attn_mma(aa, m.dh, m.nh, nseg, w.err, st);
     }
     if (rs.q == 1) {
         DISPATCH_DH(m.dh, (k_attention_single<T, DH><<<R, 256, 0, st>>>(aa)));
@@ -1233,12 +1241,14 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             g.row_seq = w.row_seq; g.row_pos = w.row_pos;
             g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
             g.err = tc->err;
+            g.v_f16 = m.v_f16;
             e = launch_gemm_tc(tc->a_zh, tc->layer[l].wqkv, g, tc->bn_qkv, st);
         } else {
             GemmArgs<T> g{};
             g.A = xb; g.W = (const T*)L.w_qkv; g.bias = L.b_qkv; g.R = R; g.N = 3 * d; g.K = 2 * d;
             g.q_out = q; g.kc = (T*)kv.k; g.vc = (T*)kv.v; g.row_seq = w.row_seq; g.row_pos = w.row_pos;
             g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+            g.v_f16 = m.v_f16;
             k_gemm<T, EPI_QKV><<<grid(3 * d), blk, 0, st>>>(g);
             e = cudaGetLastError();
         }
@@ -1251,7 +1261,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         aa.scale = 1.0f / sqrtf((float)m.dh);
         aa.attnhp = 1; aa.x = w.x; aa.hb = xb;
         PROF_MARK(prof, KC_ATTENTION, 1, st);
-        if ((e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st)) != cudaSuccess) return e;
+        if ((e = attention_launch<T>(aa, m, rs, R, nseg, w, st)) != cudaSuccess) return e;
         PROF_MARK(prof, KC_ATTENTION, 0, st);
         nl += 2;
     }
@@ -1266,6 +1276,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
             g.err = tc->err;
             g.stall = tc->stall;
+            g.v_f16 = m.v_f16;
             PROF_MARK(prof, KC_GEMM_QKV, 1, st);
             if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].wqkv, g, tc->bn_qkv, st)) != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_QKV, 0, st);
@@ -1275,7 +1286,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             aa.g0 = rs.g0; aa.d = d; aa.nh = m.nh; aa.layer = l; aa.kv = kv;
             aa.scale = 1.0f / sqrtf((float)m.dh);
             PROF_MARK(prof, KC_ATTENTION, 1, st);
-            if ((e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st)) != cudaSuccess) return e;
+            if ((e = attention_launch<T>(aa, m, rs, R, nseg, w, st)) != cudaSuccess) return e;
             PROF_MARK(prof, KC_ATTENTION, 0, st);
             if (tc->mlp) {
                 MlpArgs ma{};
@@ -1319,6 +1330,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         g.A = xb; g.W = (const T*)L.w_qkv; g.bias = L.b_qkv; g.R = R; g.N = 3 * d; g.K = d;
         g.q_out = q; g.kc = (T*)kv.k; g.vc = (T*)kv.v; g.row_seq = w.row_seq; g.row_pos = w.row_pos;
         g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+        g.v_f16 = m.v_f16;
         PROF_MARK(prof, KC_GEMM_QKV, 1, st);
         k_gemm<T, EPI_QKV><<<grid(3 * d), blk, 0, st>>>(g);
         PROF_MARK(prof, KC_GEMM_QKV, 0, st);
@@ -1329,7 +1341,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         aa.scale = 1.0f / sqrtf((float)m.dh);
         PROF_MARK(prof, KC_ATTENTION, 1, st);
         {
-            const cudaError_t e = attention_launch<T>(aa, m, rs, R, nseg, w.err, st);
+            const cudaError_t e = attention_launch<T>(aa, m, rs, R, nseg, w, st);
             if (e != cudaSuccess) return e;
         }
         PROF_MARK(prof, KC_ATTENTION, 0, st);

@@ -21,10 +21,16 @@ MARGIN_BF16 = 1e-2
 # sampled bf16 times are compared to this relative tolerance (a time is
 # exp(mu + sigma eps) with mu, sigma within TOL_BF16; several events add)
 RTOL_BF16 = 2e-2
-# bf16 sampling tests: at least this fraction of sequences must match the
-# oracle event for event (the rest may diverge only after a decision within
-# MARGIN_BF16 of its threshold)
-MIN_IDENTICAL_FRAC = 0.75
+# bf16 sampling tests on models with the workloads' weight scale: at least
+# this fraction of sequences must match the oracle event for event, and at
+# most one sequence of a small batch may diverge (only ever after a decision
+# within MARGIN_BF16 of its threshold)
+MIN_IDENTICAL_FRAC = 0.9
+
+
+def min_identical(B):
+    """Sequences of a batch of B that must match the oracle exactly."""
+    return min(B - 1, int(np.ceil(MIN_IDENTICAL_FRAC * B))) if B > 1 else 1
 
 
 def make_sampler(tcfg, dcfg, bt, bd, B, n_max, gmax):
