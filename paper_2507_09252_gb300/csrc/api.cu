@@ -632,9 +632,11 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     // cache kept in fp16.  Default: the mma.sync kernel of attn.cu (bf16 V
     // cache), measured faster at every workload shape (the decode shapes
     // leave the 128-row tensor-core products mostly idle).
-    ctx->T.dm.v_f16 = target->dtype == 1 && attn_tc_supported(target->d_model / target->heads) &&
-                      getenv("TPPSD_ATTN_TC") != nullptr;
+    const int dhT = target->d_model / target->heads;
+    ctx->T.dm.attn_tc = target->dtype == 1 && attn_tc_supported(dhT) && getenv("TPPSD_ATTN_TC") != nullptr;
+    ctx->T.dm.v_f16 = ctx->T.dm.attn_tc;
     ctx->D.dm.v_f16 = 0;
+    ctx->D.dm.attn_tc = 0;
     if (draft->encoder == 2 && !draft_team_supported(ctx->D.dm)) {
         ctx->err = "an AttNHP draft model must fit the one-CTA draft kernel (heads 1, 2 or 4, d/heads 16 or 32)";
         return TPPSD_ERR_UNSUPPORTED;
@@ -691,7 +693,7 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
         const int nq = 32;  // query columns of the tensor-core attention's products
         const long long items = (long long)B * target->heads;
         const long long ns = attn_splits(items, ctx->n_max, dh, nq, n_sm);
-        if (ctx->T.dm.v_f16 && ns > 1) need = items * ns * nq * (dh + 2) * 4;
+        if (ctx->T.dm.attn_tc && ns > 1) need = items * ns * nq * (dh + 2) * 4;
         if (need > 0) {
             TRY(dalloc(ctx, &w.attn.part, (size_t)need));
             TRY(dalloc(ctx, &w.attn.cnt, sizeof(int) * (size_t)B * target->heads));

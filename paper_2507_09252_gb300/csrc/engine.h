@@ -71,7 +71,8 @@ struct DevModel {
     int L, d, nh, dh, F, M, K, dtype;
     int enc;                 // encoder: 0 THP, 1 SAHP, 2 AttNHP (App. D.4)
     int v_f16;               // V cache stored as fp16 (the bf16-rounded values, for the
-                             // fp16 x fp16 second product of the tensor-core attention)
+                             // fp16 x fp16 second product of the tcgen05 attention)
+    int attn_tc;             // attention on the tcgen05 kernel (else the mma.sync one)
     int tenc_paired;         // dims 2i and 2i+1 share one angle (THP, AttNHP)
     const float* type_emb;   // [K][d] fp32
     // temporal encoding z_j = sin / cos (a_j + b_j t) for even / odd j:

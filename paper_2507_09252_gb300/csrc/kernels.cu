@@ -1191,7 +1191,7 @@ static cudaError_t attention_launch(const AttArgs<T>& aa, const DevModel& m, con
                                     int nseg, const Work& w, cudaStream_t st) {
     if constexpr (sizeof(T) == 2) {
         // tcgen05 form (attn_tc.cu); TPPSD_ATTN_MMA=1 selects the mma.sync form
-        if (m.v_f16) return launch_attn_tc(aa, m.dh, m.nh, nseg, rs.mode == ROWS_STEP, w.attn, w.err, st);
+        if (m.attn_tc) return launch_attn_tc(aa, m.dh, m.nh, nseg, rs.mode == ROWS_STEP, w.attn, w.err, st);
         if (m.dh >= 16) return launch_attn_mma(aa, m.dh, m.nh, nseg, w.err, st);
     }
     if (rs.q == 1) {
