@@ -389,7 +389,8 @@ def main():
     with ClockSampler(local) as clk:
         ms_sd = timed(step_sd, args.steps, args.warmup)
     _, st_sd = T.tppsd_get_stats(s.ctx)
-    ms_ar = timed(step_ar, max(1, min(args.steps, 3)), 1)
+    # the AR comparator: same warm-up, up to 10 timed steps (~70 ms each)
+    ms_ar = timed(step_ar, max(1, min(args.steps, 10)), args.warmup)
     _, st_ar = T.tppsd_get_stats(s.ctx)
 
     # Poisson draft (App. D.3) in place of the draft model, fitted by maximum

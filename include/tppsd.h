@@ -127,6 +127,7 @@ tppsd_status_t tppsd_prefill(tppsd_ctx* ctx, int32_t batch, const float* hist_ta
 #define TPPSD_FLAG_NO_BONUS 1u  /* no extra target event after a full accept */
 #define TPPSD_FLAG_HOST_LOOP 2u /* round loop driven from the host (debug) */
 #define TPPSD_FLAG_PROFILE 4u   /* host-driven loop with CUDA events around every kernel */
+#define TPPSD_FLAG_DEBUG_TRACE 8u /* record every verify decision (tppsd_get_trace) */
 
 /* TPP-SD (Sec. 4.3, Alg. 1): draws n_events events after the prefilled
  * history of each of the first `batch` sequences, with gamma drafts per
@@ -251,6 +252,24 @@ tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32_t batch, i
 tppsd_status_t tppsd_score_noalloc(tppsd_ctx* ctx, int32_t which, int32_t batch, int32_t len,
                                    const float* tau, const int32_t* marks, float* out_logg,
                                    float* out_logf, void* stream);
+
+/* Decisions of the last tppsd_sample / tppsd_sample_until /
+ * tppsd_sample_poisson(_until) call made with TPPSD_FLAG_DEBUG_TRACE (Alg. 1:
+ * the tests of Sec. 4.3, the first rejection, Theorem 1 and Eq. 4), for the
+ * first n_events generated events of each of the first `batch` sequences:
+ * out [batch][n_events][4] floats (host or device), per event
+ *   [0] u_tau - min(1, g_T / g_D) of its time test (negative: accepted)
+ *   [1] u_k - min(1, f_T / f_D) of its mark test
+ *   [2] decision code: 1 accepted draft; at the first rejection 2 (time
+ *       redrawn by Theorem 1) + 4 (mark redrawn from Eq. 4); 8 bonus event
+ *       drawn from the target (no test: [0], [1] NaN)
+ *   [3] the device round-loop iteration that decided it.
+ * The margins are the GPU's own, computed in its own precision: a sampled
+ * sequence can only differ from an exact computation after a decision
+ * whose margin is about that precision.  Events never reached read as 0.
+ * TPPSD_ERR_INVALID_ARG if the last call was not traced or the sizes
+ * exceed it. */
+tppsd_status_t tppsd_get_trace(tppsd_ctx* ctx, int32_t batch, int32_t n_events, float* out);
 
 /* Safety limits of the sampling calls that follow (diagnostics and tests).
  * resample_cap: iteration cap of the Theorem-1 resampling loop (Theorem 1

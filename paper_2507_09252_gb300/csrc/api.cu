@@ -108,6 +108,8 @@ struct tppsd_ctx {
     TcPlan tc{};          // tensor-core GEMM plan of the target model (enabled if supported)
     int* d_err = nullptr; // device error code of the current call (pipeline wait timeouts)
     int resample_cap = DEFAULT_RESAMPLE_CAP;  // Theorem-1 loop cap (tppsd_set_limits)
+    float4* d_trace = nullptr;  // [max_batch][n_max] decision records (TPPSD_FLAG_DEBUG_TRACE)
+    int trace_batch = 0, trace_hist = 0, trace_events = 0;  // extent of the last traced call
     int max_rounds = 0;   // round-loop cap below the natural N + 2 (0: none)
     std::string err;
     std::vector<void*> allocs;
@@ -680,6 +682,7 @@ static tppsd_status_t create_impl(tppsd_ctx* ctx, const tppsd_model_cfg* target,
     TRY(dalloc(ctx, &ctx->d_stats, sizeof(DevStats)));
     TRY(dalloc(ctx, &ctx->d_active, sizeof(int)));
     CK(cudaMemset(ctx->d_stats, 0, sizeof(DevStats)));
+    TRY(dalloc(ctx, &ctx->d_trace, sizeof(float4) * (size_t)B * nm));
     TRY(dalloc(ctx, &ctx->d_err, sizeof(int)));
     CK(cudaMemset(ctx->d_err, 0, sizeof(int)));
     w.err = ctx->d_err;
@@ -951,6 +954,12 @@ static tppsd_status_t run_sampler(tppsd_ctx* ctx, int mode, int B, int N, int ga
     p.max_loops = N + 2;
     if (ctx->max_rounds > 0 && ctx->max_rounds < p.max_loops) p.max_loops = ctx->max_rounds;
     p.resample_cap = ctx->resample_cap;
+    const bool traced = (flags & TPPSD_FLAG_DEBUG_TRACE) && mode != 1;
+    p.trace = traced ? ctx->d_trace : nullptr;
+    if (traced) CK(cudaMemsetAsync(ctx->d_trace, 0, sizeof(float4) * (size_t)ctx->max_batch * ctx->n_max, st));
+    ctx->trace_batch = traced ? B : 0;
+    ctx->trace_hist = H;
+    ctx->trace_events = traced ? N : 0;
     CK(cudaMemsetAsync(ctx->d_err, 0, sizeof(int), st));  // the flag reports this call only
     p.t_end = t_end;
     p.out_count = until ? (host_count ? (int*)(sb + nb * 16) : out_count) : nullptr;
@@ -1167,6 +1176,20 @@ extern "C" tppsd_status_t tppsd_score_until(tppsd_ctx* ctx, int32_t which, int32
     if (!out_logS) return TPPSD_ERR_INVALID_ARG;
     return run_score(ctx, which, batch, len, tau, marks, out_heads, out_logg, out_logf, t_end,
                      out_logS, stream);
+}
+
+extern "C" tppsd_status_t tppsd_get_trace(tppsd_ctx* ctx, int32_t batch, int32_t n_events, float* out) {
+    if (!ctx || !out || batch < 1 || n_events < 1) return TPPSD_ERR_INVALID_ARG;
+    if (batch > ctx->trace_batch || n_events > ctx->trace_events) {
+        ctx->err = "tppsd_get_trace: the last sampling call was not traced, or not that large";
+        return TPPSD_ERR_INVALID_ARG;
+    }
+    CK(cudaSetDevice(ctx->device));
+    CK(cudaEventSynchronize(ctx->done_event));
+    const size_t row = sizeof(float4) * (size_t)n_events;
+    CK(cudaMemcpy2D(out, row, ctx->d_trace + ctx->trace_hist, sizeof(float4) * (size_t)ctx->n_max, row, batch,
+                    cudaMemcpyDefault));
+    return TPPSD_OK;
 }
 
 extern "C" tppsd_status_t tppsd_set_limits(tppsd_ctx* ctx, int32_t resample_cap, int32_t max_rounds) {

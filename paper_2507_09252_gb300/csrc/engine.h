@@ -126,6 +126,9 @@ struct CallParams {
     // iteration cap of the Theorem-1 resampling loop (65 536 unless lowered
     // by tppsd_set_limits)
     int resample_cap;
+    // TPPSD_FLAG_DEBUG_TRACE: [Bmax][n_max] records of the verify decisions
+    // at each absolute position (null when off)
+    float4* trace;
 };
 
 // Device counters of the current call (mirrors tppsd_stats + status).

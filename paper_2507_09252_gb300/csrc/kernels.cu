@@ -807,9 +807,17 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
             acc_t = u.x < rt;
             acc_k = u.y < rk;
             u_mr = u.z;
+            if (P.trace)  // signed margins of the two tests (negative: accepted)
+                P.trace[sb + p] = make_float4(u.x - rt, u.y - rk, 0.f, (float)a.st->loop_iters);
         }
         const unsigned fail = __ballot_sync(0xffffffffu, lane < g && !(acc_t && acc_k));
         const int L = fail ? __ffs(fail) : g + 1;  // 1-based
+        if (P.trace && lane < g && lane < L) {
+            // decision codes: 1 accepted draft, 2 time redrawn (Theorem 1),
+            // 4 mark redrawn (Eq. 4); the first rejection may carry both
+            const int code = lane < L - 1 ? 1 : (acc_t ? 0 : 2) | (acc_k ? 0 : 4);
+            P.trace[sb + n + lane].z = (float)code;
+        }
         const int src = L <= g ? L - 1 : 0;
         const bool at = __shfl_sync(0xffffffffu, acc_t, src);
         const bool ak = __shfl_sync(0xffffffffu, acc_k, src);
@@ -963,6 +971,8 @@ __global__ void __launch_bounds__(128) k_verify_epilogue(EpiArgs a) {
         if (lane == 0) {
             const float* hT = a.th + ((size_t)s * (g + 1) + g) * a.WT;
             const U4 u = slot_uniforms(P.seed, (uint32_t)s, (uint32_t)p, 0u);
+            if (P.trace)  // 8: bonus event from the target head after the last draft
+                P.trace[sb + p] = make_float4(NAN, NAN, 8.f, (float)a.st->loop_iters);
             const float tb = draw_tau(hT, a.MT, u.x, u.y, u.z);
             ss.tau[sb + p] = tb;
             ss.t[sb + p] = ss.t[sb + p - 1] + (double)tb;

@@ -135,6 +135,12 @@ class Sampler:
     def stats(self):
         return T.tppsd_get_stats(self.ctx)
 
+    def trace(self, batch, n_events):
+        """[batch][n_events][4] verify decisions of the last call made with
+        TPPSD_FLAG_DEBUG_TRACE: time-test margin, mark-test margin, decision
+        code (1 accepted, 2 time redrawn, 4 mark redrawn, 8 bonus), round."""
+        return T.tppsd_get_trace(self.ctx, batch, n_events)
+
 
 def fit_poisson_draft(hist_tau, hist_marks, n_marks, t_window=None):
     """Maximum-likelihood Poisson draft of App. D.3 from observed sequences

@@ -24,6 +24,7 @@ TPPSD_WARN_RESAMPLE_CAP = 1
 TPPSD_FLAG_NO_BONUS = 1
 TPPSD_FLAG_HOST_LOOP = 2
 TPPSD_FLAG_PROFILE = 4
+TPPSD_FLAG_DEBUG_TRACE = 8
 TPPSD_KERNEL_CLASSES = 13
 
 
@@ -93,6 +94,7 @@ def load(build_if_missing: bool = True):
     L.tppsd_get_stats.argtypes = [_vp, C.POINTER(tppsd_stats)]
     L.tppsd_wait.argtypes = [_vp, C.c_int32]
     L.tppsd_set_limits.argtypes = [_vp, C.c_int32, C.c_int32]
+    L.tppsd_get_trace.argtypes = [_vp, C.c_int32, C.c_int32, _vp]
     L.tppsd_fit_poisson_draft.argtypes = [C.c_int32, C.c_int32, _vp, _vp, _vp, C.c_int32,
                                           C.POINTER(C.c_double), _vp]
     L.tppsd_kernel_times.argtypes = [_vp, C.POINTER(C.c_double), C.POINTER(C.c_int64)]
@@ -109,7 +111,7 @@ def load(build_if_missing: bool = True):
               "tppsd_sample_autoregressive", "tppsd_sample_until", "tppsd_sample_autoregressive_until",
               "tppsd_sample_poisson", "tppsd_sample_poisson_until",
               "tppsd_score", "tppsd_score_until", "tppsd_get_stats", "tppsd_wait",
-              "tppsd_set_limits", "tppsd_fit_poisson_draft"):
+              "tppsd_set_limits", "tppsd_fit_poisson_draft", "tppsd_get_trace"):
         getattr(L, f).restype = C.c_int
     _lib = L
     return L
@@ -353,6 +355,16 @@ def tppsd_kernel_times(ctx):
 
 def tppsd_kernel_class_name(cls):
     return load().tppsd_kernel_class_name(cls).decode()
+
+
+def tppsd_get_trace(ctx, batch, n_events, out=None):
+    """[batch][n_events][4] decision records of the last traced sampling call
+    (a new float32 numpy array unless `out` is given)."""
+    if out is None:
+        out = np.zeros((batch, n_events, 4), np.float32)
+    st = load().tppsd_get_trace(ctx, batch, n_events, _ptr(out, np.float32, batch * n_events * 4, "out"))
+    _check("tppsd_get_trace", st, ctx)
+    return out
 
 
 def tppsd_set_limits(ctx, resample_cap, max_rounds):

@@ -50,10 +50,12 @@ def first_divergence(g, o, rtol=1e-4):
     return int(idx) if bad[idx] else -1
 
 
-def compare_sequences(gpu, ora, margin_tol, rtol=1e-4):
+def compare_sequences(gpu, ora, margin_tol, rtol=1e-4, gpu_trace=None):
     """Per sequence: identical, or first divergence preceded (at or before)
-    by an oracle decision margin < margin_tol.  Returns (identical, excused,
-    failures[list of (b, idx, min_margin)])."""
+    by an oracle decision margin < margin_tol.  With gpu_trace (the
+    [B][N][4] records of a TPPSD_FLAG_DEBUG_TRACE call) the GPU's own test
+    margins count too.  Returns (identical, excused, failures[list of
+    (b, idx, min_margin)])."""
     B = gpu["k"].shape[0]
     ident, excused, fails = 0, 0, []
     for b in range(B):
@@ -64,6 +66,10 @@ def compare_sequences(gpu, ora, margin_tol, rtol=1e-4):
             ident += 1
             continue
         mm = float(np.min(ora["margin"][b, :i + 1]))
+        if gpu_trace is not None:
+            gm = np.abs(gpu_trace[b, :i + 1, :2])
+            if np.isfinite(gm).any():
+                mm = min(mm, float(np.nanmin(gm)))
         if mm < margin_tol:
             excused += 1
         else:
