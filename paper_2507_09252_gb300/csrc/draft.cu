@@ -17,6 +17,9 @@
 // written through to HBM, so all gamma steps read keys on chip.
 #include <math.h>
 
+#include <algorithm>
+#include <stdlib.h>
+
 #include "common.cuh"
 #include "engine.h"
 #include "tc_ptx.cuh"
@@ -40,7 +43,8 @@ struct DraftTeamArgs {
     DevStats* st;
     float* heads;  // [Bmax][gamma_max][W]
     int gamma, gamma_max;
-    int* err;      // set if the KV bulk load does not complete
+    int* err;      // set if a bulk copy of KV or weights does not complete
+    int ring_nst, ring_ch;  // streamed KV (k_draft_team without resident KV): stages, keys per stage
 };
 
 // DH consecutive storage-type values -> fp32, with 16-byte loads.
@@ -103,6 +107,87 @@ __device__ __forceinline__ void split_partials(const TW* __restrict__ WT, int OU
     team_sync();
 }
 
+// Floats of the partial-sum buffer of team_gemv for a model of width d and
+// FFN width F: G * OUT <= max(128 * 8, OUT) for every product of the step.
+__host__ __device__ inline int team_gp_floats(int d, int F) {
+    int g = 1024;
+    if (4 * d > g) g = 4 * d;
+    if (F > g) g = F;
+    return g;
+}
+
+// acc[v] += sum_{i0 <= i < i1} W[i][v] in[i] for the 16 bytes of weights of
+// row i at col (row stride OUT elements): eight 16-byte loads in flight.
+template <typename TW>
+__device__ __forceinline__ void gemv_slice(const TW* __restrict__ col, int OUT, const float* in, int i0, int i1,
+                                           float (&acc)[16 / sizeof(TW)]) {
+    constexpr int V = 16 / sizeof(TW), U = 8;
+    auto fma_row = [&](const uint4& w, float xv) {
+        if constexpr (sizeof(TW) == 2) {
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&w);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 f = __bfloat1622float2(h[j]);
+                acc[2 * j] = fmaf(f.x, xv, acc[2 * j]);
+                acc[2 * j + 1] = fmaf(f.y, xv, acc[2 * j + 1]);
+            }
+        } else {
+            acc[0] = fmaf(__uint_as_float(w.x), xv, acc[0]);
+            acc[1] = fmaf(__uint_as_float(w.y), xv, acc[1]);
+            acc[2] = fmaf(__uint_as_float(w.z), xv, acc[2]);
+            acc[3] = fmaf(__uint_as_float(w.w), xv, acc[3]);
+        }
+    };
+    static_assert(V == 8 || V == 4, "16-byte rows of 8 bf16 or 4 fp32 weights");
+    const TW* p = col + (size_t)i0 * OUT;
+    int i = i0;
+    for (; i + U <= i1; i += U, p += (size_t)U * OUT) {
+        uint4 w[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) w[u] = *reinterpret_cast<const uint4*>(p + (size_t)u * OUT);
+#pragma unroll
+        for (int u = 0; u < U; ++u) fma_row(w[u], in[i + u]);
+    }
+    for (; i < i1; ++i, p += OUT) fma_row(*reinterpret_cast<const uint4*>(p), in[i]);
+}
+
+// Partial sums of the product [W1 | W2]^T in (W1 [IN][OUT1], W2 [IN][OUT2],
+// [in][out] layout, OUT1 and OUT2 multiples of V = 16 bytes / weight):
+// thread t takes the V consecutive outputs of column group t % NC over input
+// slice t / NC of G (NC = (OUT1 + OUT2) / V groups; G = 128 / NC, but no
+// slice under 8 inputs; all groups per thread, G = 1, once NC >= 128).
+// part[g * OUT + o] receives slice g's sum of output o (OUT = OUT1 + OUT2).
+// Returns G; ends with a team barrier.
+template <typename TW>
+__device__ __forceinline__ int team_gemv(const TW* __restrict__ W1, int OUT1, const TW* __restrict__ W2, int OUT2,
+                                         const float* in, int IN, float* part) {
+    constexpr int V = 16 / sizeof(TW);
+    const int t = threadIdx.x & 127, OUT = OUT1 + OUT2, NC = OUT / V;
+    const int G = NC >= 128 ? 1 : max(1, min(128 / NC, IN / 8));
+    const int per = (IN + G - 1) / G;
+    for (int c = t; c < NC * G; c += 128) {
+        const int cg = c % NC, g = c / NC, o = cg * V;
+        const int i0 = g * per, i1 = min(IN, i0 + per);
+        float acc[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) acc[v] = 0.f;
+        if (o < OUT1) gemv_slice<TW>(W1 + o, OUT1, in, i0, i1, acc);
+        else gemv_slice<TW>(W2 + (o - OUT1), OUT2, in, i0, i1, acc);
+        float4* dst = reinterpret_cast<float4*>(part + (size_t)g * OUT + o);
+#pragma unroll
+        for (int v = 0; v < V; v += 4) dst[v / 4] = make_float4(acc[v], acc[v + 1], acc[v + 2], acc[v + 3]);
+    }
+    team_sync();
+    return G;
+}
+
+// Output o of a team_gemv: slice sums in slice order.
+__device__ __forceinline__ float gemv_out(const float* part, int OUT, int G, int o) {
+    float v = part[o];
+    for (int g = 1; g < G; ++g) v += part[(size_t)g * OUT + o];
+    return v;
+}
+
 // Residual add + LayerNorm of d <= 32 values by warp 0 (lane j < d holds
 // the summed output j): x = LN(x + y), xin its rounded copy.
 template <typename T>
@@ -121,34 +206,26 @@ __device__ __forceinline__ void warp_resid_ln(float yv, float* x, float* xin, in
     }
 }
 
-// Attention of one query (qs in shared memory, nh heads of DH) over keys
-// 0..n_keys-1 of K/V blocks [nh][stride][DH] (shared or global): warp w
-// takes head w % nh and key range w / nh of 4 / nh; lane-strided keys with
-// a private online softmax (exp2 units), warp merge by shuffles, then the
-// warps of a head merge through shared memory.  Softmax: the output is
-// rounded to the storage type.  attnhp (App. D.4): the normaliser is
-// 1 + sum_j f_j (an extra term exp(0)) and the fp32 output is kept.  Ends
-// with a barrier.
-template <typename T, int DH>
-__device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
-                                            int n_keys, int nh, float* out, float* scratch,
-                                            bool attnhp = false) {
-    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31;
-    const int h = warp % nh, split = warp / nh, S = 4 / nh;
-    const int per = (n_keys + S - 1) / S, lo = split * per, hi = min(n_keys, lo + per);
-    const float scale = 1.4426950408889634f / sqrtf((float)DH);
-    float q[DH];
+// Online-softmax state of one lane over the keys it has seen (exp2 units).
+template <int DH>
+struct AttState {
+    float q[DH], o[DH], mm, ll;
+    __device__ __forceinline__ void init(const float* qs, int h) {
+        const float scale = 1.4426950408889634f / sqrtf((float)DH);
 #pragma unroll
-    for (int c = 0; c < DH; ++c) q[c] = qs[h * DH + c] * scale;
-    float mm = -INFINITY, ll = 0.f, o[DH];
-#pragma unroll
-    for (int c = 0; c < DH; ++c) o[c] = 0.f;
-    const T* kh = kb + (size_t)h * stride * DH;
-    const T* vh = vb + (size_t)h * stride * DH;
-    for (int j = lo + lane; j < hi; j += 32) {
+        for (int c = 0; c < DH; ++c) {
+            q[c] = qs[h * DH + c] * scale;
+            o[c] = 0.f;
+        }
+        mm = -INFINITY;
+        ll = 0.f;
+    }
+    // one key: K row kr, V row at vp
+    template <typename T>
+    __device__ __forceinline__ void add(const T* kp, const T* vp) {
         float kr[DH], vr[DH];
-        load_row16<T, DH>(kh + (size_t)j * DH, kr);
-        load_row16<T, DH>(vh + (size_t)j * DH, vr);
+        load_row16<T, DH>(kp, kr);
+        load_row16<T, DH>(vp, vr);
         float sc = 0.f;
 #pragma unroll
         for (int c = 0; c < DH; ++c) sc = fmaf(q[c], kr[c], sc);
@@ -158,6 +235,17 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
         for (int c = 0; c < DH; ++c) o[c] = fmaf(p, vr[c], o[c] * corr);
         mm = mn;
     }
+};
+
+// Merge of the lanes' states (shuffles), then of the warps of a head
+// (shared memory), into out[nh * DH].  Softmax: the output is rounded to
+// the storage type.  attnhp (App. D.4): the normaliser is 1 + sum_j f_j (an
+// extra term exp(0)) and the fp32 output is kept.  Ends with a barrier.
+template <typename T, int DH>
+__device__ __forceinline__ void team_attend_merge(AttState<DH>& a, int nh, float* out, float* scratch,
+                                                  bool attnhp) {
+    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31, S = 4 / nh;
+    float mm = a.mm, ll = a.ll;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
         const float m2 = __shfl_xor_sync(FULL, mm, off), l2 = __shfl_xor_sync(FULL, ll, off);
@@ -170,14 +258,14 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
         }
         ll = ll * a2 + l2 * b2;
 #pragma unroll
-        for (int c = 0; c < DH; ++c) o[c] = o[c] * a2 + __shfl_xor_sync(FULL, o[c], off) * b2;
+        for (int c = 0; c < DH; ++c) a.o[c] = a.o[c] * a2 + __shfl_xor_sync(FULL, a.o[c], off) * b2;
     }
     float* sw = scratch + warp * (DH + 2);
     if (lane == 0) {
         sw[0] = mm;
         sw[1] = ll;
 #pragma unroll
-        for (int c = 0; c < DH; ++c) sw[2 + c] = o[c];
+        for (int c = 0; c < DH; ++c) sw[2 + c] = a.o[c];
     }
     team_sync();
     for (int t = threadIdx.x & 127; t < nh * DH; t += 128) {
@@ -195,6 +283,85 @@ __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const 
         out[t] = attnhp ? O / (L + exp2f(-M)) : St<T>::rnd(O / L);
     }
     team_sync();
+}
+
+// Attention of one query (qs in shared memory, nh heads of DH) over keys
+// 0..n_keys-1 of K/V blocks [nh][stride][DH] in shared memory: warp w takes
+// head w % nh and key range w / nh of 4 / nh; lane-strided keys with a
+// private online softmax, then team_attend_merge.  Ends with a barrier.
+template <typename T, int DH>
+__device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
+                                            int n_keys, int nh, float* out, float* scratch,
+                                            bool attnhp = false) {
+    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31;
+    const int h = warp % nh, split = warp / nh, S = 4 / nh;
+    const int per = (n_keys + S - 1) / S, lo = split * per, hi = min(n_keys, lo + per);
+    AttState<DH> a;
+    a.init(qs, h);
+    const T* kh = kb + (size_t)h * stride * DH;
+    const T* vh = vb + (size_t)h * stride * DH;
+    for (int j = lo + lane; j < hi; j += 32) a.template add<T>(kh + (size_t)j * DH, vh + (size_t)j * DH);
+    team_attend_merge<T, DH>(a, nh, out, scratch, attnhp);
+}
+
+// Ring of shared-memory stages through which team_attend_stream streams a
+// sequence's K/V from HBM: stage i holds ch keys of every head, K then V
+// per head ([nh][2][ch][DH]); full[i] completes when its bulk copies land.
+struct KvRing {
+    char* buf;
+    uint64_t* full;
+    int nst, ch;
+    uint32_t used;  // chunks consumed so far (the same in every thread)
+    bool ok;        // false after a wait gave up: no further copies or waits
+};
+
+// team_attend over keys 0..n_keys-1 of HBM blocks [nh][stride][DH] (the
+// draft KV cache of one layer and sequence): thread 0 keeps nst chunks of ch
+// keys in flight by bulk copies (all heads, K and V), the team consumes them
+// in order, and a team barrier after each chunk frees its stage for the
+// chunk nst ahead.  Keys written by this CTA's generic stores must be fenced
+// (fence_proxy_async_global) before the barrier that precedes the call.
+// Ends with a barrier.
+template <typename T, int DH>
+__device__ __forceinline__ void team_attend_stream(const float* qs, const T* kg, const T* vg, int stride, int n_keys,
+                                                int nh, float* out, float* scratch, KvRing& r, int* err,
+                                                bool attnhp = false) {
+    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
+    const int h = warp % nh, split = warp / nh, S = 4 / nh;
+    const int nch = (n_keys + r.ch - 1) / r.ch;
+    const size_t hs = (size_t)r.ch * DH, ss = 2 * (size_t)nh * hs;
+    auto issue = [&](int c) {
+        const uint32_t u = r.used + (uint32_t)c;
+        const int st = (int)(u % (uint32_t)r.nst);
+        const int k0 = c * r.ch, cnt = min(r.ch, n_keys - k0);
+        const uint32_t bytes = (uint32_t)cnt * DH * sizeof(T);
+        T* dst = (T*)r.buf + st * ss;
+        mbar_arrive_expect_tx(r.full + st, 2u * nh * bytes);
+        for (int hh = 0; hh < nh; ++hh) {
+            const size_t src = ((size_t)hh * stride + k0) * DH;
+            bulk_load(dst + (2 * hh) * hs, kg + src, bytes, r.full + st);
+            bulk_load(dst + (2 * hh + 1) * hs, vg + src, bytes, r.full + st);
+        }
+    };
+    if (tid == 0 && r.ok) {
+        fence_proxy_async_global();
+        for (int c = 0; c < min(r.nst, nch); ++c) issue(c);
+    }
+    AttState<DH> a;
+    a.init(qs, h);
+    for (int c = 0; c < nch; ++c) {
+        const uint32_t u = r.used + (uint32_t)c;
+        const int st = (int)(u % (uint32_t)r.nst);
+        if (r.ok) r.ok = mbar_wait(r.full + st, (u / (uint32_t)r.nst) & 1u, err, 15);
+        const int cnt = min(r.ch, n_keys - c * r.ch);
+        const int per = (cnt + S - 1) / S, lo = split * per, hi = min(cnt, lo + per);
+        const T* kh = (const T*)r.buf + st * ss + (2 * h) * hs;
+        for (int j = lo + lane; j < hi; j += 32) a.template add<T>(kh + (size_t)j * DH, kh + hs + (size_t)j * DH);
+        team_sync();
+        if (tid == 0 && r.ok && c + r.nst < nch) issue(c + r.nst);
+    }
+    r.used += (uint32_t)nch;
+    team_attend_merge<T, DH>(a, nh, out, scratch, attnhp);
 }
 
 // Warp-parallel log-softmax of n <= 32*R values v[] (shared) in place, then
@@ -306,12 +473,20 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     const DevModelT& m = WS ? msh : a.m.t;
     const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
     const int n_max = a.kv.n_max;
-    const int OPd = d <= 32 ? 32 : 64;  // output block of the few-output products
-    // team area: [resident KV][mbarrier][work vectors]
+    // team area: [resident KV][8 mbarriers][KV ring (streamed KV)][work vectors]
     const size_t kvb = KVS ? (((size_t)L * 2 * n_max * d * sizeof(T) + 15) & ~(size_t)15) : 0;
+    const size_t ringb = KVS ? 0 : (size_t)a.ring_nst * a.ring_ch * 2 * d * sizeof(T);
     T* kvs = (T*)area;
     uint64_t* bar = (uint64_t*)(area + kvb);
-    float* x = (float*)(area + kvb + 16);
+    KvRing ring{area + kvb + 64, bar + 1, a.ring_nst, a.ring_ch, 0u, true};
+    if (!KVS) {
+        if (tid == 0) {
+            for (int i = 0; i < ring.nst; ++i) mbar_init(ring.full + i, 1);
+            mbar_fence_init();
+        }
+        team_sync();
+    }
+    float* x = (float*)(area + kvb + 64 + ringb);
     float* zin = x + d;   // rounded temporal encoding; [zin | xin] is the AttNHP QKV input
     float* xin = zin + d;
     float* qkv = xin + d;
@@ -320,8 +495,8 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     float* y = hid + F;
     float* e = y + d;  // E h (3d) | tanh(V_k1 h + b_k1) (d)
     float* hd = e + 4 * d;
-    float* part = hd + ((W + 3) & ~3);
-    float* attn = part + 128;
+    float* part = hd + ((W + 3) & ~3);  // team_gemv partial sums (16-byte aligned)
+    float* attn = part + team_gp_floats(d, F);
     const SeqState& ss = a.ss;
     const int n = ss.n_emit[s], nd = ss.n_draft[s];
     auto gk = [&](int l, int w) -> T* {
@@ -343,35 +518,25 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
         team_sync();
         mbar_wait(bar, 0, a.err, 12);
     }
-    // x = LN(x + W_T in + b): few-output product, then the residual add and
-    // LayerNorm (folded into the reduction when d <= 32).  Ends synced.
+    // x = LN(x + W_T in + b): the product, then the residual add and
+    // LayerNorm (by warp 0, in registers when d <= 32).  Ends synced.
     auto proj_resid_ln = [&](const T* WT, const float* bias, const float* in, int IN, const float* g,
                              const float* b) {
-        split_partials<T>(WT, d, 0, in, IN, OPd, part);
+        const int G = team_gemv<T>(WT, d, nullptr, 0, in, IN, part);
         if (d <= 32) {
             if (warp == 0) {
-                float v = 0.f;
-                if (lane < d) {
-                    v = bias[lane];
-                    for (int gg = 0; gg < 128 / OPd; ++gg) v += part[gg * OPd + lane];
-                }
+                const float v = lane < d ? bias[lane] + gemv_out(part, d, G, lane) : 0.f;
                 warp_resid_ln<T>(v, x, xin, d, g, b);
             }
             team_sync();
             return;
         }
-        for (int ob = 0; ob < d; ob += OPd) {
-            if (ob > 0) split_partials<T>(WT, d, ob, in, IN, OPd, part);
-            if (tid < OPd && ob + tid < d) {
-                float v = bias[ob + tid];
-                for (int gg = 0; gg < 128 / OPd; ++gg) v += part[gg * OPd + tid];
-                y[ob + tid] = v;
-            }
-            team_sync();
-        }
         if (warp == 0) {
             float sum = 0.f;
-            for (int i = lane; i < d; i += 32) { x[i] += y[i]; sum += x[i]; }
+            for (int i = lane; i < d; i += 32) {
+                x[i] += bias[i] + gemv_out(part, d, G, i);
+                sum += x[i];
+            }
             const float mean = warp_sum(sum) / d;
             float var = 0.f;
             for (int i = lane; i < d; i += 32) var += (x[i] - mean) * (x[i] - mean);
@@ -384,6 +549,27 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
         }
         team_sync();
     };
+    // Q, K, V of position p from the QKV input qin (IN wide); K and V
+    // appended to the cache (and its resident copy).  Ends synced.
+    auto qkv_step = [&](const LayerW& Wl, int l, int p, const float* qin, int IN) {
+        const int G = team_gemv<T>((const T*)Wl.w_qkv, 3 * d, nullptr, 0, qin, IN, part);
+        for (int o = tid; o < 3 * d; o += 128) {
+            const float v = St<T>::rnd(Wl.b_qkv[o] + gemv_out(part, 3 * d, G, o));
+            qkv[o] = v;
+            if (o >= d) {
+                const int w = o < 2 * d ? 0 : 1, c = o - d - w * d, hh = c / DH, ee = c - hh * DH;
+                const size_t off = ((size_t)hh * n_max + p) * DH + ee;
+                St<T>::st(gk(l, w) + off, v);
+                if (KVS) St<T>::st(sk(l, w) + off, v);
+            }
+        }
+        if (!KVS) fence_proxy_async_global();  // the streamed attention reads them back by bulk copy
+        team_sync();
+    };
+    auto attend = [&](int l, int p, bool attnhp) {
+        if (KVS) team_attend<T, DH>(qkv, sk(l, 0), sk(l, 1), n_max, p + 1, NH, att, attn, attnhp);
+        else team_attend_stream<T, DH>(qkv, gk(l, 0), gk(l, 1), n_max, p + 1, NH, att, attn, ring, a.err, attnhp);
+    };
     // Layers of the encode step at position p from x / xin (set and synced
     // by the caller); leaves the final hidden state in x (synced).
     const bool att_enc = a.m.enc == 2;
@@ -392,21 +578,8 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             // AttNHP (App. D.4): q, k, v = W [z; h] + b, a = sum f v / (1 + sum f),
             // h <- h + tanh(a)
             for (int l = 0; l < L; ++l) {
-                const LayerW& Wl = m.layer[l];
-                for (int o = tid; o < 3 * d; o += 128) {
-                    const float v = St<T>::rnd(dot_col<T>((const T*)Wl.w_qkv, 3 * d, o, zin, 2 * d) + Wl.b_qkv[o]);
-                    qkv[o] = v;
-                    if (o >= d) {
-                        const int w = o < 2 * d ? 0 : 1, c = o - d - w * d, hh = c / DH, ee = c - hh * DH;
-                        const size_t off = ((size_t)hh * n_max + p) * DH + ee;
-                        St<T>::st(gk(l, w) + off, v);
-                        if (KVS) St<T>::st(sk(l, w) + off, v);
-                    }
-                }
-                team_sync();
-                const T* kb = KVS ? sk(l, 0) : gk(l, 0);
-                const T* vb = KVS ? sk(l, 1) : gk(l, 1);
-                team_attend<T, DH>(qkv, kb, vb, n_max, p + 1, NH, att, attn, true);
+                qkv_step(m.layer[l], l, p, zin, 2 * d);
+                attend(l, p, true);
                 for (int i = tid; i < d; i += 128) {
                     x[i] += tanhf(att[i]);
                     xin[i] = St<T>::rnd(x[i]);
@@ -417,25 +590,15 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
         }
         for (int l = 0; l < L; ++l) {
             const LayerW& Wl = m.layer[l];
-            // Q, K, V; K and V appended to the cache at position p
-            for (int o = tid; o < 3 * d; o += 128) {
-                const float v = St<T>::rnd(dot_col<T>((const T*)Wl.w_qkv, 3 * d, o, xin, d) + Wl.b_qkv[o]);
-                qkv[o] = v;
-                if (o >= d) {
-                    const int w = o < 2 * d ? 0 : 1, c = o - d - w * d, hh = c / DH, ee = c - hh * DH;
-                    const size_t off = ((size_t)hh * n_max + p) * DH + ee;
-                    St<T>::st(gk(l, w) + off, v);
-                    if (KVS) St<T>::st(sk(l, w) + off, v);
-                }
-            }
-            team_sync();
-            const T* kb = KVS ? sk(l, 0) : gk(l, 0);
-            const T* vb = KVS ? sk(l, 1) : gk(l, 1);
-            team_attend<T, DH>(qkv, kb, vb, n_max, p + 1, NH, att, attn);
+            qkv_step(Wl, l, p, xin, d);
+            attend(l, p, false);
             proj_resid_ln((const T*)Wl.w_o, Wl.b_o, att, d, Wl.ln1_g, Wl.ln1_b);
-            for (int o = tid; o < F; o += 128)
-                hid[o] = St<T>::rnd(fmaxf(dot_col<T>((const T*)Wl.w_1, F, o, xin, d) + Wl.b_1[o], 0.f));
-            team_sync();
+            {
+                const int G = team_gemv<T>((const T*)Wl.w_1, F, nullptr, 0, xin, d, part);
+                for (int o = tid; o < F; o += 128)
+                    hid[o] = St<T>::rnd(fmaxf(Wl.b_1[o] + gemv_out(part, F, G, o), 0.f));
+                team_sync();
+            }
             proj_resid_ln((const T*)Wl.w_2, Wl.b_2, hid, F, Wl.ln2_g, Wl.ln2_b);
         }
     };
@@ -470,10 +633,14 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     for (int l = 1; l <= a.gamma; ++l) {
         const int p = n + l - 1;  // index of the drafted event
         // head (Sec. 4.2): e = E h | a = tanh(V_k1 h + b_k1)
-        for (int o = tid; o < 4 * d; o += 128)
-            e[o] = o < 3 * d ? dot_col<float>(H.E, 3 * d, o, x, d)
-                             : tanhf(dot_col<float>(H.v_k1, d, o - 3 * d, x, d) + H.b_k1[o - 3 * d]);
-        team_sync();
+        {
+            const int G = team_gemv<float>(H.E, 3 * d, H.v_k1, d, x, d, part);
+            for (int o = tid; o < 4 * d; o += 128) {
+                const float v = gemv_out(part, 4 * d, G, o);
+                e[o] = o < 3 * d ? v : tanhf(v + H.b_k1[o - 3 * d]);
+            }
+            team_sync();
+        }
         // [w logits | mu | log sigma | mark logits] in blocks of OPh outputs;
         // output j reads its own matrix and input segment
         for (int ob = 0; ob < W; ob += OPh) {
@@ -572,10 +739,35 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
     const size_t eb = m.dtype == 1 ? 2 : 4;
     const int W = 3 * m.M + m.K;
-    const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + 128 + 4 * 66) + 16;
+    const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + team_gp_floats(m.d, m.F) + 4 * 66) + 64;
     const size_t kvb = ((size_t)m.L * 2 * kv.n_max * m.d * eb + 15) & ~(size_t)15;
-    const int kvs = kvb + fl <= 110 * 1024;
-    const size_t area = ((kvs ? kvb : 0) + fl + 15) & ~(size_t)15;
+    // TPPSD_DRAFT_STREAM=<keys>: stream the KV even where it would fit, two
+    // stages of that many keys (exercises the ring's wrap-around and ragged
+    // last chunk on small cases)
+    const char* force = getenv("TPPSD_DRAFT_STREAM");
+    const int kvs = !force && kvb + fl <= 110 * 1024;
+    size_t ringb = 0;
+    if (force) {
+        a.ring_nst = 2;
+        a.ring_ch = std::max(1, std::min(256, atoi(force)));
+        ringb = 2 * (size_t)a.ring_ch * 2 * m.d * eb;
+    } else if (!kvs) {
+        // streamed KV: as many stages of up to 64 keys as the CTAs that share
+        // an SM leave room for (at most 4 resident: the kernel holds 128
+        // registers a thread), 2 to 6 stages
+        int dev = 0, n_sm = 148;
+        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+        const int per_sm = std::min(4, std::max(1, (B + n_sm - 1) / n_sm));
+        const long long budget = std::max(0ll, (long long)(227 * 1024 / per_sm) - 2048 - (long long)fl);
+        int ch = 64;
+        auto stage = [&](int c) { return (size_t)c * 2 * m.d * eb; };
+        while (ch > 16 && 2 * stage(ch) > (size_t)budget) ch /= 2;
+        const int nst = (int)std::max<size_t>(2, std::min<size_t>(6, (size_t)budget / stage(ch)));
+        a.ring_nst = nst;
+        a.ring_ch = ch;
+        ringb = nst * stage(ch);
+    }
+    const size_t area = ((kvs ? kvb : ringb) + fl + 15) & ~(size_t)15;
     const size_t wb = m.t.bytes;  // a whole number of 16-byte chunks
     const int ws = kvs && wb % 16 == 0 && wb + 2 * area <= 224 * 1024;
     if (m.dtype == 0) {
