@@ -289,6 +289,12 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
         }
     const size_t b_ek = add(ek.data(), ek.size() * 4), b_ekb = add(ekb.data(), ekb.size() * 4);
     const size_t b_ho = add(ho.data(), ho.size() * 4), b_hob = add(hob.data(), hob.size() * 4);
+    std::vector<float> hog((size_t)d * WO);  // group by group, [d][cnt] each
+    for (int part = 0, col0 = 0; part < 4; col0 += cnt[part], ++part)
+        for (int i = 0; i < d; ++i)
+            for (int o2 = 0; o2 < cnt[part]; ++o2)
+                hog[(size_t)d * col0 + (size_t)i * cnt[part] + o2] = ho[(size_t)i * WO + col0 + o2];
+    const size_t b_hog = add(hog.data(), hog.size() * 4);
     // [E; v_k1] as a sum of two bf16 matrices (hi + lo) for the tensor-core head
     std::vector<uint16_t> ekh(ek.size()), ekl(ek.size());
     for (size_t i = 0; i < ek.size(); ++i) {
@@ -333,6 +339,7 @@ static tppsd_status_t upload_model(tppsd_ctx* ctx, HostModel& hm, const tppsd_mo
     m.head_ek_b = (const float*)(b + b_ekb);
     m.head_out_t = (const float*)(b + b_ho);
     m.head_out_b = (const float*)(b + b_hob);
+    m.head_out_g = (const float*)(b + b_hog);
     m.head_ek_hi = (const void*)(b + b_ekh);
     m.head_ek_lo = (const void*)(b + b_ekl);
     m.base = b;
@@ -560,6 +567,17 @@ static int pick_bn(int N) {
     return 0;
 }
 
+// Heads of widths other than 128 (or with the head kernel off): [E; V_k1] h
+// by the split tensor-core GEMM over the hi / lo bf16 parts of [E; V_k1].
+static void head_gemm_plan(TcPlan& p, const DevModel& m, bool ok) {
+    const int d = m.d;
+    p.bn_head = pick_bn(4 * d);
+    const int box = p.bn_head < 256 ? p.bn_head : 256;
+    p.head_g = ok && !p.head && p.bn_head && d % 64 == 0 && !getenv("TPPSD_NO_TC_HEAD") &&
+               make_tmap_bf16(&p.head_hi_g, m.head_ek_hi, d, 4 * d, box) &&
+               make_tmap_bf16(&p.head_lo_g, m.head_ek_lo, d, 4 * d, box);
+}
+
 // Tensor maps for the target model's tensor-core GEMMs (bf16 models whose
 // widths are multiples of 64 and whose heads are >= 16 wide).
 static void build_tc_plan(tppsd_ctx* ctx) {
@@ -581,6 +599,8 @@ static void build_tc_plan(tppsd_ctx* ctx) {
         p.head = ok && head_tc_supported(m) &&
                  make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
                  make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
+        ok = ok && make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128);
+        head_gemm_plan(p, m, ok);
         p.err = ctx->d_err;
         p.enabled = ok ? 1 : 0;
         return;
@@ -613,6 +633,7 @@ static void build_tc_plan(tppsd_ctx* ctx) {
     p.head = ok && head_tc_supported(m) &&
              make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
              make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
+    head_gemm_plan(p, m, ok);
     p.err = ctx->d_err;
     p.enabled = ok ? 1 : 0;
 }

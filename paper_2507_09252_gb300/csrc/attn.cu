@@ -47,6 +47,14 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2(uint32_t (&r)[2], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                  : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
@@ -130,6 +138,8 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
 
     __syncthreads();  // qpos and the mbarrier inits are visible
     const int pos_g = qpos[g], pos_g8 = qpos[g + 8];  // -1 for padding rows
+    const int pos_first = qpos[0];                    // the smallest position of the rows
+    const float scale2 = a.scale * 1.4426950408889634f;  // scores in log2 units: exp2 below
     bool ok = true;
     for (int it = 0; it < ntl && ok; ++it) {
         const int stage = it & 1;
@@ -145,33 +155,50 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
                 reinterpret_cast<uint4*>(const_cast<bf16*>(vs))[i] = make_uint4(0, 0, 0, 0);
             __syncwarp();
         }
-        // S = Q K^T for KT keys
+        // S = Q K^T for KT keys; K fragments by ldmatrix (8 keys x 8 dims a
+        // matrix; keys past the copied ones read stale rows, masked below)
         float sc[NT][4];
+        const uint32_t kbase = smem_u32(ks);
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
             sc[n][0] = sc[n][1] = sc[n][2] = sc[n][3] = 0.f;
-            const int key = 8 * n + g;
-            const bool kin = key < cnt;
 #pragma unroll
-            for (int k = 0; k < KS; ++k) {
-                const uint32_t b0 = kin ? *reinterpret_cast<const uint32_t*>(ks + key * DH + 16 * k + 2 * t4) : 0u;
-                const uint32_t b1 = kin ? *reinterpret_cast<const uint32_t*>(ks + key * DH + 16 * k + 8 + 2 * t4) : 0u;
-                mma_bf16(sc[n], qa[k], b0, b1);
+            for (int k = 0; k + 1 < KS; k += 2) {  // two k-steps (32 dims) per x4
+                uint32_t b[4];
+                ldsm_x4(b, kbase + (uint32_t)((8 * n + (lane & 7)) * DH + 16 * k + 8 * (lane >> 3)) * 2);
+                mma_bf16(sc[n], qa[k], b[0], b[1]);
+                mma_bf16(sc[n], qa[k + 1], b[2], b[3]);
+            }
+            if constexpr (KS % 2) {
+                uint32_t b[2];
+                ldsm_x2(b, kbase + (uint32_t)((8 * n + (lane & 7)) * DH + 16 * (KS - 1) + 8 * ((lane >> 3) & 1)) * 2);
+                mma_bf16(sc[n], qa[KS - 1], b[0], b[1]);
             }
         }
-        // scale, mask (keys past the copied ones, and causal), online
-        // softmax (rows g and g+8; quad reductions)
+        // scale, mask (keys past the copied ones, and causal: only tiles that
+        // reach past the first row's position need it), online softmax in
+        // log2 units (rows g and g+8; quad reductions)
         float mx0 = -INFINITY, mx1 = -INFINITY;
+        if (cnt == KT && k0 + KT - 1 <= pos_first) {
 #pragma unroll
-        for (int n = 0; n < NT; ++n) {
-            const int kt = 8 * n + 2 * t4, key = k0 + kt;
-            const bool in0 = kt < cnt, in1 = kt + 1 < cnt;
-            sc[n][0] = (in0 && key <= pos_g) ? sc[n][0] * a.scale : -INFINITY;
-            sc[n][1] = (in1 && key + 1 <= pos_g) ? sc[n][1] * a.scale : -INFINITY;
-            sc[n][2] = (in0 && key <= pos_g8) ? sc[n][2] * a.scale : -INFINITY;
-            sc[n][3] = (in1 && key + 1 <= pos_g8) ? sc[n][3] * a.scale : -INFINITY;
-            mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
-            mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
+            for (int n = 0; n < NT; ++n) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) sc[n][e] *= scale2;
+                mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
+                mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
+            }
+        } else {
+#pragma unroll
+            for (int n = 0; n < NT; ++n) {
+                const int kt = 8 * n + 2 * t4, key = k0 + kt;
+                const bool in0 = kt < cnt, in1 = kt + 1 < cnt;
+                sc[n][0] = (in0 && key <= pos_g) ? sc[n][0] * scale2 : -INFINITY;
+                sc[n][1] = (in1 && key + 1 <= pos_g) ? sc[n][1] * scale2 : -INFINITY;
+                sc[n][2] = (in0 && key <= pos_g8) ? sc[n][2] * scale2 : -INFINITY;
+                sc[n][3] = (in1 && key + 1 <= pos_g8) ? sc[n][3] * scale2 : -INFINITY;
+                mx0 = fmaxf(mx0, fmaxf(sc[n][0], sc[n][1]));
+                mx1 = fmaxf(mx1, fmaxf(sc[n][2], sc[n][3]));
+            }
         }
         mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
         mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
@@ -179,14 +206,14 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
         mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
         const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
         const float ref0 = mn0 == -INFINITY ? 0.f : mn0, ref1 = mn1 == -INFINITY ? 0.f : mn1;
-        const float c0 = expf(m0 - ref0), c1 = expf(m1 - ref1);
+        const float c0 = exp2f(m0 - ref0), c1 = exp2f(m1 - ref1);
         float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
         for (int n = 0; n < NT; ++n) {
-            sc[n][0] = expf(sc[n][0] - ref0);
-            sc[n][1] = expf(sc[n][1] - ref0);
-            sc[n][2] = expf(sc[n][2] - ref1);
-            sc[n][3] = expf(sc[n][3] - ref1);
+            sc[n][0] = exp2f(sc[n][0] - ref0);
+            sc[n][1] = exp2f(sc[n][1] - ref0);
+            sc[n][2] = exp2f(sc[n][2] - ref1);
+            sc[n][3] = exp2f(sc[n][3] - ref1);
             rs0 += sc[n][0] + sc[n][1];
             rs1 += sc[n][2] + sc[n][3];
         }
@@ -253,13 +280,13 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
         for (int w = 0; w < 4; ++w) {
             const float* p = mslot(w);
             if (p[row] == -INFINITY) continue;
-            const float e = expf(p[row] - M);
+            const float e = exp2f(p[row] - M);
             L += p[16 + row] * e;
             O += p[32 + row * DH + col] * e;
         }
         if (a.attnhp) {  // a = sum f v / (1 + sum f); h <- h + tanh(a)
             const size_t xi = (size_t)(rb + row) * a.d + h * DH + col;
-            const float hn = a.x[xi] + tanhf(O / (L + expf(-M)));
+            const float hn = a.x[xi] + tanhf(O / (L + exp2f(-M)));  // exp(-m) in log2 units
             a.x[xi] = hn;
             a.hb[(size_t)(rb + row) * 2 * a.d + a.d + h * DH + col] = __float2bfloat16_rn(hn);
         } else {

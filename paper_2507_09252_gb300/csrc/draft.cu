@@ -1227,33 +1227,48 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             for (int c = 0; c < DH; ++c) q[c] = v_q[c];
             const T* kb = sk(l, 0) + (size_t)hw * n_max * DH;
             const T* vb = sk(l, 1) + (size_t)hw * n_max * DH;
+            // keys j and j + 32 of a lane per iteration: both rows are loaded
+            // before either is used (the second is a repeat of the first
+            // when j + 32 is past the range, and its terms are dropped)
             float mx = -INFINITY;
 #pragma unroll 1
-            for (int j = lo + lane; j < hi; j += 32) {
-                float kr[DH];
+            for (int j = lo + lane; j < hi; j += 64) {
+                const bool two = j + 32 < hi;
+                float kr[DH], kr2[DH];
                 load_row16<T, DH>(kb + (size_t)j * DH, kr);
-                float s0 = 0.f, s1 = 0.f;
+                load_row16<T, DH>(kb + (size_t)(two ? j + 32 : j) * DH, kr2);
+                float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
                 for (int c = 0; c < DH; c += 2) {
                     s0 = fmaf(q[c], kr[c], s0);
                     s1 = fmaf(q[c + 1], kr[c + 1], s1);
+                    t0 = fmaf(q[c], kr2[c], t0);
+                    t1 = fmaf(q[c + 1], kr2[c + 1], t1);
                 }
-                const float sv = s0 + s1;
+                const float sv = s0 + s1, sv2 = t0 + t1;
                 sc[j - lo] = sv;
                 mx = fmaxf(mx, sv);
+                if (two) {
+                    sc[j + 32 - lo] = sv2;
+                    mx = fmaxf(mx, sv2);
+                }
             }
             mx = warp_max(mx);
             float ll = 0.f, o[DH];
 #pragma unroll
             for (int c = 0; c < DH; ++c) o[c] = 0.f;
 #pragma unroll 1
-            for (int j = lo + lane; j < hi; j += 32) {
+            for (int j = lo + lane; j < hi; j += 64) {
+                const bool two = j + 32 < hi;
                 const float pj = exp2f(sc[j - lo] - mx);
-                float vr[DH];
+                const float pj2 = two ? exp2f(sc[j + 32 - lo] - mx) : 0.f;
+                float vr[DH], vr2[DH];
                 load_row16<T, DH>(vb + (size_t)j * DH, vr);
+                load_row16<T, DH>(vb + (size_t)(two ? j + 32 : j) * DH, vr2);
                 ll += pj;
+                ll += pj2;
 #pragma unroll
-                for (int c = 0; c < DH; ++c) o[c] = fmaf(pj, vr[c], o[c]);
+                for (int c = 0; c < DH; ++c) o[c] = fmaf(pj2, vr2[c], fmaf(pj, vr[c], o[c]));
             }
             ll = warp_sum(ll);
             const float oc = warp_scatter_sum<DH>(o, lane);

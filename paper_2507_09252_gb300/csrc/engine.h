@@ -86,6 +86,7 @@ struct DevModel {
     const float* head_ek_b;  // [4d]: zeros then b_k1
     const float* head_out_t; // [d][3M+K] fp32: v_w, v_mu, v_s, v_k2 transposed side by side
     const float* head_out_b; // [3M+K]: b_w, b_mu, b_s, b_k2
+    const float* head_out_g; // the same maps group by group: [d][M] x 3, then [d][K] (contiguous)
     const void* head_ek_hi;  // [4d][d] bf16: head_ek_w = hi + lo (split of each fp32 value)
     const void* head_ek_lo;
     DevModelT t;             // transposed copy (read by the per-sequence draft kernel)
@@ -250,7 +251,7 @@ cudaError_t launch_attn_tc(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int 
                            const AttnScratch& sc, int* err, cudaStream_t st);
 
 // ---------------------------------------------------------------- tensor-core GEMM
-enum { EPI_TC_QKV = 0, EPI_TC_RELU = 1, EPI_TC_RESID_LN = 2 };
+enum { EPI_TC_QKV = 0, EPI_TC_RELU = 1, EPI_TC_RESID_LN = 2, EPI_TC_F32 = 3 };
 struct TcGemmArgs {
     int R, N, K, epi;
     const float* bias;
@@ -265,6 +266,12 @@ struct TcGemmArgs {
     int* err;  // set (first error wins) if a pipeline wait times out
     int stall; // diagnostic: wait on a barrier nothing completes, so the bounded wait runs out
     int v_f16; // EPI_TC_QKV: V stored as fp16 (of the bf16-rounded value)
+    // EPI_TC_F32: fp32 out [R][N] = acc + b
+    float* out_f;
+    // split: fp32-accurate product of fp32 operands given as bf16 pairs, as
+    // one GEMM over K' = 3K: [A_hi | A_hi | A_lo] [W_hi | W_lo | W_hi]^T
+    // (second maps: A_lo, W_lo)
+    int split;
 };
 struct TcLayerMaps {
     CUtensorMap wqkv, wo, w1, w2;      // boxes of the separate GEMMs
@@ -277,8 +284,12 @@ struct TcPlan {
     int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
     int mlp;                    // post-attention block by the fused kernel
     int mlp_cl;                 // ... in its cluster form (FFN split over F / 128 CTAs)
-    int head;                   // heads by the tensor-core head kernel
+    int head;                   // heads by the tensor-core head kernel (d = 128)
     CUtensorMap head_hi, head_lo;
+    // other widths: [E; V_k1] h by the split GEMM (A_hi = xb, A_lo = att), then
+    // the small maps by k_head_out
+    int head_g, bn_head;
+    CUtensorMap head_hi_g, head_lo_g;
     int* err;
     int stall;                  // diagnostic stall of the QKV GEMM (TcGemmArgs.stall)
     CUtensorMap a_xb, a_att, a_hid;
@@ -290,6 +301,9 @@ bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_
 PFN_cuTensorMapEncodeTiled_v12000 tmap_encoder();
 cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
                            cudaStream_t st);
+// The split form (a.split = 1): A2 = A_lo, W2 = W_lo.
+cudaError_t launch_gemm_tc_split(const CUtensorMap& A, const CUtensorMap& A2, const CUtensorMap& W,
+                                 const CUtensorMap& W2, const TcGemmArgs& a, int BN, cudaStream_t st);
 // Fused post-attention block of a layer (mlp_tc.cu): x1 = LN1(x + att W_o^T
 // + b_o); x = LN2(x1 + relu(x1 W_1^T + b_1) W_2^T + b_2); xb = bf16(x).
 struct MlpArgs {

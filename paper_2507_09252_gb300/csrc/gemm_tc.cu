@@ -12,6 +12,11 @@
 //   EPI_QKV      bias, bf16 round, Q to the row buffer, K/V scattered into the
 //                KV cache at each row's (sequence, position)
 //   EPI_RELU     bias, ReLU, bf16 round
+//   EPI_F32      bias, fp32 rows (the heads' [E; V_k1] h)
+// In the split form an fp32-accurate product of fp32 operands, each given
+// as two bf16 parts (x = x_hi + x_lo), runs as one GEMM over three times the
+// K blocks: A_hi W_hi + A_hi W_lo + A_lo W_hi (the K loop walks the three
+// pairs of maps; the dropped A_lo W_lo term is below 2^-16 of |A| |W|).
 // The residual + LayerNorm epilogue (rows of N = d) is k_gemm_ln_cl below.
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -51,7 +56,8 @@ __device__ __forceinline__ void st_bf16x16(bf16* dst, const float (&v)[16]) {
 
 template <int BN>
 __global__ void __launch_bounds__(128, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB, TcGemmArgs a) {
+    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
+              const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2, TcGemmArgs a) {
     using S = TcShape<BN>;
     pdl_wait();
     extern __shared__ unsigned char smem_raw[];
@@ -65,7 +71,7 @@ __global__ void __launch_bounds__(128, 1)
     uint32_t* tslot = (uint32_t*)(done + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int n0 = blockIdx.x * BN, m0 = blockIdx.y * S::BM;
-    const int KB = a.K / S::BK;
+    const int KB = a.K / S::BK, KBT = a.split ? 3 * KB : KB;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S::STAGES; ++s) {
@@ -94,21 +100,22 @@ __global__ void __launch_bounds__(128, 1)
 
     if (warp == 0 && lane == 0) {
         // producer: TMA loads of the A and W tiles of every K block
-        for (int kb = 0; kb < KB; ++kb) {
+        for (int kb = 0; kb < KBT; ++kb) {
             const int s = kb % S::STAGES, round = kb / S::STAGES;
             if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
             mbar_arrive_expect_tx(&full[s], S::STAGE);
             unsigned char* st = smem + s * S::STAGE;
-            tma_load_2d(st, &mapA, &full[s], kb * S::BK, m0);
+            const int pair = kb / KB, kx = (kb - pair * KB) * S::BK;  // split: (hi, hi), (hi, lo), (lo, hi)
+            tma_load_2d(st, pair == 2 ? &mapA2 : &mapA, &full[s], kx, m0);
 #pragma unroll
             for (int c = 0; c < BN; c += 256)
-                tma_load_2d(st + S::A_BYTES + c * 128, &mapB, &full[s], kb * S::BK, n0 + c);
+                tma_load_2d(st + S::A_BYTES + c * 128, pair == 1 ? &mapB2 : &mapB, &full[s], kx, n0 + c);
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
         constexpr int NI = BN < 256 ? BN : 256;
         const uint32_t idesc = idesc_bf16(128, NI);
-        for (int kb = 0; kb < KB; ++kb) {
+        for (int kb = 0; kb < KBT; ++kb) {
             const int s = kb % S::STAGES, round = kb / S::STAGES;
             if (!mbar_wait(&full[s], round & 1, a.err, 2)) break;
             tc_fence_after();
@@ -144,7 +151,19 @@ __global__ void __launch_bounds__(128, 1)
     const bool live = ok && r < a.R;
     const uint32_t tw = tmem + ((uint32_t)(warp * 32) << 16);
     if (ok) {
-        if (a.epi == EPI_TC_RELU) {
+        if (a.epi == EPI_TC_F32) {
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                float v[16];
+                tmem_ld16(tw + c0, v);
+                if (live) {
+                    float4* o = reinterpret_cast<float4*>(a.out_f + (size_t)r * a.N + n0 + c0);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        o[i] = make_float4(v[4 * i] + bias_s[c0 + 4 * i], v[4 * i + 1] + bias_s[c0 + 4 * i + 1],
+                                           v[4 * i + 2] + bias_s[c0 + 4 * i + 2], v[4 * i + 3] + bias_s[c0 + 4 * i + 3]);
+                }
+            }
+        } else if (a.epi == EPI_TC_RELU) {
             for (int c0 = 0; c0 < BN; c0 += 16) {
                 float v[16];
                 tmem_ld16(tw + c0, v);
@@ -369,12 +388,13 @@ bool make_tmap_bf16(CUtensorMap* map, const void* ptr, int K, int rows, int box_
 }
 
 template <int BN>
-static cudaError_t launch_bn(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, cudaStream_t st) {
+static cudaError_t launch_bn(const CUtensorMap& A, const CUtensorMap& W, const CUtensorMap& A2,
+                             const CUtensorMap& W2, const TcGemmArgs& a, cudaStream_t st) {
     const size_t sm = TcShape<BN>::SMEM;
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
     const dim3 grid(a.N / BN, (a.R + 127) / 128);
-    return launch_k(k_gemm_tc<BN>, grid, dim3(128), sm, st, A, W, a);
+    return launch_k(k_gemm_tc<BN>, grid, dim3(128), sm, st, A, W, A2, W2, a);
 }
 
 template <int BNC>
@@ -415,17 +435,24 @@ cudaError_t launch_gemm_ln_cluster(const CUtensorMap& A, const CUtensorMap& W, c
     return bnc == 32 ? launch_ln_bnc<32>(A, W, a, CL, st) : launch_ln_bnc<64>(A, W, a, CL, st);
 }
 
-cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
-                           cudaStream_t st) {
+cudaError_t launch_gemm_tc_split(const CUtensorMap& A, const CUtensorMap& A2, const CUtensorMap& W,
+                                 const CUtensorMap& W2, const TcGemmArgs& a, int BN, cudaStream_t st) {
     if (a.R <= 0) return cudaSuccess;
-    if (a.epi != EPI_TC_QKV && a.epi != EPI_TC_RELU) return cudaErrorInvalidValue;
+    if (a.epi != EPI_TC_QKV && a.epi != EPI_TC_RELU && a.epi != EPI_TC_F32) return cudaErrorInvalidValue;
+    if (a.K % 64 || a.N % BN) return cudaErrorInvalidValue;
     switch (BN) {
-        case 64: return launch_bn<64>(A, W, a, st);
-        case 128: return launch_bn<128>(A, W, a, st);
-        case 256: return launch_bn<256>(A, W, a, st);
-        case 512: return launch_bn<512>(A, W, a, st);
+        case 64: return launch_bn<64>(A, W, A2, W2, a, st);
+        case 128: return launch_bn<128>(A, W, A2, W2, a, st);
+        case 256: return launch_bn<256>(A, W, A2, W2, a, st);
+        case 512: return launch_bn<512>(A, W, A2, W2, a, st);
     }
     return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm_tc(const CUtensorMap& A, const CUtensorMap& W, const TcGemmArgs& a, int BN,
+                           cudaStream_t st) {
+    if (a.split) return cudaErrorInvalidValue;
+    return launch_gemm_tc_split(A, A, W, W, a, BN, st);
 }
 
 }  // namespace tppsd

@@ -11,10 +11,13 @@
 #include <math.h>
 #include <stdlib.h>
 
+#include <algorithm>
+
 #include <cuda_fp16.h>
 
 #include "common.cuh"
 #include "engine.h"
+#include "tc_ptx.cuh"
 
 namespace tppsd {
 
@@ -513,6 +516,150 @@ __global__ void __launch_bounds__(256) k_attention_single(AttArgs<T> a) {
 // (Sec. 4.2): w, mu, sigma logits from e1, e2, e3 and mark logits from
 // tanh(.), then the two log-softmaxes.  One warp per row; the output maps
 // (transposed, [d][3M+K]) are staged in shared memory when they fit.
+// Small maps of the heads (Sec. 4.2) over 16 rows of hd4 = [E h | V_k1 h +
+// b_k1] per CTA: out[o] = b[o] + sum_i act(o)[i] W_g[i][o], act = e_1, e_2,
+// e_3 or tanh(V_k1 h + b_k1) by the output's group g (w logits, mu, log
+// sigma, mark logits), then log-softmax of the w and the mark logits.  For
+// each group in turn thread 0 copies the group's map (d x cnt, contiguous
+// in head_out_g) and the 16 rows' inputs into shared memory by bulk copies
+// (rows padded by 4 floats: the two rows a warp reads sit in distinct
+// banks); thread t then takes row t / 16 and the group's outputs t % 16 +
+// 16 j, j < NJ, so a row's sixteen threads are consecutive lanes and its
+// log-softmax sums are four shuffles.
+constexpr int HR_ROWS = 16;
+__host__ __device__ inline size_t head_rows_smem(int d, int M, int K) {
+    return sizeof(float) * ((size_t)HR_ROWS * (d + 4) + (size_t)d * (M > K ? M : K)) + 16;
+}
+// acc[j] += sum_i xr[i] wg[i][sub + 16 j] for j < J (J <= NJ, outputs < cnt).
+template <int NJ, int J>
+__device__ __forceinline__ void head_rows_dot(float (&acc)[NJ], const float* xr, const float* wg, int d, int cnt,
+                                              int sub) {
+    if constexpr (J <= NJ) {
+#pragma unroll 4
+        for (int i = 0; i < d; ++i) {
+            const float xv = xr[i];
+            const float* wr = wg + i * cnt + sub;
+#pragma unroll
+            for (int j = 0; j < J; ++j)
+                if (sub + 16 * j < cnt) acc[j] = fmaf(wr[16 * j], xv, acc[j]);
+        }
+    }
+}
+
+template <int NJ>
+__global__ void __launch_bounds__(256) k_head_rows(DevModel m, Work w, int count) {
+    extern __shared__ __align__(16) float hsm[];
+    const int d = m.d, M = m.M, K = m.K, WO = 3 * M + K, ld = d + 4;
+    uint64_t* bar = (uint64_t*)hsm;
+    float* xs = hsm + 4;                // [16][d + 4]
+    float* wg = xs + HR_ROWS * ld;      // [d][cnt]: this group's map
+    const int r0 = blockIdx.x * HR_ROWS, rows = min(HR_ROWS, count - r0);
+    const int t = threadIdx.x, rr = t >> 4, sub = t & 15, r = r0 + rr;
+    const bool live = r < count && w.row_seq[r] >= 0;
+    float* dst = w.heads + (size_t)r * WO;
+    const float* xr = xs + rr * ld;
+    if (t == 0) {
+        mbar_init(bar, 1);
+        mbar_fence_init();
+    }
+    __syncthreads();
+    int col0 = 0;
+    bool ok = true;
+    for (int g = 0; g < 4; ++g) {
+        const int cnt = g < 3 ? M : K;
+        if (t == 0) {  // the previous group's rows and map are consumed (barrier below)
+            const uint32_t wbytes = (uint32_t)(d * cnt * 4), rbytes = (uint32_t)(d * 4);
+            mbar_arrive_expect_tx(bar, wbytes + rbytes * rows);
+            bulk_load(wg, m.head_out_g + (size_t)d * col0, wbytes, bar);
+            for (int q = 0; q < rows; ++q) bulk_load(xs + q * ld, w.hd4 + (size_t)(r0 + q) * 4 * d + g * d, rbytes, bar);
+        }
+        ok = mbar_wait(bar, g & 1, w.err, 6) && ok;
+        if (g == 3) {
+            for (int idx = t; idx < rows * d; idx += 256) {
+                const int q = idx / d, i = idx - q * d;
+                xs[q * ld + i] = tanhf(xs[q * ld + i]);
+            }
+            __syncthreads();
+        }
+        float acc[NJ];
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) acc[j] = 0.f;
+        if (rr < rows) {
+            // as many accumulators as the group needs (the mixture groups
+            // are narrower than the mark group)
+            const int nj = (cnt + 15) / 16;
+            if (nj == 1) head_rows_dot<NJ, 1>(acc, xr, wg, d, cnt, sub);
+            else if (nj == 2) head_rows_dot<NJ, 2>(acc, xr, wg, d, cnt, sub);
+            else if (nj <= 4) head_rows_dot<NJ, 4>(acc, xr, wg, d, cnt, sub);
+            else if (nj <= 8) head_rows_dot<NJ, 8>(acc, xr, wg, d, cnt, sub);
+            else if (nj <= 16) head_rows_dot<NJ, 16>(acc, xr, wg, d, cnt, sub);
+            else head_rows_dot<NJ, 32>(acc, xr, wg, d, cnt, sub);
+        }
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < NJ; ++j)
+            if (sub + 16 * j < cnt) {
+                acc[j] += m.head_out_b[col0 + sub + 16 * j];
+                mx = fmaxf(mx, acc[j]);
+            }
+        float lz = 0.f;
+        if (g == 0 || g == 3) {  // log-softmax over the row's sixteen threads
+#pragma unroll
+            for (int o = 1; o < 16; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            float sm = 0.f;
+#pragma unroll
+            for (int j = 0; j < NJ; ++j)
+                if (sub + 16 * j < cnt) sm += expf(acc[j] - mx);
+#pragma unroll
+            for (int o = 1; o < 16; o <<= 1) sm += __shfl_xor_sync(0xffffffffu, sm, o);
+            lz = mx + logf(sm);
+        }
+        if (live && ok) {
+#pragma unroll
+            for (int j = 0; j < NJ; ++j)
+                if (sub + 16 * j < cnt) dst[col0 + sub + 16 * j] = acc[j] - lz;
+        }
+        col0 += cnt;
+        __syncthreads();  // every thread is done with this group's shared data
+    }
+}
+
+static int head_rows_supported(const DevModel& m) {
+    const int mk = m.M > m.K ? m.M : m.K;
+    return m.d % 4 == 0 && mk <= 512 && head_rows_smem(m.d, m.M, m.K) <= 220 * 1024;
+}
+
+static cudaError_t launch_head_rows(const DevModel& m, const Work& w, int R, cudaStream_t st) {
+    const int mk = m.M > m.K ? m.M : m.K, nj = (mk + 15) / 16;
+    const size_t sm = head_rows_smem(m.d, m.M, m.K);
+    const dim3 grid((R + HR_ROWS - 1) / HR_ROWS);
+    auto go = [&](auto kern) {
+        if (sm > 48 * 1024) {
+            const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e != cudaSuccess) return e;
+        }
+        kern<<<grid, 256, sm, st>>>(m, w, R);
+        return cudaGetLastError();
+    };
+    if (nj <= 1) return go(k_head_rows<1>);
+    if (nj <= 2) return go(k_head_rows<2>);
+    if (nj <= 4) return go(k_head_rows<4>);
+    if (nj <= 8) return go(k_head_rows<8>);
+    if (nj <= 16) return go(k_head_rows<16>);
+    return go(k_head_rows<32>);
+}
+
+// x = hi + lo with hi = bf16(x), lo = bf16(x - hi), over n pairs of values.
+__global__ void k_split_rows(const float* __restrict__ x, bf16* hi, bf16* lo, long long n) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        const float2 v = reinterpret_cast<const float2*>(x)[i];
+        const __nv_bfloat162 h = __floats2bfloat162_rn(v.x, v.y);
+        const float2 hf = __bfloat1622float2(h);
+        reinterpret_cast<__nv_bfloat162*>(hi)[i] = h;
+        reinterpret_cast<__nv_bfloat162*>(lo)[i] = __floats2bfloat162_rn(v.x - hf.x, v.y - hf.y);
+    }
+}
+
 __global__ void __launch_bounds__(256) k_head_out(DevModel m, Work w, int count, int stage) {
     extern __shared__ float hsm[];
     const int d = m.d, M = m.M, K = m.K, WO = 3 * M + K;
@@ -1388,19 +1535,40 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         PROF_MARK(prof, KC_HEAD, 0, st);
         nl += 1;
     } else if (want_heads) {
-        // e | V_k1 h + b_k1 for all rows (fp32 tiled GEMM), then the small maps
         PROF_MARK(prof, KC_HEAD, 1, st);
-        GemmArgs<float> gh{};
-        gh.A = w.x; gh.W = m.head_ek_w; gh.bias = m.head_ek_b; gh.R = R; gh.N = 4 * d; gh.K = d;
-        gh.out_f = w.hd4;
-        k_gemm<float, EPI_F32><<<dim3((4 * d + 63) / 64, (R + 63) / 64), 256, 0, st>>>(gh);
-        const int WO = m.head_width();
-        const size_t wbytes = sizeof(float) * (size_t)d * WO;
-        const int stage = wbytes <= 96 * 1024;
-        const size_t sm = (stage ? wbytes : 0) + sizeof(float) * 8 * 4 * d;
-        if (sm > 48 * 1024) cudaFuncSetAttribute(k_head_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-        const int blocks = min((R + 7) / 8, 152 * 2);
-        k_head_out<<<blocks, 256, sm, st>>>(m, w, R, stage);
+        if (use_tc && tc->head_g) {
+            // e | V_k1 h + b_k1 on the tensor cores, fp32-accurate: h split
+            // into bf16 parts (hi over xb, lo over att; both free after the
+            // last layer), [E; V_k1] as stored in hi / lo parts
+            k_split_rows<<<(unsigned)std::min<long long>(((long long)R * d / 2 + 255) / 256, 152 * 8), 256, 0, st>>>(
+                w.x, (bf16*)w.xb, (bf16*)w.att, (long long)R * d / 2);
+            TcGemmArgs g{};
+            g.R = R; g.N = 4 * d; g.K = d; g.epi = EPI_TC_F32; g.bias = m.head_ek_b; g.out_f = w.hd4;
+            g.split = 1; g.err = tc->err;
+            const cudaError_t e =
+                launch_gemm_tc_split(tc->a_xb, tc->a_att, tc->head_hi_g, tc->head_lo_g, g, tc->bn_head, st);
+            if (e != cudaSuccess) return e;
+            nl += 1;
+        } else {
+            // e | V_k1 h + b_k1 for all rows (fp32 tiled GEMM)
+            GemmArgs<float> gh{};
+            gh.A = w.x; gh.W = m.head_ek_w; gh.bias = m.head_ek_b; gh.R = R; gh.N = 4 * d; gh.K = d;
+            gh.out_f = w.hd4;
+            k_gemm<float, EPI_F32><<<dim3((4 * d + 63) / 64, (R + 63) / 64), 256, 0, st>>>(gh);
+        }
+        // then the small maps
+        if (head_rows_supported(m) && !getenv("TPPSD_HEAD_OUT_WARP")) {
+            const cudaError_t e = launch_head_rows(m, w, R, st);
+            if (e != cudaSuccess) return e;
+        } else {
+            const int WO = m.head_width();
+            const size_t wbytes = sizeof(float) * (size_t)d * WO;
+            const int stage = wbytes <= 96 * 1024;
+            const size_t sm = (stage ? wbytes : 0) + sizeof(float) * 8 * 4 * d;
+            if (sm > 48 * 1024) cudaFuncSetAttribute(k_head_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            const int blocks = min((R + 7) / 8, 152 * 2);
+            k_head_out<<<blocks, 256, sm, st>>>(m, w, R, stage);
+        }
         PROF_MARK(prof, KC_HEAD, 0, st);
         nl += 2;
     }
