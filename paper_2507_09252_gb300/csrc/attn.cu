@@ -254,6 +254,7 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
         }
         __syncwarp();
     }
+    pdl_trigger();  // the next kernel may be scheduled while the partials are merged
     // per-warp partial results -> shared memory (over this warp's stages)
     auto mslot = [&](int w) { return (float*)(smem + w * S::WARP_BYTES); };
     float* mw = mslot(warp);

@@ -59,7 +59,11 @@ __global__ void __launch_bounds__(128, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
               const __grid_constant__ CUtensorMap mapA2, const __grid_constant__ CUtensorMap mapB2, TcGemmArgs a) {
     using S = TcShape<BN>;
-    pdl_wait();
+    // Before griddepcontrol.wait nothing reads what the previous kernel of
+    // the stream writes: barrier set-up, TMEM allocation and the weight
+    // tiles of the first stages (the weights are never written by a
+    // sampling kernel) overlap that kernel's tail; every role waits before
+    // its first dependent access (rows, row positions, outputs).
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     float* bias_s = (float*)(smem + S::STAGES * S::STAGE);
@@ -92,6 +96,7 @@ __global__ void __launch_bounds__(128, 1)
         // before anything is issued.  Nothing can complete it, so the bounded
         // wait runs out, records its code in *a.err and the CTA returns with
         // no copy or MMA in flight.
+        pdl_wait();
         if (threadIdx.x == 0) mbar_wait(done, 0, a.err, 9);
         __syncthreads();
         if (warp == 0) tmem_dealloc(tmem, S::TMEM_COLS);
@@ -99,17 +104,30 @@ __global__ void __launch_bounds__(128, 1)
     }
 
     if (warp == 0 && lane == 0) {
-        // producer: TMA loads of the A and W tiles of every K block
-        for (int kb = 0; kb < KBT; ++kb) {
-            const int s = kb % S::STAGES, round = kb / S::STAGES;
-            if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
-            mbar_arrive_expect_tx(&full[s], S::STAGE);
-            unsigned char* st = smem + s * S::STAGE;
+        // producer: TMA loads of the A and W tiles of every K block; the W
+        // tiles of the first stages go out before the wait
+        const int pre = KBT < S::STAGES ? KBT : S::STAGES;
+        auto load_w = [&](int kb, int s) {
             const int pair = kb / KB, kx = (kb - pair * KB) * S::BK;  // split: (hi, hi), (hi, lo), (lo, hi)
-            tma_load_2d(st, pair == 2 ? &mapA2 : &mapA, &full[s], kx, m0);
 #pragma unroll
             for (int c = 0; c < BN; c += 256)
-                tma_load_2d(st + S::A_BYTES + c * 128, pair == 1 ? &mapB2 : &mapB, &full[s], kx, n0 + c);
+                tma_load_2d(smem + s * S::STAGE + S::A_BYTES + c * 128, pair == 1 ? &mapB2 : &mapB, &full[s], kx,
+                            n0 + c);
+        };
+        for (int kb = 0; kb < pre; ++kb) {
+            mbar_arrive_expect_tx(&full[kb], S::STAGE);
+            load_w(kb, kb);
+        }
+        pdl_wait();
+        for (int kb = 0; kb < KBT; ++kb) {
+            const int s = kb % S::STAGES, round = kb / S::STAGES;
+            if (kb >= pre) {
+                if (!mbar_wait(&empty[s], (round & 1) ^ 1, a.err, 1)) break;
+                mbar_arrive_expect_tx(&full[s], S::STAGE);
+                load_w(kb, s);
+            }
+            const int pair = kb / KB, kx = (kb - pair * KB) * S::BK;
+            tma_load_2d(smem + s * S::STAGE, pair == 2 ? &mapA2 : &mapA, &full[s], kx, m0);
         }
     } else if (warp == 1 && lane == 0) {
         // MMA issuer
@@ -135,6 +153,7 @@ __global__ void __launch_bounds__(128, 1)
         // idle during the main loop: stage the epilogue's parameters
         const int t = threadIdx.x - 64;
         for (int c = t; c < BN; c += 64) bias_s[c] = a.bias[n0 + c];
+        pdl_wait();
         if (a.epi == EPI_TC_QKV) {
             for (int r = t; r < S::BM; r += 64) {
                 const bool in = m0 + r < a.R;
@@ -144,8 +163,12 @@ __global__ void __launch_bounds__(128, 1)
         }
     }
     __syncwarp();
+    if (warp < 2) pdl_wait();  // the epilogue writes what the previous kernel may read
     const bool ok = __syncthreads_and(mbar_wait(done, 0, a.err, 3)) != 0;  // CTA-uniform
     tc_fence_after();
+    // the next kernel may be scheduled now: its CTAs set up (and wait for
+    // this grid's completion) while the epilogues run
+    pdl_trigger();
 
     const int t = warp * 32 + lane, r = m0 + t;
     const bool live = ok && r < a.R;

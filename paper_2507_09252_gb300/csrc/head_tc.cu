@@ -42,7 +42,8 @@ __global__ void __launch_bounds__(320, 1)
               Work w, int R) {
     using S = HeadShape;
     constexpr int D = S::D;
-    pdl_wait();
+    // the weight tiles (never written by a sampling kernel) are requested
+    // before griddepcontrol.wait; the rows and outputs only after it
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint64_t* bars = (uint64_t*)(smem + S::OFF_BAR);
@@ -96,6 +97,7 @@ __global__ void __launch_bounds__(320, 1)
         }
     } else {
         const int tid = threadIdx.x;
+        pdl_wait();
         // A operands: h rows split into hi / lo bf16, written in the swizzled
         // K-major layout (16-byte chunk c of row r at chunk c ^ (r & 7)); all
         // 16 global loads of a thread are issued before the first store
@@ -155,6 +157,7 @@ __global__ void __launch_bounds__(320, 1)
         const bool live = t < rows && w.row_seq[m0 + t] >= 0;
         mbar_wait(done, 0, w.err, 53);
         tc_fence_after();
+        pdl_trigger();  // the next kernel may be scheduled while the outputs are formed
         float v[64];
         tmem_ld64(tmem + ((uint32_t)(q * 32) << 16) + 64 * hf, v);
         if (nb == 3) {

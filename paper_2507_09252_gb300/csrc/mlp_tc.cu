@@ -394,7 +394,9 @@ __global__ void __launch_bounds__(320, 1)
              const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2, MlpArgs a) {
     using S = MlpClShape;
     constexpr int D = S::D;
-    pdl_wait();
+    // griddepcontrol.wait comes after everything that reads no output of the
+    // previous kernel: barrier set-up, TMEM allocation, the weight tiles and
+    // the bias / LayerNorm parameters (never written by a sampling kernel)
     extern __shared__ unsigned char smem_raw[];
     unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* A = smem + S::OFF_A;
@@ -436,9 +438,6 @@ __global__ void __launch_bounds__(320, 1)
 
     if (warp == 8) {
         if (lane == 0) {  // every tile of this CTA at once: nothing is reused
-            mbar_arrive_expect_tx(abar, 2 * S::TILE);
-            tma_load_2d(A, &mapAtt, abar, 0, m0);
-            tma_load_2d(A + S::TILE, &mapAtt, abar, 64, m0);
             const CUtensorMap* maps[S::NT] = {&mapWo, &mapWo, &mapW1, &mapW1, &mapW2, &mapW2};
             const int xs[S::NT] = {0, 64, 0, 64, c * S::CH, c * S::CH + 64};
             const int ys[S::NT] = {0, 0, c * S::CH, c * S::CH, 0, 0};
@@ -447,6 +446,10 @@ __global__ void __launch_bounds__(320, 1)
                 tma_load_2d(Wt + i * S::TILE, maps[i], &full[i], xs[i], ys[i]);
             }
             if (NCL > 1) mbar_arrive_expect_tx(rbar, (uint32_t)(NCL - 1) * S::SLICE_BYTES(NCL));
+            pdl_wait();  // the attention rows are the previous kernel's output
+            mbar_arrive_expect_tx(abar, 2 * S::TILE);
+            tma_load_2d(A, &mapAtt, abar, 0, m0);
+            tma_load_2d(A + S::TILE, &mapAtt, abar, 64, m0);
         }
         __syncwarp();
     } else if (warp == 9) {
@@ -485,15 +488,8 @@ __global__ void __launch_bounds__(320, 1)
         // epilogue warps 0-7: row t = 32 (warp % 4) + lane, columns cb..cb+63
         const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * 64;
         const bool live = t < rows;
-        {   // residual tile and parameters; all loads issued before any store
-            constexpr int NV = S::BM * D / 4 / 256;
-            float4 v[NV];
-#pragma unroll
-            for (int k = 0; k < NV; ++k) {
-                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
-                v[k] = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
-                                : make_float4(0.f, 0.f, 0.f, 0.f);
-            }
+        {   // parameters, then (after the wait) the residual tile; all loads
+            // issued before any store
             const float* src[6] = {a.b_o, a.ln1_g, a.ln1_b, a.b_2, a.ln2_g, a.ln2_b};
             float pv[3];
 #pragma unroll
@@ -502,6 +498,15 @@ __global__ void __launch_bounds__(320, 1)
                 pv[k] = src[i / D][i % D];
             }
             const float b1v = tid < S::CH ? a.b_1[c * S::CH + tid] : 0.f;
+            pdl_wait();
+            constexpr int NV = S::BM * D / 4 / 256;
+            float4 v[NV];
+#pragma unroll
+            for (int k = 0; k < NV; ++k) {
+                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                v[k] = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
+                                : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
 #pragma unroll
             for (int k = 0; k < NV; ++k) {
                 const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
@@ -589,6 +594,7 @@ __global__ void __launch_bounds__(320, 1)
     // every partial of the cluster is in shared memory and every CTA's
     // weight region is free
     cluster_sync();
+    pdl_trigger();  // the next kernel may be scheduled while the rows are finished
     if (threadIdx.x == 0 && NCL > 1) {  // slice p of this partial -> slot c of CTA p's weight region
         for (int p = 0; p < NCL; ++p)
             if (p != c)
