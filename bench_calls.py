@@ -54,6 +54,15 @@ def _time_calls(torch, fn, flush, reps=3, warm=2):
     return tot / reps
 
 
+def _hbm_peak():
+    """Measured HBM copy bandwidth of this machine (GB/s), else the fallback."""
+    try:
+        with open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"])
+    except (OSError, KeyError, ValueError):
+        return 6800.0
+
+
 def _shape(cfg, fields):
     return " ".join(f"{n}{getattr(cfg, f)}" for n, f in fields)
 
@@ -121,6 +130,28 @@ def main(argv=None):
         ms_sd = _time_calls(torch, sd, flush)
         _, st_sd = T.tppsd_get_stats(s.ctx)
         ms_ar = _time_calls(torch, ar, flush, reps=2, warm=1)
+        # the draft kernel against HBM: one profiled call gives its time per
+        # round; its bytes are the draft K/V it reads per round (every key of
+        # the context once per encoded position when the cache is streamed,
+        # SURVEY's "streamed" bytes; once per round when it stays in shared
+        # memory), counted by the kernel (draft_keys, per layer)
+        draft = None
+        if not a.poisson:
+            T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
+            sample_call(T.TPPSD_FLAG_PROFILE)
+            torch.cuda.synchronize()
+            _, st_p = T.tppsd_get_stats(s.ctx)
+            kms, kn = T.tppsd_kernel_times(s.ctx).get("draft", (0.0, 0))
+            if kn:
+                eb = 2 if wl.draft.dtype == CF.BF16 else 4
+                dcfg = wl.draft
+                kv = st_p["draft_keys"] * dcfg.layers * 2 * dcfg.d_model * eb
+                gbs = kv / (kms / 1e3) / 1e9
+                peak = _hbm_peak()
+                draft = {"us_per_round": round(1e3 * kms / kn, 2),
+                         "kv_bytes_per_round": int(kv / kn),
+                         "achieved_GBps": round(gbs, 1), "frac_of_hbm": round(gbs / peak, 4),
+                         "peak_GBps": peak}
         layer = (("L", "layers"), ("d", "d_model"), ("h", "heads"), ("F", "d_ffn"))
         print(json.dumps({
             "workload": wl.name, "batch": B, "gamma": g, "n_events": N, "hist_len": H,
@@ -132,7 +163,8 @@ def main(argv=None):
             "speedup_vs_ar": round(ms_ar / ms_sd, 3),
             "mean_accepted_per_verify": round(st_sd["accepted"] / max(st_sd["rounds"], 1), 3),
             "alpha": round(st_sd["accepted"] / max(st_sd["drafted"], 1), 4),
-            "rounds": st_sd["loop_iters"], "note": "prefill included in both timed calls"}), flush=True)
+            "rounds": st_sd["loop_iters"], "draft_kernel": draft,
+            "note": "prefill included in both timed calls"}), flush=True)
         s.close()
         return 0
     flags = T.TPPSD_FLAG_HOST_LOOP if a.host_loop else T.TPPSD_FLAG_PROFILE

@@ -630,6 +630,16 @@ static void build_tc_plan(tppsd_ctx* ctx) {
                 make_tmap_bf16(&p.layer[l].w1_m, L.w_1, d, F, 128) &&
                 make_tmap_bf16(&p.layer[l].w2_m, L.w_2, F, d, 128);
     }
+    // TPPSD_QKV_FOLD=1: the cluster form also computes the next layer's Q,
+    // K, V (W_qkv maps with boxes of its per-CTA column count).  Off by
+    // default: with programmatic dependent launch the separate QKV GEMM is
+    // already resident and waiting when the block ends, and the fold's
+    // in-kernel row exchange measured slower (14.98 against 14.82 ms per
+    // headline call).
+    const int nq = p.mlp && p.mlp_cl ? mlp_cl_qkv_cols(d, F) : 0;
+    p.qkv_fold = nq > 0 && getenv("TPPSD_QKV_FOLD") != nullptr;
+    for (int l = 0; l < m.L && p.qkv_fold; ++l)
+        p.qkv_fold = make_tmap_bf16(&p.layer[l].wqkv_f, m.layer[l].w_qkv, d, 3 * d, nq);
     p.head = ok && head_tc_supported(m) &&
              make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
              make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);

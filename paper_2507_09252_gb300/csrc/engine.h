@@ -276,6 +276,7 @@ struct TcGemmArgs {
 struct TcLayerMaps {
     CUtensorMap wqkv, wo, w1, w2;      // boxes of the separate GEMMs
     CUtensorMap wo_m, w1_m, w2_m;      // boxes of 128 rows for the fused block
+    CUtensorMap wqkv_f;                // W_qkv with boxes of mlp_cl_qkv_cols rows (folded QKV)
 };
 // Tensor maps of one bf16 model's weights and of the row-workspace buffers it
 // reads (rows = Work.R), built once per context.
@@ -284,6 +285,7 @@ struct TcPlan {
     int bn_qkv, bn_o, bn_ffn1;  // bn_o: columns per CTA of the cluster LayerNorm GEMMs
     int mlp;                    // post-attention block by the fused kernel
     int mlp_cl;                 // ... in its cluster form (FFN split over F / 128 CTAs)
+    int qkv_fold;               // ... which also computes the next layer's Q, K, V
     int head;                   // heads by the tensor-core head kernel (d = 128)
     CUtensorMap head_hi, head_lo;
     // other widths: [E; V_k1] h by the split GEMM (A_hi = xb, A_lo = att), then
@@ -312,11 +314,22 @@ struct MlpArgs {
     float* x;             // [R][d] residual in, LN2 output out
     __nv_bfloat16* xb;    // [R][d] bf16 copy of the output
     int* err;
+    // qkv (cluster form): also the next layer's Q, K, V from the output rows,
+    // stored as the QKV GEMM's epilogue stores them
+    int qkv;
+    const float* b_qkv;   // [3d] the next layer's bias
+    __nv_bfloat16* q_out; __nv_bfloat16* kc; __nv_bfloat16* vc;
+    const int* row_seq; const int* row_pos;
+    int nh, dh, layer, Bmax, n_max, v_f16;
 };
 int mlp_tc_supported(int d, int F);
 int mlp_cl_supported(int d, int F);
+// Columns of W_qkv per CTA when the cluster form can fold the next layer's
+// QKV GEMM in (0: it cannot); the W_qkv tensor map then has boxes of that
+// many rows.
+int mlp_cl_qkv_cols(int d, int F);
 cudaError_t launch_mlp_cl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
-                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st);
+                          const CUtensorMap& w2, const CUtensorMap& wq, const MlpArgs& a, cudaStream_t st);
 // att: tensor map of the attention output rows (box 64 x 128); wo / w1 / w2:
 // weight maps with boxes of 64 x 128.
 cudaError_t launch_mlp_tc(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,

@@ -42,17 +42,6 @@ struct TcShape {
     static constexpr size_t SMEM = (size_t)STAGES * STAGE + PARAM_BYTES + 1024 + 256;
 };
 
-__device__ __forceinline__ void st_bf16x16(bf16* dst, const float (&v)[16]) {
-    uint32_t w[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
-        w[i] = *reinterpret_cast<const uint32_t*>(&p);
-    }
-    uint4* d = reinterpret_cast<uint4*>(dst);
-    d[0] = make_uint4(w[0], w[1], w[2], w[3]);
-    d[1] = make_uint4(w[4], w[5], w[6], w[7]);
-}
 
 template <int BN>
 __global__ void __launch_bounds__(128, 1)
@@ -210,21 +199,8 @@ __global__ void __launch_bounds__(128, 1)
                 } else if (s >= 0) {
                     const int h = cc / a.dh, e = cc - h * a.dh;
                     const size_t o = ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
-                    if (which == 2 && a.v_f16) {
-                        // fp16 of the bf16-rounded value (exact in the fp16 range)
-                        uint32_t w[8];
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const __half2 p2 = __floats2half2_rn(__bfloat162float(__float2bfloat16_rn(v[2 * i])),
-                                                                 __bfloat162float(__float2bfloat16_rn(v[2 * i + 1])));
-                            w[i] = *reinterpret_cast<const uint32_t*>(&p2);
-                        }
-                        uint4* d4 = reinterpret_cast<uint4*>(a.vc + o);
-                        d4[0] = make_uint4(w[0], w[1], w[2], w[3]);
-                        d4[1] = make_uint4(w[4], w[5], w[6], w[7]);
-                    } else {
-                        st_bf16x16((which == 1 ? a.kc : a.vc) + o, v);
-                    }
+                    if (which == 2 && a.v_f16) st_f16x16_of_bf16(a.vc + o, v);
+                    else st_bf16x16((which == 1 ? a.kc : a.vc) + o, v);
                 }
             }
         }

@@ -1422,21 +1422,26 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
         PROF_MARK(prof, KC_ATTENTION, 0, st);
         nl += 2;
     }
+    // the fused block of layer l computes layer l + 1's Q, K, V (folded QKV)
+    const bool fold = use_tc && tc->mlp && tc->mlp_cl && tc->qkv_fold;
     for (int l = 0; l < m.L && m.enc != 2; ++l) {
         const LayerW& L = m.layer[l];
         if (use_tc) {
             cudaError_t e;
-            TcGemmArgs g{};
-            g.R = R; g.N = 3 * d; g.K = d; g.epi = EPI_TC_QKV; g.bias = L.b_qkv;
-            g.q_out = (bf16*)q; g.kc = (bf16*)kv.k; g.vc = (bf16*)kv.v;
-            g.row_seq = w.row_seq; g.row_pos = w.row_pos;
-            g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
-            g.err = tc->err;
-            g.stall = tc->stall;
-            g.v_f16 = m.v_f16;
-            PROF_MARK(prof, KC_GEMM_QKV, 1, st);
-            if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].wqkv, g, tc->bn_qkv, st)) != cudaSuccess) return e;
-            PROF_MARK(prof, KC_GEMM_QKV, 0, st);
+            if (!(fold && l > 0)) {
+                TcGemmArgs g{};
+                g.R = R; g.N = 3 * d; g.K = d; g.epi = EPI_TC_QKV; g.bias = L.b_qkv;
+                g.q_out = (bf16*)q; g.kc = (bf16*)kv.k; g.vc = (bf16*)kv.v;
+                g.row_seq = w.row_seq; g.row_pos = w.row_pos;
+                g.d = d; g.nh = m.nh; g.dh = m.dh; g.layer = l; g.Bmax = kv.Bmax; g.n_max = kv.n_max;
+                g.err = tc->err;
+                g.stall = tc->stall;
+                g.v_f16 = m.v_f16;
+                PROF_MARK(prof, KC_GEMM_QKV, 1, st);
+                if ((e = launch_gemm_tc(tc->a_xb, tc->layer[l].wqkv, g, tc->bn_qkv, st)) != cudaSuccess) return e;
+                PROF_MARK(prof, KC_GEMM_QKV, 0, st);
+                ++nl;
+            }
             AttArgs<T> aa{};
             aa.q = q; aa.kc = (const T*)kv.k; aa.vc = (const T*)kv.v; aa.out = att;
             aa.row_seq = w.row_seq; aa.row_pos = w.row_pos; aa.count = R; aa.q_per_seq = rs.q;
@@ -1450,12 +1455,21 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
                 ma.R = R; ma.F = F; ma.b_o = L.b_o; ma.ln1_g = L.ln1_g; ma.ln1_b = L.ln1_b;
                 ma.b_1 = L.b_1; ma.b_2 = L.b_2; ma.ln2_g = L.ln2_g; ma.ln2_b = L.ln2_b;
                 ma.x = w.x; ma.xb = (bf16*)xb; ma.err = tc->err;
+                const int ln = l + 1 < m.L ? l + 1 : l;  // the layer whose Q, K, V are folded in
+                if (fold && l + 1 < m.L) {
+                    ma.qkv = 1; ma.b_qkv = m.layer[ln].b_qkv;
+                    ma.q_out = (bf16*)q; ma.kc = (bf16*)kv.k; ma.vc = (bf16*)kv.v;
+                    ma.row_seq = w.row_seq; ma.row_pos = w.row_pos;
+                    ma.nh = m.nh; ma.dh = m.dh; ma.layer = ln; ma.Bmax = kv.Bmax; ma.n_max = kv.n_max;
+                    ma.v_f16 = m.v_f16;
+                }
                 PROF_MARK(prof, KC_GEMM_FFN2, 1, st);
-                e = tc->mlp_cl ? launch_mlp_cl(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st)
+                e = tc->mlp_cl ? launch_mlp_cl(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m,
+                                               ma.qkv ? tc->layer[ln].wqkv_f : tc->layer[l].w2_m, ma, st)
                                : launch_mlp_tc(tc->a_att, tc->layer[l].wo_m, tc->layer[l].w1_m, tc->layer[l].w2_m, ma, st);
                 if (e != cudaSuccess) return e;
                 PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
-                nl += 3;
+                nl += 2;
                 continue;
             }
             TcGemmArgs go{};
@@ -1480,7 +1494,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
             e = launch_gemm_ln_cluster(tc->a_hid, tc->layer[l].w2, g2, st);
             if (e != cudaSuccess) return e;
             PROF_MARK(prof, KC_GEMM_FFN2, 0, st);
-            nl += 5;
+            nl += 4;
             continue;
         }
         GemmArgs<T> g{};

@@ -367,7 +367,17 @@ __global__ void __launch_bounds__(320, 1)
 // thus one FFN1 chunk and one FFN2 chunk instead of F / 128 of each, and
 // the weights a CTA streams drop to W_o plus 1/n of W_1 and W_2 (six tiles,
 // all in flight at once).  TMEM: 0-127 the output projection, then the
-// FFN2 partial; 128-255 the FFN1 chunk; 256-383 x1 in fp32.
+// FFN2 partial; 128-255 the FFN1 chunk; 256-383 x1 in fp32; 384.. the next
+// layer's Q, K, V slice.
+//
+// With a.qkv the block also computes the next layer's Q, K and V (the QKV
+// GEMM of the next layer folded in): CTA c writes its finished rows (bf16)
+// into the A tile at their row offset, sends that slice (one contiguous
+// 128-byte-per-row block per k-block under the 128-byte swizzle) to every
+// peer by bulk copy, and once the whole 128-row tile is in place multiplies
+// it by columns c NQ .. (c+1) NQ - 1 of W_qkv (NQ = 3d / n, prefetched at
+// start); the epilogue adds the bias, rounds to bf16 and scatters Q to the
+// row buffer and K, V into the cache, as the QKV GEMM does.
 struct MlpClShape {
     static constexpr int D = 128, BM = 128, BK = 64, CH = 128;
     static constexpr int TILE = BM * BK * 2;
@@ -380,18 +390,37 @@ struct MlpClShape {
     static constexpr int OFF_P = OFF_W + NT * TILE;        // b_o g1 be1 b_2 g2 be2 (D each), b_1 chunk
     static constexpr int OFF_RED = OFF_P + (6 * D + CH) * 4;
     static constexpr int OFF_B = OFF_RED + 4 * BM * 4;
-    static constexpr int NBAR = 14;
+    static constexpr int NBAR = 18;
     __host__ __device__ static constexpr int SLICE_BYTES(int ncl) { return (BM / ncl) * RLD * 4; }
     static_assert(NT * TILE >= BM * RLD * 4, "the partial slices fit in the weight region");
-    static constexpr size_t SMEM = (size_t)OFF_B + NBAR * 8 + 16 + 1024;
+    // next layer's W_qkv columns of this CTA: 3D / ncl rows of 128 B per k-block
+    static constexpr int OFF_Q = ((OFF_B + NBAR * 8 + 16 + 1023) / 1024) * 1024;
+    __host__ __device__ static constexpr int NQ(int ncl) { return 3 * D / ncl; }
+    __host__ __device__ static constexpr bool QKV_OK(int ncl) { return ncl == 4 || ncl == 8; }
+    static constexpr size_t SMEM = (size_t)OFF_Q + 2 * 96 * 128 + 1024;  // room for NQ <= 96
     static_assert(R_BYTES >= 2 * TILE, "the activation tile fits in the residual region");
     static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
+// 8 consecutive columns c0.. (c0 % 8 == 0) of row t of a pair of
+// 128-byte-swizzled 64-column tiles, rounded to bf16.
+__device__ __forceinline__ void st_swizzled8(unsigned char* tiles, int t, int c0, const float* v) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
+    unsigned char* row = tiles + kb * MlpShape::TILE + t * 128;
+    *reinterpret_cast<uint4*>(row + ((ch ^ (t & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 template <int NCL>
 __global__ void __launch_bounds__(320, 1)
     k_mlp_cl(const __grid_constant__ CUtensorMap mapAtt, const __grid_constant__ CUtensorMap mapWo,
-             const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2, MlpArgs a) {
+             const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2,
+             const __grid_constant__ CUtensorMap mapWq, MlpArgs a) {
     using S = MlpClShape;
     constexpr int D = S::D;
     // griddepcontrol.wait comes after everything that reads no output of the
@@ -414,7 +443,14 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t* e2_done = bars + 10;    // chunk activations written (256 arrivals)
     uint64_t* y_done = bars + 11;     // FFN2 partial in TMEM
     uint64_t* rbar = bars + 12;       // the other CTAs' partial slices landed
-    uint32_t* tslot = (uint32_t*)(bars + 13);
+    uint64_t* wqbar = bars + 13;      // next layer's W_qkv columns landed
+    uint64_t* qa_local = bars + 14;   // this CTA's rows written into the A tile (256 arrivals)
+    uint64_t* qa_remote = bars + 15;  // the other CTAs' rows landed in the A tile
+    uint64_t* q_done = bars + 16;     // next layer's Q, K, V slice in TMEM
+    uint32_t* tslot = (uint32_t*)(bars + 17);
+    unsigned char* Wq = smem + S::OFF_Q;
+    constexpr int NQ = S::NQ(NCL), RW = S::BM / NCL;
+    const bool qkv = S::QKV_OK(NCL) && a.qkv;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = (int)cluster_ctarank();
     const int m0 = blockIdx.y * S::BM, rows = min(S::BM, a.R - m0);
@@ -428,6 +464,10 @@ __global__ void __launch_bounds__(320, 1)
         mbar_init(e2_done, 256);
         mbar_init(y_done, 1);
         mbar_init(rbar, 1);
+        mbar_init(wqbar, 1);
+        mbar_init(qa_local, 256);
+        mbar_init(qa_remote, 1);
+        mbar_init(q_done, 1);
         mbar_fence_init();
     }
     if (warp == 0) tmem_alloc(tslot, 512);
@@ -446,6 +486,12 @@ __global__ void __launch_bounds__(320, 1)
                 tma_load_2d(Wt + i * S::TILE, maps[i], &full[i], xs[i], ys[i]);
             }
             if (NCL > 1) mbar_arrive_expect_tx(rbar, (uint32_t)(NCL - 1) * S::SLICE_BYTES(NCL));
+            if (qkv) {
+                mbar_arrive_expect_tx(wqbar, 2 * NQ * 128);
+                tma_load_2d(Wq, &mapWq, wqbar, 0, c * NQ);
+                tma_load_2d(Wq + NQ * 128, &mapWq, wqbar, 64, c * NQ);
+                mbar_arrive_expect_tx(qa_remote, (uint32_t)(NCL - 1) * 2 * RW * 128);
+            }
             pdl_wait();  // the attention rows are the previous kernel's output
             mbar_arrive_expect_tx(abar, 2 * S::TILE);
             tma_load_2d(A, &mapAtt, abar, 0, m0);
@@ -643,6 +689,16 @@ __global__ void __launch_bounds__(320, 1)
 #pragma unroll
         for (int o = TPR >> 1; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
         const float inv = 1.0f / sqrtf(sq / D + LN_EPS);
+        if (qkv) {  // this row slice of the next layer's A tile (zeros past the rows)
+            float o[CPT];
+#pragma unroll
+            for (int j = 0; j < CPT; ++j)
+                o[j] = r < rows ? (v[j] - mean) * inv * p_g2[col + j] + p_be2[col + j] : 0.f;
+            if constexpr (CPT == 16) st_swizzled16(A, r, col, o);
+            else if constexpr (CPT == 8) st_swizzled8(A, r, col, o);
+            fence_proxy_async_smem();
+            mbar_arrive(qa_local);
+        }
         if (r < rows) {
             float* xo = a.x + (size_t)(m0 + r) * D + col;
             bf16* xbo = a.xb + (size_t)(m0 + r) * D + col;
@@ -663,9 +719,63 @@ __global__ void __launch_bounds__(320, 1)
             }
         }
     }
+    if (qkv) {
+        if (threadIdx.x == 0) {  // this CTA's finished rows -> the same rows of every peer's A tile
+            mbar_wait(qa_local, 0, a.err, 69);
+            for (int p = 0; p < NCL; ++p)
+                if (p != c)
+                    for (int kb = 0; kb < 2; ++kb) {
+                        unsigned char* blk = A + kb * S::TILE + c * RW * 128;
+                        bulk_s2peer(blk, blk, (uint32_t)(RW * 128), qa_remote, (uint32_t)p);
+                    }
+            bulk_commit();
+        } else if (warp == 9 && lane == 0) {
+            bool ok = mbar_wait(wqbar, 0, a.err, 70);
+            ok = ok && mbar_wait(qa_local, 0, a.err, 71);
+            ok = ok && mbar_wait(qa_remote, 0, a.err, 72);
+            tc_fence_after();
+            if (ok) {
+                const uint32_t idesc = idesc_bf16(128, NQ), a0 = smem_u32(A), q0 = smem_u32(Wq);
+                for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+                    for (int kk = 0; kk < S::BK / 16; ++kk)
+                        tc_mma_bf16(tmem + 384, sw128_desc(a0 + kb * S::TILE + kk * 32),
+                                    sw128_desc(q0 + kb * NQ * 128 + kk * 32), idesc, (kb | kk) ? 1u : 0u);
+            }
+            tc_commit(q_done);
+        }
+        __syncwarp();
+        if (warp < 8) {
+            // rows t = 32 (warp % 4) + lane; the column halves of the slice by
+            // warps 0-3 / 4-7 when they split into 16-column groups
+            constexpr int HALF = (NQ / 2) % 16 == 0 ? NQ / 2 : NQ;
+            const int q = warp & 3, hh = warp >> 2, t = q * 32 + lane, r = m0 + t;
+            const bool ok = mbar_wait(q_done, 0, a.err, 73);
+            tc_fence_after();
+            const bool mine = HALF == NQ ? hh == 0 : true;
+            const int s = t < rows ? a.row_seq[r] : -1, pos = t < rows ? a.row_pos[r] : 0;
+            const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16) + 384;
+            for (int c0 = hh * HALF; mine && c0 < hh * HALF + HALF; c0 += 16) {
+                float v[16];
+                tmem_ld16(tl + c0, v);
+                if (!ok || t >= rows) continue;
+                const int col = c * NQ + c0, which = col / D, cc = col - which * D;
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[i] += a.b_qkv[col + i];
+                if (which == 0) {
+                    st_bf16x16(a.q_out + (size_t)r * D + cc, v);
+                } else if (s >= 0) {
+                    const int h = cc / a.dh, e = cc - h * a.dh;
+                    const size_t o = ((((size_t)a.layer * a.Bmax + s) * a.nh + h) * (size_t)a.n_max + pos) * a.dh + e;
+                    if (which == 2 && a.v_f16) st_f16x16_of_bf16(a.vc + o, v);
+                    else st_bf16x16((which == 1 ? a.kc : a.vc) + o, v);
+                }
+            }
+        }
+    }
     // the sources of this CTA's bulk copies have been read before it exits;
-    // its own slots were all filled (rbar) before the sums above
-    if (threadIdx.x == 0 && NCL > 1) bulk_wait_read_all();
+    // its own slots were all filled (rbar, qa_remote) before they were read
+    if (threadIdx.x == 0 && (NCL > 1 || qkv)) bulk_wait_read_all();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tmem, 512);
@@ -679,7 +789,7 @@ int mlp_cl_supported(int d, int F) {
 
 template <int NCL>
 static cudaError_t launch_mlp_ncl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
-                                  const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st) {
+                                  const CUtensorMap& w2, const CUtensorMap& wq, const MlpArgs& a, cudaStream_t st) {
     const size_t sm = MlpClShape::SMEM;
     cudaError_t e = cudaFuncSetAttribute(k_mlp_cl<NCL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
@@ -698,18 +808,25 @@ static cudaError_t launch_mlp_ncl(const CUtensorMap& att, const CUtensorMap& wo,
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = at;
     cfg.numAttrs = g_pdl ? 2 : 1;
-    return cudaLaunchKernelEx(&cfg, k_mlp_cl<NCL>, att, wo, w1, w2, a);
+    return cudaLaunchKernelEx(&cfg, k_mlp_cl<NCL>, att, wo, w1, w2, wq, a);
+}
+
+int mlp_cl_qkv_cols(int d, int F) {
+    if (!mlp_cl_supported(d, F)) return 0;
+    const int n = F / MlpClShape::CH;
+    return MlpClShape::QKV_OK(n) ? MlpClShape::NQ(n) : 0;
 }
 
 cudaError_t launch_mlp_cl(const CUtensorMap& att, const CUtensorMap& wo, const CUtensorMap& w1,
-                          const CUtensorMap& w2, const MlpArgs& a, cudaStream_t st) {
+                          const CUtensorMap& w2, const CUtensorMap& wq, const MlpArgs& a, cudaStream_t st) {
     if (a.R <= 0) return cudaSuccess;
     if (!mlp_cl_supported(MlpClShape::D, a.F)) return cudaErrorInvalidValue;
+    if (a.qkv && !mlp_cl_qkv_cols(MlpClShape::D, a.F)) return cudaErrorInvalidValue;
     switch (a.F / MlpClShape::CH) {
-        case 1: return launch_mlp_ncl<1>(att, wo, w1, w2, a, st);
-        case 2: return launch_mlp_ncl<2>(att, wo, w1, w2, a, st);
-        case 4: return launch_mlp_ncl<4>(att, wo, w1, w2, a, st);
-        case 8: return launch_mlp_ncl<8>(att, wo, w1, w2, a, st);
+        case 1: return launch_mlp_ncl<1>(att, wo, w1, w2, wq, a, st);
+        case 2: return launch_mlp_ncl<2>(att, wo, w1, w2, wq, a, st);
+        case 4: return launch_mlp_ncl<4>(att, wo, w1, w2, wq, a, st);
+        case 8: return launch_mlp_ncl<8>(att, wo, w1, w2, wq, a, st);
     }
     return cudaErrorInvalidValue;
 }

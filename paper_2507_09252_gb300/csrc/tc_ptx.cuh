@@ -5,6 +5,8 @@
 // kernel can stop, release its TMEM and return instead of hanging.
 #pragma once
 #include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -188,6 +190,33 @@ __device__ __forceinline__ void tmem_st64(uint32_t taddr, const float* v) {
           "r"(__float_as_uint(v[56])), "r"(__float_as_uint(v[57])), "r"(__float_as_uint(v[58])), "r"(__float_as_uint(v[59])),
           "r"(__float_as_uint(v[60])), "r"(__float_as_uint(v[61])), "r"(__float_as_uint(v[62])), "r"(__float_as_uint(v[63]))
         : "memory");
+}
+
+// 16 consecutive values rounded to bf16 (32 bytes, 16-byte aligned dst).
+__device__ __forceinline__ void st_bf16x16(__nv_bfloat16* dst, const float (&v)[16]) {
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const __nv_bfloat162 p = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+        w[i] = *reinterpret_cast<const uint32_t*>(&p);
+    }
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    d[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+// The same values rounded to bf16 and stored as fp16 (exact in the fp16
+// range): the fp16 V cache of the tensor-core attention.
+__device__ __forceinline__ void st_f16x16_of_bf16(__nv_bfloat16* dst, const float (&v)[16]) {
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        const __half2 p2 = __floats2half2_rn(__bfloat162float(__float2bfloat16_rn(v[2 * i])),
+                                             __bfloat162float(__float2bfloat16_rn(v[2 * i + 1])));
+        w[i] = *reinterpret_cast<const uint32_t*>(&p2);
+    }
+    uint4* d = reinterpret_cast<uint4*>(dst);
+    d[0] = make_uint4(w[0], w[1], w[2], w[3]);
+    d[1] = make_uint4(w[4], w[5], w[6], w[7]);
 }
 
 // ---------------------------------------------------------------- clusters

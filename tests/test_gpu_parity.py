@@ -261,6 +261,30 @@ def test_sequence_parity_bf16_prefix():
     assert ident >= 3
 
 
+def test_folded_qkv_is_bit_identical(monkeypatch):
+    """TPPSD_QKV_FOLD=1: the fused post-attention block of layer l also
+    computes layer l + 1's Q, K and V (the rows it finishes exchanged
+    inside the cluster).  The products, the bias add and the bf16 rounding
+    are those of the separate QKV GEMM, so sampled sequences are
+    bit-identical to the default path at the headline target shape."""
+    wl = CF.C2
+    bt, bd, tau, mk = IN.workload_inputs(wl.with_(batch=12, hist_len=40))
+    def run():
+        s = G.make_sampler(wl.target, wl.draft, bt, bd, 12, 40 + 48 + wl.gamma + 4, wl.gamma)
+        s.prefill(tau, mk)
+        out = G.to_np(s.sample(48, wl.gamma, 5))
+        st, stats = s.stats()
+        s.close()
+        return out, st, stats
+    base, st0, stats0 = run()
+    monkeypatch.setenv("TPPSD_QKV_FOLD", "1")
+    fold, st1, stats1 = run()
+    assert st0 == T.TPPSD_OK and st1 == T.TPPSD_OK
+    for k in ("tau", "t", "k"):
+        assert np.array_equal(base[k], fold[k]), k
+    assert stats0["kernel_launches"] > stats1["kernel_launches"]
+
+
 def test_identical_draft_gives_autoregressive_output():
     tcfg, _, bt, _ = G.small_models(gain=1.5)
     tau, mk = G.hist(8, 5, 3, 1)
