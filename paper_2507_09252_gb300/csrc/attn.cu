@@ -3,8 +3,10 @@
 //
 // CTA = (up to 16 query rows of one sequence, one head), four warps.  The
 // K and V of one (sequence, layer, head) are contiguous [position][d_head]
-// in HBM, so every key tile is one bulk copy (cp.async.bulk) into the
-// warp's own double-buffered shared stage, completing on an mbarrier.  The
+// in HBM, so every key tile is one copy into the warp's own double-buffered
+// shared stage, completing on an mbarrier: a TMA tensor-map box with the
+// row-width swizzle for d_head >= 32 (conflict-free ldmatrix over
+// consecutive keys), a linear bulk copy (cp.async.bulk) for d_head 16.  The
 // keys 0..maxpos are cut into four contiguous ranges of equal length (a
 // multiple of 8 keys), one per warp, so all four warps work even when the
 // context is a single tile; each warp keeps its own online-softmax state
@@ -32,13 +34,31 @@ struct AttnShape {
     static constexpr int KT = TB / (2 * DH) < 16 ? 16 : TB / (2 * DH);
     static constexpr int TILE_BYTES = KT * DH * 2;
     static constexpr int STAGE_BYTES = 2 * TILE_BYTES;
-    static constexpr int WARP_BYTES = 2 * STAGE_BYTES + 32;  // two stages + two mbarriers
+    // warp w's two stages at (2w + s) STAGE_BYTES from a 1024-byte aligned
+    // base (the swizzle pattern of a tile repeats within 1 KB), then the
+    // eight mbarriers and the row positions
+    static constexpr int WARP_BYTES = 2 * STAGE_BYTES;
+    static constexpr int OFF_BAR = 4 * WARP_BYTES;
     // a warp's partial result (max, sum, 16 x DH numerators), written over
     // its own stages once its last tile is consumed
     static constexpr int MERGE_FLOATS = 16 * DH + 32;
     static_assert(MERGE_FLOATS * 4 <= 2 * STAGE_BYTES, "partial result must fit the warp's stages");
-    static constexpr int SMEM = 4 * WARP_BYTES + 16 * 4 + 64;
+    static_assert(TILE_BYTES % 1024 == 0 || DH < 32, "swizzled tiles start on 1 KB boundaries");
+    static constexpr int SMEM = OFF_BAR + 64 + 16 * 4 + 1024;
+    // d_head >= 32: tiles by TMA tensor maps with the row-width swizzle (32,
+    // 64 or 128 bytes, 16-byte chunk c of row r at c ^ ((r * rowb) >> 7)),
+    // so ldmatrix phases over consecutive keys meet no bank conflicts;
+    // d_head = 16 keeps linear bulk copies
+    static constexpr bool TMA = DH >= 32;
 };
+
+// Byte offset of 16-byte chunk c of row r of a tile of DH-wide bf16 rows
+// as the tensor map's swizzle lays it out (linear when not swizzled).
+template <int DH, bool SWZ>
+__device__ __forceinline__ uint32_t tile_off(int r, int c) {
+    constexpr int ROWB = DH * 2, MASK = ROWB == 128 ? 7 : ROWB == 64 ? 3 : 1;
+    return SWZ ? (uint32_t)(r * ROWB + ((c ^ (((r * ROWB) >> 7) & MASK)) << 4)) : (uint32_t)(r * ROWB + (c << 4));
+}
 
 __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
     asm volatile(
@@ -71,11 +91,14 @@ __device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& hi, uin
 // TB = 1024: small footprint, seven CTAs per SM (d_head <= 32); TB = 2048:
 // fewer tiles per key range, four CTAs per SM.
 template <int DH, int TB>
-__global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_mma(AttArgs<bf16> a, int* err) {
+__global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7)
+    k_attn_mma(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap, AttArgs<bf16> a,
+               int* err) {
     using S = AttnShape<DH, TB>;
     constexpr int KT = S::KT, NT = KT / 8, KS = DH / 16;
     pdl_wait();
-    extern __shared__ __align__(128) unsigned char smem[];
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    unsigned char* smem = (unsigned char*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane >> 2, t4 = lane & 3;
     const int h = blockIdx.y;
@@ -90,23 +113,29 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
     if (s < 0) return;  // rows of one sequence are all active or all inactive
     const int nq = re - rb;
     unsigned char* wbase = smem + warp * S::WARP_BYTES;
-    uint64_t* bars = (uint64_t*)(wbase + 2 * S::STAGE_BYTES);
-    int* qpos = (int*)(smem + 4 * S::WARP_BYTES);
+    uint64_t* bars = (uint64_t*)(smem + S::OFF_BAR) + 2 * warp;
+    int* qpos = (int*)(smem + S::OFF_BAR + 64);
     // this warp's key range [klo, khi)
     const int nkeys = maxpos + 1;
     const int share = (((nkeys + 3) / 4) + 7) & ~7;
     const int klo = min(nkeys, warp * share), khi = min(nkeys, klo + share);
     const int ntl = (khi - klo + KT - 1) / KT;
-    const size_t base = ((((size_t)a.layer * a.kv.Bmax + s) * a.nh + h) * (size_t)a.kv.n_max) * DH;
-    const bf16* kg = a.kc + base;
-    const bf16* vg = a.vc + base;
+    const long long yrow = (((long long)a.layer * a.kv.Bmax + s) * a.nh + h) * a.kv.n_max;  // tensor-map row of key 0
+    const bf16* kg = a.kc + (size_t)yrow * DH;
+    const bf16* vg = a.vc + (size_t)yrow * DH;
     auto issue = [&](int tile, int stage) {
         const int k0 = klo + tile * KT, cnt = min(KT, khi - k0);
-        const uint32_t bytes = (uint32_t)cnt * DH * 2;
         unsigned char* st = wbase + stage * S::STAGE_BYTES;
-        mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
-        bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
-        bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
+        if constexpr (S::TMA) {  // whole boxes: keys past the range are masked, V rows zeroed
+            mbar_arrive_expect_tx(&bars[stage], 2 * S::TILE_BYTES);
+            tma_load_2d(st, &kmap, &bars[stage], 0, (int)(yrow + k0));
+            tma_load_2d(st + S::TILE_BYTES, &vmap, &bars[stage], 0, (int)(yrow + k0));
+        } else {
+            const uint32_t bytes = (uint32_t)cnt * DH * 2;
+            mbar_arrive_expect_tx(&bars[stage], 2 * bytes);
+            bulk_load(st, kg + (size_t)k0 * DH, bytes, &bars[stage]);
+            bulk_load(st + S::TILE_BYTES, vg + (size_t)k0 * DH, bytes, &bars[stage]);
+        }
     };
     // the first tile's copy is in flight before anything else is loaded
     if (lane == 0) {
@@ -150,9 +179,10 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
         const bf16* ks = (const bf16*)st;
         const bf16* vs = (const bf16*)(st + S::TILE_BYTES);
         const int k0 = klo + it * KT, cnt = min(KT, khi - k0);
-        if (cnt < KT) {  // V rows past the copied keys -> 0 (their P is 0, and 0 * NaN bits is NaN)
+        if (cnt < KT) {  // V rows past the range -> 0 (their P is 0, and 0 * NaN bits is NaN)
             for (int i = cnt * DH / 8 + lane; i < KT * DH / 8; i += 32)
                 reinterpret_cast<uint4*>(const_cast<bf16*>(vs))[i] = make_uint4(0, 0, 0, 0);
+            fence_proxy_async_smem();  // before the stage is refilled by the async proxy
             __syncwarp();
         }
         // S = Q K^T for KT keys; K fragments by ldmatrix (8 keys x 8 dims a
@@ -165,13 +195,13 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
 #pragma unroll
             for (int k = 0; k + 1 < KS; k += 2) {  // two k-steps (32 dims) per x4
                 uint32_t b[4];
-                ldsm_x4(b, kbase + (uint32_t)((8 * n + (lane & 7)) * DH + 16 * k + 8 * (lane >> 3)) * 2);
+                ldsm_x4(b, kbase + tile_off<DH, S::TMA>(8 * n + (lane & 7), 2 * k + (lane >> 3)));
                 mma_bf16(sc[n], qa[k], b[0], b[1]);
                 mma_bf16(sc[n], qa[k + 1], b[2], b[3]);
             }
             if constexpr (KS % 2) {
                 uint32_t b[2];
-                ldsm_x2(b, kbase + (uint32_t)((8 * n + (lane & 7)) * DH + 16 * (KS - 1) + 8 * ((lane >> 3) & 1)) * 2);
+                ldsm_x2(b, kbase + tile_off<DH, S::TMA>(8 * n + (lane & 7), 2 * (KS - 1) + ((lane >> 3) & 1)));
                 mma_bf16(sc[n], qa[KS - 1], b[0], b[1]);
             }
         }
@@ -245,7 +275,7 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
                 const int key = 16 * kk + (lane & 15);
                 const int col = 8 * n + (lane >> 4) * 8;
                 uint32_t vb[4];
-                ldsm_x4_trans(vb, vbase + (uint32_t)(key * DH + col) * 2);
+                ldsm_x4_trans(vb, vbase + tile_off<DH, S::TMA>(key, col >> 3));
                 mma_bf16(o[n], ph, vb[0], vb[1]);
                 mma_bf16(o[n], pl, vb[0], vb[1]);
                 mma_bf16(o[n + 1], ph, vb[2], vb[3]);
@@ -299,9 +329,17 @@ __global__ void __launch_bounds__(128, (DH >= 64 || TB > 1024) ? 4 : 7) k_attn_m
 
 template <int DH, int TB>
 static cudaError_t launch_attn_t(const AttArgs<bf16>& a, dim3 grid, int* err, cudaStream_t st) {
-    const int sm = AttnShape<DH, TB>::SMEM;
+    using S = AttnShape<DH, TB>;
+    const int sm = S::SMEM;
     cudaFuncSetAttribute(k_attn_mma<DH, TB>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm);
-    return launch_k(k_attn_mma<DH, TB>, grid, dim3(128), sm, st, a, err);
+    CUtensorMap mk{}, mv{};
+    if (S::TMA) {
+        // the caches of layers 0..layer as [(layer, sequence, head, position)][d_head]
+        const long long items = (long long)(a.layer + 1) * a.kv.Bmax * a.nh;
+        if (!kv_tile_map(&mk, a.kc, DH, a.kv.n_max, items, S::KT) || !kv_tile_map(&mv, a.vc, DH, a.kv.n_max, items, S::KT))
+            return cudaErrorInvalidValue;
+    }
+    return launch_k(k_attn_mma<DH, TB>, grid, dim3(128), sm, st, mk, mv, a, err);
 }
 
 cudaError_t launch_attn_mma(const AttArgs<bf16>& a, int dh, int nh, int nseg, int* err, cudaStream_t st) {

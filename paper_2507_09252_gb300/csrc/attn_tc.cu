@@ -622,18 +622,19 @@ static CUtensorMapSwizzle swz_enum(int rowb) {
     return rowb == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : rowb == 64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B;
 }
 
-// KV cache [items * n_max rows][dh] as a 2-D map, boxes of 128 rows.
-static bool kv_map(CUtensorMap* m, const void* base, int dh, int n_max, long long items,
-                   CUtensorMapDataType dt = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
+// KV cache [items * n_max rows][dh] as a 2-D map, boxes of box_rows rows,
+// swizzled by the row width (32, 64 or 128 bytes).
+bool kv_tile_map(CUtensorMap* m, const void* base, int dh, int n_max, long long items, int box_rows, int f16) {
     auto enc = tmap_encoder();
     if (!enc || ((uintptr_t)base & 15) || items * n_max >= (1LL << 31)) return false;
+    if (!(dh == 16 || dh == 32 || dh == 64) || box_rows < 1 || box_rows > 256) return false;
     cuuint64_t dims[2] = {(cuuint64_t)dh, (cuuint64_t)(items * n_max)};
     cuuint64_t strides[1] = {(cuuint64_t)dh * 2};
-    cuuint32_t box[2] = {(cuuint32_t)dh, 128};
+    cuuint32_t box[2] = {(cuuint32_t)dh, (cuuint32_t)box_rows};
     cuuint32_t estr[2] = {1, 1};
-    return enc(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, swz_enum(dh * 2), CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    return enc(m, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base),
+               dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz_enum(dh * 2),
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Q rows [R][d] as a 2-D map, boxes of nq rows x dh columns.
@@ -690,7 +691,7 @@ cudaError_t launch_attn_tc(const AttArgs<bf16>& aa, int dh, int nh, int nseg, bo
     const long long items = (long long)qblocks * nh * nseg;
     const long long kv_items = (long long)(aa.layer + 1) * aa.kv.Bmax * nh;  // items up to this layer
     CUtensorMap mk, mv, mq;
-    if (!kv_map(&mk, aa.kc, dh, aa.kv.n_max, kv_items) || !kv_map(&mv, aa.vc, dh, aa.kv.n_max, kv_items, CU_TENSOR_MAP_DATA_TYPE_FLOAT16) ||
+    if (!kv_tile_map(&mk, aa.kc, dh, aa.kv.n_max, kv_items, 128) || !kv_tile_map(&mv, aa.vc, dh, aa.kv.n_max, kv_items, 128, 1) ||
         !q_map(&mq, aa.q, aa.d, aa.count, dh, NQ))
         return cudaErrorInvalidValue;
     AttTcArgs a{};

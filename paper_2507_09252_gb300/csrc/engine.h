@@ -222,6 +222,9 @@ struct AttArgs {
     float* x;
     T* hb;
 };
+// KV cache [items * n_max rows][dh] (bf16, or fp16 with f16) as a 2-D
+// tensor map with boxes of box_rows rows, swizzled by the row width.
+bool kv_tile_map(CUtensorMap* m, const void* base, int dh, int n_max, long long items, int box_rows, int f16 = 0);
 cudaError_t launch_attn_mma(const AttArgs<__nv_bfloat16>& a, int dh, int nh, int nseg, int* err,
                             cudaStream_t st);
 
