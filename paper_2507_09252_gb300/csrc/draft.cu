@@ -883,32 +883,36 @@ __device__ __forceinline__ float lane_ln(float v, int lane, float inv_d, int d, 
     return live ? c * inv * g[lane] + b[lane] : 0.f;
 }
 
-// Log-softmax of v[0..n) (shared, n <= NMAX) in place by one thread, and
-// the smallest index whose running sum of probabilities reaches u * total
-// (the same rule as warp_logsoftmax_pick, summed in index order).
+// Log-softmax of v[0..n) (shared, n <= NMAX) in place, and the smallest
+// index whose running sum of probabilities reaches u * total, with every
+// sum taken in index order (the same rule as warp_logsoftmax_pick, whose
+// scans sum in tree order).  By a whole warp: lane i < n evaluates the
+// exponentials of value i, and every lane forms the ordered sums itself
+// from shuffled copies, so all lanes hold the same sums and the same pick.
+// Ends with __syncwarp.
 template <int NMAX>
-__device__ __forceinline__ int serial_logsoftmax_pick(float* v, int n, float u) {
-    float x[NMAX], p[NMAX];
+__device__ __forceinline__ int lane_logsoftmax_pick(float* v, int n, float u) {
+    const int lane = threadIdx.x & 31;
+    const float xi = lane < n ? v[lane] : -INFINITY;
     float mx = -INFINITY;
 #pragma unroll
-    for (int i = 0; i < NMAX; ++i) {
-        x[i] = i < n ? v[i] : -INFINITY;
-        mx = fmaxf(mx, x[i]);
-    }
+    for (int i = 0; i < NMAX; ++i) mx = fmaxf(mx, __shfl_sync(FULL, xi, i));
+    const float ei = lane < n ? expf(xi - mx) : 0.f;
     float sm = 0.f;
 #pragma unroll
-    for (int i = 0; i < NMAX; ++i) sm += i < n ? expf(x[i] - mx) : 0.f;
+    for (int i = 0; i < NMAX; ++i) sm += __shfl_sync(FULL, ei, i);
     const float lz = mx + logf(sm);
-    float tot = 0.f;
+    float pi = 0.f;
+    if (lane < n) {
+        const float xn = xi - lz;
+        v[lane] = xn;
+        pi = expf(xn);
+    }
+    float pr[NMAX], tot = 0.f;
 #pragma unroll
     for (int i = 0; i < NMAX; ++i) {
-        p[i] = 0.f;
-        if (i < n) {
-            x[i] -= lz;
-            v[i] = x[i];
-            p[i] = expf(x[i]);
-        }
-        tot += p[i];
+        pr[i] = __shfl_sync(FULL, pi, i);
+        tot += pr[i];
     }
     const float target = u * tot;
     float run = 0.f;
@@ -916,12 +920,13 @@ __device__ __forceinline__ int serial_logsoftmax_pick(float* v, int n, float u) 
     bool found = false;
 #pragma unroll
     for (int i = 0; i < NMAX; ++i) {
-        run += p[i];
+        run += pr[i];
         if (!found && i < n && run >= target) {
             pick = i;
             found = true;
         }
     }
+    __syncwarp();
     return pick;
 }
 
@@ -1125,7 +1130,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                 __syncwarp();
                 int z;
                 if (M <= 8) {
-                    z = lane == 0 ? serial_logsoftmax_pick<8>(hd, M, v_rng[2 * l]) : 0;
+                    z = lane_logsoftmax_pick<8>(hd, M, v_rng[2 * l]);
                 } else {
                     z = warp_logsoftmax_pick<2>(hd, M, v_rng[2 * l]);
                 }
@@ -1150,7 +1155,7 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                 __syncwarp();
                 int k;
                 if (K <= 8) {
-                    k = lane == 0 ? serial_logsoftmax_pick<8>(hd + 3 * M, K, v_rng[2 * l]) : 0;
+                    k = lane_logsoftmax_pick<8>(hd + 3 * M, K, v_rng[2 * l]);
                 } else {
                     k = warp_logsoftmax_pick<8>(hd + 3 * M, K, v_rng[2 * l]);
                 }
