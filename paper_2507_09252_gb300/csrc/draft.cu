@@ -28,11 +28,17 @@ namespace tppsd {
 
 constexpr unsigned FULL = 0xffffffffu;
 
-// Barrier of the 128 threads that work on one sequence (named barrier 1 or
-// 2: a CTA holds one or two such teams).
+// Barrier of the NT threads that work on one sequence: 128-thread teams use
+// named barrier 1 or 2 (a CTA holds one or two such teams), a 256-thread
+// team named barrier 1.
+template <int NT = 128>
 __device__ __forceinline__ void team_sync() {
-    if (threadIdx.x < 128) asm volatile("bar.sync 1, 128;" ::: "memory");
-    else asm volatile("bar.sync 2, 128;" ::: "memory");
+    if constexpr (NT == 256) {
+        asm volatile("bar.sync 1, 256;" ::: "memory");
+    } else {
+        if (threadIdx.x < 128) asm volatile("bar.sync 1, 128;" ::: "memory");
+        else asm volatile("bar.sync 2, 128;" ::: "memory");
+    }
 }
 
 struct DraftTeamArgs {
@@ -90,27 +96,12 @@ __device__ __forceinline__ float dot_range(const TW* __restrict__ WT, int OUT, i
     for (; i < i1; ++i, w += OUT) a0 = fmaf(St<TW>::ld(w), xs[i], a0);
     return (a0 + a1) + (a2 + a3);
 }
-template <typename TW>
-__device__ __forceinline__ float dot_col(const TW* __restrict__ WT, int OUT, int o, const float* xs, int IN) {
-    return dot_range<TW>(WT, OUT, o, xs, 0, IN);
-}
-
-// Partial sums of a product with few outputs: thread t takes output
-// ob + t % OP over input slice t / OP of 128 / OP; part[t] receives its sum.
-// Ends with a block barrier; the caller reduces part[g * OP + j] over g.
-template <typename TW>
-__device__ __forceinline__ void split_partials(const TW* __restrict__ WT, int OUT, int ob, const float* xs,
-                                               int IN, int OP, float* part) {
-    const int t = threadIdx.x & 127, G = 128 / OP, o = ob + t % OP, g = t / OP;
-    const int per = (IN + G - 1) / G, i0 = g * per, i1 = min(IN, i0 + per);
-    part[t] = o < OUT ? dot_range<TW>(WT, OUT, o, xs, i0, i1) : 0.f;
-    team_sync();
-}
 
 // Floats of the partial-sum buffer of team_gemv for a model of width d and
-// FFN width F: G * OUT <= max(128 * 8, OUT) for every product of the step.
-__host__ __device__ inline int team_gp_floats(int d, int F) {
-    int g = 1024;
+// FFN width F and a team of NT threads: G * OUT <= max(NT * 8, OUT) for
+// every product of the step.
+__host__ __device__ inline int team_gp_floats(int d, int F, int NT = 128) {
+    int g = 8 * NT;
     if (4 * d > g) g = 4 * d;
     if (F > g) g = F;
     return g;
@@ -158,14 +149,14 @@ __device__ __forceinline__ void gemv_slice(const TW* __restrict__ col, int OUT, 
 // slice under 8 inputs; all groups per thread, G = 1, once NC >= 128).
 // part[g * OUT + o] receives slice g's sum of output o (OUT = OUT1 + OUT2).
 // Returns G; ends with a team barrier.
-template <typename TW>
+template <typename TW, int NT = 128>
 __device__ __forceinline__ int team_gemv(const TW* __restrict__ W1, int OUT1, const TW* __restrict__ W2, int OUT2,
                                          const float* in, int IN, float* part) {
     constexpr int V = 16 / sizeof(TW);
-    const int t = threadIdx.x & 127, OUT = OUT1 + OUT2, NC = OUT / V;
-    const int G = NC >= 128 ? 1 : max(1, min(128 / NC, IN / 8));
+    const int t = threadIdx.x & (NT - 1), OUT = OUT1 + OUT2, NC = OUT / V;
+    const int G = NC >= NT ? 1 : max(1, min(NT / NC, IN / 8));
     const int per = (IN + G - 1) / G;
-    for (int c = t; c < NC * G; c += 128) {
+    for (int c = t; c < NC * G; c += NT) {
         const int cg = c % NC, g = c / NC, o = cg * V;
         const int i0 = g * per, i1 = min(IN, i0 + per);
         float acc[V];
@@ -177,7 +168,7 @@ __device__ __forceinline__ int team_gemv(const TW* __restrict__ W1, int OUT1, co
 #pragma unroll
         for (int v = 0; v < V; v += 4) dst[v / 4] = make_float4(acc[v], acc[v + 1], acc[v + 2], acc[v + 3]);
     }
-    team_sync();
+    team_sync<NT>();
     return G;
 }
 
@@ -241,10 +232,10 @@ struct AttState {
 // (shared memory), into out[nh * DH].  Softmax: the output is rounded to
 // the storage type.  attnhp (App. D.4): the normaliser is 1 + sum_j f_j (an
 // extra term exp(0)) and the fp32 output is kept.  Ends with a barrier.
-template <typename T, int DH>
+template <typename T, int DH, int NT = 128>
 __device__ __forceinline__ void team_attend_merge(AttState<DH>& a, int nh, float* out, float* scratch,
                                                   bool attnhp) {
-    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31, S = 4 / nh;
+    const int warp = (threadIdx.x & (NT - 1)) >> 5, lane = threadIdx.x & 31, S = NT / 32 / nh;
     float mm = a.mm, ll = a.ll;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
@@ -267,8 +258,8 @@ __device__ __forceinline__ void team_attend_merge(AttState<DH>& a, int nh, float
 #pragma unroll
         for (int c = 0; c < DH; ++c) sw[2 + c] = a.o[c];
     }
-    team_sync();
-    for (int t = threadIdx.x & 127; t < nh * DH; t += 128) {
+    team_sync<NT>();
+    for (int t = threadIdx.x & (NT - 1); t < nh * DH; t += NT) {
         const int hh = t / DH, c = t % DH;
         float M = -INFINITY;
         for (int sp = 0; sp < S; ++sp) M = fmaxf(M, scratch[(sp * nh + hh) * (DH + 2)]);
@@ -282,26 +273,26 @@ __device__ __forceinline__ void team_attend_merge(AttState<DH>& a, int nh, float
         }
         out[t] = attnhp ? O / (L + exp2f(-M)) : St<T>::rnd(O / L);
     }
-    team_sync();
+    team_sync<NT>();
 }
 
 // Attention of one query (qs in shared memory, nh heads of DH) over keys
 // 0..n_keys-1 of K/V blocks [nh][stride][DH] in shared memory: warp w takes
 // head w % nh and key range w / nh of 4 / nh; lane-strided keys with a
 // private online softmax, then team_attend_merge.  Ends with a barrier.
-template <typename T, int DH>
+template <typename T, int DH, int NT = 128>
 __device__ __forceinline__ void team_attend(const float* qs, const T* kb, const T* vb, int stride,
                                             int n_keys, int nh, float* out, float* scratch,
                                             bool attnhp = false) {
-    const int warp = (threadIdx.x & 127) >> 5, lane = threadIdx.x & 31;
-    const int h = warp % nh, split = warp / nh, S = 4 / nh;
+    const int warp = (threadIdx.x & (NT - 1)) >> 5, lane = threadIdx.x & 31;
+    const int h = warp % nh, split = warp / nh, S = NT / 32 / nh;
     const int per = (n_keys + S - 1) / S, lo = split * per, hi = min(n_keys, lo + per);
     AttState<DH> a;
     a.init(qs, h);
     const T* kh = kb + (size_t)h * stride * DH;
     const T* vh = vb + (size_t)h * stride * DH;
     for (int j = lo + lane; j < hi; j += 32) a.template add<T>(kh + (size_t)j * DH, vh + (size_t)j * DH);
-    team_attend_merge<T, DH>(a, nh, out, scratch, attnhp);
+    team_attend_merge<T, DH, NT>(a, nh, out, scratch, attnhp);
 }
 
 // Ring of shared-memory stages through which team_attend_stream streams a
@@ -322,12 +313,12 @@ struct KvRing {
 // chunk nst ahead.  Keys written by this CTA's generic stores must be fenced
 // (fence_proxy_async_global) before the barrier that precedes the call.
 // Ends with a barrier.
-template <typename T, int DH>
+template <typename T, int DH, int NT = 128>
 __device__ __forceinline__ void team_attend_stream(const float* qs, const T* kg, const T* vg, int stride, int n_keys,
                                                 int nh, float* out, float* scratch, KvRing& r, int* err,
                                                 bool attnhp = false) {
-    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
-    const int h = warp % nh, split = warp / nh, S = 4 / nh;
+    const int tid = threadIdx.x & (NT - 1), warp = tid >> 5, lane = tid & 31;
+    const int h = warp % nh, split = warp / nh, S = NT / 32 / nh;
     const int nch = (n_keys + r.ch - 1) / r.ch;
     const size_t hs = (size_t)r.ch * DH, ss = 2 * (size_t)nh * hs;
     auto issue = [&](int c) {
@@ -357,11 +348,11 @@ __device__ __forceinline__ void team_attend_stream(const float* qs, const T* kg,
         const int per = (cnt + S - 1) / S, lo = split * per, hi = min(cnt, lo + per);
         const T* kh = (const T*)r.buf + st * ss + (2 * h) * hs;
         for (int j = lo + lane; j < hi; j += 32) a.template add<T>(kh + (size_t)j * DH, kh + hs + (size_t)j * DH);
-        team_sync();
+        team_sync<NT>();
         if (tid == 0 && r.ok && c + r.nst < nch) issue(c + r.nst);
     }
     r.used += (uint32_t)nch;
-    team_attend_merge<T, DH>(a, nh, out, scratch, attnhp);
+    team_attend_merge<T, DH, NT>(a, nh, out, scratch, attnhp);
 }
 
 // Warp-parallel log-softmax of n <= 32*R values v[] (shared) in place, then
@@ -437,11 +428,14 @@ __device__ void rebase_model(DevModelT& m, const DevModelT& src, int L, const ch
     m.base = dst;
 }
 
-// TEAMS sequences per CTA, 128 threads each.  With WS the draft model is
-// staged once per CTA in shared memory (shared by its teams), so no weight
-// read leaves the SM; otherwise weights are read through L1.
-template <typename T, int DH, bool KVS, bool WS>
-__global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, int area_bytes) {
+// TEAMS sequences per CTA, NT threads each (128, or 256 when there are
+// fewer sequences than SMs, so that each sequence's chain of products and
+// key ranges is split twice as finely).  With WS the draft model is staged
+// once per CTA in shared memory (shared by its two 128-thread teams), so no
+// weight read leaves the SM; otherwise weights are read through L1.
+template <typename T, int DH, bool KVS, bool WS, int NT>
+__global__ void __launch_bounds__(WS ? 256 : NT) k_draft_team(DraftTeamArgs a, int area_bytes) {
+    static_assert(!WS || NT == 128, "two teams of 128 share a staged model");
     constexpr int TEAMS = WS ? 2 : 1;
     pdl_wait();
     extern __shared__ __align__(16) char smem[];
@@ -449,7 +443,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     __shared__ int k_new_s[TEAMS];
     __shared__ DevModelT msh;
     __shared__ uint64_t wbar;
-    const int team = threadIdx.x >> 7;
+    const int team = threadIdx.x / NT;
     const int s = blockIdx.x * TEAMS + team;
     const CallParams& P = *a.P;
     char* area = smem;
@@ -469,7 +463,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     if (s >= P.B || a.ss.done[s]) return;  // the rest synchronises within the team only
     double& t_new = t_new_s[team];
     int& k_new = k_new_s[team];
-    const int tid = threadIdx.x & 127, warp = tid >> 5, lane = tid & 31;
+    const int tid = threadIdx.x & (NT - 1), warp = tid >> 5, lane = tid & 31;
     const DevModelT& m = WS ? msh : a.m.t;
     const int d = a.m.d, F = a.m.F, M = a.m.M, K = a.m.K, W = 3 * M + K, L = a.m.L, NH = d / DH;
     const int n_max = a.kv.n_max;
@@ -484,7 +478,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             for (int i = 0; i < ring.nst; ++i) mbar_init(ring.full + i, 1);
             mbar_fence_init();
         }
-        team_sync();
+        team_sync<NT>();
     }
     float* x = (float*)(area + kvb + 64 + ringb);
     float* zin = x + d;   // rounded temporal encoding; [zin | xin] is the AttNHP QKV input
@@ -496,7 +490,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     float* e = y + d;  // E h (3d) | tanh(V_k1 h + b_k1) (d)
     float* hd = e + 4 * d;
     float* part = hd + ((W + 3) & ~3);  // team_gemv partial sums (16-byte aligned)
-    float* attn = part + team_gp_floats(d, F);
+    float* attn = part + team_gp_floats(d, F, NT);
     const SeqState& ss = a.ss;
     const int n = ss.n_emit[s], nd = ss.n_draft[s];
     auto gk = [&](int l, int w) -> T* {
@@ -515,20 +509,20 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
                     for (int h = 0; h < NH; ++h)
                         bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
         }
-        team_sync();
+        team_sync<NT>();
         mbar_wait(bar, 0, a.err, 12);
     }
     // x = LN(x + W_T in + b): the product, then the residual add and
     // LayerNorm (by warp 0, in registers when d <= 32).  Ends synced.
     auto proj_resid_ln = [&](const T* WT, const float* bias, const float* in, int IN, const float* g,
                              const float* b) {
-        const int G = team_gemv<T>(WT, d, nullptr, 0, in, IN, part);
+        const int G = team_gemv<T, NT>(WT, d, nullptr, 0, in, IN, part);
         if (d <= 32) {
             if (warp == 0) {
                 const float v = lane < d ? bias[lane] + gemv_out(part, d, G, lane) : 0.f;
                 warp_resid_ln<T>(v, x, xin, d, g, b);
             }
-            team_sync();
+            team_sync<NT>();
             return;
         }
         if (warp == 0) {
@@ -547,13 +541,13 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
                 xin[i] = St<T>::rnd(v);
             }
         }
-        team_sync();
+        team_sync<NT>();
     };
     // Q, K, V of position p from the QKV input qin (IN wide); K and V
     // appended to the cache (and its resident copy).  Ends synced.
     auto qkv_step = [&](const LayerW& Wl, int l, int p, const float* qin, int IN) {
-        const int G = team_gemv<T>((const T*)Wl.w_qkv, 3 * d, nullptr, 0, qin, IN, part);
-        for (int o = tid; o < 3 * d; o += 128) {
+        const int G = team_gemv<T, NT>((const T*)Wl.w_qkv, 3 * d, nullptr, 0, qin, IN, part);
+        for (int o = tid; o < 3 * d; o += NT) {
             const float v = St<T>::rnd(Wl.b_qkv[o] + gemv_out(part, 3 * d, G, o));
             qkv[o] = v;
             if (o >= d) {
@@ -564,11 +558,11 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             }
         }
         if (!KVS) fence_proxy_async_global();  // the streamed attention reads them back by bulk copy
-        team_sync();
+        team_sync<NT>();
     };
     auto attend = [&](int l, int p, bool attnhp) {
-        if (KVS) team_attend<T, DH>(qkv, sk(l, 0), sk(l, 1), n_max, p + 1, NH, att, attn, attnhp);
-        else team_attend_stream<T, DH>(qkv, gk(l, 0), gk(l, 1), n_max, p + 1, NH, att, attn, ring, a.err, attnhp);
+        if (KVS) team_attend<T, DH, NT>(qkv, sk(l, 0), sk(l, 1), n_max, p + 1, NH, att, attn, attnhp);
+        else team_attend_stream<T, DH, NT>(qkv, gk(l, 0), gk(l, 1), n_max, p + 1, NH, att, attn, ring, a.err, attnhp);
     };
     // Layers of the encode step at position p from x / xin (set and synced
     // by the caller); leaves the final hidden state in x (synced).
@@ -580,11 +574,11 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             for (int l = 0; l < L; ++l) {
                 qkv_step(m.layer[l], l, p, zin, 2 * d);
                 attend(l, p, true);
-                for (int i = tid; i < d; i += 128) {
+                for (int i = tid; i < d; i += NT) {
                     x[i] += tanhf(att[i]);
                     xin[i] = St<T>::rnd(x[i]);
                 }
-                team_sync();
+                team_sync<NT>();
             }
             return;
         }
@@ -594,10 +588,10 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
             attend(l, p, false);
             proj_resid_ln((const T*)Wl.w_o, Wl.b_o, att, d, Wl.ln1_g, Wl.ln1_b);
             {
-                const int G = team_gemv<T>((const T*)Wl.w_1, F, nullptr, 0, xin, d, part);
-                for (int o = tid; o < F; o += 128)
+                const int G = team_gemv<T, NT>((const T*)Wl.w_1, F, nullptr, 0, xin, d, part);
+                for (int o = tid; o < F; o += NT)
                     hid[o] = St<T>::rnd(fmaxf(Wl.b_1[o] + gemv_out(part, F, G, o), 0.f));
-                team_sync();
+                team_sync<NT>();
             }
             proj_resid_ln((const T*)Wl.w_2, Wl.b_2, hid, F, Wl.ln2_g, Wl.ln2_b);
         }
@@ -606,7 +600,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     // z_i = sin / cos (a_i + b_i t), angle reduced mod 2 pi in fp64, plus the
     // mark embedding); zin = rounded z.  Not synced.
     auto embed = [&](double t, int k) {
-        for (int i = tid; i < d; i += 128) {
+        for (int i = tid; i < d; i += NT) {
             const double ang = m.tenc[i] + m.tenc[d + i] * t;
             const double red = fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
             float sv, cv;
@@ -621,7 +615,7 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
     for (int p = nd; p < n; ++p) {  // catch-up over events already emitted
         const size_t so = (size_t)s * ss.n_max + p;
         embed(ss.t[so], min(max(ss.k[so], 0), K - 1));
-        team_sync();
+        team_sync<NT>();
         layers(p);
     }
     if (tid == 0) {
@@ -634,18 +628,18 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
         const int p = n + l - 1;  // index of the drafted event
         // head (Sec. 4.2): e = E h | a = tanh(V_k1 h + b_k1)
         {
-            const int G = team_gemv<float>(H.E, 3 * d, H.v_k1, d, x, d, part);
-            for (int o = tid; o < 4 * d; o += 128) {
+            const int G = team_gemv<float, NT>(H.E, 3 * d, H.v_k1, d, x, d, part);
+            for (int o = tid; o < 4 * d; o += NT) {
                 const float v = gemv_out(part, 4 * d, G, o);
                 e[o] = o < 3 * d ? v : tanhf(v + H.b_k1[o - 3 * d]);
             }
-            team_sync();
+            team_sync<NT>();
         }
         // [w logits | mu | log sigma | mark logits] in blocks of OPh outputs;
         // output j reads its own matrix and input segment
         for (int ob = 0; ob < W; ob += OPh) {
             {
-                const int G = 128 / OPh, o = ob + tid % OPh, g = tid / OPh;
+                const int G = NT / OPh, o = ob + tid % OPh, g = tid / OPh;
                 const int per = (d + G - 1) / G, i0 = g * per, i1 = min(d, i0 + per);
                 float acc = 0.f;
                 if (o < W) {
@@ -660,14 +654,14 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
                 }
                 part[tid] = acc;
             }
-            team_sync();
+            team_sync<NT>();
             if (tid < OPh && ob + tid < W) {
                 const int o = ob + tid;
                 float v = o < M ? H.b_w[o] : o < 2 * M ? H.b_mu[o - M] : o < 3 * M ? H.b_s[o - 2 * M] : H.b_k2[o - 3 * M];
-                for (int gg = 0; gg < 128 / OPh; ++gg) v += part[gg * OPh + tid];
+                for (int gg = 0; gg < NT / OPh; ++gg) v += part[gg * OPh + tid];
                 hd[o] = v;
             }
-            team_sync();
+            team_sync<NT>();
         }
         // direct sample: warp 0 the time (component, Box-Muller), warp 1 the
         // mark; both normalise their logits in place
@@ -692,33 +686,38 @@ __global__ void __launch_bounds__(WS ? 256 : 128) k_draft_team(DraftTeamArgs a, 
                 }
             }
         }
-        team_sync();
+        team_sync<NT>();
         float* rec = a.heads + ((size_t)s * a.gamma_max + (l - 1)) * W;
-        for (int i = tid; i < W; i += 128) rec[i] = hd[i];
+        for (int i = tid; i < W; i += NT) rec[i] = hd[i];
         if (l < a.gamma) {
             embed(t_new, k_new);
-            team_sync();
+            team_sync<NT>();
             layers(p);
         }
     }
     pdl_trigger();
 }
 
-template <typename T, int DH, bool KVS, bool WS>
+template <typename T, int DH, bool KVS, bool WS, int NT>
 static cudaError_t launch_t(DraftTeamArgs& a, int B, int area, size_t sm, cudaStream_t st) {
     constexpr int TEAMS = WS ? 2 : 1;
-    cudaError_t e = cudaFuncSetAttribute(k_draft_team<T, DH, KVS, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)sm);
+    cudaError_t e = cudaFuncSetAttribute(k_draft_team<T, DH, KVS, WS, NT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
     if (e != cudaSuccess) return e;
-    return launch_k(k_draft_team<T, DH, KVS, WS>, dim3((B + TEAMS - 1) / TEAMS), dim3(128 * TEAMS), sm, st, a,
+    return launch_k(k_draft_team<T, DH, KVS, WS, NT>, dim3((B + TEAMS - 1) / TEAMS), dim3(NT * TEAMS), sm, st, a,
                     area);
 }
 
 template <typename T, int DH>
-static cudaError_t launch_team(DraftTeamArgs& a, int B, int kvs, int ws, size_t area, size_t wb, cudaStream_t st) {
-    if (ws) return launch_t<T, DH, true, true>(a, B, (int)area, wb + 2 * area, st);
-    if (kvs) return launch_t<T, DH, true, false>(a, B, (int)area, area, st);
-    return launch_t<T, DH, false, false>(a, B, (int)area, area, st);
+static cudaError_t launch_team(DraftTeamArgs& a, int B, int kvs, int ws, int nt, size_t area, size_t wb,
+                               cudaStream_t st) {
+    if (ws) return launch_t<T, DH, true, true, 128>(a, B, (int)area, wb + 2 * area, st);
+    if (nt == 256) {
+        if (kvs) return launch_t<T, DH, true, false, 256>(a, B, (int)area, area, st);
+        return launch_t<T, DH, false, false, 256>(a, B, (int)area, area, st);
+    }
+    if (kvs) return launch_t<T, DH, true, false, 128>(a, B, (int)area, area, st);
+    return launch_t<T, DH, false, false, 128>(a, B, (int)area, area, st);
 }
 
 int draft_team_supported(const DevModel& m) {
@@ -739,7 +738,14 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
     const size_t eb = m.dtype == 1 ? 2 : 4;
     const int W = 3 * m.M + m.K;
-    const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + team_gp_floats(m.d, m.F) + 4 * 66) + 64;
+    int dev = 0, n_sm = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    // 256-thread teams when every sequence can have an SM of its own
+    // (TPPSD_DRAFT_NT=128|256 forces a size)
+    int nt = B <= n_sm ? 256 : 128;
+    if (const char* f = getenv("TPPSD_DRAFT_NT")) nt = atoi(f) == 256 ? 256 : 128;
+    const size_t fl = sizeof(float) * (12 * (size_t)m.d + m.F + ((W + 3) & ~3) + team_gp_floats(m.d, m.F, nt) +
+                                       (size_t)(nt / 32) * 66) + 64;
     const size_t kvb = ((size_t)m.L * 2 * kv.n_max * m.d * eb + 15) & ~(size_t)15;
     // TPPSD_DRAFT_STREAM=<keys>: stream the KV even where it would fit, two
     // stages of that many keys (exercises the ring's wrap-around and ragged
@@ -755,9 +761,7 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
         // streamed KV: as many stages of up to 64 keys as the CTAs that share
         // an SM leave room for (at most 4 resident: the kernel holds 128
         // registers a thread), 2 to 6 stages
-        int dev = 0, n_sm = 148;
-        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-        const int per_sm = std::min(4, std::max(1, (B + n_sm - 1) / n_sm));
+        const int per_sm = nt == 256 ? 1 : std::min(4, std::max(1, (B + n_sm - 1) / n_sm));
         const long long budget = std::max(0ll, (long long)(227 * 1024 / per_sm) - 2048 - (long long)fl);
         int ch = 64;
         auto stage = [&](int c) { return (size_t)c * 2 * m.d * eb; };
@@ -769,13 +773,15 @@ cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqSta
     }
     const size_t area = ((kvs ? kvb : ringb) + fl + 15) & ~(size_t)15;
     const size_t wb = m.t.bytes;  // a whole number of 16-byte chunks
-    const int ws = kvs && wb % 16 == 0 && wb + 2 * area <= 224 * 1024;
+    // two 128-thread teams sharing a staged model, unless each sequence gets
+    // its own SM
+    const int ws = nt == 128 && kvs && wb % 16 == 0 && wb + 2 * area <= 224 * 1024;
     if (m.dtype == 0) {
-        if (m.dh == 16) return launch_team<float, 16>(a, B, kvs, ws, area, wb, st);
-        return launch_team<float, 32>(a, B, kvs, ws, area, wb, st);
+        if (m.dh == 16) return launch_team<float, 16>(a, B, kvs, ws, nt, area, wb, st);
+        return launch_team<float, 32>(a, B, kvs, ws, nt, area, wb, st);
     }
-    if (m.dh == 16) return launch_team<bf16, 16>(a, B, kvs, ws, area, wb, st);
-    return launch_team<bf16, 32>(a, B, kvs, ws, area, wb, st);
+    if (m.dh == 16) return launch_team<bf16, 16>(a, B, kvs, ws, nt, area, wb, st);
+    return launch_team<bf16, 32>(a, B, kvs, ws, nt, area, wb, st);
 }
 
 

@@ -174,20 +174,30 @@ def test_sequence_parity_fp32_with_rejections(gamma, flags):
         assert stats["resample_iters"] == ostats[:, 3].sum()
 
 
-@pytest.mark.parametrize("form", ["lane", "team", "team_stream"])
+def _set_draft_form(monkeypatch, form):
+    """Environment switches of a draft kernel form (read when the context's
+    graphs are captured)."""
+    if form.startswith("team"):
+        monkeypatch.setenv("TPPSD_DRAFT_TEAM", "1")
+    if form.startswith("team128"):
+        monkeypatch.setenv("TPPSD_DRAFT_NT", "128")
+    if form.endswith("_stream"):
+        monkeypatch.setenv("TPPSD_DRAFT_STREAM", "13")
+
+
+@pytest.mark.parametrize("form", ["lane", "team", "team_stream", "team128", "team128_stream"])
 @pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
 def test_draft_kernel_forms_match_oracle(form, dtype, monkeypatch):
     """Both forms of the per-sequence draft kernel on a d = 32, two-head
     draft (lane form: one hidden component per lane, the default for
     d <= 32; team form: TPPSD_DRAFT_TEAM=1) reproduce the oracle's
-    sequences, rejections and resampling included.  team_stream: the team
-    form with its KV streamed from HBM through two 13-key shared-memory
-    stages (TPPSD_DRAFT_STREAM=13), so the ring wraps several times per
-    attention and every last chunk is ragged."""
-    if form.startswith("team"):
-        monkeypatch.setenv("TPPSD_DRAFT_TEAM", "1")
-    if form == "team_stream":
-        monkeypatch.setenv("TPPSD_DRAFT_STREAM", "13")
+    sequences, rejections and resampling included.  The team form runs
+    with 256 threads per sequence here (fewer sequences than SMs); team128
+    forces the 128-thread teams that large batches use
+    (TPPSD_DRAFT_NT=128).  *_stream: the KV streamed from HBM through two
+    13-key shared-memory stages (TPPSD_DRAFT_STREAM=13), so the ring wraps
+    several times per attention and every last chunk is ragged."""
+    _set_draft_form(monkeypatch, form)
     dcfg = CF.ModelCfg(1, 32, 2, 128, 4, 3, dtype)
     tcfg = None if dtype == CF.FP32 else CF.ModelCfg(2, 128, 4, 512, 4, 3, dtype)
     tcfg, dcfg, bt, bd = G.small_models(gain=1.5, dtype=dtype, tcfg=tcfg, dcfg=dcfg)
@@ -201,16 +211,13 @@ def test_draft_kernel_forms_match_oracle(form, dtype, monkeypatch):
     assert st == T.TPPSD_OK and stats["accepted"] < stats["drafted"]
 
 
-@pytest.mark.parametrize("form", ["lane", "team", "team_stream"])
+@pytest.mark.parametrize("form", ["lane", "team", "team_stream", "team128"])
 @pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
 def test_draft_kernel_wide_heads_match_oracle(form, dtype, monkeypatch):
     """M = 12 mixture components and K = 20 marks: the draft kernels draw
     the component and the mark with the warp-wide log-softmax (more than
     eight values), and the sequences still follow the oracle."""
-    if form.startswith("team"):
-        monkeypatch.setenv("TPPSD_DRAFT_TEAM", "1")
-    if form == "team_stream":
-        monkeypatch.setenv("TPPSD_DRAFT_STREAM", "13")
+    _set_draft_form(monkeypatch, form)
     dcfg = CF.ModelCfg(1, 32, 2, 128, 12, 20, dtype)
     tcfg = CF.ModelCfg(2, 32, 2, 64, 12, 20, dtype) if dtype == CF.FP32 else CF.ModelCfg(2, 128, 4, 512, 12, 20, dtype)
     tcfg, dcfg, bt, bd = G.small_models(gain=1.5, dtype=dtype, tcfg=tcfg, dcfg=dcfg)
