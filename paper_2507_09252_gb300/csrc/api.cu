@@ -569,9 +569,9 @@ static int pick_bn(int N) {
 
 // Heads of widths other than 128 (or with the head kernel off): [E; V_k1] h
 // by the split tensor-core GEMM over the hi / lo bf16 parts of [E; V_k1].
-static void head_gemm_plan(TcPlan& p, const DevModel& m, bool ok) {
+static void head_gemm_plan(TcPlan& p, const DevModel& m, bool ok, int bn) {
     const int d = m.d;
-    p.bn_head = pick_bn(4 * d);
+    p.bn_head = bn;
     const int box = p.bn_head < 256 ? p.bn_head : 256;
     p.head_g = ok && !p.head && p.bn_head && d % 64 == 0 && !getenv("TPPSD_NO_TC_HEAD") &&
                make_tmap_bf16(&p.head_hi_g, m.head_ek_hi, d, 4 * d, box) &&
@@ -600,16 +600,30 @@ static void build_tc_plan(tppsd_ctx* ctx) {
                  make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
                  make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
         ok = ok && make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128);
-        head_gemm_plan(p, m, ok);
+        head_gemm_plan(p, m, ok, pick_bn(4 * d));
         p.err = ctx->d_err;
         p.enabled = ok ? 1 : 0;
         return;
     }
     if (d % 64 || F % 64 || m.dh < 16 || !(d == 64 || d == 128 || d == 256 || d == 512)) return;
-    // QKV: 64-column tiles up to d = 128 (more CTAs, each with a shorter
-    // epilogue; measured 9.6 -> 8.5 us per launch at 2 304 rows, d = 128)
-    p.bn_qkv = d <= 128 ? 64 : pick_bn(3 * d);
-    p.bn_ffn1 = pick_bn(F);
+    // QKV and FFN1 tiles: the widest of 256 / 128 / 64 / 32 columns whose
+    // grid over the context's row capacity still covers every SM (more CTAs,
+    // each with a shorter epilogue: at 2 304 rows, d = 128, 128 -> 64
+    // columns took the QKV launch from 9.6 to 8.5 us, and 64 -> 32 the
+    // headline call from 14.41 to 14.22 ms).  TPPSD_QKV_BN / TPPSD_FFN1_BN
+    // force a width.
+    int n_sm = 148;
+    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, ctx->device);
+    const long long tiles = (w.R + 127) / 128;
+    auto fill_bn = [&](int N) {
+        for (int bn = 256; bn >= 32; bn /= 2)
+            if (N % bn == 0 && (N / bn) * tiles >= n_sm) return bn;
+        return N % 32 == 0 ? 32 : pick_bn(N);
+    };
+    p.bn_qkv = fill_bn(3 * d);
+    p.bn_ffn1 = fill_bn(F);
+    if (const char* f = getenv("TPPSD_QKV_BN")) p.bn_qkv = atoi(f);
+    if (const char* f = getenv("TPPSD_FFN1_BN")) p.bn_ffn1 = atoi(f);
     p.bn_o = ln_cluster_cols(d);
     if (!p.bn_qkv || !p.bn_ffn1 || !p.bn_o) return;
     bool ok = make_tmap_bf16(&p.a_xb, w.xb, d, w.R, 128) && make_tmap_bf16(&p.a_att, w.att, d, w.R, 128) &&
@@ -643,7 +657,7 @@ static void build_tc_plan(tppsd_ctx* ctx) {
     p.head = ok && head_tc_supported(m) &&
              make_tmap_bf16(&p.head_hi, m.head_ek_hi, d, 4 * d, 128) &&
              make_tmap_bf16(&p.head_lo, m.head_ek_lo, d, 4 * d, 128);
-    head_gemm_plan(p, m, ok);
+    head_gemm_plan(p, m, ok, fill_bn(4 * d));
     p.err = ctx->d_err;
     p.enabled = ok ? 1 : 0;
 }

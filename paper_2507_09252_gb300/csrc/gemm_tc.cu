@@ -440,6 +440,7 @@ cudaError_t launch_gemm_tc_split(const CUtensorMap& A, const CUtensorMap& A2, co
     if (a.epi != EPI_TC_QKV && a.epi != EPI_TC_RELU && a.epi != EPI_TC_F32) return cudaErrorInvalidValue;
     if (a.K % 64 || a.N % BN) return cudaErrorInvalidValue;
     switch (BN) {
+        case 32: return launch_bn<32>(A, W, A2, W2, a, st);
         case 64: return launch_bn<64>(A, W, A2, W2, a, st);
         case 128: return launch_bn<128>(A, W, A2, W2, a, st);
         case 256: return launch_bn<256>(A, W, A2, W2, a, st);
