@@ -863,10 +863,18 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
     } else if (mode == 0) {
         PROF_MARK(prof, KC_DRAFT, 1, st);
         const bool team = draft_team_supported(ctx->D.dm) && (ctx->D.dm.enc == 2 || !getenv("TPPSD_DRAFT_CTA"));
-        if (team && draft_lane_supported(ctx->D.dm, ctx->kvD.n_max, ctx->max_gamma) && !getenv("TPPSD_DRAFT_TEAM"))
+        // the lane form also writes the target's verify rows (same storage
+        // type, THP / SAHP layout), so the forward below has no embedding
+        // launch (TPPSD_NO_EMBED_FUSION keeps it)
+        bool fused = false;
+        if (team && draft_lane_supported(ctx->D.dm, ctx->kvD.n_max, ctx->max_gamma) && !getenv("TPPSD_DRAFT_TEAM")) {
+            const DevModel& tm = ctx->T.dm;
+            DraftEmbed emb{tm.tenc, tm.type_emb, w.x, w.xb, w.row_seq, w.row_pos, tm.d, tm.K, tm.tenc_paired};
+            fused = tm.dtype == ctx->D.dm.dtype && tm.enc != 2 && !getenv("TPPSD_NO_EMBED_FUSION");
             CK(launch_draft_lane(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
-                                 ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
-        else if (team)
+                                 ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st,
+                                 fused ? &emb : nullptr));
+        } else if (team)
             CK(launch_draft_team(ctx->D.dm, ctx->kvD, ctx->ss, ctx->d_params, B, gamma,
                                  ctx->draft_heads, ctx->max_gamma, ctx->d_stats, ctx->d_err, st));
         else
@@ -874,7 +882,7 @@ static tppsd_status_t record_round(tppsd_ctx* ctx, int mode, int B, int gamma, c
                             ctx->max_gamma, ctx->d_stats, st));
         PROF_MARK(prof, KC_DRAFT, 0, st);
         ++n;
-        RowSpec rs{ROWS_STEP, gamma + 1, B * (gamma + 1), 0};
+        RowSpec rs{ROWS_STEP, gamma + 1, B * (gamma + 1), 0, fused ? 1 : 0};
         CK(launch_forward(ctx->T.dm, ctx->kvT, ctx->ss, w, rs, true, st, &n, prof, &ctx->tc));
         PROF_MARK(prof, KC_EPILOGUE, 1, st);
         CK(launch_verify_epilogue(ctx->T.dm, ctx->D.dm, ctx->ss, ctx->d_params, B, gamma, w.heads,

@@ -42,6 +42,23 @@ template <> struct St<bf16> {
 // key is bumped by the Weyl constants between rounds.
 struct U4 { float x, y, z, w; };
 
+// Temporal encoding (App. D.4) of a model with encoding table tenc (a_j,
+// then b_j; fp64) and width d: the angle a_j + b_j t formed and reduced mod
+// 2 pi in fp64, then fp32 sin / cos.  Dimensions 2i, 2i+1 share one angle
+// (one sincos) when paired (THP, AttNHP); SAHP's have their own.
+__device__ __forceinline__ float tenc_angle(const double* tenc, int d, int j, double t) {
+    const double ang = tenc[j] + tenc[d + j] * t;
+    return (float)fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
+}
+__device__ __forceinline__ void tenc_pair_of(const double* tenc, int d, int paired, double t, int i, float* z0,
+                                             float* z1) {
+    float sv, cv;
+    sincosf(tenc_angle(tenc, d, 2 * i, t), &sv, &cv);
+    if (!paired) cv = cosf(tenc_angle(tenc, d, 2 * i + 1, t));
+    *z0 = sv;
+    *z1 = cv;
+}
+
 __device__ __forceinline__ uint4 philox(uint4 c, uint32_t k0, uint32_t k1) {
 #pragma unroll
     for (int r = 0; r < 10; ++r) {

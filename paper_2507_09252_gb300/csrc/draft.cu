@@ -51,6 +51,7 @@ struct DraftTeamArgs {
     int gamma, gamma_max;
     int* err;      // set if a bulk copy of KV or weights does not complete
     int ring_nst, ring_ch;  // streamed KV (k_draft_team without resident KV): stages, keys per stage
+    DraftEmbed emb;         // lane form: the target's verify rows (emb.x null: not written here)
 };
 
 // DH consecutive storage-type values -> fp32, with 16-byte loads.
@@ -986,6 +987,35 @@ __host__ __device__ inline int lane_team_floats(int W, int G, int sc) {
     return ((W + 3) & ~3) + 2 * 4 * 36 + 128 + 4 + 4 * lane_warp_floats(G, sc);
 }
 
+// Pairs i0, i0 + stride, ... of the target's embedding of verify row r
+// (event (t, k) at position pos of sequence s, THP or SAHP layout): the
+// same arithmetic as the forward's embedding kernel, whose launch the lane
+// form replaces.  live == false writes the inactive row (zeros, s = -1).
+template <typename T>
+__device__ __forceinline__ void draft_embed_row(const DraftEmbed& e, int r, int s, int pos, double t, int k,
+                                                bool live, int i0, int stride) {
+    const int half = e.d / 2;
+    k = min(max(k, 0), e.K - 1);
+    T* xb = (T*)e.xb;
+    for (int i = i0; i < half; i += stride) {
+        float z0 = 0.f, z1 = 0.f, e0 = 0.f, e1 = 0.f;
+        if (live) {
+            tenc_pair_of(e.tenc, e.d, e.paired, t, i, &z0, &z1);
+            e0 = e.type_emb[(size_t)k * e.d + 2 * i];
+            e1 = e.type_emb[(size_t)k * e.d + 2 * i + 1];
+        }
+        const size_t xo = (size_t)r * e.d + 2 * i;
+        e.x[xo] = z0 + e0;
+        e.x[xo + 1] = z1 + e1;
+        St<T>::st(xb + xo, z0 + e0);
+        St<T>::st(xb + xo + 1, z1 + e1);
+    }
+    if (i0 == 0) {
+        e.row_seq[r] = live ? s : -1;
+        e.row_pos[r] = pos;
+    }
+}
+
 // D: the draft width (16 or 32), a compile-time constant so that the
 // product loops, lane predicates and head splits are fixed.
 template <typename T, int DH, int D>
@@ -1041,7 +1071,14 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                     bulk_load(sk(l, w) + (size_t)h * n_max * DH, gk(l, w) + (size_t)h * n_max * DH, bytes, bar);
     }
     __syncthreads();
+    const bool emb = a.emb.x != nullptr;
+    const int q = a.gamma + 1;  // verify rows per sequence
     if (!live) {
+        if (emb && s < P.B) {  // the sequence's verify rows, inactive
+            const int ne = ss.n_emit[s];
+            for (int l = 0; l < q; ++l)
+                draft_embed_row<T>(a.emb, s * q + l, s, ne - 1 + l, 0.0, 0, false, tid, 128);
+        }
         // a CTA may not exit while the model copy still writes its shared memory
         mbar_wait(&wbar, 0, a.err, 14);
         return;  // the rest synchronises within the team only
@@ -1085,11 +1122,15 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
         k_cu[i] = min(max(ss.k[so], 0), K - 1);
     }
     double t64 = ss.t[(size_t)s * ss.n_max + n - 1];  // fp64 time of the last event (warp 1)
+    int k_emb = 0;  // mark of the last drawn event (warp 1)
     if (tid == 0) {  // its pair form, which the first draft adds to
         const F2 t2 = f2_from_double(t64);
         ev[0] = t2.h;
         ev[1] = t2.l;
     }
+    if (emb)  // verify row 0: the last emitted event, at position n - 1
+        draft_embed_row<T>(a.emb, s * q, s, n - 1, t64, min(max(ss.k[(size_t)s * ss.n_max + n - 1], 0), a.emb.K - 1),
+                           true, tid, 128);
     mbar_wait(&wbar, 0, a.err, 14);
     if (nd > 0) mbar_wait(bar, 0, a.err, 12);
     const float* type_emb = (const float*)sm(mp.type_emb);
@@ -1169,6 +1210,10 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
                     ss.k[so] = k;
                     ev[3] = __int_as_float(k);
                 }
+            } else if (warp == 1 && emb && l >= 1) {
+                // idle while warps 0 and 3 draw: the target's verify row of the
+                // previous draft (row l, position p - 1)
+                draft_embed_row<T>(a.emb, s * q + l, s, p - 1, t64, k_emb, true, lane, 32);
             }
             team_sync();
             tp = {ev[0], ev[1]};
@@ -1176,12 +1221,15 @@ __global__ void __launch_bounds__(256) k_draft_lane(DraftTeamArgs a, int area_by
             if (warp == 1) {
                 float* rec = a.heads + ((size_t)s * a.gamma_max + l) * W;
                 for (int i = lane; i < W; i += 32) rec[i] = hd[i];
-                if (lane == 0) {  // the fp64 time of the event, as the target reads it
-                    t64 += (double)ev[2];
-                    ss.t[so] = t64;
-                }
+                t64 += (double)ev[2];  // the fp64 time of the event, as the target reads it
+                k_emb = kp;
+                if (lane == 0) ss.t[so] = t64;
             }
-            if (p == p_last) break;
+            if (p == p_last) {
+                if (warp == 1 && emb)  // the last draft's verify row (row gamma)
+                    draft_embed_row<T>(a.emb, s * q + q - 1, s, p, t64, k_emb, true, lane, 32);
+                break;
+            }
         } else {
             const int i = p - nd;
             double t;
@@ -1376,10 +1424,12 @@ int draft_lane_supported(const DevModel& m, int n_max, int gamma_max) {
 
 cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
-                              int gamma_max, DevStats* stats, int* err, cudaStream_t st) {
+                              int gamma_max, DevStats* stats, int* err, cudaStream_t st,
+                              const DraftEmbed* emb) {
     DraftTeamArgs a{};
     a.m = m; a.kv = kv; a.ss = ss; a.P = dp; a.st = stats; a.heads = draft_heads;
     a.gamma = gamma; a.gamma_max = gamma_max; a.err = err;
+    if (emb) a.emb = *emb;
     int sc = 0, G = 0;
     const size_t area = lane_area(m, kv.n_max, gamma_max, &sc, &G);
     const size_t sm = m.p.bytes + 2 * area;

@@ -201,6 +201,7 @@ struct RowSpec {
     int q;      // rows per sequence
     int count;  // rows in this pass
     int g0;
+    int pre_embedded;  // ROWS_STEP: the rows (x, xb, row_seq, row_pos) were written by the draft kernel
 };
 
 // Arguments of one attention launch (rows of q_per_seq queries per sequence).
@@ -384,9 +385,24 @@ int draft_team_supported(const DevModel& m);
 // Lane form of the draft kernel (draft.cu) for d <= 32 models whose packed
 // copy and two sequences' draft KV fit in shared memory.
 int draft_lane_supported(const DevModel& m, int n_max, int gamma_max);
+// The target's embedding of the verify rows (THP / SAHP layout), written by
+// the lane draft kernel in place of the forward's embedding kernel: row
+// s (gamma + 1) + l is the event at position n_emit[s] - 1 + l.
+struct DraftEmbed {
+    const double* tenc;     // the target's encoding table (a_j, then b_j)
+    const float* type_emb;  // [K][d]
+    float* x;               // [rows][d] fp32
+    void* xb;               // [rows][d] storage type (the draft's, equal to the target's)
+    int* row_seq;
+    int* row_pos;
+    int d, K, paired;
+};
+// emb: null, or the target rows to write (then the forward skips its
+// embedding kernel: RowSpec.pre_embedded).
 cudaError_t launch_draft_lane(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
-                              int gamma_max, DevStats* stats, int* err, cudaStream_t st);
+                              int gamma_max, DevStats* stats, int* err, cudaStream_t st,
+                              const DraftEmbed* emb = nullptr);
 cudaError_t launch_draft_team(const DevModel& m, const KVCache& kv, const SeqState& ss,
                               const CallParams* dp, int B, int gamma, float* draft_heads,
                               int gamma_max, DevStats* stats, int* err, cudaStream_t st);

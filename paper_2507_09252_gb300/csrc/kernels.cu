@@ -34,21 +34,11 @@ __device__ __forceinline__ void load_row(const T* p, float* out, int n) {
     for (int c = 0; c < n; ++c) out[c] = St<T>::ld(p + c);
 }
 
-// Angle a + b t in fp64, reduced mod 2 pi in fp64 (then fp32 sin / cos).
-__device__ __forceinline__ float tenc_angle(const double* tenc, int d, int j, double t) {
-    const double ang = tenc[j] + tenc[d + j] * t;
-    return (float)fma(-6.283185307179586476925, rint(ang * 0.15915494309189533577), ang);
-}
-
 // Temporal encoding (App. D.4: z_j = sin / cos (a_j + b_j t) for even / odd
 // j) of dimensions 2i, 2i+1.  THP and AttNHP pairs share one angle (one
 // sincos); SAHP's dimensions have their own.
 __device__ __forceinline__ void tenc_pair(const DevModel& m, double t, int i, float* z0, float* z1) {
-    float sv, cv;
-    sincosf(tenc_angle(m.tenc, m.d, 2 * i, t), &sv, &cv);
-    if (!m.tenc_paired) cv = cosf(tenc_angle(m.tenc, m.d, 2 * i + 1, t));
-    *z0 = sv;
-    *z1 = cv;
+    tenc_pair_of(m.tenc, m.d, m.tenc_paired, t, i, z0, z1);
 }
 
 // Temporal encoding + type embedding (Sec. 4.2) of pair i.  Marks outside
@@ -1367,7 +1357,7 @@ static cudaError_t forward_t(const DevModel& m, const KVCache& kv, const SeqStat
     const int R = rs.count, d = m.d, F = m.F;
     if (R <= 0) return cudaSuccess;
     int nl = 0;
-    {
+    if (!rs.pre_embedded) {
         const long long total = (long long)R * (d / 2);
         const long long want = (total + 255) / 256;
         const int blocks = (int)(want < 152 * 16 ? want : 152 * 16);
