@@ -292,6 +292,31 @@ def test_folded_qkv_is_bit_identical(monkeypatch):
     assert stats0["kernel_launches"] > stats1["kernel_launches"]
 
 
+@pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
+def test_fused_verify_rows_are_bit_identical(dtype, monkeypatch):
+    """The lane draft kernel writes the target's verify rows (the embedding
+    of the last emitted event and of every draft) in place of the
+    forward's embedding kernel: the same arithmetic, so sampled sequences
+    are bit-identical to the unfused path (TPPSD_NO_EMBED_FUSION=1), with
+    one launch fewer per round."""
+    tcfg, dcfg, bt, bd = G.small_models(gain=1.5, dtype=dtype)
+    tau, mk = G.hist(13, 9, 3, 6)
+    def run():
+        s = G.make_sampler(tcfg, dcfg, bt, bd, 13, 9 + 40 + 6 + 4, 6)
+        s.prefill(tau, mk)
+        out = G.to_np(s.sample(40, 6, 9))
+        st, stats = s.stats()
+        s.close()
+        return out, st, stats
+    fused, st0, stats0 = run()
+    monkeypatch.setenv("TPPSD_NO_EMBED_FUSION", "1")
+    plain, st1, stats1 = run()
+    assert st0 == T.TPPSD_OK and st1 == T.TPPSD_OK
+    for k in ("tau", "t", "k"):
+        assert np.array_equal(fused[k], plain[k]), k
+    assert stats0["kernel_launches"] + stats0["loop_iters"] == stats1["kernel_launches"]
+
+
 def test_identical_draft_gives_autoregressive_output():
     tcfg, _, bt, _ = G.small_models(gain=1.5)
     tau, mk = G.hist(8, 5, 3, 1)
