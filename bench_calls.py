@@ -132,9 +132,9 @@ def main(argv=None):
         ms_ar = _time_calls(torch, ar, flush, reps=2, warm=1)
         # the draft kernel against HBM: one profiled call gives its time per
         # round; its bytes are the draft K/V it reads per round (every key of
-        # the context once per encoded position when the cache is streamed,
-        # SURVEY's "streamed" bytes; once per round when it stays in shared
-        # memory), counted by the kernel (draft_keys, per layer)
+        # the context once per encoded position when the cache is streamed;
+        # once per round when it stays in shared memory), counted by the
+        # kernel (draft_keys, per layer)
         draft = None
         if not a.poisson:
             T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
