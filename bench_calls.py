@@ -3,7 +3,7 @@ workload shape.
 
     python bench_calls.py [--workload c2] [--calls 2] [--mode sd|ar] [--host-loop]
     python bench_calls.py --time --workload c3 [--gamma 4] [--batch 16] [--draft 0]
-                          [--encoder attnhp]
+                          [--encoder attnhp] [--hist-len 4096] [--n-events 256]
 
 Builds the workload's models and histories (seeded, synthetic) and prefills.
 
@@ -17,8 +17,11 @@ are not visible to it.
 --time: TPP-SD and target-only AR events/s of the graph-launched calls
 (CUDA events, inputs resident, 2 warm-up + 3 timed calls each, L2 flushed
 before each timed call), mean accepted drafts per verify and acceptance
-rate, as one JSON line.  --gamma / --batch / --draft override the workload's
-gamma, batch and draft model (an index into the workload's draft sweep).
+rate, as one JSON line, with the draft and target-attention kernels against
+the HBM peak (from one profiled call).  --gamma / --batch / --draft override
+the workload's gamma, batch and draft model (an index into the workload's
+draft sweep); --hist-len / --n-events its history and generated lengths
+(a long history puts every round's context past that many keys).
 --poisson: the draft is the Poisson process of App. D.3, fitted by maximum
 likelihood on a pilot AR sample of the target (64 events per sequence).
 """
@@ -80,6 +83,8 @@ def main(argv=None):
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--draft", type=int, default=None)
     ap.add_argument("--poisson", action="store_true")
+    ap.add_argument("--hist-len", type=int, default=None)
+    ap.add_argument("--n-events", type=int, default=None)
     ap.add_argument("--encoder", default=None, choices=["thp", "sahp", "attnhp"],
                     help="history encoder of both models (App. D.4); default: the workload's")
     a = ap.parse_args(argv)
@@ -91,6 +96,10 @@ def main(argv=None):
         wl = wl.with_(batch=a.batch)
     if a.draft is not None:
         wl = wl.with_(draft=wl.drafts[a.draft])
+    if a.hist_len is not None:
+        wl = wl.with_(hist_len=a.hist_len)
+    if a.n_events is not None:
+        wl = wl.with_(n_events=a.n_events)
     if a.encoder is not None:
         enc = {"thp": CF.THP, "sahp": CF.SAHP, "attnhp": CF.ATTNHP}[a.encoder]
         wl = wl.with_(target=CF.ModelCfg(**{**wl.target.__dict__, "encoder": enc}),
@@ -135,13 +144,28 @@ def main(argv=None):
         # the context once per encoded position when the cache is streamed;
         # once per round when it stays in shared memory), counted by the
         # kernel (draft_keys, per layer)
-        draft = None
+        # The target's attention against HBM, from the same profiled call:
+        # K and V of every cached key once per (sequence, layer), counted by
+        # the kernels (target_keys), plus the Q rows read and the output
+        # rows written (CUDA-event time per launch, launch gap included)
+        draft = attn = None
         if not a.poisson:
             T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
             sample_call(T.TPPSD_FLAG_PROFILE)
             torch.cuda.synchronize()
             _, st_p = T.tppsd_get_stats(s.ctx)
-            kms, kn = T.tppsd_kernel_times(s.ctx).get("draft", (0.0, 0))
+            kt = T.tppsd_kernel_times(s.ctx)
+            ams, an = kt.get("attention", (0.0, 0))
+            if an:
+                tc = wl.target
+                teb = 2 if tc.dtype == CF.BF16 else 4
+                rows = st_p["rounds"] * (g + 1)
+                by = (st_p["target_keys"] + rows) * tc.layers * 2 * tc.d_model * teb
+                gbs = by / (ams / 1e3) / 1e9
+                attn = {"us_per_launch": round(1e3 * ams / an, 2), "bytes_per_launch": int(by / an),
+                        "mean_keys_per_sequence": round(st_p["target_keys"] / max(st_p["rounds"], 1), 1),
+                        "achieved_GBps": round(gbs, 1), "frac_of_hbm": round(gbs / _hbm_peak(), 4)}
+            kms, kn = kt.get("draft", (0.0, 0))
             if kn:
                 eb = 2 if wl.draft.dtype == CF.BF16 else 4
                 dcfg = wl.draft
@@ -163,7 +187,7 @@ def main(argv=None):
             "speedup_vs_ar": round(ms_ar / ms_sd, 3),
             "mean_accepted_per_verify": round(st_sd["accepted"] / max(st_sd["rounds"], 1), 3),
             "alpha": round(st_sd["accepted"] / max(st_sd["drafted"], 1), 4),
-            "rounds": st_sd["loop_iters"], "draft_kernel": draft,
+            "rounds": st_sd["loop_iters"], "draft_kernel": draft, "attention_kernel": attn,
             "note": "prefill included in both timed calls"}), flush=True)
         s.close()
         return 0
