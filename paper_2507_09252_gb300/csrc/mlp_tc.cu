@@ -67,6 +67,9 @@ __device__ __forceinline__ void st_swizzled16(unsigned char* tiles, int t, int c
 __device__ __forceinline__ void epi_sync() {  // the 256 epilogue threads only
     asm volatile("bar.sync 1, 256;" ::: "memory");
 }
+__device__ __forceinline__ void epi_sync512() {  // the cluster form's 512 epilogue threads
+    asm volatile("bar.sync 1, 512;" ::: "memory");
+}
 
 __global__ void __launch_bounds__(320, 1)
     k_mlp_tc(const __grid_constant__ CUtensorMap mapAtt, const __grid_constant__ CUtensorMap mapWo,
@@ -366,7 +369,10 @@ __global__ void __launch_bounds__(320, 1)
 // applies LN2 and writes them.  The dependent chain of one CTA is
 // thus one FFN1 chunk and one FFN2 chunk instead of F / 128 of each, and
 // the weights a CTA streams drop to W_o plus 1/n of W_1 and W_2 (six tiles,
-// all in flight at once).  TMEM: 0-127 the output projection, then the
+// all in flight at once).  Eighteen warps: sixteen epilogue warps (warp w
+// reads TMEM lanes 32 (w % 4).. and takes 32 of its rows' 128 columns, so
+// each element-wise phase is a quarter row per thread), a producer warp
+// (TMA) and an MMA warp.  TMEM: 0-127 the output projection, then the
 // FFN2 partial; 128-255 the FFN1 chunk; 256-383 x1 in fp32; 384.. the next
 // layer's Q, K, V slice.
 //
@@ -389,7 +395,10 @@ struct MlpClShape {
     static constexpr int OFF_W = OFF_R + R_BYTES;
     static constexpr int OFF_P = OFF_W + NT * TILE;        // b_o g1 be1 b_2 g2 be2 (D each), b_1 chunk
     static constexpr int OFF_RED = OFF_P + (6 * D + CH) * 4;
-    static constexpr int OFF_B = OFF_RED + 4 * BM * 4;
+    static constexpr int OFF_B = OFF_RED + 8 * BM * 4;     // LN1 partials: [sum, centred squares][4][BM]
+    // sixteen epilogue warps (lane quarter q = warp % 4, column quarter
+    // warp / 4: 32 columns per thread), then the producer and MMA warps
+    static constexpr int EW = 16, ET = 32 * EW, CW = D / (EW / 4), THREADS = 32 * (EW + 2);
     static constexpr int NBAR = 18;
     __host__ __device__ static constexpr int SLICE_BYTES(int ncl) { return (BM / ncl) * RLD * 4; }
     static_assert(NT * TILE >= BM * RLD * 4, "the partial slices fit in the weight region");
@@ -399,6 +408,7 @@ struct MlpClShape {
     __host__ __device__ static constexpr bool QKV_OK(int ncl) { return ncl == 4 || ncl == 8; }
     static constexpr size_t SMEM = (size_t)OFF_Q + 2 * 96 * 128 + 1024;  // room for NQ <= 96
     static_assert(R_BYTES >= 2 * TILE, "the activation tile fits in the residual region");
+    static_assert(SMEM <= 227 * 1024, "shared memory");
     static_assert(SMEM <= 227 * 1024, "shared memory");
 };
 
@@ -416,8 +426,18 @@ __device__ __forceinline__ void st_swizzled8(unsigned char* tiles, int t, int c0
     *reinterpret_cast<uint4*>(row + ((ch ^ (t & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+// 4 consecutive columns c0.. (c0 % 4 == 0) of row t, the same layout.
+__device__ __forceinline__ void st_swizzled4(unsigned char* tiles, int t, int c0, const float* v) {
+    const __nv_bfloat162 p0 = __floats2bfloat162_rn(v[0], v[1]);
+    const __nv_bfloat162 p1 = __floats2bfloat162_rn(v[2], v[3]);
+    const int kb = c0 >> 6, ch = (c0 & 63) >> 3;
+    unsigned char* row = tiles + kb * MlpShape::TILE + t * 128;
+    *reinterpret_cast<uint2*>(row + ((ch ^ (t & 7)) << 4) + (c0 & 4) * 2) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&p0), *reinterpret_cast<const uint32_t*>(&p1));
+}
+
 template <int NCL>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(MlpClShape::THREADS, 1)
     k_mlp_cl(const __grid_constant__ CUtensorMap mapAtt, const __grid_constant__ CUtensorMap mapWo,
              const __grid_constant__ CUtensorMap mapW1, const __grid_constant__ CUtensorMap mapW2,
              const __grid_constant__ CUtensorMap mapWq, MlpArgs a) {
@@ -438,18 +458,19 @@ __global__ void __launch_bounds__(320, 1)
     uint64_t* full = bars;            // [NT] weight tile i landed
     uint64_t* abar = bars + 6;        // attention tile landed
     uint64_t* o_done = bars + 7;      // output projection in TMEM
-    uint64_t* x1_ready = bars + 8;    // x1 operand written (256 arrivals)
+    uint64_t* x1_ready = bars + 8;    // x1 operand written (ET arrivals)
     uint64_t* h_done = bars + 9;      // FFN1 chunk in TMEM
-    uint64_t* e2_done = bars + 10;    // chunk activations written (256 arrivals)
+    uint64_t* e2_done = bars + 10;    // chunk activations written (ET arrivals)
     uint64_t* y_done = bars + 11;     // FFN2 partial in TMEM
     uint64_t* rbar = bars + 12;       // the other CTAs' partial slices landed
     uint64_t* wqbar = bars + 13;      // next layer's W_qkv columns landed
-    uint64_t* qa_local = bars + 14;   // this CTA's rows written into the A tile (256 arrivals)
+    uint64_t* qa_local = bars + 14;   // this CTA's rows written into the A tile (ET arrivals)
     uint64_t* qa_remote = bars + 15;  // the other CTAs' rows landed in the A tile
     uint64_t* q_done = bars + 16;     // next layer's Q, K, V slice in TMEM
     uint32_t* tslot = (uint32_t*)(bars + 17);
     unsigned char* Wq = smem + S::OFF_Q;
     constexpr int NQ = S::NQ(NCL), RW = S::BM / NCL;
+    constexpr int ET = S::ET, CW = S::CW, WP = S::EW, WM = S::EW + 1;  // producer, MMA warps
     const bool qkv = S::QKV_OK(NCL) && a.qkv;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int c = (int)cluster_ctarank();
@@ -459,13 +480,13 @@ __global__ void __launch_bounds__(320, 1)
         for (int i = 0; i < S::NT; ++i) mbar_init(&full[i], 1);
         mbar_init(abar, 1);
         mbar_init(o_done, 1);
-        mbar_init(x1_ready, 256);
+        mbar_init(x1_ready, ET);
         mbar_init(h_done, 1);
-        mbar_init(e2_done, 256);
+        mbar_init(e2_done, ET);
         mbar_init(y_done, 1);
         mbar_init(rbar, 1);
         mbar_init(wqbar, 1);
-        mbar_init(qa_local, 256);
+        mbar_init(qa_local, ET);
         mbar_init(qa_remote, 1);
         mbar_init(q_done, 1);
         mbar_fence_init();
@@ -476,7 +497,7 @@ __global__ void __launch_bounds__(320, 1)
     tc_fence_after();
     const uint32_t tmem = *tslot;
 
-    if (warp == 8) {
+    if (warp == WP) {
         if (lane == 0) {  // every tile of this CTA at once: nothing is reused
             const CUtensorMap* maps[S::NT] = {&mapWo, &mapWo, &mapW1, &mapW1, &mapW2, &mapW2};
             const int xs[S::NT] = {0, 64, 0, 64, c * S::CH, c * S::CH + 64};
@@ -498,7 +519,7 @@ __global__ void __launch_bounds__(320, 1)
             tma_load_2d(A + S::TILE, &mapAtt, abar, 64, m0);
         }
         __syncwarp();
-    } else if (warp == 9) {
+    } else if (warp == WM) {
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16(128, 128);
             bool ok = true;
@@ -531,109 +552,112 @@ __global__ void __launch_bounds__(320, 1)
         }
         __syncwarp();
     } else {
-        // epilogue warps 0-7: row t = 32 (warp % 4) + lane, columns cb..cb+63
-        const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * 64;
+        // epilogue warps 0-15: row t = 32 (warp % 4) + lane, columns cb..cb+CW-1
+        const int tid = threadIdx.x, q = warp & 3, hh = warp >> 2, t = q * 32 + lane, cb = hh * CW;
         const bool live = t < rows;
         {   // parameters, then (after the wait) the residual tile; all loads
             // issued before any store
             const float* src[6] = {a.b_o, a.ln1_g, a.ln1_b, a.b_2, a.ln2_g, a.ln2_b};
-            float pv[3];
+            constexpr int NP = (6 * D + ET - 1) / ET;
+            float pv[NP];
 #pragma unroll
-            for (int k = 0; k < 3; ++k) {
-                const int i = tid + 256 * k;
-                pv[k] = src[i / D][i % D];
+            for (int k = 0; k < NP; ++k) {
+                const int i = tid + ET * k;
+                pv[k] = i < 6 * D ? src[i / D][i % D] : 0.f;
             }
             const float b1v = tid < S::CH ? a.b_1[c * S::CH + tid] : 0.f;
             pdl_wait();
-            constexpr int NV = S::BM * D / 4 / 256;
+            constexpr int NV = S::BM * D / 4 / ET;
             float4 v[NV];
 #pragma unroll
             for (int k = 0; k < NV; ++k) {
-                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                const int f = tid + ET * k, r = f >> 5, c4 = f & 31;
                 v[k] = r < rows ? *reinterpret_cast<const float4*>(a.x + (size_t)(m0 + r) * D + 4 * c4)
                                 : make_float4(0.f, 0.f, 0.f, 0.f);
             }
 #pragma unroll
             for (int k = 0; k < NV; ++k) {
-                const int f = tid + 256 * k, r = f >> 5, c4 = f & 31;
+                const int f = tid + ET * k, r = f >> 5, c4 = f & 31;
                 *reinterpret_cast<float4*>(res + r * S::RLD + 4 * c4) = v[k];
             }
 #pragma unroll
-            for (int k = 0; k < 3; ++k) prm[tid + 256 * k] = pv[k];
+            for (int k = 0; k < NP; ++k)
+                if (tid + ET * k < 6 * D) prm[tid + ET * k] = pv[k];
             if (tid < S::CH) prm[6 * D + tid] = b1v;
         }
-        epi_sync();
+        epi_sync512();
         const float *p_bo = prm + cb, *p_g1 = prm + D + cb, *p_be1 = prm + 2 * D + cb, *p_b2 = prm + 3 * D + cb;
         const float* p_b1 = prm + 6 * D + cb;
         const uint32_t tl = tmem + ((uint32_t)(q * 32) << 16);
         float* xr = res + t * S::RLD + cb;
-        float y[64];
+        float y[CW];
         mbar_wait(o_done, 0, a.err, 65);
         tc_fence_after();
-        tmem_ld64(tl + cb, y);
+        tmem_ld32(tl + cb, y);
 #pragma unroll
-        for (int cc = 0; cc < 64; cc += 4) {
+        for (int cc = 0; cc < CW; cc += 4) {
             const float4 r4 = *reinterpret_cast<const float4*>(xr + cc);
             y[cc] += p_bo[cc] + r4.x;
             y[cc + 1] += p_bo[cc + 1] + r4.y;
             y[cc + 2] += p_bo[cc + 2] + r4.z;
             y[cc + 3] += p_bo[cc + 3] + r4.w;
         }
-        {   // LN1 (row halves held by the thread pairs hh = 0 / 1)
+        {   // LN1 (row quarters held by the four warps of lane quarter q)
             float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-            for (int cc = 0; cc < 64; cc += 4) {
+            for (int cc = 0; cc < CW; cc += 4) {
                 s0 += y[cc];
                 s1 += y[cc + 1];
                 s2 += y[cc + 2];
                 s3 += y[cc + 3];
             }
             red[hh * S::BM + t] = (s0 + s1) + (s2 + s3);
-            epi_sync();
-            const float mean = (red[t] + red[S::BM + t]) / D;
+            epi_sync512();
+            const float mean = ((red[t] + red[S::BM + t]) + (red[2 * S::BM + t] + red[3 * S::BM + t])) / D;
             s0 = s1 = s2 = s3 = 0.f;
 #pragma unroll
-            for (int cc = 0; cc < 64; cc += 4) {
+            for (int cc = 0; cc < CW; cc += 4) {
                 s0 = fmaf(y[cc] - mean, y[cc] - mean, s0);
                 s1 = fmaf(y[cc + 1] - mean, y[cc + 1] - mean, s1);
                 s2 = fmaf(y[cc + 2] - mean, y[cc + 2] - mean, s2);
                 s3 = fmaf(y[cc + 3] - mean, y[cc + 3] - mean, s3);
             }
-            red[(2 + hh) * S::BM + t] = (s0 + s1) + (s2 + s3);
-            epi_sync();  // also ends every read of the residual tile
-            const float inv = 1.0f / sqrtf((red[2 * S::BM + t] + red[3 * S::BM + t]) / D + LN_EPS);
+            red[(4 + hh) * S::BM + t] = (s0 + s1) + (s2 + s3);
+            epi_sync512();  // also ends every read of the residual tile
+            const float var = ((red[4 * S::BM + t] + red[5 * S::BM + t]) + (red[6 * S::BM + t] + red[7 * S::BM + t])) / D;
+            const float inv = 1.0f / sqrtf(var + LN_EPS);
 #pragma unroll
-            for (int cc = 0; cc < 64; ++cc) y[cc] = live ? (y[cc] - mean) * inv * p_g1[cc] + p_be1[cc] : 0.f;
+            for (int cc = 0; cc < CW; ++cc) y[cc] = live ? (y[cc] - mean) * inv * p_g1[cc] + p_be1[cc] : 0.f;
         }
-        tmem_st64(tl + 256 + cb, y);
+        tmem_st32(tl + 256 + cb, y);
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(A, t, cb + c0, y + c0);
+        for (int c0 = 0; c0 < CW; c0 += 16) st_swizzled16(A, t, cb + c0, y + c0);
         fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(x1_ready);
         // FFN1 chunk c: ReLU(H + b_1) -> bf16 operand of FFN2 (residual region)
         mbar_wait(h_done, 0, a.err, 66);
         tc_fence_after();
-        tmem_ld64(tl + 128 + cb, y);
+        tmem_ld32(tl + 128 + cb, y);
 #pragma unroll
-        for (int cc = 0; cc < 64; ++cc) y[cc] = fmaxf(y[cc] + p_b1[cc], 0.f);
+        for (int cc = 0; cc < CW; ++cc) y[cc] = fmaxf(y[cc] + p_b1[cc], 0.f);
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 16) st_swizzled16(Rg, t, cb + c0, y + c0);
+        for (int c0 = 0; c0 < CW; c0 += 16) st_swizzled16(Rg, t, cb + c0, y + c0);
         fence_proxy_async_smem();
         tc_fence_before();
         mbar_arrive(e2_done);
         // this CTA's FFN2 partial (CTA 0: + b_2 + x1) into the residual region
         mbar_wait(y_done, 0, a.err, 67);
         tc_fence_after();
-        tmem_ld64(tl + cb, y);
+        tmem_ld32(tl + cb, y);
         if (c == 0) {
-            float x1[64];
-            tmem_ld64(tl + 256 + cb, x1);
+            float x1[CW];
+            tmem_ld32(tl + 256 + cb, x1);
 #pragma unroll
-            for (int cc = 0; cc < 64; ++cc) y[cc] += p_b2[cc] + x1[cc];
+            for (int cc = 0; cc < CW; ++cc) y[cc] += p_b2[cc] + x1[cc];
         }
 #pragma unroll
-        for (int cc = 0; cc < 64; cc += 4)
+        for (int cc = 0; cc < CW; cc += 4)
             *reinterpret_cast<float4*>(xr + cc) = make_float4(y[cc], y[cc + 1], y[cc + 2], y[cc + 3]);
         fence_proxy_async_smem();  // the bulk copies below read these writes
     }
@@ -648,9 +672,9 @@ __global__ void __launch_bounds__(320, 1)
                             (uint32_t)S::SLICE_BYTES(NCL), rbar, (uint32_t)p);
         bulk_commit();
     }
-    if (warp < 8) {
+    if (warp < S::EW) {
         // rows c RW .. c RW + RW - 1 of the tile: TPR threads per row, CPT columns each
-        constexpr int RW = S::BM / NCL, TPR = 256 / RW, CPT = D / TPR;
+        constexpr int RW = S::BM / NCL, TPR = ET / RW, CPT = D / TPR;
         const int tid = threadIdx.x, rr = tid / TPR, col = (tid % TPR) * CPT, r = c * RW + rr;
         const float *p_g2 = prm + 4 * D, *p_be2 = prm + 5 * D;
         // slice of CTA pr: this CTA's own partial for pr = c, else slot pr
@@ -696,6 +720,7 @@ __global__ void __launch_bounds__(320, 1)
                 o[j] = r < rows ? (v[j] - mean) * inv * p_g2[col + j] + p_be2[col + j] : 0.f;
             if constexpr (CPT == 16) st_swizzled16(A, r, col, o);
             else if constexpr (CPT == 8) st_swizzled8(A, r, col, o);
+            else if constexpr (CPT == 4) st_swizzled4(A, r, col, o);
             fence_proxy_async_smem();
             mbar_arrive(qa_local);
         }
@@ -729,7 +754,7 @@ __global__ void __launch_bounds__(320, 1)
                         bulk_s2peer(blk, blk, (uint32_t)(RW * 128), qa_remote, (uint32_t)p);
                     }
             bulk_commit();
-        } else if (warp == 9 && lane == 0) {
+        } else if (warp == WM && lane == 0) {
             bool ok = mbar_wait(wqbar, 0, a.err, 70);
             ok = ok && mbar_wait(qa_local, 0, a.err, 71);
             ok = ok && mbar_wait(qa_remote, 0, a.err, 72);
@@ -747,7 +772,8 @@ __global__ void __launch_bounds__(320, 1)
         __syncwarp();
         if (warp < 8) {
             // rows t = 32 (warp % 4) + lane; the column halves of the slice by
-            // warps 0-3 / 4-7 when they split into 16-column groups
+            // warps 0-3 / 4-7 when they split into 16-column groups (warps
+            // 8-15 have no part here)
             constexpr int HALF = (NQ / 2) % 16 == 0 ? NQ / 2 : NQ;
             const int q = warp & 3, hh = warp >> 2, t = q * 32 + lane, r = m0 + t;
             const bool ok = mbar_wait(q_done, 0, a.err, 73);
@@ -796,7 +822,7 @@ static cudaError_t launch_mlp_ncl(const CUtensorMap& att, const CUtensorMap& wo,
     const int ncl = NCL;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(ncl, (a.R + 127) / 128, 1);
-    cfg.blockDim = dim3(320, 1, 1);
+    cfg.blockDim = dim3(MlpClShape::THREADS, 1, 1);
     cfg.dynamicSmemBytes = sm;
     cfg.stream = st;
     cudaLaunchAttribute at[2];
