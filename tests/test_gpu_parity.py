@@ -292,6 +292,30 @@ def test_folded_qkv_is_bit_identical(monkeypatch):
     assert stats0["kernel_launches"] > stats1["kernel_launches"]
 
 
+def test_folded_qkv_is_bit_identical_eight_ctas(monkeypatch):
+    """The folded QKV GEMM with an eight-CTA cluster (d = 128, F = 1024:
+    each CTA finishes 16 rows, four columns per thread) against the
+    separate GEMM: bit-identical sampled sequences."""
+    tcfg = CF.ModelCfg(2, 128, 4, 1024, 8, 5, CF.BF16)
+    dcfg = CF.ModelCfg(1, 32, 2, 128, 8, 5, CF.BF16)
+    bt, bd = IN.model_blob(tcfg, 4, 0), IN.model_blob(dcfg, 4, 1)
+    tau, mk = G.hist(10, 30, 5, 3)
+    def run():
+        s = G.make_sampler(tcfg, dcfg, bt, bd, 10, 30 + 40 + 8 + 4, 8)
+        s.prefill(tau, mk)
+        out = G.to_np(s.sample(40, 8, 5))
+        st, stats = s.stats()
+        s.close()
+        return out, st, stats
+    base, st0, stats0 = run()
+    monkeypatch.setenv("TPPSD_QKV_FOLD", "1")
+    fold, st1, stats1 = run()
+    assert st0 == T.TPPSD_OK and st1 == T.TPPSD_OK
+    for k in ("tau", "t", "k"):
+        assert np.array_equal(base[k], fold[k]), k
+    assert stats0["kernel_launches"] > stats1["kernel_launches"]
+
+
 @pytest.mark.parametrize("dtype", [CF.FP32, CF.BF16])
 def test_fused_verify_rows_are_bit_identical(dtype, monkeypatch):
     """The lane draft kernel writes the target's verify rows (the embedding
