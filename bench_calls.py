@@ -66,6 +66,16 @@ def _hbm_peak():
         return 6800.0
 
 
+def attention_roofline(ms, launches, stats, wl):
+    """The target attention class of one profiled call against the HBM
+    peak, by bench.py's per-class formula."""
+    import bench
+    r = bench.class_roofline("attention", ms, launches, stats, wl, {"hbm_gbs": _hbm_peak()}, False)
+    return {"us_per_launch": round(1e3 * ms / launches, 2), "bytes_per_launch": int(r["algorithmic_per_launch"]),
+            "mean_keys_per_sequence": round(stats["target_keys"] / max(stats["rounds"], 1), 1),
+            "achieved_GBps": r["achieved"], "frac_of_hbm": r["frac"]}
+
+
 def _shape(cfg, fields):
     return " ".join(f"{n}{getattr(cfg, f)}" for n, f in fields)
 
@@ -144,10 +154,11 @@ def main(argv=None):
         # the context once per encoded position when the cache is streamed;
         # once per round when it stays in shared memory), counted by the
         # kernel (draft_keys, per layer)
-        # The target's attention against HBM, from the same profiled call:
-        # K and V of every cached key once per (sequence, layer), counted by
-        # the kernels (target_keys), plus the Q rows read and the output
-        # rows written (CUDA-event time per launch, launch gap included)
+        # The target's attention against HBM, from the same profiled call,
+        # by bench.py's formula: K and V of every cached key once per
+        # (sequence, layer), counted by the kernels (target_keys), plus the
+        # Q rows read and the output rows written (CUDA-event time per
+        # launch, launch gap included)
         draft = attn = None
         if not a.poisson:
             T.tppsd_prefill(s.ctx, B, tau, mk, H, st)
@@ -157,14 +168,7 @@ def main(argv=None):
             kt = T.tppsd_kernel_times(s.ctx)
             ams, an = kt.get("attention", (0.0, 0))
             if an:
-                tc = wl.target
-                teb = 2 if tc.dtype == CF.BF16 else 4
-                rows = st_p["rounds"] * (g + 1)
-                by = (st_p["target_keys"] + rows) * tc.layers * 2 * tc.d_model * teb
-                gbs = by / (ams / 1e3) / 1e9
-                attn = {"us_per_launch": round(1e3 * ams / an, 2), "bytes_per_launch": int(by / an),
-                        "mean_keys_per_sequence": round(st_p["target_keys"] / max(st_p["rounds"], 1), 1),
-                        "achieved_GBps": round(gbs, 1), "frac_of_hbm": round(gbs / _hbm_peak(), 4)}
+                attn = attention_roofline(ams, an, st_p, wl)
             kms, kn = kt.get("draft", (0.0, 0))
             if kn:
                 eb = 2 if wl.draft.dtype == CF.BF16 else 4

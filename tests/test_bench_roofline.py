@@ -62,3 +62,17 @@ def test_path_roofline():
     assert 0.05 < pr["frac"] < 0.3
     att = per["attention"]
     assert att["algorithmic_per_launch"] * 280 / (att["peak"] * 1e9) * 1e3 > 0.5 * pr["ideal_ms"]
+
+
+def test_bench_calls_attention_figure_and_length_overrides():
+    """bench_calls' attention figure is bench.py's attention class (one
+    formula), and --hist-len / --n-events reshape the workload so that a
+    long history puts every round's context past that many keys."""
+    import bench_calls
+    r = bench_calls.attention_roofline(5.167, 280, STATS, CF.C2)
+    _, per = bench.roofline(KT, STATS, CF.C2, {"hbm_gbs": bench_calls._hbm_peak(), "bf16_tflops_sustained": 1772.7})
+    assert r["achieved_GBps"] == pytest.approx(per["attention"]["achieved"], rel=1e-6)
+    assert r["bytes_per_launch"] == int(per["attention"]["algorithmic_per_launch"])
+    assert r["mean_keys_per_sequence"] == pytest.approx(STATS["target_keys"] / STATS["rounds"], abs=0.05)
+    wl = CF.C4.with_(hist_len=4096, n_events=256)
+    assert (wl.hist_len, wl.n_events, wl.batch, wl.gamma) == (4096, 256, CF.C4.batch, CF.C4.gamma)
